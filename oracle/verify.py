@@ -161,9 +161,11 @@ def _spectr_step(rec, q, dists, X, seed, b, j):
 
 
 def verify_sequence(b, target_logits, draft_logits, draft_model_id, draft_tokens, temperatures,
-                    scheme, seed, wis_s=5, is_h=0.25):
-    """Walk sequence b.  Returns (tokens [L+1] with -1 padding, accept_len,
-    list of DepthRecord)."""
+                    scheme, seed, wis_s=5, is_h=0.25, draw_id=None):
+    """Walk the sequence stored at index b of the arrays; its Philox draws use
+    sequence id ``draw_id`` (default b).  Returns (tokens [L+1] with -1
+    padding, accept_len, list of DepthRecord)."""
+    sid = b if draw_id is None else int(draw_id)
     K = target_logits.shape[1]
     L = draft_tokens.shape[2]
     out = np.full(L + 1, -1, dtype=np.int64)
@@ -184,20 +186,20 @@ def verify_sequence(b, target_logits, draft_logits, draft_model_id, draft_tokens
         dists = [rows[int(draft_model_id[k])] for k in valid]
         if scheme == "single":
             Y, pI = X[0], dists[0]
-            Z = _speculative_step(rec, q, pI, Y, philox.uniform(seed, b, j, DRAW_ACCEPT),
-                                  philox.uniform(seed, b, j, DRAW_RESIDUAL))
+            Z = _speculative_step(rec, q, pI, Y, philox.uniform(seed, sid, j, DRAW_ACCEPT),
+                                  philox.uniform(seed, sid, j, DRAW_RESIDUAL))
         elif scheme == "IS":
             mids = [int(draft_model_id[k]) for k in valid]
-            Y, pI = is_laplace.is_select(rec, q, rows, mids, X, philox.uniform(seed, b, j, DRAW_SELECT), is_h)
-            Z = _speculative_step(rec, q, pI, Y, philox.uniform(seed, b, j, DRAW_ACCEPT),
-                                  philox.uniform(seed, b, j, DRAW_RESIDUAL))
+            Y, pI = is_laplace.is_select(rec, q, rows, mids, X, philox.uniform(seed, sid, j, DRAW_SELECT), is_h)
+            Z = _speculative_step(rec, q, pI, Y, philox.uniform(seed, sid, j, DRAW_ACCEPT),
+                                  philox.uniform(seed, sid, j, DRAW_RESIDUAL))
         elif scheme == "WIS":
-            us = [philox.uniform(seed, b, j, DRAW_SELECT + m) for m in range(max(0, len(X) - 1))]
+            us = [philox.uniform(seed, sid, j, DRAW_SELECT + m) for m in range(max(0, len(X) - 1))]
             Y, pI = wis_mod.wis_select(rec, q, dists, X, us, wis_s)
-            Z = _speculative_step(rec, q, pI, Y, philox.uniform(seed, b, j, DRAW_ACCEPT),
-                                  philox.uniform(seed, b, j, DRAW_RESIDUAL))
+            Z = _speculative_step(rec, q, pI, Y, philox.uniform(seed, sid, j, DRAW_ACCEPT),
+                                  philox.uniform(seed, sid, j, DRAW_RESIDUAL))
         elif scheme == "SpecTr":
-            Z = _spectr_step(rec, q, dists, X, seed, b, j)
+            Z = _spectr_step(rec, q, dists, X, seed, sid, j)
         else:
             raise ValueError(f"unknown scheme {scheme!r}")
         rec.Z = int(Z)
@@ -211,7 +213,7 @@ def verify_sequence(b, target_logits, draft_logits, draft_model_id, draft_tokens
     rec = DepthRecord(L)
     records.append(rec)
     q = softmax_t(target_logits[b, valid[0], L], temperatures[b, 0])
-    z, m = inverse_cdf(q, philox.uniform(seed, b, L, DRAW_BONUS))
+    z, m = inverse_cdf(q, philox.uniform(seed, sid, L, DRAW_BONUS))
     rec.note("cdf", m, BAND_CDF)
     rec.Z = int(z)
     out[L] = z
@@ -219,7 +221,7 @@ def verify_sequence(b, target_logits, draft_logits, draft_model_id, draft_tokens
 
 
 def oracle_verify(target_logits, draft_logits, draft_model_id, draft_tokens, temperatures,
-                  scheme, seed, wis_s=5, is_h=0.25, seqs=None):
+                  scheme, seed, wis_s=5, is_h=0.25, seqs=None, seq_ids=None):
     """Oracle over a batch.
 
     target_logits  [B, K, L+1, V] (any real dtype; upcast exactly to fp64)
@@ -228,18 +230,30 @@ def oracle_verify(target_logits, draft_logits, draft_model_id, draft_tokens, tem
     draft_tokens   [B, K, L] ints
     temperatures   [B, 1+K] (target, then per branch)
     seqs           optional iterable of sequence indices to evaluate
+    seq_ids        optional global sequence ids of the B stored sequences (a
+                   sample of a larger batch); Philox draws use these ids and
+                   the results are keyed by them
 
-    Returns (out_tokens [B, L+1], accept_len [B], records {b: [DepthRecord]});
-    rows of sequences not in ``seqs`` are left at -1."""
+    Returns (out_tokens, accept_len, records {id: [DepthRecord]}).  Without
+    seq_ids the arrays are [B, L+1] and [B] and rows of sequences not in
+    ``seqs`` are -1; with seq_ids they are dicts keyed by the global id."""
     target_logits = np.asarray(target_logits)
     B, K = target_logits.shape[0], target_logits.shape[1]
     L = np.asarray(draft_tokens).shape[2]
     out = np.full((B, L + 1), -1, dtype=np.int64)
     acc = np.full(B, -1, dtype=np.int64)
     recs = {}
+    temps = np.asarray(temperatures, dtype=np.float64)
+    if seq_ids is not None:
+        out_d, acc_d = {}, {}
+        for i, sid in enumerate(seq_ids):
+            o, a, r = verify_sequence(i, target_logits, draft_logits, draft_model_id, draft_tokens, temps,
+                                      scheme, seed, wis_s, is_h, draw_id=sid)
+            out_d[int(sid)], acc_d[int(sid)], recs[int(sid)] = o, a, r
+        return out_d, acc_d, recs
     for b in (range(B) if seqs is None else seqs):
         o, a, r = verify_sequence(b, target_logits, draft_logits, draft_model_id, draft_tokens,
-                                  np.asarray(temperatures, dtype=np.float64), scheme, seed, wis_s, is_h)
+                                  temps, scheme, seed, wis_s, is_h)
         out[b] = o
         acc[b] = a
         recs[b] = r

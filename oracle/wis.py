@@ -38,16 +38,22 @@ K > 2 drafts (Remark 4): stage 1 pairs (X_1, X_2) -> Y_1, stage m pairs
 (Y_{m-1}, X_{m+1}) -> Y_m, with a = law of Y_{m-1} and b = law of X_{m+1};
 every stage maximises against the same target q (reading).
 
-Augmenting-path order.  Omega_1 is indexed by increasing token id.  Pairs
-are indexed lexicographically over index pairs (i, j), i < j; side 0 of a
-pair is its lower index.  A breadth-first search starts from every pair with
-remaining supply > eps in pair order; dequeuing a pair visits its side-0 then
-side-1 token; dequeuing a token ends the search if its remaining demand is
-> eps, else it visits, in pair order, every unvisited pair through which flow
-> eps reaches this token (the reverse edge).  The path's bottleneck is the
-minimum of the first pair's remaining supply, the last token's remaining
-demand and the reverse-edge flows on the way; it is pushed and the search
-repeats until no path exists.
+Flow order (reading; any maximum flow is an LP optimum).  Omega_1 is indexed
+by increasing token id; pair (i, j), i < j, are taken lexicographically.
+(a) Direct pass: each pair in order gives what it can to its lower-index
+    token, then to its higher-index token (each while both the pair's supply
+    and the token's remaining demand exceed eps).
+(b) Augmenting paths in token space: a token is a source if some pair
+    containing it has supply > eps (its source pair: the first such pair);
+    token u leads to token v if pair {u, v} currently gives flow > eps to u
+    (that flow can be moved to v).  Breadth-first from all sources, level by
+    level, tokens in increasing index within a level, each token's parent the
+    first frontier token (increasing index) that reaches it; the path ends at
+    the first token in that order whose remaining demand exceeds eps.  The
+    bottleneck (source pair supply, moved flows, end demand) is pushed and
+    the search repeats until no path exists.
+(c) Pair mass left over is split 1/2 - 1/2.
+Residuals at or below eps = 1e-6 * sum_{Omega_1}(q_k + base_k) count as zero.
 """
 import numpy as np
 
@@ -65,77 +71,78 @@ class Stage:
 
 
 def _max_flow(d, m_pairs, ends, eps, note):
-    """Breadth-first augmenting paths on the pair/token graph (order in the
-    module docstring).  Returns (flow [P][2], remaining supply [P])."""
+    """Maximum flow on the pair/token network in the fixed order of the
+    module docstring.  Returns (flow [P][2] to (lower, higher) token,
+    remaining supply [P])."""
     P = len(m_pairs)
     n = len(d)
     rs = np.array(m_pairs, dtype=np.float64)
     rd = np.array(d, dtype=np.float64)
     f = np.zeros((P, 2), dtype=np.float64)
-    pairs_of = [[] for _ in range(n)]
+    pair_of = {}
     for e, (i, j) in enumerate(ends):
-        pairs_of[i].append((e, 0))
-        pairs_of[j].append((e, 1))
+        pair_of[(i, j)] = e
+        pair_of[(j, i)] = e
 
     def pos(val):
         note("lp", abs(val - eps), BAND_LP * eps)
         return val > eps
 
-    for _ in range(LP_MAX_AUGMENT):
-        seen_pair = [False] * P
-        seen_tok = [False] * n
-        parent_tok = [None] * n      # (pair e, side) through which token was reached
-        parent_pair = [None] * P     # None: from the source; else token index (reverse edge)
-        queue = []
-        for e in range(P):
-            if pos(rs[e]):
-                seen_pair[e] = True
-                queue.append(("p", e))
-        sink_tok = -1
-        head = 0
-        while head < len(queue):
-            kind, v = queue[head]
-            head += 1
-            if kind == "p":
-                for side in (0, 1):
-                    t = ends[v][side]
-                    if not seen_tok[t]:
-                        seen_tok[t] = True
-                        parent_tok[t] = (v, side)
-                        queue.append(("t", t))
-            else:
-                if pos(rd[v]):
-                    sink_tok = v
-                    break
-                for e, side in pairs_of[v]:
-                    if not seen_pair[e] and pos(f[e, side]):
-                        seen_pair[e] = True
-                        parent_pair[e] = v
-                        queue.append(("p", e))
-        if sink_tok < 0:
-            return f, rs
-        # trace the path back to the source and find the bottleneck
-        steps = []   # (pair e, side entered, side left or None)
-        t = sink_tok
-        delta = rd[t]
-        while True:
-            e, side = parent_tok[t]
-            back = parent_pair[e]
-            if back is None:
-                steps.append((e, side, None))
-                delta = min(delta, rs[e])
-                break
-            back_side = 0 if ends[e][0] == back else 1
-            steps.append((e, side, back_side))
-            delta = min(delta, f[e, back_side])
-            t = back
-        for e, side, back_side in steps:
-            f[e, side] += delta
-            if back_side is None:
+    # (a) direct pass
+    for e, (i, j) in enumerate(ends):
+        for side, t in ((0, i), (1, j)):
+            if pos(rs[e]) and pos(rd[t]):
+                delta = min(rs[e], rd[t])
+                f[e, side] += delta
                 rs[e] -= delta
-            else:
-                f[e, back_side] -= delta
-        rd[sink_tok] -= delta
+                rd[t] -= delta
+    # (b) augmenting paths in token space
+    for _ in range(LP_MAX_AUGMENT):
+        src_pair = [-1] * n
+        for e, (i, j) in enumerate(ends):
+            if pos(rs[e]):
+                for t in (i, j):
+                    if src_pair[t] < 0:
+                        src_pair[t] = e
+        parent = [-1] * n
+        visited = [src_pair[t] >= 0 for t in range(n)]
+        frontier = [t for t in range(n) if visited[t]]
+        sink = next((t for t in frontier if pos(rd[t])), -1)
+        while sink < 0 and frontier:
+            nxt = []
+            for u in frontier:
+                for v in range(n):
+                    if v == u or visited[v] or v in nxt:
+                        continue
+                    e = pair_of[(u, v)]
+                    side_u = 0 if ends[e][0] == u else 1
+                    if pos(f[e, side_u]):
+                        parent[v] = u
+                        nxt.append(v)
+            nxt.sort()
+            for v in nxt:
+                visited[v] = True
+            frontier = nxt
+            sink = next((t for t in frontier if pos(rd[t])), -1)
+        if sink < 0:
+            return f, rs
+        # path sink <- ... <- t0 (a source); bottleneck
+        path = [sink]
+        while parent[path[-1]] >= 0:
+            path.append(parent[path[-1]])
+        path.reverse()
+        e0 = src_pair[path[0]]
+        delta = min(rs[e0], rd[sink])
+        for u, v in zip(path[:-1], path[1:]):
+            e = pair_of[(u, v)]
+            delta = min(delta, f[e, 0 if ends[e][0] == u else 1])
+        rs[e0] -= delta
+        f[e0, 0 if ends[e0][0] == path[0] else 1] += delta
+        for u, v in zip(path[:-1], path[1:]):
+            e = pair_of[(u, v)]
+            f[e, 0 if ends[e][0] == u else 1] -= delta
+            f[e, 0 if ends[e][0] == v else 1] += delta
+        rd[sink] -= delta
     note("lp_cap", 0.0, 1.0)   # iteration cap reached: flag the depth
     return f, rs
 

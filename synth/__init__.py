@@ -156,9 +156,15 @@ def make_workload(spec: WorkloadSpec, device="cpu", seed=None) -> Workload:
     return Workload(spec, target, drafts, tokens, temps, list(spec.model_ids))
 
 
-def host_copy(w: Workload):
-    """numpy views for the oracle: fp32 logits (exact upcast of the stored
-    values), int64 tokens, float32 temperatures."""
-    target = w.target.float().cpu().numpy()
-    drafts = [w.drafts[k].float().cpu().numpy() for k in range(w.spec.K)]
-    return target, drafts, list(w.model_ids), w.tokens.cpu().numpy().astype("int64"), w.temps.cpu().numpy()
+def host_copy(w: Workload, seqs=None):
+    """numpy arrays for the oracle: fp32 logits (exact upcast of the stored
+    values), int64 tokens, float32 temperatures.  With ``seqs`` only those
+    sequences are copied (in that order)."""
+    if seqs is None:
+        sel = slice(None)
+    else:
+        sel = torch.as_tensor(list(seqs), dtype=torch.long, device=w.target.device)
+    target = w.target[sel].float().cpu().numpy()
+    drafts = [w.drafts[k][sel].float().cpu().numpy() for k in range(w.spec.K)]
+    return (target, drafts, list(w.model_ids), w.tokens[sel].cpu().numpy().astype("int64"),
+            w.temps[sel].cpu().numpy())
