@@ -1,0 +1,385 @@
+"""Benchmark of batched multi-draft verification on GB300.
+
+One step = one call of the verification kernel over the whole batch of a
+synthetic workload (every sequence walked along its draft tree: softmaxes,
+importance step, speculative step, residual or bonus draw).  Prints ONE JSON
+line (rank 0).
+
+Metric: verified vocab-rows per second (a vocab-row is one length-V logit row
+the walk consumed: the target row and one row per distinct draft model at
+every visited depth, the target row at the bonus depth), with the achieved
+HBM bandwidth of the verification kernel against the measured GB300 peak and
+the oracle's agreement on sampled sequences.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--scheme S]
+  python bench.py --impl reference ...   (the CPU oracle on host cores)
+
+Multi-GPU (torchrun, one rank per GPU): every rank verifies its own batch of
+the same shape (sequences are independent: no collective on the data path);
+the value is the sum over ranks divided by the slowest rank's time.
+"""
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "verified vocab-rows/sec and achieved HBM GB/s vs GB300 peak; oracle agreement"
+UNIT = "vocab-rows/s"
+DEFAULT_WORKLOAD = "llama3-128k"
+FALLBACK_HBM = 6800.0
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="native", choices=["native", "reference"])
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--scheme", default=None)
+    ap.add_argument("--cluster", type=int, default=0)
+    ap.add_argument("--B", type=int, default=0, help="override the batch (profiling on a small case)")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-parity", action="store_true")
+    ap.add_argument("--no-clocks", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0, help="budget of the oracle sample")
+    return ap.parse_args()
+
+
+# ----------------------------------------------------------------- accounting
+
+
+def walk_accounting(tokens, model_ids, out_tokens, acc, V, esize):
+    """Rows the walk consumed per sequence, replayed from the outputs:
+    returns (vocab_rows, algorithmic_bytes) summed over the batch."""
+    B, K, L = tokens.shape
+    mids = np.asarray(model_ids)
+    rows = 0
+    for b in range(B):
+        valid = np.arange(K)
+        for j in range(int(acc[b]) + 1):
+            if j == L:
+                rows += 1
+                break
+            rows += 1 + len(np.unique(mids[valid]))
+            z = out_tokens[b, j]
+            valid = valid[tokens[b, valid, j] == z]
+            if len(valid) == 0:
+                break
+    per_seq_io = 4 * (K * L + (1 + K) + (L + 1) + 1)
+    return rows, rows * V * esize + B * per_seq_io
+
+
+# ----------------------------------------------------------------- clocks
+
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.proc = None
+        self.path = os.path.join("/tmp", f"mds_clocks_{os.getpid()}.csv")
+        self.gpu = gpu_index
+
+    def start(self):
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"], stdout=self.f,
+                                         stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.f.close()
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx = float(parts[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        os.unlink(self.path)
+        if not sm:
+            return None
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ----------------------------------------------------------------- peaks / traffic
+
+
+def hbm_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        d = json.load(open(path))
+        return float(d["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM, "fallback"
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2410_18234_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        h.update(open(os.path.join(csrc, name), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(workload, scheme):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken
+    on the current kernel source; else None."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        d = json.load(open(path))
+    except (OSError, ValueError):
+        return None
+    e = d.get(f"{workload}/{scheme}")
+    if not e or e.get("kernel_hash") != kernel_source_hash():
+        return None
+    return e.get("dram_bytes_per_launch")
+
+
+# ----------------------------------------------------------------- oracle leg
+
+
+def oracle_rate(w, scheme, seconds, seqs=None):
+    """The oracle, as it stands, over a bounded prefix of the workload's
+    sequences (host cores).  Returns (vocab_rows/s, sample description,
+    outputs) for the sequences it finished."""
+    from oracle.verify import oracle_verify
+    from synth import host_copy
+    spec = w.spec
+    es = 4 if spec.dtype == "f32" else 2
+    done, rows, t_total = [], 0, 0.0
+    outs = {}
+    order = list(range(spec.B)) if seqs is None else list(seqs)
+    for b in order:
+        host = host_copy(w, [b])
+        t0 = time.perf_counter()
+        o, a, recs = oracle_verify(*host, scheme, spec.verify_seed, seq_ids=[b])
+        t_total += time.perf_counter() - t0
+        out = np.asarray(o[b])[None]
+        r, _ = walk_accounting(host[3], w.model_ids, out, np.array([a[b]]), spec.V, es)
+        rows += r
+        done.append(b)
+        outs[b] = (o[b], a[b], recs[b])
+        if t_total >= seconds:
+            break
+    return rows / t_total, f"{len(done)} of {spec.B} sequences (first {len(done)}), {t_total:.1f} s", outs
+
+
+def agreement(g_tok, g_acc, outs):
+    """GPU vs oracle on the sequences the oracle finished: identical, within
+    the band (first differing decision flagged by the oracle), or mismatched."""
+    same = band = bad = 0
+    for b, (o, a, recs) in outs.items():
+        if np.array_equal(g_tok[b], np.asarray(o)) and int(g_acc[b]) == int(a):
+            same += 1
+            continue
+        diff = np.flatnonzero(g_tok[b] != np.asarray(o))
+        j = int(diff[0]) if len(diff) else min(int(g_acc[b]), int(a))
+        if any(r.band for r in recs[: j + 1]):
+            band += 1
+        else:
+            bad += 1
+    return {"sequences": len(outs), "identical": same, "band": band, "mismatch": bad}
+
+
+# ----------------------------------------------------------------- main
+
+
+def main():
+    args = parse()
+    import torch
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    from synth import WORKLOADS, make_workload
+    spec = WORKLOADS[args.workload]
+    if args.B:
+        spec = spec.with_(B=args.B)
+    scheme = args.scheme or spec.schemes[0]
+    es = 4 if spec.dtype == "f32" else 2
+
+    if args.impl == "reference":
+        if world > 1 and rank != 0:
+            return 0
+        dev = "cuda:0" if torch.cuda.is_available() else "cpu"
+        w = make_workload(spec, device=dev)
+        # each step: the oracle over a bounded sample of the workload
+        per_step = max(2.0, args.cpu_seconds / max(1, args.steps + args.warmup))
+        for _ in range(args.warmup):
+            oracle_rate(w, scheme, per_step / 4)
+        rates = []
+        desc = ""
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            r, desc, _ = oracle_rate(w, scheme, per_step)
+            rates.append(r)
+        wall = time.perf_counter() - t0
+        value = float(np.mean(rates))
+        line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": 1,
+                "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * wall / args.steps,
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+                "data": "synthetic",
+                "config": {"workload": spec.name, "B": spec.B, "K": spec.K, "L": spec.L, "V": spec.V,
+                           "logits": spec.dtype, "scheme": scheme},
+                "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                                 "sample": f"per step {desc}"},
+                "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+        print(json.dumps(line))
+        return 0
+
+    # ------------------------------------------------------------- native
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local if world > 1 else 0)
+    torch.cuda.set_device(dev)
+    from paper_2410_18234_gb300 import mds
+    w = make_workload(spec, device=dev, seed=spec.data_seed + 7919 * rank)
+    v = mds.Verifier(spec.B, spec.K, spec.L, spec.V, dtype=spec.dtype, cluster=args.cluster, device=dev.index)
+    drafts = w.draft_list()
+    out_tokens = torch.empty(spec.B, spec.L + 1, dtype=torch.int32, device=dev)
+    out_acc = torch.empty(spec.B, dtype=torch.int32, device=dev)
+    flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)   # > L2 (129 MB)
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        mds.mds_verify(v.ctx, w.target, drafts, w.model_ids, w.tokens, w.temps, scheme, spec.verify_seed,
+                       out_tokens, out_acc, None, stream)
+
+    for _ in range(max(args.warmup, 0)):
+        flush.fill_(1.0)
+        step()
+    torch.cuda.synchronize()
+    bits, msg = v.status()
+    if bits:
+        print(f"status after warm-up: {bits} {msg}", file=sys.stderr)
+
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    clocks = None if args.no_clocks else ClockSampler(dev.index)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    if clocks:
+        clocks.start()
+        time.sleep(0.3)
+    for i in range(args.steps):
+        flush.fill_(1.0)                       # evict L2 between timed launches
+        starts[i].record(stream)
+        step()
+        ends[i].record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clk = clocks.stop() if clocks else None
+    times = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    ms = float(np.mean(times))
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+
+    tok = w.tokens.cpu().numpy()
+    o_tok = out_tokens.cpu().numpy()
+    o_acc = out_acc.cpu().numpy()
+    rows, abytes = walk_accounting(tok, w.model_ids, o_tok, o_acc, spec.V, es)
+    value = rows * world / (ms * 1e-3)
+    achieved = abytes / (ms * 1e-3) / 1e9
+    peak, peak_kind = hbm_peak()
+
+    # ------------------------------------------------------------- e2e through the host-buffer entry
+    e2e = None
+    if not args.no_e2e:
+        h_target = w.target.cpu().pin_memory()
+        h_drafts = [d.cpu().pin_memory() for d in drafts]
+        h_tokens = w.tokens.cpu().pin_memory()
+        h_temps = w.temps.cpu().pin_memory()
+        h_out = torch.empty(spec.B, spec.L + 1, dtype=torch.int32).pin_memory()
+        h_acc = torch.empty(spec.B, dtype=torch.int32).pin_memory()
+        e2e_steps = max(1, min(args.steps, 5))
+        mds.mds_verify_host(v.ctx, h_target, h_drafts, w.model_ids, h_tokens, h_temps, scheme,
+                            spec.verify_seed, h_out, h_acc, None, stream)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for _ in range(e2e_steps):
+            mds.mds_verify_host(v.ctx, h_target, h_drafts, w.model_ids, h_tokens, h_temps, scheme,
+                                spec.verify_seed, h_out, h_acc, None, stream)
+        e2e_s = (time.perf_counter() - t0) / e2e_steps
+        assert np.array_equal(h_out.numpy(), o_tok) and np.array_equal(h_acc.numpy(), o_acc)
+        h2d = (h_target.numel() * h_target.element_size() + sum(d.numel() * d.element_size() for d in h_drafts)
+               + h_tokens.numel() * 4 + h_temps.numel() * 4)
+        d2h = h_out.numel() * 4 + h_acc.numel() * 4
+        e2e = {"value": rows * world / e2e_s, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+               "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_s * 1e3}
+
+    # ------------------------------------------------------------- oracle agreement + cpu baseline
+    cpu = None
+    parity = None
+    if rank == 0 and world == 1 and not (args.no_cpu_baseline and args.no_parity):
+        rate, desc, outs = oracle_rate(w, scheme, args.cpu_seconds)
+        parity = agreement(o_tok, o_acc, outs)
+        if not args.no_cpu_baseline:
+            cpu = {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc}
+
+    bits, msg = v.status()
+    cn = v.cluster_size
+    v.close()
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": spec.name, "B": spec.B, "K": spec.K, "L": spec.L, "V": spec.V,
+                       "logits": spec.dtype, "scheme": scheme, "cluster": cn, "l2_flush": True,
+                       "parallelism": f"sequence-sharded x{world}", "seed": spec.verify_seed},
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak, "peak_kind": peak_kind,
+                         "traffic": recorded_traffic(spec.name, scheme),
+                         "algorithmic_bytes_per_launch": int(abytes), "kernel": "verify_kernel"},
+            "cpu_baseline": cpu,
+            "e2e": e2e,
+            "gpu_launches": args.steps,
+            "clocks": clk,
+            "vocab_rows_per_step": rows,
+            "block_efficiency": float(np.mean(o_acc + 1)),
+            "oracle_agreement": parity,
+            "status_bits": bits,
+        }
+        print(json.dumps(line))
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,154 @@
+/*
+ * mds.h -- C ABI of the GB300 multi-draft speculative verification library.
+ *
+ * The library verifies K draft branches of L tokens per sequence against a
+ * target model, as in "Multi-Draft Speculative Sampling: Canonical
+ * Decomposition and Theoretical Limits" (arXiv 2410.18234).  For every depth
+ * j of every sequence b it computes the temperature softmax of the target row
+ * and of one row per distinct draft model (Section 3), chooses one
+ * intermediate token Y among the valid draft tokens with an importance step
+ * (Definition 1; Theorem 1's canonical decomposition), applies the
+ * single-draft speculative step to Y (Appendix A, Algorithm 1: accept with
+ * probability min(1, q(Y)/p_I(Y)), else resample the normalised residual
+ * max(0, q - p_I)), and walks the draft tree: the walk continues while the
+ * output token is one of the valid draft tokens (the event Z in S of
+ * Problem 1), and after L accepted positions a bonus token is drawn from the
+ * target row at depth L.
+ *
+ * Notation follows the paper: q is the target distribution, p a draft
+ * distribution, p_I the law of the intermediate token.
+ *
+ * Random numbers: Philox4x32-10 (Salmon et al., SC'11) with counter
+ * (b, j, draw, 0) and key (seed low 32 bits, seed high 32 bits); the uniform
+ * is (word0 >> 8) * 2^-24.  Draw ids: 0..15 importance-step selection (stage
+ * m of the pairwise stages uses m), 16..31 accept (the sequential-rejection
+ * baseline's round i uses 16 + i), 32 residual, 33 bonus.
+ *
+ * Threading: a context may be used from one host thread at a time and its
+ * calls must not overlap on the GPU (they share a work counter and a status
+ * word).  All device work is issued on the caller's stream; mds_verify does
+ * not synchronise.
+ */
+#ifndef MDS_H
+#define MDS_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- return codes (synchronous argument/launch errors) ---------------- */
+#define MDS_OK 0
+#define MDS_EINVAL (-1)   /* null pointer, bad enum, misaligned pointer     */
+#define MDS_ESHAPE (-2)   /* B, K, L or V outside the supported range       */
+#define MDS_EVOCAB (-3)   /* V does not fit the shared-memory budget        */
+#define MDS_ECUDA (-4)    /* a CUDA runtime call failed                     */
+#define MDS_EUNSUP (-5)   /* unsupported combination (see mds_verify)       */
+
+/* ---- device status bits (read and cleared by mds_status) -------------- */
+#define MDS_ST_NONFINITE 1u   /* a row had NaN logits or a zero/inf normaliser */
+#define MDS_ST_BADTEMP 2u     /* a temperature was <= 0 or not finite          */
+#define MDS_ST_ZERO_RESID 4u  /* residual mass was 0 after a rejection (only by
+                                 rounding); the target row was sampled instead */
+#define MDS_ST_TIMEOUT 8u     /* a bounded wait on a bulk copy gave up         */
+#define MDS_ST_LP_CAP 16u     /* the stage LP hit its augmentation cap         */
+#define MDS_ST_BADTOKEN 32u   /* a draft token was outside [0, V) (token 0 used) */
+
+/* ---- limits ------------------------------------------------------------ */
+#define MDS_MAX_K 16      /* draft branches per sequence                    */
+#define MDS_MAX_L 64      /* draft positions per branch                     */
+#define MDS_MAX_S 8       /* LP truncation threshold s (|Omega_1|)          */
+#define MDS_MAX_IS_MODELS 4  /* distinct draft models for plain IS          */
+
+typedef struct mds_ctx mds_ctx;
+
+/* Importance step.  MDS_SINGLE: Algorithm 1 on the lowest valid branch.
+ * MDS_IS: classical importance sampling, Pr(I = i) proportional to
+ * q(X_i)/p(X_i) (Section 3, after Definition 1).  MDS_WIS: the paper's
+ * weighted importance sampling with the variant truncated LP (appendix
+ * "Variant of Truncated LP", Eq. heur2), pairwise stages for K > 2
+ * (Remark 4) and the non-iid key q - p_1 p_2 (non-iid appendix).
+ * MDS_SPECTR: sequential-rejection baseline (Algorithm 1 applied to the
+ * valid drafts in turn against the running residual target). */
+typedef enum { MDS_SINGLE = 0, MDS_IS = 1, MDS_WIS = 2, MDS_SPECTR = 3 } mds_scheme;
+
+/* Storage type of the logits. */
+typedef enum { MDS_F32 = 0, MDS_BF16 = 1 } mds_dtype;
+
+typedef struct {
+  int max_B;       /* largest batch a call may pass (>= 1)                    */
+  int K;           /* draft branches, 1..MDS_MAX_K                            */
+  int L;           /* draft positions per branch, 1..MDS_MAX_L                */
+  int V;           /* vocabulary size, 1..2^24                                */
+  mds_dtype dtype; /* storage type of every logit buffer                      */
+  int wis_s;       /* LP truncation threshold s, 1..MDS_MAX_S (0: 5, the value
+                      of the paper's experiments, Section 5)                  */
+  float is_h;      /* trapezoid step in ln t for plain IS (0: 0.25)           */
+  int cluster;     /* CTAs per sequence: 1, 2, 4, 8 or 16 (0: chosen from V)  */
+} mds_config;
+
+/* Create a context on CUDA device `device`.  Allocates the context's device
+ * workspace (a work counter and the status word) and, lazily, the staging
+ * buffers of mds_verify_host.  Returns MDS_OK and stores the context in *out,
+ * or a negative code (nothing allocated). */
+int mds_create(mds_ctx** out, const mds_config* cfg, int device);
+
+/* Verify B sequences (0 <= B <= max_B) on `stream` (a cudaStream_t; NULL for
+ * the legacy default stream).  All buffers are caller-owned DEVICE memory in
+ * row-major layout:
+ *   target_logits  [B][K][L+1][V] dtype: target logits of the node reached by
+ *                  branch k after j draft tokens (branches with equal prefixes
+ *                  must hold equal rows; the walk reads the lowest valid one)
+ *   draft_logits   HOST array of K device pointers, each [B][L][V] dtype:
+ *                  branch k's draft-model logits at depth j
+ *   draft_model_id HOST array [K] of ids in 0..MDS_MAX_K-1: branches with equal
+ *                  ids are i.i.d. drafts of one model (equal rows at equal
+ *                  prefixes, equal temperatures)
+ *   draft_tokens   [B][K][L] int32 in [0, V)
+ *   temperatures   [B][1+K] float32 > 0: target, then one per branch
+ *   out_tokens     [B][L+1] int32: the emitted tokens (accepted tokens then the
+ *                  correction or bonus token), -1 after them
+ *   out_accept_len [B] int32 in [0, L]: accepted draft positions
+ *   out_diag       optional [B][L+1][4] float32: per depth q(Y), p_I(Y), the
+ *                  residual mass (0 if accepted) and Y; NULL to skip
+ * Pointers must be aligned to the element size; rows whose byte length is a
+ * multiple of 16 at 16-byte-aligned bases are fetched with bulk copies.
+ * Plain IS supports at most MDS_MAX_IS_MODELS distinct draft models
+ * (MDS_EUNSUP otherwise).  Returns MDS_OK after the launch was issued, or a
+ * negative code with nothing launched.  Data-dependent anomalies are reported
+ * through the status word (mds_status). */
+int mds_verify(mds_ctx* ctx, const void* target_logits, const void* const* draft_logits,
+               const int32_t* draft_model_id, const int32_t* draft_tokens, const float* temperatures,
+               int scheme, uint64_t philox_seed, int32_t* out_tokens, int32_t* out_accept_len,
+               float* out_diag, int B, void* stream);
+
+/* Same as mds_verify with every buffer in HOST memory (pinned memory gives
+ * the fastest copies).  The context stages the inputs into device buffers it
+ * owns (allocated on first use, grown as needed), runs the verification and
+ * copies the outputs back, all on `stream`, and synchronises the stream
+ * before returning. */
+int mds_verify_host(mds_ctx* ctx, const void* target_logits, const void* const* draft_logits,
+                    const int32_t* draft_model_id, const int32_t* draft_tokens, const float* temperatures,
+                    int scheme, uint64_t philox_seed, int32_t* out_tokens, int32_t* out_accept_len,
+                    float* out_diag, int B, void* stream);
+
+/* Synchronise the device, read and clear the status word.  Returns the
+ * MDS_ST_* bits (>= 0) or a negative code; *msg (if not NULL) receives a
+ * static description of the highest set bit. */
+int mds_status(mds_ctx* ctx, const char** msg);
+
+/* Number of CTAs per sequence the context launches with (for reporting). */
+int mds_cluster_size(const mds_ctx* ctx);
+
+/* Static text for a return code. */
+const char* mds_error_string(int code);
+
+/* Free the context and everything it allocated. */
+void mds_destroy(mds_ctx* ctx);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MDS_H */

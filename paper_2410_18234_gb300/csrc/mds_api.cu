@@ -1,0 +1,355 @@
+// C ABI of the verification library (declared in include/mds.h): argument
+// validation, launch geometry, workspace and the host-buffer entry point.
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <vector>
+
+#include "mds_internal.h"
+
+struct mds_ctx {
+  mds_config cfg;
+  int device;
+  unsigned* work;          // [0] status word, [1] work counter (monotonic tickets)
+  unsigned tickets;        // tickets consumed by earlier launches
+  int last_cn;
+  // occupancy cache: (cn, dynamic smem) -> max active clusters
+  struct Occ {
+    int cn;
+    size_t smem;
+    int dtype;
+    int clusters;
+  };
+  std::vector<Occ> occ;
+  // staging buffers of mds_verify_host
+  void* h_buf;
+  size_t h_bytes;
+};
+
+namespace {
+
+constexpr size_t kSmemTarget = 66 * 1024;  // dynamic part; with the static state, three CTAs per SM
+
+struct DeviceGuard {
+  int prev = -1;
+  explicit DeviceGuard(int dev) {
+    cudaGetDevice(&prev);
+    if (prev != dev) cudaSetDevice(dev);
+  }
+  ~DeviceGuard() {
+    int cur = -1;
+    cudaGetDevice(&cur);
+    if (prev >= 0 && cur != prev) cudaSetDevice(prev);
+  }
+};
+
+int esize_of(int dtype) { return dtype == MDS_F32 ? 4 : 2; }
+
+size_t round_up(size_t x, size_t m) { return (x + m - 1) / m * m; }
+
+thread_local char g_cuda_detail[256] = "";
+
+// Remember the CUDA error behind an MDS_ECUDA return (per host thread).
+int cuda_fail(cudaError_t e, const char* where) {
+  std::snprintf(g_cuda_detail, sizeof(g_cuda_detail), "CUDA runtime error in %s: %s", where,
+                cudaGetErrorString(e));
+  cudaGetLastError();
+  return MDS_ECUDA;
+}
+
+bool configured[2] = {false, false};
+std::mutex config_mu;
+
+int ensure_configured(int dtype) {
+  std::lock_guard<std::mutex> lk(config_mu);
+  if (!configured[dtype]) {
+    const cudaError_t e = mds::configure_kernel(dtype);
+    if (e != cudaSuccess) return cuda_fail(e, "kernel configuration");
+    configured[dtype] = true;
+  }
+  return MDS_OK;
+}
+
+int optin_smem(int device) {
+  int v = 0;
+  cudaDeviceGetAttribute(&v, cudaDevAttrMaxSharedMemoryPerBlockOptin, device);
+  return v;
+}
+
+// Fill the launch geometry (cluster size, slice, row stride) for n_models
+// distinct draft models.  Returns MDS_OK or MDS_EVOCAB.
+int geometry(const mds_ctx* ctx, int scheme, int n_models, mds::Params& p) {
+  const mds_config& c = ctx->cfg;
+  p.esize = esize_of(c.dtype);
+  p.rows_max = 1 + n_models;
+  p.scheme = scheme;
+  // WIS candidate lists (target + up to 3 draft models); the merged list
+  // shares its memory with the special-token bitmap, so it is sized to at
+  // least 64 entries and otherwise to the bitmap's bytes
+  const bool lists = scheme == MDS_WIS && p.rows_max <= 4;
+  const size_t limit = (size_t)optin_smem(ctx->device) - 12 * 1024;  // static shared state
+  auto fill = [&](int cn) {
+    p.cn = cn;
+    p.slice = (int)round_up((size_t)((c.V + cn - 1) / cn), 8);
+    p.row_stride = (int)round_up((size_t)p.slice * p.esize, 128);
+    if (lists) {
+      const int bm_bytes = (p.slice + 31) / 32 * 4;
+      p.cand_cap = bm_bytes / (4 * (3 + p.rows_max));
+      if (p.cand_cap < 64) p.cand_cap = 64;
+      if (p.cand_cap > 512) p.cand_cap = 512;
+      p.cand_cap_cta = p.cand_cap < 64 ? p.cand_cap : 64;
+    } else {
+      p.cand_cap = p.cand_cap_cta = 0;
+    }
+    return mds::smem_bytes(p);
+  };
+  if (c.cluster > 0) {
+    if (fill(c.cluster) > limit) return MDS_EVOCAB;
+    return MDS_OK;
+  }
+  for (int cn = 1; cn <= mds::kMaxCluster; cn *= 2) {
+    if (cn > 1 && (c.V + cn - 1) / cn < 8) break;
+    if (fill(cn) <= kSmemTarget) return MDS_OK;
+  }
+  for (int cn = 1; cn <= mds::kMaxCluster; cn *= 2)
+    if (fill(cn) <= limit) return MDS_OK;
+  return MDS_EVOCAB;
+}
+
+int clusters_for(mds_ctx* ctx, const mds::Params& p) {
+  const size_t smem = mds::smem_bytes(p);
+  for (const auto& o : ctx->occ)
+    if (o.cn == p.cn && o.smem == smem && o.dtype == p.dtype) return o.clusters;
+  int n = mds::max_active_clusters(p);
+  if (n < 1) n = 1;
+  ctx->occ.push_back({p.cn, smem, p.dtype, n});
+  return n;
+}
+
+bool aligned(const void* ptr, size_t a) { return ((uintptr_t)ptr % a) == 0; }
+
+}  // namespace
+
+extern "C" {
+
+const char* mds_error_string(int code) {
+  switch (code) {
+    case MDS_OK: return "ok";
+    case MDS_EINVAL: return "invalid argument (null pointer, bad enum or misaligned buffer)";
+    case MDS_ESHAPE: return "B, K, L or V outside the supported range";
+    case MDS_EVOCAB: return "vocabulary does not fit the shared-memory budget";
+    case MDS_ECUDA: return g_cuda_detail[0] ? g_cuda_detail : "CUDA runtime error";
+    case MDS_EUNSUP: return "unsupported combination of arguments";
+    default: return "unknown error";
+  }
+}
+
+int mds_create(mds_ctx** out, const mds_config* cfg, int device) {
+  if (!out || !cfg) return MDS_EINVAL;
+  *out = nullptr;
+  mds_config c = *cfg;
+  if (c.wis_s == 0) c.wis_s = 5;
+  if (c.is_h == 0.f) c.is_h = 0.25f;
+  if (c.max_B < 1 || c.K < 1 || c.K > MDS_MAX_K || c.L < 1 || c.L > MDS_MAX_L || c.V < 1 || c.V > (1 << 24))
+    return MDS_ESHAPE;
+  if (c.dtype != MDS_F32 && c.dtype != MDS_BF16) return MDS_EINVAL;
+  if (c.wis_s < 1 || c.wis_s > MDS_MAX_S || !(c.is_h > 0.f) || c.is_h > 4.f) return MDS_EINVAL;
+  if (c.cluster != 0 && c.cluster != 1 && c.cluster != 2 && c.cluster != 4 && c.cluster != 8 && c.cluster != 16)
+    return MDS_EINVAL;
+  int ndev = 0;
+  const cudaError_t de = cudaGetDeviceCount(&ndev);
+  if (de != cudaSuccess) return cuda_fail(de, "cudaGetDeviceCount");
+  if (device < 0 || device >= ndev) return cuda_fail(cudaErrorInvalidDevice, "mds_create");
+  DeviceGuard g(device);
+  if (ensure_configured(c.dtype) != MDS_OK) return MDS_ECUDA;
+  mds_ctx* ctx = new mds_ctx();
+  ctx->cfg = c;
+  ctx->device = device;
+  ctx->last_cn = 0;
+  ctx->tickets = 0u;
+  ctx->h_buf = nullptr;
+  ctx->h_bytes = 0;
+  cudaError_t me = cudaMalloc(&ctx->work, 256);
+  if (me == cudaSuccess) me = cudaMemset(ctx->work, 0, 256);
+  if (me != cudaSuccess) {
+    delete ctx;
+    return cuda_fail(me, "workspace allocation");
+  }
+  *out = ctx;
+  return MDS_OK;
+}
+
+int mds_verify(mds_ctx* ctx, const void* target_logits, const void* const* draft_logits,
+               const int32_t* draft_model_id, const int32_t* draft_tokens, const float* temperatures,
+               int scheme, uint64_t philox_seed, int32_t* out_tokens, int32_t* out_accept_len,
+               float* out_diag, int B, void* stream) {
+  if (!ctx) return MDS_EINVAL;
+  const mds_config& c = ctx->cfg;
+  if (scheme < MDS_SINGLE || scheme > MDS_SPECTR) return MDS_EINVAL;
+  if (B < 0 || B > c.max_B) return MDS_ESHAPE;
+  if (B == 0) return MDS_OK;
+  if (!target_logits || !draft_logits || !draft_model_id || !draft_tokens || !temperatures || !out_tokens ||
+      !out_accept_len)
+    return MDS_EINVAL;
+  const int es = esize_of(c.dtype);
+  if (!aligned(target_logits, es) || !aligned(draft_tokens, 4) || !aligned(temperatures, 4) ||
+      !aligned(out_tokens, 4) || !aligned(out_accept_len, 4) || (out_diag && !aligned(out_diag, 4)))
+    return MDS_EINVAL;
+  mds::Params p{};
+  int remap[MDS_MAX_K];
+  for (int m = 0; m < MDS_MAX_K; ++m) remap[m] = -1;
+  int n_models = 0;
+  bool tma_ok = ((size_t)c.V * es) % 16 == 0 && aligned(target_logits, 16);
+  for (int k = 0; k < c.K; ++k) {
+    if (!draft_logits[k] || !aligned(draft_logits[k], es)) return MDS_EINVAL;
+    tma_ok = tma_ok && aligned(draft_logits[k], 16);
+    const int m = draft_model_id[k];
+    if (m < 0 || m >= MDS_MAX_K) return MDS_EINVAL;
+    if (remap[m] < 0) remap[m] = n_models++;
+    p.model_of[k] = (int8_t)remap[m];
+    p.drafts[k] = static_cast<const char*>(draft_logits[k]);
+  }
+  if (scheme == MDS_IS && n_models > MDS_MAX_IS_MODELS) return MDS_EUNSUP;
+  p.dtype = c.dtype;
+  int rc = geometry(ctx, scheme, n_models, p);
+  if (rc != MDS_OK) return rc;
+  p.target = static_cast<const char*>(target_logits);
+  p.tokens = draft_tokens;
+  p.temps = temperatures;
+  p.out_tokens = out_tokens;
+  p.out_accept = out_accept_len;
+  p.out_diag = out_diag;
+  p.status = ctx->work;
+  p.queue = ctx->work + 1;
+  p.seed = philox_seed;
+  p.B = B;
+  p.K = c.K;
+  p.L = c.L;
+  p.V = c.V;
+  p.wis_s = c.wis_s;
+  p.is_h = c.is_h;
+  p.n_models = n_models;
+  p.tma_ok = tma_ok ? 1 : 0;
+  DeviceGuard g(ctx->device);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  int clusters = clusters_for(ctx, p);
+  if (clusters > B) clusters = B;
+  // Every cluster takes tickets until one maps past B: a launch consumes
+  // exactly B + clusters tickets, so the next launch's base is known here and
+  // the counter never needs a reset.
+  p.ticket0 = ctx->tickets;
+  const cudaError_t e = mds::launch(p, clusters, st);
+  if (e != cudaSuccess) return cuda_fail(e, "kernel launch");
+  ctx->tickets += (unsigned)(B + clusters);
+  ctx->last_cn = p.cn;
+  return MDS_OK;
+}
+
+int mds_verify_host(mds_ctx* ctx, const void* target_logits, const void* const* draft_logits,
+                    const int32_t* draft_model_id, const int32_t* draft_tokens, const float* temperatures,
+                    int scheme, uint64_t philox_seed, int32_t* out_tokens, int32_t* out_accept_len,
+                    float* out_diag, int B, void* stream) {
+  if (!ctx) return MDS_EINVAL;
+  const mds_config& c = ctx->cfg;
+  if (B < 0 || B > c.max_B) return MDS_ESHAPE;
+  if (B == 0) return MDS_OK;
+  if (!target_logits || !draft_logits || !draft_model_id || !draft_tokens || !temperatures || !out_tokens ||
+      !out_accept_len)
+    return MDS_EINVAL;
+  for (int k = 0; k < c.K; ++k)
+    if (!draft_logits[k]) return MDS_EINVAL;
+  const size_t es = (size_t)esize_of(c.dtype);
+  const size_t n_tgt = round_up((size_t)B * c.K * (c.L + 1) * c.V * es, 256);
+  const size_t n_drf = round_up((size_t)B * c.L * c.V * es, 256);
+  const size_t n_tok = round_up((size_t)B * c.K * c.L * 4, 256);
+  const size_t n_tmp = round_up((size_t)B * (1 + c.K) * 4, 256);
+  const size_t n_out = round_up((size_t)B * (c.L + 1) * 4, 256);
+  const size_t n_acc = round_up((size_t)B * 4, 256);
+  const size_t n_dg = out_diag ? round_up((size_t)B * (c.L + 1) * 16, 256) : 0;
+  const size_t total = n_tgt + c.K * n_drf + n_tok + n_tmp + n_out + n_acc + n_dg;
+  DeviceGuard g(ctx->device);
+  if (total > ctx->h_bytes) {
+    if (ctx->h_buf) cudaFree(ctx->h_buf);
+    ctx->h_buf = nullptr;
+    ctx->h_bytes = 0;
+    if (cudaMalloc(&ctx->h_buf, total) != cudaSuccess) {
+      cudaGetLastError();
+      return MDS_ECUDA;
+    }
+    ctx->h_bytes = total;
+  }
+  char* base = static_cast<char*>(ctx->h_buf);
+  char* d_tgt = base;
+  char* d_drf = d_tgt + n_tgt;
+  char* d_tok = d_drf + c.K * n_drf;
+  char* d_tmp = d_tok + n_tok;
+  char* d_out = d_tmp + n_tmp;
+  char* d_acc = d_out + n_out;
+  char* d_dg = d_acc + n_acc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const void* dptr[MDS_MAX_K];
+  bool ok = cudaMemcpyAsync(d_tgt, target_logits, (size_t)B * c.K * (c.L + 1) * c.V * es, cudaMemcpyHostToDevice,
+                            st) == cudaSuccess;
+  for (int k = 0; k < c.K && ok; ++k) {
+    dptr[k] = d_drf + k * n_drf;
+    ok = cudaMemcpyAsync(d_drf + k * n_drf, draft_logits[k], (size_t)B * c.L * c.V * es, cudaMemcpyHostToDevice,
+                         st) == cudaSuccess;
+  }
+  ok = ok && cudaMemcpyAsync(d_tok, draft_tokens, (size_t)B * c.K * c.L * 4, cudaMemcpyHostToDevice, st) == cudaSuccess;
+  ok = ok && cudaMemcpyAsync(d_tmp, temperatures, (size_t)B * (1 + c.K) * 4, cudaMemcpyHostToDevice, st) == cudaSuccess;
+  if (!ok) {
+    cudaGetLastError();
+    return MDS_ECUDA;
+  }
+  int rc = mds_verify(ctx, d_tgt, dptr, draft_model_id, reinterpret_cast<const int32_t*>(d_tok),
+                      reinterpret_cast<const float*>(d_tmp), scheme, philox_seed, reinterpret_cast<int32_t*>(d_out),
+                      reinterpret_cast<int32_t*>(d_acc), out_diag ? reinterpret_cast<float*>(d_dg) : nullptr, B, stream);
+  if (rc != MDS_OK) {
+    cudaStreamSynchronize(st);
+    return rc;
+  }
+  ok = cudaMemcpyAsync(out_tokens, d_out, (size_t)B * (c.L + 1) * 4, cudaMemcpyDeviceToHost, st) == cudaSuccess;
+  ok = ok && cudaMemcpyAsync(out_accept_len, d_acc, (size_t)B * 4, cudaMemcpyDeviceToHost, st) == cudaSuccess;
+  if (out_diag)
+    ok = ok && cudaMemcpyAsync(out_diag, d_dg, (size_t)B * (c.L + 1) * 16, cudaMemcpyDeviceToHost, st) == cudaSuccess;
+  ok = (cudaStreamSynchronize(st) == cudaSuccess) && ok;
+  if (!ok) {
+    cudaGetLastError();
+    return MDS_ECUDA;
+  }
+  return MDS_OK;
+}
+
+int mds_status(mds_ctx* ctx, const char** msg) {
+  if (!ctx) return MDS_EINVAL;
+  DeviceGuard g(ctx->device);
+  unsigned st = 0;
+  if (cudaDeviceSynchronize() != cudaSuccess || cudaMemcpy(&st, ctx->work, sizeof(st), cudaMemcpyDeviceToHost) != cudaSuccess ||
+      cudaMemset(ctx->work, 0, sizeof(st)) != cudaSuccess) {
+    cudaGetLastError();
+    if (msg) *msg = "CUDA runtime error while reading the status word";
+    return MDS_ECUDA;
+  }
+  if (msg) {
+    if (st & MDS_ST_BADTOKEN) *msg = "draft token outside [0, V); token 0 used";
+    else if (st & MDS_ST_LP_CAP) *msg = "stage LP reached its augmentation cap";
+    else if (st & MDS_ST_TIMEOUT) *msg = "a bounded wait on a bulk copy gave up";
+    else if (st & MDS_ST_ZERO_RESID) *msg = "zero residual mass after a rejection; target row sampled";
+    else if (st & MDS_ST_BADTEMP) *msg = "temperature <= 0 or not finite (1.0 used)";
+    else if (st & MDS_ST_NONFINITE) *msg = "non-finite logits or normaliser";
+    else *msg = "ok";
+  }
+  return (int)st;
+}
+
+int mds_cluster_size(const mds_ctx* ctx) { return ctx ? ctx->last_cn : 0; }
+
+void mds_destroy(mds_ctx* ctx) {
+  if (!ctx) return;
+  DeviceGuard g(ctx->device);
+  if (ctx->h_buf) cudaFree(ctx->h_buf);
+  if (ctx->work) cudaFree(ctx->work);
+  delete ctx;
+}
+
+}  // extern "C"

@@ -1,0 +1,61 @@
+// Internal interface between the C ABI (mds_api.cu) and the verification
+// kernel (mds_kernel.cu).  Not installed; not part of the public ABI.
+#pragma once
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "../../include/mds.h"
+
+namespace mds {
+
+constexpr int kThreads = 256;          // threads per CTA
+constexpr int kMaxRows = 1 + MDS_MAX_K; // target + one row per distinct draft model
+constexpr int kMaxSpecial = MDS_MAX_S * (MDS_MAX_K - 1);
+constexpr int kIsNodesMax = 1024;      // trapezoid nodes for plain IS
+constexpr int kIsChunk = 16;           // nodes accumulated per pass
+constexpr int kXch = 34;               // floats one CTA contributes to a cluster exchange
+constexpr int kMaxCluster = 16;
+
+struct Params {
+  const char* target;                  // [B][K][L+1][V]
+  const char* drafts[MDS_MAX_K];       // K x [B][L][V]
+  const int32_t* tokens;               // [B][K][L]
+  const float* temps;                  // [B][1+K]
+  int32_t* out_tokens;                 // [B][L+1]
+  int32_t* out_accept;                 // [B]
+  float* out_diag;                     // [B][L+1][4] or null
+  unsigned* status;                    // status word (workspace)
+  unsigned* queue;                     // work counter (workspace): monotonic tickets
+  unsigned ticket0;                    // counter value when this launch starts
+  unsigned long long seed;
+  int B, K, L, V;
+  int scheme;
+  int dtype;                           // MDS_F32 / MDS_BF16
+  int esize;                           // bytes per logit
+  int wis_s;
+  float is_h;
+  int cn;                              // CTAs per cluster
+  int slice;                           // tokens per CTA (multiple of 8)
+  int row_stride;                      // bytes per smem row (multiple of 128)
+  int rows_max;                        // smem rows (1 + distinct models)
+  int n_models;                        // distinct draft models (ids are 0..n_models-1 after remap)
+  int tma_ok;                          // rows are 16-byte aligned with 16-byte-multiple length
+  int cand_cap_cta;                    // WIS candidate list capacity per CTA (0: no candidate path)
+  int cand_cap;                        // WIS merged candidate list capacity per cluster
+  int8_t model_of[MDS_MAX_K];          // remapped model id per branch
+};
+
+// Dynamic shared memory bytes the kernel needs for `p`.
+size_t smem_bytes(const Params& p);
+
+// Configure the kernel attributes once per process (dynamic smem limit,
+// non-portable cluster size).  Returns a CUDA error code.
+cudaError_t configure_kernel(int dtype);
+
+// Largest number of co-resident clusters for this configuration.
+int max_active_clusters(const Params& p);
+
+// Launch the persistent verification kernel with `clusters` clusters.
+cudaError_t launch(const Params& p, int clusters, cudaStream_t stream);
+
+}  // namespace mds

@@ -1,0 +1,218 @@
+"""ctypes binding of the verification library (C ABI in include/mds.h).
+
+Argument marshalling only: every step of the verification runs in the CUDA
+kernels of libmds.so.  PyTorch tensors serve as owners of device memory and
+streams.  If the library is missing the import of this module fails loudly;
+there is no fallback.
+
+The module mirrors the C entry points under the same names (``mds_create``,
+``mds_verify``, ``mds_verify_host``, ``mds_status``, ``mds_destroy``) and adds
+a small ``Verifier`` convenience wrapper.
+"""
+import ctypes
+import os
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "_lib", "libmds.so")
+
+MDS_SINGLE, MDS_IS, MDS_WIS, MDS_SPECTR = 0, 1, 2, 3
+SCHEMES = {"single": MDS_SINGLE, "IS": MDS_IS, "WIS": MDS_WIS, "SpecTr": MDS_SPECTR}
+MDS_F32, MDS_BF16 = 0, 1
+DTYPES = {"f32": MDS_F32, "bf16": MDS_BF16}
+TORCH_DTYPES = {MDS_F32: torch.float32, MDS_BF16: torch.bfloat16}
+
+MDS_OK, MDS_EINVAL, MDS_ESHAPE, MDS_EVOCAB, MDS_ECUDA, MDS_EUNSUP = 0, -1, -2, -3, -4, -5
+MDS_ST_NONFINITE, MDS_ST_BADTEMP, MDS_ST_ZERO_RESID, MDS_ST_TIMEOUT, MDS_ST_LP_CAP, MDS_ST_BADTOKEN = \
+    1, 2, 4, 8, 16, 32
+MDS_MAX_K = 16
+
+# every symbol include/mds.h declares
+EXPORTS = ("mds_create", "mds_verify", "mds_verify_host", "mds_status", "mds_cluster_size",
+           "mds_error_string", "mds_destroy")
+
+
+class MdsConfig(ctypes.Structure):
+    _fields_ = [("max_B", ctypes.c_int), ("K", ctypes.c_int), ("L", ctypes.c_int), ("V", ctypes.c_int),
+                ("dtype", ctypes.c_int), ("wis_s", ctypes.c_int), ("is_h", ctypes.c_float),
+                ("cluster", ctypes.c_int)]
+
+
+class MdsError(RuntimeError):
+    def __init__(self, code, where):
+        self.code = code
+        super().__init__(f"{where}: {error_string(code)} ({code})")
+
+
+def load_library(path=LIB_PATH):
+    if not os.path.exists(path):
+        raise ImportError(f"{path} is missing: build it with __graft_entry__.build() "
+                          "(python -m paper_2410_18234_gb300.build)")
+    lib = ctypes.CDLL(path)
+    vp, i32p, f32p = ctypes.c_void_p, ctypes.POINTER(ctypes.c_int32), ctypes.c_void_p
+    lib.mds_create.argtypes = [ctypes.POINTER(vp), ctypes.POINTER(MdsConfig), ctypes.c_int]
+    lib.mds_create.restype = ctypes.c_int
+    verify_args = [vp, vp, ctypes.POINTER(vp), i32p, vp, vp, ctypes.c_int, ctypes.c_uint64, vp, vp, f32p,
+                   ctypes.c_int, vp]
+    lib.mds_verify.argtypes = verify_args
+    lib.mds_verify.restype = ctypes.c_int
+    lib.mds_verify_host.argtypes = verify_args
+    lib.mds_verify_host.restype = ctypes.c_int
+    lib.mds_status.argtypes = [vp, ctypes.POINTER(ctypes.c_char_p)]
+    lib.mds_status.restype = ctypes.c_int
+    lib.mds_cluster_size.argtypes = [vp]
+    lib.mds_cluster_size.restype = ctypes.c_int
+    lib.mds_error_string.argtypes = [ctypes.c_int]
+    lib.mds_error_string.restype = ctypes.c_char_p
+    lib.mds_destroy.argtypes = [vp]
+    lib.mds_destroy.restype = None
+    return lib
+
+
+_lib = load_library()
+
+
+def error_string(code):
+    return _lib.mds_error_string(int(code)).decode()
+
+
+# ----------------------------------------------------------- C entry points
+
+
+def mds_create(max_B, K, L, V, dtype="bf16", wis_s=5, is_h=0.25, cluster=0, device=0):
+    cfg = MdsConfig(int(max_B), int(K), int(L), int(V), DTYPES[dtype] if isinstance(dtype, str) else int(dtype),
+                    int(wis_s), float(is_h), int(cluster))
+    h = ctypes.c_void_p()
+    rc = _lib.mds_create(ctypes.byref(h), ctypes.byref(cfg), int(device))
+    if rc != MDS_OK:
+        raise MdsError(rc, "mds_create")
+    return h
+
+
+def _ptr(t):
+    return ctypes.c_void_p(t.data_ptr()) if t is not None else ctypes.c_void_p(0)
+
+
+def _draft_ptrs(drafts, K):
+    arr = (ctypes.c_void_p * K)()
+    for k in range(K):
+        arr[k] = drafts[k].data_ptr()
+    return arr
+
+
+def _ids(model_ids, K):
+    arr = (ctypes.c_int32 * K)()
+    for k in range(K):
+        arr[k] = int(model_ids[k])
+    return arr
+
+
+def mds_verify(ctx, target, drafts, model_ids, tokens, temps, scheme, seed, out_tokens, out_accept,
+               out_diag=None, stream=None):
+    """Device-buffer entry point.  ``drafts`` is a sequence of K device
+    tensors (or a [K, B, L, V] tensor); ``stream`` a torch.cuda.Stream, a raw
+    handle, or None for torch's current stream."""
+    K = len(model_ids)
+    B = int(tokens.shape[0])
+    if stream is None:
+        stream = torch.cuda.current_stream().cuda_stream
+    elif isinstance(stream, torch.cuda.Stream):
+        stream = stream.cuda_stream
+    keep = _draft_ptrs(drafts, K)
+    rc = _lib.mds_verify(ctx, _ptr(target), keep, _ids(model_ids, K), _ptr(tokens), _ptr(temps),
+                         SCHEMES[scheme] if isinstance(scheme, str) else int(scheme), ctypes.c_uint64(int(seed)),
+                         _ptr(out_tokens), _ptr(out_accept), _ptr(out_diag), B, ctypes.c_void_p(int(stream)))
+    if rc != MDS_OK:
+        raise MdsError(rc, "mds_verify")
+
+
+def mds_verify_host(ctx, target, drafts, model_ids, tokens, temps, scheme, seed, out_tokens, out_accept,
+                    out_diag=None, stream=None):
+    """Host-buffer entry point: CPU tensors (pinned for speed); copies in and
+    out happen inside the call, which returns after the stream synchronised."""
+    K = len(model_ids)
+    B = int(tokens.shape[0])
+    if stream is None:
+        stream = torch.cuda.current_stream().cuda_stream
+    elif isinstance(stream, torch.cuda.Stream):
+        stream = stream.cuda_stream
+    keep = _draft_ptrs(drafts, K)
+    rc = _lib.mds_verify_host(ctx, _ptr(target), keep, _ids(model_ids, K), _ptr(tokens), _ptr(temps),
+                              SCHEMES[scheme] if isinstance(scheme, str) else int(scheme),
+                              ctypes.c_uint64(int(seed)), _ptr(out_tokens), _ptr(out_accept), _ptr(out_diag), B,
+                              ctypes.c_void_p(int(stream)))
+    if rc != MDS_OK:
+        raise MdsError(rc, "mds_verify_host")
+
+
+def mds_status(ctx):
+    msg = ctypes.c_char_p()
+    rc = _lib.mds_status(ctx, ctypes.byref(msg))
+    if rc < 0:
+        raise MdsError(rc, "mds_status")
+    return rc, (msg.value or b"").decode()
+
+
+def mds_cluster_size(ctx):
+    return _lib.mds_cluster_size(ctx)
+
+
+def mds_destroy(ctx):
+    if ctx:
+        _lib.mds_destroy(ctx)
+
+
+# ----------------------------------------------------------- convenience
+
+
+class Verifier:
+    """Owns one context; allocates outputs with torch on the context's device."""
+
+    def __init__(self, max_B, K, L, V, dtype="bf16", wis_s=5, is_h=0.25, cluster=0, device=0):
+        self.max_B, self.K, self.L, self.V = int(max_B), int(K), int(L), int(V)
+        self.dtype = dtype
+        self.device = torch.device("cuda", device)
+        self.ctx = mds_create(max_B, K, L, V, dtype, wis_s, is_h, cluster, device)
+
+    def verify(self, target, drafts, model_ids, tokens, temps, scheme, seed, diag=False, out=None, stream=None):
+        B = int(tokens.shape[0])
+        if out is None:
+            out_tokens = torch.empty(B, self.L + 1, dtype=torch.int32, device=self.device)
+            out_accept = torch.empty(B, dtype=torch.int32, device=self.device)
+            out_diag = torch.empty(B, self.L + 1, 4, dtype=torch.float32, device=self.device) if diag else None
+        else:
+            out_tokens, out_accept, out_diag = out
+        mds_verify(self.ctx, target, drafts, model_ids, tokens, temps, scheme, seed, out_tokens, out_accept,
+                   out_diag, stream)
+        return out_tokens, out_accept, out_diag
+
+    def verify_host(self, target, drafts, model_ids, tokens, temps, scheme, seed, out=None, stream=None):
+        B = int(tokens.shape[0])
+        if out is None:
+            out_tokens = torch.empty(B, self.L + 1, dtype=torch.int32).pin_memory()
+            out_accept = torch.empty(B, dtype=torch.int32).pin_memory()
+            out_diag = None
+        else:
+            out_tokens, out_accept, out_diag = out
+        mds_verify_host(self.ctx, target, drafts, model_ids, tokens, temps, scheme, seed, out_tokens, out_accept,
+                        out_diag, stream)
+        return out_tokens, out_accept, out_diag
+
+    def status(self):
+        return mds_status(self.ctx)
+
+    @property
+    def cluster_size(self):
+        return mds_cluster_size(self.ctx)
+
+    def close(self):
+        if self.ctx:
+            mds_destroy(self.ctx)
+            self.ctx = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

@@ -1,0 +1,144 @@
+"""CUDA path vs the oracle, through the C ABI.
+
+Small cases span several tiles and a ragged tail (oracle finishes in
+seconds); full-size workloads run in the launch configuration the bench
+uses and are compared on sampled sequences.  Edge cases: vocabularies of
+1..9 tokens, K = 1, L = 1, duplicated draft tokens, one-hot targets,
+non-unit temperatures, rows whose byte length is not a multiple of 16 (plain
+loads instead of bulk copies), every cluster size.
+"""
+import numpy as np
+import pytest
+import torch
+
+pytestmark = pytest.mark.gpu
+
+if not torch.cuda.is_available():
+    pytest.skip("needs a CUDA GPU", allow_module_level=True)
+
+from paper_2410_18234_gb300 import mds  # noqa: E402
+from synth import WORKLOADS, WorkloadSpec, make_workload, host_copy  # noqa: E402
+from oracle.verify import oracle_verify  # noqa: E402
+from parity import compare, check  # noqa: E402
+
+DEV = "cuda:0"
+
+
+def run_both(spec, scheme, seed, cluster=0, seqs=None, wis_s=5):
+    w = make_workload(spec, device=DEV)
+    v = mds.Verifier(spec.B, spec.K, spec.L, spec.V, dtype=spec.dtype, wis_s=wis_s, cluster=cluster)
+    out, acc, diag = v.verify(w.target, w.draft_list(), w.model_ids, w.tokens, w.temps, scheme, seed, diag=True)
+    torch.cuda.synchronize()
+    bits, msg = v.status()
+    cn = v.cluster_size
+    v.close()
+    if seqs is None:
+        o_out, o_acc, recs = oracle_verify(*host_copy(w), scheme, seed, wis_s=wis_s)
+    else:
+        o_out, o_acc, recs = oracle_verify(*host_copy(w, seqs), scheme, seed, wis_s=wis_s, seq_ids=seqs)
+    res = compare(out.cpu().numpy(), acc.cpu().numpy(), o_out, o_acc, recs, g_diag=diag.cpu().numpy(),
+                  scheme=scheme)
+    res["status"] = bits
+    res["cn"] = cn
+    return res
+
+
+def small(name, **kw):
+    return WORKLOADS[name].with_(**kw)
+
+
+SMALL_CASES = [
+    ("tiny", dict(), ["IS", "single", "WIS", "SpecTr"]),
+    ("llama2-32k", dict(B=12, V=5003), ["IS", "WIS", "single", "SpecTr"]),
+    ("two-models-50k", dict(B=16, V=7001), ["WIS", "SpecTr", "single", "IS"]),
+    ("llama3-128k", dict(B=12, V=9000), ["WIS", "single", "SpecTr"]),
+    ("serving-152k", dict(B=12, V=6007, L=5), ["single", "IS", "WIS", "SpecTr"]),
+]
+
+
+@pytest.mark.parametrize("name,kw,schemes", SMALL_CASES, ids=[c[0] for c in SMALL_CASES])
+def test_small_workloads_match_oracle(name, kw, schemes):
+    spec = small(name, **kw)
+    for scheme in schemes:
+        res = run_both(spec, scheme, seed=11)
+        check(res, scheme)
+        assert res["status"] == 0
+
+
+@pytest.mark.parametrize("cluster", [1, 2, 4, 8, 16])
+def test_every_cluster_size(cluster):
+    spec = small("llama2-32k", B=6, V=4099, K=3, model_ids=[0, 0, 0])
+    for scheme in ("WIS", "single", "SpecTr"):
+        res = run_both(spec, scheme, seed=5, cluster=cluster)
+        assert res["cn"] == cluster
+        check(res, scheme)
+
+
+@pytest.mark.parametrize("V", [1, 2, 3, 5, 7, 8, 9, 17, 100])
+def test_tiny_vocabularies(V):
+    for dtype in ("f32", "bf16"):
+        spec = WorkloadSpec(f"v{V}", B=24, K=3, L=3, V=V, dtype=dtype, model_ids=[0, 0, 1], target_scale=2.0,
+                            draft_sigma=[0.5, 1.0], t_target=1.0, t_draft=[1.0, 1.3], data_seed=V)
+        for scheme in ("single", "IS", "WIS", "SpecTr"):
+            res = run_both(spec, scheme, seed=V + 1, wis_s=min(5, max(1, V)))
+            check(res, scheme)
+
+
+def test_k1_l1_and_s_values():
+    spec = WorkloadSpec("k1", B=16, K=1, L=1, V=3001, dtype="bf16", model_ids=[0], target_scale=3.0,
+                        draft_sigma=[1.0], t_target=0.8, t_draft=[1.1], data_seed=9)
+    for scheme in ("single", "IS", "WIS", "SpecTr"):
+        check(run_both(spec, scheme, seed=2), scheme)
+    spec = small("llama3-128k", B=8, V=3000)
+    for s in (1, 2, 3, 8):
+        check(run_both(spec, "WIS", seed=4, wis_s=s), "WIS")
+
+
+def test_duplicated_tokens_and_peaked_target():
+    # very peaked distributions make most draft tokens coincide
+    spec = WorkloadSpec("peaked", B=16, K=6, L=4, V=2048, dtype="bf16", model_ids=[0] * 6, target_scale=12.0,
+                        draft_sigma=[0.2], t_target=0.5, t_draft=[0.5], data_seed=3)
+    for scheme in ("WIS", "IS", "SpecTr", "single"):
+        check(run_both(spec, scheme, seed=8), scheme)
+
+
+def test_ragged_rows_without_bulk_copies():
+    # V * 2 bytes is not a multiple of 16: every row is fetched with plain loads
+    spec = small("two-models-50k", B=8, V=4097)
+    for scheme in ("WIS", "SpecTr"):
+        check(run_both(spec, scheme, seed=6), scheme)
+    spec = small("tiny", V=1001)        # f32, 4004-byte rows
+    for scheme in ("IS", "WIS"):
+        check(run_both(spec, scheme, seed=6), scheme)
+
+
+def test_mixed_models_and_temperatures():
+    spec = WorkloadSpec("mixed", B=16, K=4, L=4, V=3000, dtype="bf16", model_ids=[0, 1, 0, 2], target_scale=4.0,
+                        draft_sigma=[0.5, 1.5, 1.0], t_target=0.9, t_draft=[1.0, 2.0, 0.7], data_seed=17)
+    for scheme in ("WIS", "IS", "SpecTr", "single"):
+        check(run_both(spec, scheme, seed=13), scheme)
+
+
+FULL = [
+    ("tiny", ["IS", "WIS", "single", "SpecTr"], None),
+    ("llama2-32k", ["IS", "WIS"], [0, 1, 31, 63]),
+    ("two-models-50k", ["WIS", "SpecTr"], [0, 1, 64, 127]),
+    ("llama3-128k", ["WIS"], [0, 1, 100, 255]),
+]
+
+
+@pytest.mark.parametrize("name,schemes,seqs", FULL, ids=[f[0] for f in FULL])
+def test_full_size_workloads_sampled(name, schemes, seqs):
+    spec = WORKLOADS[name]
+    for scheme in schemes:
+        res = run_both(spec, scheme, seed=spec.verify_seed, seqs=seqs)
+        check(res, scheme)
+        assert res["status"] == 0
+
+
+def test_full_size_serving_sampled():
+    spec = WORKLOADS["serving-152k"]
+    for scheme, seqs in (("single", [0, 1, 2, 1023]), ("WIS", [0, 1, 2, 511]), ("SpecTr", [0, 1, 2]),
+                         ("IS", [0, 1])):
+        res = run_both(spec, scheme, seed=1, seqs=seqs)
+        check(res, scheme)
