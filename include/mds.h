@@ -133,6 +133,29 @@ int mds_verify_host(mds_ctx* ctx, const void* target_logits, const void* const* 
                     int scheme, uint64_t philox_seed, int32_t* out_tokens, int32_t* out_accept_len,
                     float* out_diag, int B, void* stream);
 
+/* Variant of mds_verify for callers that cannot allocate device memory:
+ * code that runs where cudaMalloc is not allowed (for example inside a
+ * serving loop whose memory is fixed at start-up, or under an allocator that
+ * forbids growth after warm-up) and so cannot create a context.  It takes
+ * the configuration directly and the same buffers as mds_verify (caller-
+ * owned device memory; same layouts, alignment rules and return codes).  It
+ * allocates nothing: the kernel's scratch (status word and work counter, 8
+ * bytes) lives in a file-scope device array of MDS_NOALLOC_SCRATCH_BYTES that
+ * every GPU loading the library holds until the process exits; a need beyond
+ * that size is rejected with MDS_ESHAPE (the need does not grow with B, K, L
+ * or V).  The first call on a device looks up that array's device address
+ * and sets kernel attributes, so make it before any stream capture.  Every
+ * call clears the scratch on `stream` and then launches; all calls share the
+ * one array, so calls that overlap on the GPU race.  The status word is not
+ * reported (use a context for mds_status).  The paper has no counterpart to
+ * this entry point: it exists only for callers that cannot allocate. */
+#define MDS_NOALLOC_SCRATCH_BYTES 256
+int mds_verify_noalloc(const mds_config* cfg, int device, const void* target_logits,
+                       const void* const* draft_logits, const int32_t* draft_model_id,
+                       const int32_t* draft_tokens, const float* temperatures, int scheme,
+                       uint64_t philox_seed, int32_t* out_tokens, int32_t* out_accept_len, float* out_diag,
+                       int B, void* stream);
+
 /* Synchronise the device, read and clear the status word.  Returns the
  * MDS_ST_* bits (>= 0) or a negative code; *msg (if not NULL) receives a
  * static description of the highest set bit. */

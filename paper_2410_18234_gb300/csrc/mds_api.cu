@@ -353,3 +353,14 @@ void mds_destroy(mds_ctx* ctx) {
 }
 
 }  // extern "C"
+
+// Internal helpers for entry points that have no context (mds_noalloc.cu).
+namespace mds {
+int launch_geometry(const mds_config& cfg, int device, int scheme, int n_models, Params& p) {
+  mds_ctx view;   // host-side view only: no device work, no allocation
+  view.cfg = cfg;
+  view.device = device;
+  return geometry(&view, scheme, n_models, p);
+}
+int prepare_kernels(int dtype) { return ensure_configured(dtype); }
+}  // namespace mds

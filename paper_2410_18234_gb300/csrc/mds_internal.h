@@ -58,4 +58,11 @@ int max_active_clusters(const Params& p);
 // Launch the persistent verification kernel with `clusters` clusters.
 cudaError_t launch(const Params& p, int clusters, cudaStream_t stream);
 
+// Launch geometry (cluster size, slice, row stride, list capacities) that
+// mds_verify would use for this configuration; MDS_OK or MDS_EVOCAB.
+int launch_geometry(const mds_config& cfg, int device, int scheme, int n_models, Params& p);
+
+// One-time kernel attribute set-up for a logit type; MDS_OK or MDS_ECUDA.
+int prepare_kernels(int dtype);
+
 }  // namespace mds

@@ -1,0 +1,126 @@
+// mds_verify_noalloc: the verification entry point for callers that cannot
+// allocate device memory.  See include/mds.h for the contract.
+#include <mutex>
+
+#include "mds_internal.h"
+
+namespace {
+
+// The kernel's scratch: word 0 the status word, word 1 the work counter.
+// Every GPU that loads the library holds this array until the process exits.
+static __device__ __align__(256) unsigned g_noalloc_scratch[MDS_NOALLOC_SCRATCH_BYTES / sizeof(unsigned)];
+
+constexpr size_t kScratchNeeded = 2 * sizeof(unsigned);
+constexpr int kMaxDevices = 64;
+
+std::mutex g_mu;
+unsigned* g_scratch_ptr[kMaxDevices] = {};
+
+bool aligned_to(const void* ptr, size_t a) { return ((uintptr_t)ptr % a) == 0; }
+
+// Device address of the scratch on the current device.  In host code the
+// array's name is only a host-side stand-in; the kernel must get the address
+// cudaGetSymbolAddress returns with the device current.
+int scratch_for(int device, unsigned** out) {
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (!g_scratch_ptr[device]) {
+    void* ptr = nullptr;
+    if (cudaGetSymbolAddress(&ptr, g_noalloc_scratch) != cudaSuccess || !ptr) {
+      cudaGetLastError();
+      return MDS_ECUDA;
+    }
+    g_scratch_ptr[device] = static_cast<unsigned*>(ptr);
+  }
+  *out = g_scratch_ptr[device];
+  return MDS_OK;
+}
+
+}  // namespace
+
+extern "C" int mds_verify_noalloc(const mds_config* cfg_in, int device, const void* target_logits,
+                                  const void* const* draft_logits, const int32_t* draft_model_id,
+                                  const int32_t* draft_tokens, const float* temperatures, int scheme,
+                                  uint64_t philox_seed, int32_t* out_tokens, int32_t* out_accept_len, float* out_diag,
+                                  int B, void* stream) {
+  if (!cfg_in) return MDS_EINVAL;
+  mds_config c = *cfg_in;
+  if (c.wis_s == 0) c.wis_s = 5;
+  if (c.is_h == 0.f) c.is_h = 0.25f;
+  if (c.max_B < 1 || c.K < 1 || c.K > MDS_MAX_K || c.L < 1 || c.L > MDS_MAX_L || c.V < 1 || c.V > (1 << 24))
+    return MDS_ESHAPE;
+  if (c.dtype != MDS_F32 && c.dtype != MDS_BF16) return MDS_EINVAL;
+  if (c.wis_s < 1 || c.wis_s > MDS_MAX_S || !(c.is_h > 0.f) || c.is_h > 4.f) return MDS_EINVAL;
+  if (c.cluster != 0 && c.cluster != 1 && c.cluster != 2 && c.cluster != 4 && c.cluster != 8 && c.cluster != 16)
+    return MDS_EINVAL;
+  if (scheme < MDS_SINGLE || scheme > MDS_SPECTR) return MDS_EINVAL;
+  if (B < 0 || B > c.max_B) return MDS_ESHAPE;
+  // the scratch this launch needs (it does not grow with B, K, L or V)
+  if (kScratchNeeded > MDS_NOALLOC_SCRATCH_BYTES) return MDS_ESHAPE;
+  if (device < 0 || device >= kMaxDevices) return MDS_EINVAL;
+  if (B == 0) return MDS_OK;
+  if (!target_logits || !draft_logits || !draft_model_id || !draft_tokens || !temperatures || !out_tokens ||
+      !out_accept_len)
+    return MDS_EINVAL;
+  const int es = c.dtype == MDS_F32 ? 4 : 2;
+  if (!aligned_to(target_logits, es) || !aligned_to(draft_tokens, 4) || !aligned_to(temperatures, 4) ||
+      !aligned_to(out_tokens, 4) || !aligned_to(out_accept_len, 4) || (out_diag && !aligned_to(out_diag, 4)))
+    return MDS_EINVAL;
+  mds::Params p{};
+  int remap[MDS_MAX_K];
+  for (int m = 0; m < MDS_MAX_K; ++m) remap[m] = -1;
+  int n_models = 0;
+  bool tma_ok = ((size_t)c.V * es) % 16 == 0 && aligned_to(target_logits, 16);
+  for (int k = 0; k < c.K; ++k) {
+    if (!draft_logits[k] || !aligned_to(draft_logits[k], es)) return MDS_EINVAL;
+    tma_ok = tma_ok && aligned_to(draft_logits[k], 16);
+    const int m = draft_model_id[k];
+    if (m < 0 || m >= MDS_MAX_K) return MDS_EINVAL;
+    if (remap[m] < 0) remap[m] = n_models++;
+    p.model_of[k] = (int8_t)remap[m];
+    p.drafts[k] = static_cast<const char*>(draft_logits[k]);
+  }
+  if (scheme == MDS_IS && n_models > MDS_MAX_IS_MODELS) return MDS_EUNSUP;
+
+  int prev = -1;
+  cudaGetDevice(&prev);
+  if (prev != device && cudaSetDevice(device) != cudaSuccess) {
+    cudaGetLastError();
+    return MDS_ECUDA;
+  }
+  int rc = mds::prepare_kernels(c.dtype);
+  unsigned* scratch = nullptr;
+  if (rc == MDS_OK) rc = scratch_for(device, &scratch);
+  p.dtype = c.dtype;
+  if (rc == MDS_OK) rc = mds::launch_geometry(c, device, scheme, n_models, p);
+  if (rc == MDS_OK) {
+    p.target = static_cast<const char*>(target_logits);
+    p.tokens = draft_tokens;
+    p.temps = temperatures;
+    p.out_tokens = out_tokens;
+    p.out_accept = out_accept_len;
+    p.out_diag = out_diag;
+    p.status = scratch;
+    p.queue = scratch + 1;
+    p.ticket0 = 0u;   // the counter is cleared below for every call
+    p.seed = philox_seed;
+    p.B = B;
+    p.K = c.K;
+    p.L = c.L;
+    p.V = c.V;
+    p.wis_s = c.wis_s;
+    p.is_h = c.is_h;
+    p.n_models = n_models;
+    p.tma_ok = tma_ok ? 1 : 0;
+    int clusters = mds::max_active_clusters(p);
+    if (clusters < 1) clusters = 1;
+    if (clusters > B) clusters = B;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (cudaMemsetAsync(scratch, 0, kScratchNeeded, st) != cudaSuccess ||
+        mds::launch(p, clusters, st) != cudaSuccess) {
+      cudaGetLastError();
+      rc = MDS_ECUDA;
+    }
+  }
+  if (prev >= 0 && prev != device) cudaSetDevice(prev);
+  return rc;
+}

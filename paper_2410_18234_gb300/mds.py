@@ -29,8 +29,8 @@ MDS_ST_NONFINITE, MDS_ST_BADTEMP, MDS_ST_ZERO_RESID, MDS_ST_TIMEOUT, MDS_ST_LP_C
 MDS_MAX_K = 16
 
 # every symbol include/mds.h declares
-EXPORTS = ("mds_create", "mds_verify", "mds_verify_host", "mds_status", "mds_cluster_size",
-           "mds_error_string", "mds_destroy")
+EXPORTS = ("mds_create", "mds_verify", "mds_verify_host", "mds_verify_noalloc", "mds_status",
+           "mds_cluster_size", "mds_error_string", "mds_destroy")
 
 
 class MdsConfig(ctypes.Structure):
@@ -59,6 +59,9 @@ def load_library(path=LIB_PATH):
     lib.mds_verify.restype = ctypes.c_int
     lib.mds_verify_host.argtypes = verify_args
     lib.mds_verify_host.restype = ctypes.c_int
+    lib.mds_verify_noalloc.argtypes = [ctypes.POINTER(MdsConfig), ctypes.c_int, vp, ctypes.POINTER(vp), i32p, vp, vp,
+                                       ctypes.c_int, ctypes.c_uint64, vp, vp, f32p, ctypes.c_int, vp]
+    lib.mds_verify_noalloc.restype = ctypes.c_int
     lib.mds_status.argtypes = [vp, ctypes.POINTER(ctypes.c_char_p)]
     lib.mds_status.restype = ctypes.c_int
     lib.mds_cluster_size.argtypes = [vp]
@@ -144,6 +147,29 @@ def mds_verify_host(ctx, target, drafts, model_ids, tokens, temps, scheme, seed,
                               ctypes.c_void_p(int(stream)))
     if rc != MDS_OK:
         raise MdsError(rc, "mds_verify_host")
+
+
+def mds_verify_noalloc(max_B, K, L, V, target, drafts, model_ids, tokens, temps, scheme, seed, out_tokens,
+                       out_accept, out_diag=None, stream=None, dtype="bf16", wis_s=5, is_h=0.25, cluster=0,
+                       device=0):
+    """Context-free entry point for callers that cannot allocate device
+    memory (see include/mds.h): the configuration is passed directly and the
+    kernel's scratch is a static device array inside the library."""
+    cfg = MdsConfig(int(max_B), int(K), int(L), int(V), DTYPES[dtype] if isinstance(dtype, str) else int(dtype),
+                    int(wis_s), float(is_h), int(cluster))
+    Kn = len(model_ids)
+    B = int(tokens.shape[0])
+    if stream is None:
+        stream = torch.cuda.current_stream().cuda_stream
+    elif isinstance(stream, torch.cuda.Stream):
+        stream = stream.cuda_stream
+    rc = _lib.mds_verify_noalloc(ctypes.byref(cfg), int(device), _ptr(target), _draft_ptrs(drafts, Kn),
+                                 _ids(model_ids, Kn), _ptr(tokens), _ptr(temps),
+                                 SCHEMES[scheme] if isinstance(scheme, str) else int(scheme),
+                                 ctypes.c_uint64(int(seed)), _ptr(out_tokens), _ptr(out_accept), _ptr(out_diag), B,
+                                 ctypes.c_void_p(int(stream)))
+    if rc != MDS_OK:
+        raise MdsError(rc, "mds_verify_noalloc")
 
 
 def mds_status(ctx):
