@@ -85,7 +85,7 @@ typedef struct {
   int wis_s;       /* LP truncation threshold s, 1..MDS_MAX_S (0: 5, the value
                       of the paper's experiments, Section 5)                  */
   float is_h;      /* trapezoid step in ln t for plain IS (0: 0.25)           */
-  int cluster;     /* CTAs per sequence: 1, 2, 4, 8 or 16 (0: chosen from V)  */
+  int cluster;     /* CTAs per sequence: 1, 2, 4, 8 or 16 (0: chosen from max_B and the device) */
 } mds_config;
 
 /* Create a context on CUDA device `device`.  Allocates the context's device

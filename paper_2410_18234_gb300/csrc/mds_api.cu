@@ -28,7 +28,7 @@ struct mds_ctx {
 
 namespace {
 
-constexpr size_t kSmemTarget = 66 * 1024;  // dynamic part; with the static state, three CTAs per SM
+constexpr int kRingBytes = 64 * 1024;   // streaming rings: 8 warps x 4 stages of 2 KB
 
 struct DeviceGuard {
   int prev = -1;
@@ -76,44 +76,47 @@ int optin_smem(int device) {
   return v;
 }
 
-// Fill the launch geometry (cluster size, slice, row stride) for n_models
-// distinct draft models.  Returns MDS_OK or MDS_EVOCAB.
+// Fill the launch geometry (cluster size, slice, ring and list sizes) for
+// n_models distinct draft models.  Rows stream through per-warp rings, so
+// shared memory grows with V only through the special-token bitmap and the
+// segment sums; the cluster size sets the slice each CTA streams per depth.
+// Returns MDS_OK or MDS_EVOCAB.
 int geometry(const mds_ctx* ctx, int scheme, int n_models, mds::Params& p) {
   const mds_config& c = ctx->cfg;
   p.esize = esize_of(c.dtype);
   p.rows_max = 1 + n_models;
   p.scheme = scheme;
-  // WIS candidate lists (target + up to 3 draft models); the merged list
-  // shares its memory with the special-token bitmap, so it is sized to at
-  // least 64 entries and otherwise to the bitmap's bytes
+  p.ring_bytes = kRingBytes;
   const bool lists = scheme == MDS_WIS && p.rows_max <= 4;
-  const size_t limit = (size_t)optin_smem(ctx->device) - 12 * 1024;  // static shared state
   auto fill = [&](int cn) {
     p.cn = cn;
     p.slice = (int)round_up((size_t)((c.V + cn - 1) / cn), 8);
-    p.row_stride = (int)round_up((size_t)p.slice * p.esize, 128);
     if (lists) {
-      const int bm_bytes = (p.slice + 31) / 32 * 4;
-      p.cand_cap = bm_bytes / (4 * (3 + p.rows_max));
-      if (p.cand_cap < 64) p.cand_cap = 64;
-      if (p.cand_cap > 512) p.cand_cap = 512;
-      p.cand_cap_cta = p.cand_cap < 64 ? p.cand_cap : 64;
+      p.cand_cap = mds::kListN;
+      p.cand_stage = cn * mds::kListN;
     } else {
-      p.cand_cap = p.cand_cap_cta = 0;
+      p.cand_cap = p.cand_stage = 0;
     }
     return mds::smem_bytes(p);
   };
-  if (c.cluster > 0) {
-    if (fill(c.cluster) > limit) return MDS_EVOCAB;
-    return MDS_OK;
+  const size_t limit = (size_t)optin_smem(ctx->device) - 12 * 1024;  // static shared state
+  int cn = c.cluster;
+  if (cn <= 0) {
+    // Every sequence is a serial chain of depths, so as many sequences as
+    // possible should be in flight: the largest cluster with cn * max_B
+    // within the co-resident CTAs (two per SM), then larger while two CTAs
+    // per SM would not fit the shared memory.
+    int sms = 0, per_sm = 0;
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, ctx->device);
+    cudaDeviceGetAttribute(&per_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, ctx->device);
+    const long slots = 2L * (sms > 0 ? sms : 1);
+    cn = 1;
+    while (cn < mds::kMaxCluster && 2L * cn * (c.max_B > 0 ? c.max_B : 1) <= slots) cn *= 2;
+    while (cn < mds::kMaxCluster && 2 * (fill(cn) + 12 * 1024) > (size_t)per_sm) cn *= 2;
+    while (cn > 1 && (c.V + cn - 1) / cn < 8) cn /= 2;
   }
-  for (int cn = 1; cn <= mds::kMaxCluster; cn *= 2) {
-    if (cn > 1 && (c.V + cn - 1) / cn < 8) break;
-    if (fill(cn) <= kSmemTarget) return MDS_OK;
-  }
-  for (int cn = 1; cn <= mds::kMaxCluster; cn *= 2)
-    if (fill(cn) <= limit) return MDS_OK;
-  return MDS_EVOCAB;
+  if (fill(cn) > limit) return MDS_EVOCAB;
+  return MDS_OK;
 }
 
 int clusters_for(mds_ctx* ctx, const mds::Params& p) {

@@ -15,6 +15,7 @@ constexpr int kIsNodesMax = 1024;      // trapezoid nodes for plain IS
 constexpr int kIsChunk = 16;           // nodes accumulated per pass
 constexpr int kXch = 34;               // floats one CTA contributes to a cluster exchange
 constexpr int kMaxCluster = 16;
+constexpr int kListN = 32;             // WIS candidate list: the largest target logits of a sequence
 
 struct Params {
   const char* target;                  // [B][K][L+1][V]
@@ -36,12 +37,12 @@ struct Params {
   float is_h;
   int cn;                              // CTAs per cluster
   int slice;                           // tokens per CTA (multiple of 8)
-  int row_stride;                      // bytes per smem row (multiple of 128)
-  int rows_max;                        // smem rows (1 + distinct models)
+  int ring_bytes;                      // streaming ring (kStages stages)
+  int rows_max;                        // rows per depth at most (1 + distinct models)
   int n_models;                        // distinct draft models (ids are 0..n_models-1 after remap)
   int tma_ok;                          // rows are 16-byte aligned with 16-byte-multiple length
-  int cand_cap_cta;                    // WIS candidate list capacity per CTA (0: no candidate path)
-  int cand_cap;                        // WIS merged candidate list capacity per cluster
+  int cand_cap;                        // WIS candidate list capacity (kListN; 0: no candidate path)
+  int cand_stage;                      // WIS staging capacity (every CTA's list: cn * kListN)
   int8_t model_of[MDS_MAX_K];          // remapped model id per branch
 };
 

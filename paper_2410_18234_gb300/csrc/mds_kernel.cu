@@ -4,22 +4,26 @@
 // sequences taken from a work counter (a persistent kernel sized to the
 // co-resident clusters).  CTA r of the cluster owns tokens
 // [r*slice, (r+1)*slice) of every row.  Per depth j of the walk it
-//   1. bulk-copies (cp.async.bulk, mbarrier completion) its slice of the
-//      target row and of one row per distinct draft model into shared memory,
-//   2. computes the temperature-softmax statistics (max, sum of exp) of each
-//      row and combines them across the cluster through distributed shared
-//      memory,
-//   3. runs the importance step of the selected scheme (Definition 1 /
-//      Theorem 1), reading the rows from shared memory,
-//   4. applies Algorithm 1 (accept with probability min(1, q(Y)/p_I(Y)), else
-//      an inverse-CDF draw from max(0, q - p_I) in token order), and
-//   5. advances the walk: continue while the output is one of the valid draft
+//   1. streams its slice of the target row and of one row per distinct draft
+//      model through a small shared-memory ring (cp.async.bulk with mbarrier
+//      completion), computing the temperature-softmax statistics online and,
+//      for the weighted scheme, collecting the candidate tokens; one exchange
+//      over distributed shared memory combines the cluster,
+//   2. runs the importance step of the selected scheme (Definition 1 /
+//      Theorem 1) -- for the weighted scheme on the candidate list alone
+//      whenever that list provably holds every stage's Omega_1,
+//   3. applies Algorithm 1 (accept with probability min(1, q(Y)/p_I(Y)), else
+//      an inverse-CDF draw from max(0, q - p_I) in token order, streaming the
+//      rows again, typically from L2), and
+//   4. advances the walk: continue while the output is one of the valid draft
 //      tokens (Problem 1's event Z in S); after L accepted positions draw the
 //      bonus token from the target row at depth L.
-// Every decision is taken redundantly and identically by every CTA of the
-// cluster from cluster-combined values, so control flow stays uniform and
-// the cluster barriers always match.  There are no spin-waits across CTAs;
-// the only wait is on this CTA's own bulk copies and it is bounded.
+// Rows are not kept resident, so shared memory does not bound how many
+// sequences are in flight.  Every decision is taken redundantly and
+// identically by every CTA of the cluster from cluster-combined values, so
+// control flow stays uniform and the cluster barriers always match.  No CTA
+// waits on another CTA's flag; the only waits are on this CTA's own bulk
+// copies and they are bounded.
 #include <cuda_bf16.h>
 #include <cooperative_groups.h>
 
@@ -38,8 +42,17 @@ constexpr int kLpMaxAugment = 4096;
 constexpr float kLpEpsRel = 1e-6f;
 constexpr long long kWaitLimit = 1ll << 24;
 constexpr int kFastRows = 4;            // WIS candidate path: target + up to 3 draft models
-constexpr int kCandLevels = 4;          // candidate levels: q >= q_max * 2^-(12, 10, 8, 6)
-__host__ __device__ constexpr float cand_log2(int level) { return 12.f - 2.f * (float)level; }
+constexpr int kWStages = 4;             // stages of each warp's streaming ring
+constexpr int kWarpApp = 128;           // candidate tokens one warp can hold during the stats pass
+
+// Order-preserving map of floats (not NaN) to unsigned; every key is > 0.
+__device__ __forceinline__ unsigned ord_key(float f) {
+  const unsigned u = __float_as_uint(f);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ float ord_val(unsigned k) {
+  return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);
+}
 
 // ------------------------------------------------------------------ PTX helpers
 
@@ -72,8 +85,8 @@ __device__ __forceinline__ void st_dsmem(int* local, uint32_t rank, int v) {
 }
 __device__ __forceinline__ void mbar_init(uint64_t* bar) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(bar)));
-  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
 }
+__device__ __forceinline__ void mbar_init_fence() { asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory"); }
 __device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes) : "memory");
 }
@@ -138,6 +151,13 @@ struct Elt<MDS_F32> {
   __device__ static __forceinline__ float global(const char* row, int x) {
     return __ldg(reinterpret_cast<const float*>(row) + x);
   }
+  __device__ static __forceinline__ void unit_global(const char* at, float* v) {
+    const float4 x = __ldg(reinterpret_cast<const float4*>(at));
+    v[0] = x.x;
+    v[1] = x.y;
+    v[2] = x.z;
+    v[3] = x.w;
+  }
 };
 template <>
 struct Elt<MDS_BF16> {
@@ -155,6 +175,17 @@ struct Elt<MDS_BF16> {
   }
   __device__ static __forceinline__ float global(const char* row, int x) {
     return __uint_as_float((uint32_t)__ldg(reinterpret_cast<const unsigned short*>(row) + x) << 16);
+  }
+  __device__ static __forceinline__ void unit_global(const char* at, float* v) {
+    const uint4 x = __ldg(reinterpret_cast<const uint4*>(at));
+    v[0] = __uint_as_float(x.x << 16);
+    v[1] = __uint_as_float(x.x & 0xffff0000u);
+    v[2] = __uint_as_float(x.y << 16);
+    v[3] = __uint_as_float(x.y & 0xffff0000u);
+    v[4] = __uint_as_float(x.z << 16);
+    v[5] = __uint_as_float(x.z & 0xffff0000u);
+    v[6] = __uint_as_float(x.w << 16);
+    v[7] = __uint_as_float(x.w & 0xffff0000u);
   }
 };
 
@@ -198,7 +229,9 @@ struct State {
   float xch[2][kXch];
   float gat[kMaxCluster * kXch];
   // block reduction scratch
-  float red[kWarps * 2 * kMaxRows];
+  float red[kWarps * 3 * kMaxRows];
+  float wthr[kWarps];        // per warp: bound on the target logits outside its list
+  float wtau[kWarps];        // per warp: largest target logit dropped at a merge
   Cand wcand[kWarps * kTop];
   Cand blk[kTop];
   Cand fin[kTop];
@@ -217,7 +250,6 @@ struct State {
   float pc[kMaxRows];        // complement exp mass per row
   int ncand, cand_all, fast_ok;
   float cand_q;
-  int wlev[kWarps * kCandLevels];
   // SpecTr: inverse residual masses of rejected rounds
   float sp_invR[MDS_MAX_K];
   int sp_rows[MDS_MAX_K];
@@ -228,7 +260,10 @@ struct State {
   // CDF search
   int owner, seg;
   float run, T;
-  uint64_t mbar;
+  // streaming: one ring per warp, one mbarrier per stage
+  uint64_t wbar[kWarps][kWStages];
+  int wapp[kWarps];          // tokens each warp set aside (may exceed kWarpApp: overflow)
+  float thr_cta;
 };
 
 // ------------------------------------------------------------------ reductions
@@ -353,6 +388,35 @@ __device__ __forceinline__ void cand_insert(Cand (&top)[kTop], const Cand& c, fl
 
 // ------------------------------------------------------------------ the kernel
 
+// Unit lu of row r in the current ring stage (rows of the pass in mask order).
+template <int DT>
+struct StageLoad {
+  const char* base;
+  uint32_t mask;
+  int cb;
+  int lu;
+  __device__ __forceinline__ void operator()(int r, float* v) const {
+    Elt<DT>::unit(base + __popc(mask & ((1u << r) - 1u)) * cb, lu, v);
+  }
+};
+// Unit gu of row r straight from global memory (logits past V read -inf);
+// one 16-byte load when the rows are 16-byte aligned and the unit is whole.
+template <int DT>
+struct GlobalLoad {
+  const char* const* gptr;
+  int tok0, V, gu;
+  bool aligned;
+  __device__ __forceinline__ void operator()(int r, float* v) const {
+    const int t0 = tok0 + gu * Elt<DT>::VE;
+    if (aligned && t0 + Elt<DT>::VE <= V) {
+      Elt<DT>::unit_global(gptr[r] + (size_t)t0 * (16 / Elt<DT>::VE), v);
+      return;
+    }
+#pragma unroll
+    for (int e = 0; e < Elt<DT>::VE; ++e) v[e] = (t0 + e < V) ? Elt<DT>::global(gptr[r], t0 + e) : kNegInf;
+  }
+};
+
 template <int DT, int SCHEME>
 struct Kernel {
   using E = Elt<DT>;
@@ -360,147 +424,599 @@ struct Kernel {
 
   const Params& p;
   State& S;
-  char* rows;          // rows_max x row_stride
+  char* ring;          // streaming rings: kWarps x kWStages stages
   uint32_t* bitmap;    // special-token bits of this CTA's slice
   float* segsum;       // per-segment residual sums
   float* isW;          // IS: weights [rows][kIsNodesMax]
   float* isT;          // IS: nodes t_n
-  int* cl_id;          // WIS: this CTA's candidates (token order) ...
-  float* cl_e;         //      ... and their exp values per row [rows][cap_cta]
+  char* cl_base;       // WIS: this CTA's buffered tokens and their logits per row,
+                       //      two alternating copies of [cap_cta] ids + [rows][cap_cta] logits
+  int* ap_id;          // WIS: tokens each warp set aside during the stats pass ...
+  float* ap_l;         //      ... and their logits per row [rows][kWarps * kWarpApp]
+  int* cs_id;          // WIS: every CTA's kept tokens (rank order) ...
+  float* cs_l;         //      ... their logits [rows][stage]
+  float* cs_x;         //      ... and the target's scaled log-ratio
   int* cm_id;          // WIS: the cluster's merged candidates (token order) ...
   float* cm_e;         //      ... exp values per row [rows][cap]
   float* cm_a;         //      ... current law value of special tokens
   int* cm_sp;          //      ... special flag
-  int rank, cn, tok0, nvalid, U, nseg, bm_words;
+  int rank, cn, tok0, nvalid, Uv, Uw, nseg, nsegv, bm_words;   // nseg: layout (slice); nsegv: written (valid units)
   int xbuf;
-  uint32_t mphase;
-
-  __device__ const char* srow(int r) const { return rows + (size_t)r * p.row_stride; }
+  int clbuf;           // which copy of the CTA list the next candidate pass publishes
+  uint32_t wphase;     // parity of each stage of this warp's ring
 
   __device__ float prob_row(int r, int x) const {
     return prob_of(E::global(S.gptr[r], x), S.M[r], S.c[r], S.invZ[r]);
   }
 
-  // ---------------------------------------------------------------- loads
-  __device__ void load_rows() {
-    const int nr = S.nrows;
-    const int tid = threadIdx.x;
-    const int vbytes = nvalid * p.esize;
-    const int tma_bytes = p.tma_ok ? (vbytes & ~15) : 0;
-    // padding (tokens past V) reads as -inf; plain loads for what bulk copies skip
-    for (int r = 0; r < nr; ++r) {
-      char* dst = rows + (size_t)r * p.row_stride;
-      const char* src = S.gptr[r] + (size_t)tok0 * p.esize;
-      for (int i = tid; i < p.slice - nvalid; i += kThreads) {
-        const int t = nvalid + i;
-        if (DT == MDS_F32)
-          reinterpret_cast<float*>(dst)[t] = kNegInf;
-        else
-          reinterpret_cast<unsigned short*>(dst)[t] = 0xff80u;
-      }
-      for (int byte = tma_bytes + tid * p.esize; byte < vbytes; byte += kThreads * p.esize) {
-        if (DT == MDS_F32)
-          *reinterpret_cast<float*>(dst + byte) = __ldg(reinterpret_cast<const float*>(src + byte));
-        else
-          *reinterpret_cast<unsigned short*>(dst + byte) = __ldg(reinterpret_cast<const unsigned short*>(src + byte));
-      }
+  // ---------------------------------------------------------------- streaming engine
+  // Warp w owns units [w*Uw, min((w+1)*Uw, Uv)) of the CTA's slice (Uw a
+  // multiple of 32) and walks them in groups of 32, one unit per lane:
+  // fn(gu, valid, L) is called by all 32 lanes together, gu the unit's index
+  // in the slice (a group starts at a multiple of 32) and L(r, v) loading
+  // unit gu of row r.  With 16-byte aligned rows the rows of `mask` flow
+  // through the warp's own ring of kWStages stages (cp.async.bulk issued by
+  // lane 0 up to kWStages stages ahead, completion counted on the stage's
+  // mbarrier); otherwise, or when a stage could not hold a group of every
+  // row, units are loaded straight from global memory.  No block barrier is
+  // taken inside a pass, nor at its end: a caller synchronises the block
+  // before reading what other warps wrote.  Every wait is bounded.
+  __device__ __forceinline__ int stage_units(int nrm) const {
+    return ((p.ring_bytes / kWarps / kWStages) / (16 * nrm)) & ~31;
+  }
+
+  __device__ __forceinline__ void issue_stage(int c, uint32_t mask, int su, int u0, int u1) {
+    const int warp = threadIdx.x >> 5;
+    const int stage = c % kWStages;
+    char* dst = ring + (size_t)(warp * kWStages + stage) * (p.ring_bytes / kWarps / kWStages);
+    const int cu0 = u0 + c * su;
+    const int bytes = (min(cu0 + su, u1) - cu0) * 16;
+    mbar_expect_tx(&S.wbar[warp][stage], (uint32_t)(bytes * __popc(mask)));
+    int pos = 0;
+    for (int r = 0; r < S.nrows; ++r) {
+      if (!(mask >> r & 1u)) continue;
+      bulk_copy(dst + pos * su * 16, S.gptr[r] + ((size_t)tok0 + (size_t)cu0 * VE) * p.esize, (uint32_t)bytes,
+                &S.wbar[warp][stage]);
+      ++pos;
     }
-    if (tma_bytes > 0) {
-      if (tid == 0) {
-        fence_proxy_async();
-        mbar_expect_tx(&S.mbar, (uint32_t)(tma_bytes * nr));
-        for (int r = 0; r < nr; ++r)
-          bulk_copy(rows + (size_t)r * p.row_stride, S.gptr[r] + (size_t)tok0 * p.esize, (uint32_t)tma_bytes,
-                    &S.mbar);
+  }
+
+  template <class FN>
+  __device__ void stream(uint32_t mask, FN&& fn) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int u0 = warp * Uw, u1 = min(u0 + Uw, Uv);
+    if (u0 >= u1) return;
+    const int nrm = __popc(mask);
+    const int su = stage_units(nrm);
+    if (!p.tma_ok || su < 32) {
+      for (int g = u0; g < u1; g += 32) {
+        const int gu = g + lane;
+        fn(gu, gu < u1, GlobalLoad<DT>{S.gptr, tok0, p.V, gu, p.tma_ok != 0});
       }
+      return;
+    }
+    const int nch = (u1 - u0 + su - 1) / su;
+    if (lane == 0) {
+      fence_proxy_async();
+      for (int c = 0; c < nch && c < kWStages; ++c) issue_stage(c, mask, su, u0, u1);
+    }
+    __syncwarp();
+    for (int c = 0; c < nch; ++c) {
+      const int stage = c % kWStages;
+      const char* base = ring + (size_t)(warp * kWStages + stage) * (p.ring_bytes / kWarps / kWStages);
       long long spins = 0;
-      while (!mbar_try_wait(&S.mbar, mphase)) {
+      while (!mbar_try_wait(&S.wbar[warp][stage], (wphase >> stage) & 1u)) {
         if (++spins > kWaitLimit) {
-          if (tid == 0) atomicOr(p.status, MDS_ST_TIMEOUT);
+          if (lane == 0) atomicOr(p.status, MDS_ST_TIMEOUT);
           break;
         }
       }
-      mphase ^= 1u;
+      wphase ^= 1u << stage;
+      const int cu0 = u0 + c * su, cu1 = min(cu0 + su, u1);
+      for (int g = cu0; g < cu1; g += 32) {
+        const int gu = g + lane;
+        fn(gu, gu < cu1, StageLoad<DT>{base, mask, su * 16, g - cu0 + lane});
+      }
+      __syncwarp();
+      if (lane == 0 && c + kWStages < nch) {
+        fence_proxy_async();
+        issue_stage(c + kWStages, mask, su, u0, u1);
+      }
+      __syncwarp();
     }
-    __syncthreads();
   }
 
-  // ---------------------------------------------------------------- stats
-  // Softmax statistics of every loaded row: M = max logit, Z = sum exp((l-M)/T).
-  __device__ void row_stats() {
-    const int nr = S.nrows;
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    for (int r = 0; r < nr; ++r) {
-      const char* row = srow(r);
-      const float c = S.c[r];
-      float m = kNegInf;
-      for (int u = threadIdx.x; u < U; u += kThreads) {
-        float v[VE];
-        E::unit(row, u, v);
+  // ---------------------------------------------------------------- softmax statistics
+  // Candidate order: larger target logit first, then smaller token id.
+  __device__ __forceinline__ static bool cand_before(float la, int ia, float lb, int ib) {
+    return la > lb || (la == lb && ia < ib);
+  }
+
+  // Warp-wide: raise `theta` to the kListN-th largest target logit among the
+  // warp's set-aside list and the tokens of the current group flagged in
+  // `aside` (bisection on order-preserving keys), drop the list entries at
+  // or below it (their exp values join the warp's pruned sums: reference
+  // max pm, sum ps, both warp-uniform; the reference only grows and every
+  // logit of the list is <= the warp's running max of its row) and unflag
+  // the group's tokens at or below it.  Fewer than kListN entries remain,
+  // so the flagged tokens fit.  Returns the new length.
+  template <int R>
+  __device__ int prune_warp_list(int napp, float& theta, uint32_t& aside, const float (&v0)[VE], const float (&m)[R],
+                                 const float (&cr)[R], float (&pm)[R], float (&ps)[R], int* wa_id, float* wa_l) {
+    const int lane = threadIdx.x & 31;
+    constexpr int kPer = kWarpApp / 32;
+    unsigned lk[kPer], gk[VE];
 #pragma unroll
-        for (int e = 0; e < VE; ++e) m = fmaxf(m, v[e]);
+    for (int k = 0; k < kPer; ++k) lk[k] = (k * 32 + lane < napp) ? ord_key(wa_l[k * 32 + lane]) : 0u;
+#pragma unroll
+    for (int e = 0; e < VE; ++e) gk[e] = ((aside >> e) & 1u) ? ord_key(v0[e]) : 0u;
+    // the largest key with at least kListN keys >= it (0: fewer keys); the
+    // low 16 bits of a key are zero for bf16 logits
+    unsigned t = 0u;
+#pragma unroll 1
+    for (int bit = 31; bit >= (DT == MDS_BF16 ? 16 : 0); --bit) {
+      const unsigned c = t | (1u << bit);
+      int cnt = 0;
+#pragma unroll
+      for (int k = 0; k < kPer; ++k) cnt += (lk[k] >= c) ? 1 : 0;
+#pragma unroll
+      for (int e = 0; e < VE; ++e) cnt += (gk[e] >= c) ? 1 : 0;
+      if (__reduce_add_sync(0xffffffffu, cnt) >= kListN) t = c;
+    }
+    if (t != 0u) theta = fmaxf(theta, ord_val(t));
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      float wm = m[r];
+#pragma unroll
+      for (int o = 16; o; o >>= 1) wm = fmaxf(wm, __shfl_xor_sync(0xffffffffu, wm, o));
+      if (wm > pm[r]) {
+        ps[r] = (pm[r] == kNegInf) ? 0.f : __fmul_rn(ps[r], ex2(__fmul_rn(__fsub_rn(pm[r], wm), cr[r])));
+        pm[r] = wm;
       }
-      float s = 0.f;
-      if (m != kNegInf) {
-        for (int u = threadIdx.x; u < U; u += kThreads) {
-          float v[VE];
-          E::unit(row, u, v);
+    }
+    float add[R];
 #pragma unroll
-          for (int e = 0; e < VE; ++e) s += ex2(__fmul_rn(__fsub_rn(v[e], m), c));
+    for (int r = 0; r < R; ++r) add[r] = 0.f;
+    int outp = 0;
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) {
+      // entries move only towards the front: read this slice, then write it
+      const int i = k * 32 + lane;
+      const bool present = i < napp;
+      int id = 0;
+      float l[R];
+#pragma unroll
+      for (int r = 0; r < R; ++r) l[r] = kNegInf;
+      if (present) {
+        id = wa_id[i];
+#pragma unroll
+        for (int r = 0; r < R; ++r) l[r] = wa_l[r * kWarps * kWarpApp + i];
+      }
+      const bool keep = present && l[0] > theta;
+      const uint32_t bal = __ballot_sync(0xffffffffu, keep);
+      __syncwarp();
+      if (keep) {
+        const int pos = outp + __popc(bal & ((1u << lane) - 1u));
+        wa_id[pos] = id;
+#pragma unroll
+        for (int r = 0; r < R; ++r) wa_l[r * kWarps * kWarpApp + pos] = l[r];
+      } else if (present) {
+#pragma unroll
+        for (int r = 0; r < R; ++r)
+          if (l[r] > kNegInf) add[r] = __fadd_rn(add[r], ex2(__fmul_rn(__fsub_rn(l[r], pm[r]), cr[r])));
+      }
+      outp += __popc(bal);
+      __syncwarp();
+    }
+#pragma unroll
+    for (int r = 0; r < R; ++r) ps[r] = __fadd_rn(ps[r], warp_sum(add[r]));
+#pragma unroll
+    for (int e = 0; e < VE; ++e)
+      if (!(v0[e] > theta)) aside &= ~(1u << e);
+    return outp;
+  }
+
+  // One streaming pass over rows [r0, r0 + R): per thread an online max and a
+  // sum of exp((l - m) c) per row, rescaled once per unit.  With CAND (WIS,
+  // R = all rows) the pass also finds the kListN largest target logits of the
+  // sequence (ties: smaller token id first), which are kept out of the sums:
+  // each warp sets aside every token above `theta`, the kListN-th largest
+  // target logit it kept so far, and prunes its list back to kListN when it
+  // fills; the CTA keeps the first kListN of its warps' lists and the
+  // cluster the first kListN of its CTAs' lists.  Every pruned or never
+  // set-aside token has a target logit <= tau, the last kept one.  One
+  // cluster exchange gives every CTA M and Z of each row, the candidate list
+  // (by token id, exp values per row) and the complement's exp mass per row
+  // (S.pc), so Omega_2 masses need no 1 - sum.
+  template <int R, bool CAND>
+  __device__ void stats_pass(int r0) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    float m[R], sc[R], cr[R];
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      m[r] = kNegInf;
+      sc[r] = 0.f;
+      cr[r] = S.c[r0 + r];
+    }
+    float theta = kNegInf;              // warp-uniform
+    int napp = 0;                       // this warp's set-aside tokens (warp-uniform)
+    float pm[R], ps[R];                 // pruned set-aside tokens: reference max and sum (warp-uniform)
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      pm[r] = kNegInf;
+      ps[r] = 0.f;
+    }
+    int* wa_id = ap_id + warp * kWarpApp;
+    float* wa_l = ap_l + warp * kWarpApp;   // row r at wa_l[r * kWarps * kWarpApp + i]
+    const uint32_t mask = ((1u << R) - 1u) << r0;
+    stream(mask, [&](int gu, bool valid, const auto& L) {
+      // row 0 first: its values decide which tokens are set aside
+      float v0[VE];
+      if (valid) {
+        L(r0, v0);
+      } else {
+#pragma unroll
+        for (int e = 0; e < VE; ++e) v0[e] = kNegInf;
+      }
+      uint32_t aside = 0u;
+      if constexpr (CAND) {
+        float mu = v0[0];
+#pragma unroll
+        for (int e = 1; e < VE; ++e) mu = fmaxf(mu, v0[e]);
+        const int t0 = tok0 + gu * VE;
+#pragma unroll
+        for (int e = 0; e < VE; ++e)
+          if (t0 + e < p.V && v0[e] > theta) aside |= 1u << e;
+        const int nadd = __reduce_add_sync(0xffffffffu, __popc(aside));
+        if (nadd) {
+          if (napp + nadd > kWarpApp) {
+            if (mu > m[0]) {   // keep the running maxima current for the pruned sums
+              sc[0] = (m[0] == kNegInf) ? 0.f : __fmul_rn(sc[0], ex2(__fmul_rn(__fsub_rn(m[0], mu), cr[0])));
+              m[0] = mu;
+            }
+            napp = prune_warp_list<R>(napp, theta, aside, v0, m, cr, pm, ps, wa_id, wa_l);
+          }
+          // append in lane order, each lane its flagged tokens in token order;
+          // the other rows' logits are re-read from the unit
+          int cnt = __popc(aside), incl = cnt;
+#pragma unroll
+          for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += y;
+          }
+          int pos = napp + incl - cnt;
+          if (aside) {
+            float vr[VE];
+#pragma unroll
+            for (int e = 0; e < VE; ++e)
+              if ((aside >> e) & 1u) {
+                wa_id[pos] = t0 + e;
+                wa_l[pos] = v0[e];
+                ++pos;
+              }
+#pragma unroll
+            for (int r = 1; r < R; ++r) {
+              L(r0 + r, vr);
+              int q = napp + incl - cnt;
+#pragma unroll
+              for (int e = 0; e < VE; ++e)
+                if ((aside >> e) & 1u) wa_l[r * kWarps * kWarpApp + q++] = vr[e];
+            }
+          }
+          napp += __shfl_sync(0xffffffffu, incl, 31);
         }
       }
 #pragma unroll
+      for (int r = 0; r < R; ++r) {
+        float v[VE];
+        if (r == 0) {
+#pragma unroll
+          for (int e = 0; e < VE; ++e) v[e] = v0[e];
+        } else if (valid) {
+          L(r0 + r, v);
+        } else {
+#pragma unroll
+          for (int e = 0; e < VE; ++e) v[e] = kNegInf;
+        }
+        float mu = v[0];
+#pragma unroll
+        for (int e = 1; e < VE; ++e) mu = fmaxf(mu, v[e]);
+        if (mu > m[r]) {
+          sc[r] = (m[r] == kNegInf) ? 0.f : __fmul_rn(sc[r], ex2(__fmul_rn(__fsub_rn(m[r], mu), cr[r])));
+          m[r] = mu;
+        }
+#pragma unroll
+        for (int e = 0; e < VE; ++e)
+          if (!((aside >> e) & 1u) && v[e] > kNegInf) sc[r] = __fadd_rn(sc[r], ex2(__fmul_rn(__fsub_rn(v[e], m[r]), cr[r])));
+      }
+    });
+    if constexpr (CAND) {
+      __syncwarp();
+      if (napp > kListN) {   // at most kListN entries per warp for the CTA merge
+        uint32_t none = 0u;
+        float nv[VE];
+#pragma unroll
+        for (int e = 0; e < VE; ++e) nv[e] = kNegInf;
+        napp = prune_warp_list<R>(napp, theta, none, nv, m, cr, pm, ps, wa_id, wa_l);
+      }
+    }
+    // block: combine (max, sum) per row
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      float mm = m[r], ss = sc[r];
+      if (CAND && lane == 0) combine_ms(mm, ss, pm[r], ps[r], cr[r]);
+#pragma unroll
       for (int o = 16; o; o >>= 1) {
-        const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
-        const float s2 = __shfl_xor_sync(0xffffffffu, s, o);
-        combine_ms(m, s, m2, s2, c);
+        const float m2 = __shfl_xor_sync(0xffffffffu, mm, o);
+        const float s2 = __shfl_xor_sync(0xffffffffu, ss, o);
+        combine_ms(mm, ss, m2, s2, cr[r]);
       }
       if (lane == 0) {
-        S.red[(warp * kMaxRows + r) * 2] = m;
-        S.red[(warp * kMaxRows + r) * 2 + 1] = s;
+        S.red[(warp * kMaxRows + r) * 2] = mm;
+        S.red[(warp * kMaxRows + r) * 2 + 1] = ss;
       }
     }
+    if (CAND && lane == 0) {
+      S.wapp[warp] = napp;
+      S.wthr[warp] = theta;   // every token of the warp outside its list has a target logit <= theta
+    }
     __syncthreads();
-    if (threadIdx.x < nr) {
+    constexpr int nx = CAND ? 3 * R + 2 : 2 * R;
+    constexpr int sx = CAND ? 3 : 2;   // exchange stride per row: max, complement sum[, list sum]
+    if (threadIdx.x < R) {
       const int r = threadIdx.x;
-      float m = kNegInf, s = 0.f;
+      float mm = kNegInf, ss = 0.f;
       for (int w = 0; w < kWarps; ++w)
-        combine_ms(m, s, S.red[(w * kMaxRows + r) * 2], S.red[(w * kMaxRows + r) * 2 + 1], S.c[r]);
-      S.xch[xbuf][2 * r] = m;
-      S.xch[xbuf][2 * r + 1] = s;
+        combine_ms(mm, ss, S.red[(w * kMaxRows + r) * 2], S.red[(w * kMaxRows + r) * 2 + 1], cr[r]);
+      S.xch[xbuf][sx * r] = mm;
+      S.xch[xbuf][sx * r + 1] = ss;
     }
-    cluster_gather(S, 2 * nr, xbuf, cn);
-    if (threadIdx.x < nr) {
-      const int r = threadIdx.x;
-      float m = kNegInf, s = 0.f;
-      for (int q = 0; q < cn; ++q) combine_ms(m, s, S.gat[q * 2 * nr + 2 * r], S.gat[q * 2 * nr + 2 * r + 1], S.c[r]);
-      if (!(m > kNegInf) || !(s > 0.f) || !(s < kPosInf) || m != m) {
-        atomicOr(p.status, MDS_ST_NONFINITE);
-        if (m != m || m == kNegInf) m = 0.f;
-        if (!(s > 0.f) || s != s) s = 1.f;
+    if constexpr (CAND) {
+      __syncthreads();
+      // CTA list: the first kListN of the warps' lists (entry t: warp t / 32,
+      // slot t % 32); the others join the CTA's complement sums, the kept ones
+      // its list sums (both relative to the CTA's row max)
+      float pr_s[R], kp_s[R];
+#pragma unroll
+      for (int r = 0; r < R; ++r) {
+        pr_s[r] = 0.f;
+        kp_s[r] = 0.f;
       }
-      S.M[r] = m;
-      S.invZ[r] = __frcp_rn(s);
+      int* cl_id = reinterpret_cast<int*>(cl_base) + clbuf * kListN * (1 + p.rows_max);
+      float* cl_l = reinterpret_cast<float*>(cl_id + kListN);
+      float tau_t = kNegInf;   // largest target logit this thread drops
+      {
+        const int w = threadIdx.x >> 5, slot = threadIdx.x & 31;
+        static_assert(kListN == 32 && kWarps * 32 == kThreads, "one warp-list entry per thread");
+        if (slot < S.wapp[w]) {
+          const int i = w * kWarpApp + slot;
+          const float l0 = ap_l[i];
+          const int id = ap_id[i];
+          int rk = 0;
+          for (int w2 = 0; w2 < kWarps; ++w2) {
+            const int n2 = S.wapp[w2];
+            for (int j = 0; j < n2; ++j)
+              rk += cand_before(ap_l[w2 * kWarpApp + j], ap_id[w2 * kWarpApp + j], l0, id) ? 1 : 0;
+          }
+#pragma unroll
+          for (int r = 0; r < R; ++r) {
+            const float l = ap_l[r * kWarps * kWarpApp + i];
+            const float ev = (l > kNegInf) ? ex2(__fmul_rn(__fsub_rn(l, S.xch[xbuf][sx * r]), cr[r])) : 0.f;
+            if (rk < kListN)
+              kp_s[r] = ev;
+            else
+              pr_s[r] = ev;
+          }
+          if (rk < kListN) {
+            cl_id[rk] = id;
+#pragma unroll
+            for (int r = 0; r < R; ++r) cl_l[r * kListN + rk] = ap_l[r * kWarps * kWarpApp + i];
+          } else {
+            tau_t = l0;
+          }
+        }
+      }
+#pragma unroll
+      for (int o = 16; o; o >>= 1) tau_t = fmaxf(tau_t, __shfl_xor_sync(0xffffffffu, tau_t, o));
+      int nk = 0;
+      for (int w = 0; w < kWarps; ++w) nk += S.wapp[w];
+      nk = min(nk, kListN);
+#pragma unroll
+      for (int r = 0; r < R; ++r) {
+        pr_s[r] = warp_sum(pr_s[r]);
+        kp_s[r] = warp_sum(kp_s[r]);
+      }
+      __syncthreads();   // S.red reads above are done; cl_* written
+#pragma unroll
+      for (int r = 0; r < R; ++r)
+        if (lane == 0) {
+          S.red[(warp * kMaxRows + r) * 2] = pr_s[r];
+          S.red[(warp * kMaxRows + r) * 2 + 1] = kp_s[r];
+        }
+      if (lane == 0) S.wtau[warp] = tau_t;
+      __syncthreads();
+      if (threadIdx.x < R) {
+        const int r = threadIdx.x;
+        float ss = S.xch[xbuf][sx * r + 1], bs = 0.f;
+        for (int w = 0; w < kWarps; ++w) {
+          ss = __fadd_rn(ss, S.red[(w * kMaxRows + r) * 2]);
+          bs = __fadd_rn(bs, S.red[(w * kMaxRows + r) * 2 + 1]);
+        }
+        S.xch[xbuf][sx * r + 1] = ss;
+        S.xch[xbuf][sx * r + 2] = bs;
+      }
+      if (threadIdx.x == 0) {
+        float tc = kNegInf;
+        for (int w = 0; w < kWarps; ++w) tc = fmaxf(tc, fmaxf(S.wthr[w], S.wtau[w]));
+        S.xch[xbuf][3 * R] = __int_as_float(nk);
+        S.xch[xbuf][3 * R + 1] = tc;   // bound on every target logit of this CTA outside its list
+      }
     }
-    __syncthreads();
+    cluster_gather(S, nx, xbuf, cn);   // also publishes cl_* to the cluster
+    // every CTA: M, Z and the complement sum of each row (rank order)
+    if (threadIdx.x < R) {
+      const int r = threadIdx.x;
+      float mm = kNegInf;
+      for (int q = 0; q < cn; ++q) mm = fmaxf(mm, S.gat[q * nx + sx * r]);
+      float ss = 0.f, zz = 0.f;
+      if (mm > kNegInf)
+        for (int q = 0; q < cn; ++q) {
+          const float mq = S.gat[q * nx + sx * r];
+          if (!(mq > kNegInf)) continue;
+          const float f = ex2(__fmul_rn(__fsub_rn(mq, mm), cr[r]));
+          const float sq = S.gat[q * nx + sx * r + 1];
+          ss = __fadd_rn(ss, __fmul_rn(sq, f));
+          zz = __fadd_rn(zz, __fmul_rn(CAND ? __fadd_rn(sq, S.gat[q * nx + sx * r + 2]) : sq, f));
+        }
+      if (!(mm > kNegInf) || mm != mm) {
+        atomicOr(p.status, MDS_ST_NONFINITE);
+        mm = 0.f;
+      }
+      S.M[r0 + r] = mm;
+      S.pc[r0 + r] = ss;
+      finish_row(r0 + r, zz);
+    }
+    if constexpr (!CAND) {
+      if (threadIdx.x == 0) S.ncand = -1;
+      __syncthreads();
+      return;
+    } else {
+      __syncthreads();
+      // stage every CTA's list (rank order)
+      int ntot = 0;
+      for (int q = 0; q < cn; ++q) ntot += __float_as_int(S.gat[q * nx + 3 * R]);
+      {
+        int base = 0;
+        for (int q = 0; q < cn; ++q) {
+          const int c = __float_as_int(S.gat[q * nx + 3 * R]);
+          const int* qid = reinterpret_cast<const int*>(cl_base) + clbuf * kListN * (1 + p.rows_max);
+          const float* ql = reinterpret_cast<const float*>(qid + kListN);
+          for (int i = threadIdx.x; i < c; i += kThreads) {
+            if (cn > 1) {
+              cs_id[base + i] = __float_as_int(ld_dsmem(reinterpret_cast<const float*>(qid) + i, (uint32_t)q));
+              for (int r = 0; r < R; ++r) cs_l[r * p.cand_stage + base + i] = ld_dsmem(ql + r * kListN + i, (uint32_t)q);
+            } else {
+              cs_id[base + i] = qid[i];
+              for (int r = 0; r < R; ++r) cs_l[r * p.cand_stage + base + i] = ql[r * kListN + i];
+            }
+          }
+          base += c;
+        }
+      }
+      __syncthreads();
+      // the cluster list: the first kListN staged entries, by token id; the
+      // others join the complement.  Ranks first (candidate order), then
+      // each kept entry's position among the kept by token id.
+      const int n = min(ntot, kListN);
+      int* rank = reinterpret_cast<int*>(cs_x);
+      for (int i = threadIdx.x; i < ntot; i += kThreads) {
+        const float l0 = cs_l[i];
+        const int id = cs_id[i];
+        int rk = 0;
+        for (int j = 0; j < ntot; ++j) rk += cand_before(cs_l[j], cs_id[j], l0, id) ? 1 : 0;
+        rank[i] = rk;
+      }
+      __syncthreads();
+      float add[R];
+#pragma unroll
+      for (int r = 0; r < R; ++r) add[r] = 0.f;
+      float tau_t2 = kNegInf;
+      for (int i = threadIdx.x; i < ntot; i += kThreads) {
+        if (rank[i] < kListN) {
+          const int id = cs_id[i];
+          int pos = 0;
+          for (int j = 0; j < ntot; ++j) pos += (rank[j] < kListN && cs_id[j] < id) ? 1 : 0;
+          cm_id[pos] = id;
+#pragma unroll
+          for (int r = 0; r < R; ++r) {
+            const float l = cs_l[r * p.cand_stage + i];
+            cm_e[r * p.cand_cap + pos] = (l > kNegInf) ? ex2(__fmul_rn(__fsub_rn(l, S.M[r0 + r]), cr[r])) : 0.f;
+          }
+          cm_sp[pos] = 0;
+          cm_a[pos] = 0.f;
+        } else {
+          tau_t2 = fmaxf(tau_t2, cs_l[i]);
+#pragma unroll
+          for (int r = 0; r < R; ++r) {
+            const float l = cs_l[r * p.cand_stage + i];
+            if (l > kNegInf) add[r] = __fadd_rn(add[r], ex2(__fmul_rn(__fsub_rn(l, S.M[r0 + r]), cr[r])));
+          }
+        }
+      }
+#pragma unroll
+      for (int o = 16; o; o >>= 1) tau_t2 = fmaxf(tau_t2, __shfl_xor_sync(0xffffffffu, tau_t2, o));
+      if (lane == 0) S.wtau[warp] = tau_t2;
+#pragma unroll
+      for (int r = 0; r < R; ++r) {
+        add[r] = warp_sum(add[r]);
+        if (lane == 0) S.red[warp * R + r] = add[r];
+      }
+      __syncthreads();
+      if (threadIdx.x < R) {
+        const int r = threadIdx.x;
+        float ss = S.pc[r0 + r];
+        for (int w = 0; w < kWarps; ++w) ss = __fadd_rn(ss, S.red[w * R + r]);
+        S.pc[r0 + r] = ss;
+      }
+      if (threadIdx.x == 0) {
+        // every token outside the list has a target logit <= tau
+        float tau = kNegInf;
+        for (int q = 0; q < cn; ++q) tau = fmaxf(tau, S.gat[q * nx + 3 * R + 1]);
+        for (int w = 0; w < kWarps; ++w) tau = fmaxf(tau, S.wtau[w]);
+        S.ncand = n;
+        S.cand_all = (n == p.V) ? 1 : 0;
+        S.cand_q = (tau > kNegInf) ? ex2(__fmul_rn(__fsub_rn(tau, S.M[r0]), cr[0])) : 0.f;
+      }
+      clbuf ^= 1;
+      __syncthreads();
+    }
+  }
+
+  __device__ __forceinline__ void finish_row(int r, float Z) {
+    if (!(Z > 0.f) || !(Z < kPosInf) || Z != Z) {
+      atomicOr(p.status, MDS_ST_NONFINITE);
+      Z = 1.f;
+    }
+    S.invZ[r] = __frcp_rn(Z);
+  }
+
+  // Statistics of every row loaded at this depth (candidates for WIS).
+  __device__ void depth_stats(bool cand) {
+    const int nr = S.nrows;
+    if (cand && nr <= kFastRows && p.cand_cap > 0) {
+      switch (nr) {
+        case 2: stats_pass<2, true>(0); return;
+        case 3: stats_pass<3, true>(0); return;
+        case 4: stats_pass<4, true>(0); return;
+        default: break;
+      }
+    }
+    for (int r0 = 0; r0 < nr; r0 += 4) {
+      switch (min(4, nr - r0)) {
+        case 1: stats_pass<1, false>(r0); break;
+        case 2: stats_pass<2, false>(r0); break;
+        case 3: stats_pass<3, false>(r0); break;
+        default: stats_pass<4, false>(r0); break;
+      }
+    }
   }
 
   // ---------------------------------------------------------------- residual / CDF sampling
   // Inverse-CDF draw over this sequence's vocabulary from the nonnegative
-  // weights rf(u, r[VE]) in token order: the smallest token whose running sum
-  // exceeds u * (total).  Sums are formed per 32-unit segment (lane partial
-  // sums, warp inclusive scan), segments in order per CTA, CTAs in rank order;
-  // the search re-walks the same sums.  Returns the token (cluster-uniform)
-  // and the total mass in *total.
+  // weights rf(gu, L, r[VE]) in token order: the smallest token whose running
+  // sum exceeds u * (total).  A streaming pass over the rows in `mask` forms
+  // the sum of every 32-unit segment (lane partial sums, warp inclusive
+  // scan); segments are added in order per CTA and CTAs in rank order; the
+  // owner CTA re-reads its one segment from global memory and re-walks the
+  // same sums.  Returns the token (cluster-uniform) and the total mass.
   template <class RF>
-  __device__ int sample_cdf(const RF& rf, float u01, float* total) {
+  __device__ int sample_cdf(uint32_t mask, const RF& rf, float u01, float* total) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    for (int u0 = warp * 32; u0 < U; u0 += kThreads) {
-      const int uu = u0 + lane;
+    stream(mask, [&](int gu, bool valid, const auto& L) {
       float part = 0.f;
-      if (uu < U) {
+      if (valid) {
         float r[VE];
-        rf(uu, r);
+        rf(gu, L, r);
 #pragma unroll
         for (int e = 0; e < VE; ++e) part = __fadd_rn(part, r[e]);
       }
@@ -509,12 +1025,12 @@ struct Kernel {
         const float t = __shfl_up_sync(0xffffffffu, part, o);
         if (lane >= o) part = __fadd_rn(part, t);
       }
-      if (lane == 31) segsum[u0 >> 5] = part;
-    }
-    __syncthreads();
+      if (lane == 31) segsum[gu >> 5] = part;   // groups start at multiples of 32 units
+    });
+    __syncthreads();   // every warp's segment sums
     if (threadIdx.x == 0) {
       float tot = 0.f;
-      for (int g = 0; g < nseg; ++g) tot = __fadd_rn(tot, segsum[g]);
+      for (int g = 0; g < nsegv; ++g) tot = __fadd_rn(tot, segsum[g]);
       S.xch[xbuf][0] = tot;
     }
     cluster_gather(S, 1, xbuf, cn);
@@ -526,10 +1042,8 @@ struct Kernel {
     if (threadIdx.x == 0) {
       // owner CTA: first whose cumulative total exceeds T (else the last with mass)
       float run = 0.f;
-      int owner = -1;
-      float run_owner = 0.f;
-      int last = -1;
-      float run_last = 0.f;
+      int owner = -1, last = -1;
+      float run_owner = 0.f, run_last = 0.f;
       for (int q = 0; q < cn; ++q) {
         const float tq = S.gat[q];
         if (tq > 0.f) {
@@ -548,7 +1062,6 @@ struct Kernel {
       }
       S.owner = owner;
       S.run = run_owner;
-      S.T = T;
     }
     __syncthreads();
     const int owner = S.owner;
@@ -557,7 +1070,7 @@ struct Kernel {
         float run = S.run;
         int g = -1, glast = -1;
         float run_g = 0.f, run_last = 0.f;
-        for (int h = 0; h < nseg; ++h) {
+        for (int h = 0; h < nsegv; ++h) {
           if (segsum[h] > 0.f) {
             glast = h;
             run_last = run;
@@ -579,13 +1092,13 @@ struct Kernel {
       if (warp == 0) {
         const int g = S.seg;
         const float base = S.run;
-        const int uu = g * 32 + lane;
+        const int gu = g * 32 + lane;
         float r[VE];
 #pragma unroll
         for (int e = 0; e < VE; ++e) r[e] = 0.f;
         float part = 0.f;
-        if (uu < U) {
-          rf(uu, r);
+        if (gu < Uv) {
+          rf(gu, GlobalLoad<DT>{S.gptr, tok0, p.V, gu, p.tma_ok != 0}, r);
 #pragma unroll
           for (int e = 0; e < VE; ++e) part = __fadd_rn(part, r[e]);
         }
@@ -598,7 +1111,7 @@ struct Kernel {
         const float Pprev = __shfl_up_sync(0xffffffffu, P, 1);
         const unsigned hit = __ballot_sync(0xffffffffu, __fadd_rn(base, P) > T);
         const unsigned pos = __ballot_sync(0xffffffffu, part > 0.f);
-        int l = hit ? __ffs(hit) - 1 : (pos ? 31 - __clz(pos) : 0);
+        const int l = hit ? __ffs(hit) - 1 : (pos ? 31 - __clz(pos) : 0);
         if (lane == l) {
           float acc = (l > 0) ? __fadd_rn(base, Pprev) : base;
           int e_hit = -1, e_last = -1;
@@ -609,7 +1122,7 @@ struct Kernel {
             if (e_hit < 0 && acc > T && r[e] > 0.f) e_hit = e;
           }
           if (e_hit < 0) e_hit = e_last < 0 ? 0 : e_last;
-          const int tok = min(tok0 + uu * VE + e_hit, p.V - 1);
+          const int tok = min(tok0 + gu * VE + e_hit, p.V - 1);
           for (int q = 0; q < cn; ++q) {
             if (cn > 1)
               st_dsmem(&S.Zslot, (uint32_t)q, tok);
@@ -935,13 +1448,17 @@ struct Kernel {
     for (int t = 0; t < kTop; ++t) top[t] = CAND_NONE;
     float suma = 0.f, sumb = 0.f;   // masses of tokens dropped from this thread's list
     const int nr = S.nrows;
-    for (int uu = threadIdx.x; uu < U; uu += kThreads) {
+    uint32_t mask = 1u | (1u << rb);
+    for (int r = 1; r < nr; ++r)
+      if (S.gamma[r] != 0.f) mask |= 1u << r;
+    stream(mask, [&](int gu, bool valid, const auto& L) {
+      if (!valid) return;
+      const int uu = gu;
       const int tbase = tok0 + uu * VE;
-      if (tbase >= p.V) break;
       float q[VE], a[VE], bb[VE];
       {
         float v[VE];
-        E::unit(srow(0), uu, v);
+        L(0, v);
 #pragma unroll
         for (int e = 0; e < VE; ++e) q[e] = prob_of(v[e], S.M[0], S.c[0], S.invZ[0]);
       }
@@ -951,7 +1468,7 @@ struct Kernel {
         const float g = S.gamma[r];
         if (g == 0.f && r != rb) continue;
         float v[VE];
-        E::unit(srow(r), uu, v);
+        L(r, v);
 #pragma unroll
         for (int e = 0; e < VE; ++e) {
           const float pr = prob_of(v[e], S.M[r], S.c[r], S.invZ[r]);
@@ -970,7 +1487,7 @@ struct Kernel {
         if (tbase + e >= p.V) break;
         cand_insert(top, Cand{__fmaf_rn(-a[e], bb[e], q[e]), tbase + e, a[e], bb[e]}, suma, sumb);
       }
-    }
+    });
     // merge: lanes -> warp -> CTA -> cluster, popping s entries at each level;
     // every entry not popped adds its a and b to the Omega_2 masses
     {
@@ -1080,250 +1597,6 @@ struct Kernel {
     }
     __syncthreads();
     return S.Y;
-  }
-
-  // ---------------------------------------------------------------- WIS: candidate list
-  // Softmax statistics for a WIS depth with more than one valid draft, plus
-  // the candidate list C = {k : q_k >= q_max 2^-kCandLog2} gathered to every
-  // CTA in token order.  Every stage key q - a b is <= q, so whenever the
-  // s-th best key in C exceeds the largest q outside C, Omega_1 lies in C and
-  // the stage can run on C alone.  Two cluster exchanges: the row maxima,
-  // then the per-CTA exp sums (split into candidates and complement) and the
-  // candidate counts.  Units are mapped to warps in contiguous chunks so the
-  // candidates come out in token order with a single block barrier.
-  __device__ void wis_prepare() {
-    const int nr = S.nrows;
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    // pass A: maxima; then, against this CTA's target max (<= the global
-    // max, so these are upper bounds), counts of tokens at each candidate level
-    for (int r = 0; r < nr; ++r) {
-      float m = kNegInf;
-      for (int u = threadIdx.x; u < U; u += kThreads) {
-        float v[VE];
-        E::unit(srow(r), u, v);
-#pragma unroll
-        for (int e = 0; e < VE; ++e) m = fmaxf(m, v[e]);
-      }
-#pragma unroll
-      for (int o = 16; o; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
-      if (lane == 0) S.red[warp * kMaxRows + r] = m;
-    }
-    __syncthreads();
-    float mcta = kNegInf;
-    for (int w = 0; w < kWarps; ++w) mcta = fmaxf(mcta, S.red[w * kMaxRows]);
-    int lc[kCandLevels];
-#pragma unroll
-    for (int l = 0; l < kCandLevels; ++l) lc[l] = 0;
-    if (mcta > kNegInf) {
-      const float c0 = S.c[0];
-      for (int u = threadIdx.x; u < U; u += kThreads) {
-        if (tok0 + u * VE >= p.V) break;
-        float v[VE];
-        E::unit(srow(0), u, v);
-#pragma unroll
-        for (int e = 0; e < VE; ++e) {
-          const float x = __fmul_rn(__fsub_rn(v[e], mcta), c0);
-#pragma unroll
-          for (int l = 0; l < kCandLevels; ++l) lc[l] += (x >= -cand_log2(l)) ? 1 : 0;
-        }
-      }
-    }
-#pragma unroll
-    for (int l = 0; l < kCandLevels; ++l) lc[l] = __reduce_add_sync(0xffffffffu, lc[l]);
-    if (lane == 0)
-#pragma unroll
-      for (int l = 0; l < kCandLevels; ++l) S.wlev[warp * kCandLevels + l] = lc[l];
-    __syncthreads();
-    if (threadIdx.x < nr) {
-      float m = kNegInf;
-      for (int w = 0; w < kWarps; ++w) m = fmaxf(m, S.red[w * kMaxRows + threadIdx.x]);
-      S.xch[xbuf][threadIdx.x] = m;
-    }
-    if (threadIdx.x < kCandLevels) {
-      int c = 0;
-      for (int w = 0; w < kWarps; ++w) c += S.wlev[w * kCandLevels + threadIdx.x];
-      S.xch[xbuf][nr + threadIdx.x] = __int_as_float(c);
-    }
-    const int n1 = nr + kCandLevels;
-    cluster_gather(S, n1, xbuf, cn);
-    if (threadIdx.x < nr) {
-      float m = kNegInf;
-      for (int q = 0; q < cn; ++q) m = fmaxf(m, S.gat[q * n1 + threadIdx.x]);
-      if (!(m > kNegInf) || m != m) {
-        atomicOr(p.status, MDS_ST_NONFINITE);
-        m = 0.f;
-      }
-      S.M[threadIdx.x] = m;
-    }
-    // the most permissive level whose bounded counts fit the lists
-    int level = -1;
-    if (p.cand_cap > 0) {
-      for (int l = 0; l < kCandLevels && level < 0; ++l) {
-        int tot = 0, worst = 0;
-        for (int q = 0; q < cn; ++q) {
-          const int c = __float_as_int(S.gat[q * n1 + nr + l]);
-          tot += c;
-          worst = max(worst, c);
-        }
-        if (tot <= p.cand_cap && worst <= p.cand_cap_cta) level = l;
-      }
-    }
-    __syncthreads();
-    const float xthr = (level >= 0) ? -cand_log2(level) : 0.f;   // level < 0: no list (overflow)
-    // pass B over this warp's chunk: exp sums split by candidacy, counts
-    const int chunk = ((U + kWarps - 1) / kWarps + 31) & ~31;
-    const int ubeg = min(U, warp * chunk), uend = min(U, ubeg + chunk);
-    const float M0 = S.M[0], c0 = S.c[0];
-    float comp[kFastRows], cand[kFastRows];
-#pragma unroll
-    for (int r = 0; r < kFastRows; ++r) comp[r] = cand[r] = 0.f;
-    int cnt = 0;
-    for (int u = ubeg + lane; u < uend; u += 32) {
-      float x0[VE];
-      {
-        float v[VE];
-        E::unit(srow(0), u, v);
-#pragma unroll
-        for (int e = 0; e < VE; ++e) x0[e] = __fmul_rn(__fsub_rn(v[e], M0), c0);
-      }
-      uint32_t isc = 0u;
-#pragma unroll
-      for (int e = 0; e < VE; ++e) {
-        const bool c = (level >= 0) && (x0[e] >= xthr) && (tok0 + u * VE + e < p.V);
-        isc |= (c ? 1u : 0u) << e;
-        const float ex = ex2(x0[e]);
-        if (c) cand[0] += ex; else comp[0] += ex;
-      }
-      cnt += __popc(isc);
-#pragma unroll
-      for (int r = 1; r < kFastRows; ++r) {
-        if (r >= nr) break;
-        const float Mr = S.M[r], cr = S.c[r];
-        float v[VE];
-        E::unit(srow(r), u, v);
-#pragma unroll
-        for (int e = 0; e < VE; ++e) {
-          const float ex = ex2(__fmul_rn(__fsub_rn(v[e], Mr), cr));
-          if (isc >> e & 1u) cand[r] += ex; else comp[r] += ex;
-        }
-      }
-    }
-#pragma unroll
-    for (int r = 0; r < kFastRows; ++r) {
-      comp[r] = warp_sum(comp[r]);
-      cand[r] = warp_sum(cand[r]);
-    }
-    const int wtot = __reduce_add_sync(0xffffffffu, cnt);
-    if (lane == 0) {
-      S.wcnt[warp] = wtot;
-#pragma unroll
-      for (int r = 0; r < kFastRows; ++r) {
-        S.red[(warp * kFastRows + r) * 2] = comp[r];
-        S.red[(warp * kFastRows + r) * 2 + 1] = cand[r];
-      }
-    }
-    __syncthreads();
-    int woff = 0, total = 0;
-    for (int w = 0; w < kWarps; ++w) {
-      if (w < warp) woff += S.wcnt[w];
-      total += S.wcnt[w];
-    }
-    // candidate write pass (compare-only; exps just for the candidates)
-    if (level >= 0 && total <= p.cand_cap_cta && wtot > 0) {
-      int run = woff;
-      for (int u = ubeg + lane; u - lane < uend; u += 32) {
-        float v0[VE];
-        uint32_t isc = 0u;
-        if (u < uend) {
-          E::unit(srow(0), u, v0);
-#pragma unroll
-          for (int e = 0; e < VE; ++e)
-            isc |= ((__fmul_rn(__fsub_rn(v0[e], M0), c0) >= xthr && tok0 + u * VE + e < p.V) ? 1u : 0u) << e;
-        }
-        const int c = __popc(isc);
-        int inc = c;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-          const int t = __shfl_up_sync(0xffffffffu, inc, o);
-          if (lane >= o) inc += t;
-        }
-        if (c) {
-          int pos = run + inc - c;
-#pragma unroll
-          for (int e = 0; e < VE; ++e) {
-            if (!(isc >> e & 1u)) continue;
-            cl_id[pos] = tok0 + u * VE + e;
-            cl_e[pos] = ex2(__fmul_rn(__fsub_rn(v0[e], M0), c0));
-            for (int r = 1; r < nr; ++r) {
-              float v[VE];
-              E::unit(srow(r), u, v);
-              cl_e[r * p.cand_cap_cta + pos] = ex2(__fmul_rn(__fsub_rn(v[e], S.M[r]), S.c[r]));
-            }
-            ++pos;
-          }
-        }
-        run += __shfl_sync(0xffffffffu, inc, 31);
-      }
-    }
-    if (threadIdx.x < kFastRows) {
-      float a0 = 0.f, a1 = 0.f;
-      for (int w = 0; w < kWarps; ++w) {
-        a0 = __fadd_rn(a0, S.red[(w * kFastRows + threadIdx.x) * 2]);
-        a1 = __fadd_rn(a1, S.red[(w * kFastRows + threadIdx.x) * 2 + 1]);
-      }
-      S.xch[xbuf][2 * threadIdx.x] = a0;
-      S.xch[xbuf][2 * threadIdx.x + 1] = a1;
-    }
-    if (threadIdx.x == 0) S.xch[xbuf][2 * kFastRows] = __int_as_float(total);
-    const int nx = 2 * kFastRows + 1;
-    cluster_gather(S, nx, xbuf, cn);   // also publishes cl_* to the cluster
-    // totals, complement masses, the merged list (every CTA, rank order)
-    int ntot = 0, overflow = level >= 0 ? 0 : 1;
-    for (int q = 0; q < cn; ++q) {
-      const int c = __float_as_int(S.gat[q * nx + 2 * kFastRows]);
-      if (c > p.cand_cap_cta) overflow = 1;
-      ntot += c;
-    }
-    if (ntot > p.cand_cap) overflow = 1;
-    if (threadIdx.x < nr) {
-      const int r = threadIdx.x;
-      float comp_t = 0.f, cand_t = 0.f;
-      for (int q = 0; q < cn; ++q) {
-        comp_t = __fadd_rn(comp_t, S.gat[q * nx + 2 * r]);
-        cand_t = __fadd_rn(cand_t, S.gat[q * nx + 2 * r + 1]);
-      }
-      const float Z = __fadd_rn(comp_t, cand_t);
-      if (!(Z > 0.f) || !(Z < kPosInf)) atomicOr(p.status, MDS_ST_NONFINITE);
-      S.invZ[r] = (Z > 0.f && Z < kPosInf) ? __frcp_rn(Z) : 1.f;
-      S.pc[r] = comp_t;                  // complement exp mass (times invZ: probability)
-    }
-    if (!overflow) {
-      int off = 0;
-      for (int q = 0; q < cn; ++q) {
-        const int c = __float_as_int(S.gat[q * nx + 2 * kFastRows]);
-        for (int i = threadIdx.x; i < c; i += kThreads) {
-          if (cn > 1) {
-            cm_id[off + i] = __float_as_int(ld_dsmem(reinterpret_cast<const float*>(cl_id) + i, (uint32_t)q));
-            for (int r = 0; r < nr; ++r)
-              cm_e[r * p.cand_cap + off + i] = ld_dsmem(cl_e + r * p.cand_cap_cta + i, (uint32_t)q);
-          } else {
-            cm_id[off + i] = cl_id[i];
-            for (int r = 0; r < nr; ++r) cm_e[r * p.cand_cap + off + i] = cl_e[r * p.cand_cap_cta + i];
-          }
-          cm_sp[off + i] = 0;
-          cm_a[off + i] = 0.f;
-        }
-        off += c;
-      }
-    }
-    if (threadIdx.x == 0) {
-      S.ncand = overflow ? -1 : ntot;
-      S.cand_all = (!overflow && ntot == p.V) ? 1 : 0;
-      S.cand_q = (level >= 0) ? ex2(xthr) : 0.f;   // every non-candidate has q < cand_q / Z
-    }
-    __syncthreads();
-    // Other CTAs read this CTA's cl_* right after the exchange; the next write
-    // to cl_* is a depth later, behind at least one more cluster barrier.
   }
 
   // One stage on the merged candidate list, by warp 0 of every CTA.
@@ -1442,18 +1715,22 @@ struct Kernel {
     __syncthreads();
     // range of rho = q / p_r over tokens with q > 0 and p_r > 0
     float lo = kPosInf, hi = 0.f;
-    for (int uu = threadIdx.x; uu < U; uu += kThreads) {
+    uint32_t mask = 1u;
+    for (int r = 1; r < S.nrows; ++r)
+      if (S.is_cnt[r]) mask |= 1u << r;
+    stream(mask, [&](int, bool valid, const auto& L) {
+      if (!valid) return;
       float q[VE];
       {
         float v[VE];
-        E::unit(srow(0), uu, v);
+        L(0, v);
 #pragma unroll
         for (int e = 0; e < VE; ++e) q[e] = prob_of(v[e], S.M[0], S.c[0], S.invZ[0]);
       }
       for (int r = 1; r < S.nrows; ++r) {
         if (!S.is_cnt[r]) continue;
         float v[VE];
-        E::unit(srow(r), uu, v);
+        L(r, v);
 #pragma unroll
         for (int e = 0; e < VE; ++e) {
           const float pr = prob_of(v[e], S.M[r], S.c[r], S.invZ[r]);
@@ -1464,7 +1741,7 @@ struct Kernel {
           }
         }
       }
-    }
+    });
 #pragma unroll
     for (int o = 16; o; o >>= 1) {
       lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
@@ -1519,14 +1796,15 @@ struct Kernel {
           acc[i] = 0.f;
           tl[i] = (n0 + i < nn) ? __fmul_rn(isT[n0 + i], -kLog2e) : 0.f;
         }
-        for (int uu = threadIdx.x; uu < U; uu += kThreads) {
+        stream(1u | (1u << r), [&](int, bool valid, const auto& L) {
+          if (!valid) return;
           float q[VE], pr[VE];
           {
             float v[VE];
-            E::unit(srow(0), uu, v);
+            L(0, v);
 #pragma unroll
             for (int e = 0; e < VE; ++e) q[e] = prob_of(v[e], S.M[0], S.c[0], S.invZ[0]);
-            E::unit(srow(r), uu, v);
+            L(r, v);
 #pragma unroll
             for (int e = 0; e < VE; ++e) pr[e] = prob_of(v[e], S.M[r], S.c[r], S.invZ[r]);
           }
@@ -1537,7 +1815,7 @@ struct Kernel {
 #pragma unroll
             for (int i = 0; i < kIsChunk; ++i) acc[i] = __fmaf_rn(pr[e], ex2(__fmul_rn(tl[i], rho)), acc[i]);
           }
-        }
+        });
 #pragma unroll
         for (int i = 0; i < kIsChunk; ++i) {
           const float v = warp_sum(acc[i]);
@@ -1680,7 +1958,7 @@ struct Kernel {
   }
 
   // ---------------------------------------------------------------- one sequence
-  __device__ void run_sequence(int b) {
+  __device__ __forceinline__ void run_sequence(int b) {
     const int K = p.K, L = p.L, V = p.V;
     const int tid = threadIdx.x;
     unsigned valid = (K >= 32) ? 0xffffffffu : ((1u << K) - 1u);
@@ -1736,21 +2014,17 @@ struct Kernel {
         S.R = 0.f;
       }
       __syncthreads();
-      load_rows();
-      if (SCHEME == MDS_WIS && !bonus && S.nv > 1 && S.nrows <= kFastRows)
-        wis_prepare();
-      else
-        row_stats();
-      if (threadIdx.x == 0 && !(SCHEME == MDS_WIS && !bonus && S.nv > 1 && S.nrows <= kFastRows)) S.ncand = -1;
+      depth_stats(SCHEME == MDS_WIS && !bonus && S.nv > 1);
       int Z;
       float qY = 0.f, pIY = 0.f, Rdiag = 0.f;
       int Ydiag = -1;
       if (bonus) {
         float tot;
         Z = sample_cdf(
-            [&](int uu, float* r) {
+            1u,
+            [&](int, const auto& L, float* r) {
               float v[VE];
-              E::unit(srow(0), uu, v);
+              L(0, v);
 #pragma unroll
               for (int e = 0; e < VE; ++e) r[e] = prob_of(v[e], S.M[0], S.c[0], S.invZ[0]);
             },
@@ -1790,23 +2064,30 @@ struct Kernel {
           bool done = false;
           if constexpr (SCHEME == MDS_WIS) {
             if (S.nv > 1) {
-              Z = sample_cdf([&](int uu, float* r) { residual_wis(uu, r); }, ures, &tot);
+              uint32_t mask = 1u;
+              for (int r = 1; r < S.nrows; ++r)
+                if (S.gamma[r] != 0.f) mask |= 1u << r;
+              Z = sample_cdf(mask, [&](int gu, const auto& L, float* r) { residual_wis(gu, L, r); }, ures, &tot);
               done = true;
             }
           }
           if constexpr (SCHEME == MDS_IS) {
             if (S.nv > 1) {
-              Z = sample_cdf([&](int uu, float* r) { residual_is(uu, r); }, ures, &tot);
+              uint32_t mask = 1u;
+              for (int r = 1; r < S.nrows; ++r)
+                if (S.is_cnt[r]) mask |= 1u << r;
+              Z = sample_cdf(mask, [&](int, const auto& L, float* r) { residual_is(L, r); }, ures, &tot);
               done = true;
             }
           }
           if (!done) {
             const int r1 = S.vrow[0];
             Z = sample_cdf(
-                [&](int uu, float* r) {
+                1u | (1u << r1),
+                [&](int, const auto& L, float* r) {
                   float v[VE], w[VE];
-                  E::unit(srow(0), uu, v);
-                  E::unit(srow(r1), uu, w);
+                  L(0, v);
+                  L(r1, w);
 #pragma unroll
                   for (int e = 0; e < VE; ++e)
                     r[e] = fmaxf(0.f, __fsub_rn(prob_of(v[e], S.M[0], S.c[0], S.invZ[0]),
@@ -1818,9 +2099,10 @@ struct Kernel {
           if (Z < 0) {
             if (tid == 0) atomicOr(p.status, MDS_ST_ZERO_RESID);
             Z = sample_cdf(
-                [&](int uu, float* r) {
+                1u,
+                [&](int, const auto& L, float* r) {
                   float v[VE];
-                  E::unit(srow(0), uu, v);
+                  L(0, v);
 #pragma unroll
                   for (int e = 0; e < VE; ++e) r[e] = prob_of(v[e], S.M[0], S.c[0], S.invZ[0]);
                 },
@@ -1860,27 +2142,28 @@ struct Kernel {
   }
 
   // residual weight max(0, q - p_I) for WIS (generic gamma law + special table)
-  __device__ __forceinline__ void residual_wis(int uu, float* r) const {
-    const int tbase = tok0 + uu * VE;
+  template <class LD>
+  __device__ __forceinline__ void residual_wis(int gu, const LD& L, float* r) const {
+    const int tbase = tok0 + gu * VE;
     float q[VE], a[VE];
     {
       float v[VE];
-      E::unit(srow(0), uu, v);
+      L(0, v);
 #pragma unroll
       for (int e = 0; e < VE; ++e) {
         q[e] = prob_of(v[e], S.M[0], S.c[0], S.invZ[0]);
         a[e] = 0.f;
       }
     }
-    for (int r = 1; r < S.nrows; ++r) {
-      const float g = S.gamma[r];
+    for (int rr = 1; rr < S.nrows; ++rr) {
+      const float g = S.gamma[rr];
       if (g == 0.f) continue;
       float v[VE];
-      E::unit(srow(r), uu, v);
+      L(rr, v);
 #pragma unroll
-      for (int e = 0; e < VE; ++e) a[e] = __fmaf_rn(g, prob_of(v[e], S.M[r], S.c[r], S.invZ[r]), a[e]);
+      for (int e = 0; e < VE; ++e) a[e] = __fmaf_rn(g, prob_of(v[e], S.M[rr], S.c[rr], S.invZ[rr]), a[e]);
     }
-    const uint32_t bits = (bitmap[(uu * VE) >> 5] >> ((uu * VE) & 31)) & ((1u << VE) - 1u);
+    const uint32_t bits = (bitmap[(gu * VE) >> 5] >> ((gu * VE) & 31)) & ((1u << VE) - 1u);
     if (bits) {
 #pragma unroll
       for (int e = 0; e < VE; ++e)
@@ -1891,11 +2174,12 @@ struct Kernel {
   }
 
   // residual weight max(0, q - p_I) for plain IS (Laplace identity)
-  __device__ __forceinline__ void residual_is(int uu, float* r) const {
+  template <class LD>
+  __device__ __forceinline__ void residual_is(const LD& L, float* r) const {
     float q[VE];
     {
       float v[VE];
-      E::unit(srow(0), uu, v);
+      L(0, v);
 #pragma unroll
       for (int e = 0; e < VE; ++e) q[e] = prob_of(v[e], S.M[0], S.c[0], S.invZ[0]);
     }
@@ -1903,7 +2187,7 @@ struct Kernel {
     for (int rr = 1; rr < S.nrows; ++rr) {
       if (!S.is_cnt[rr]) continue;
       float v[VE];
-      E::unit(srow(rr), uu, v);
+      L(rr, v);
 #pragma unroll
       for (int e = 0; e < VE; ++e) {
         const float pv = prob_of(v[e], S.M[rr], S.c[rr], S.invZ[rr]);
@@ -1955,14 +2239,17 @@ struct Kernel {
       // residual mass of this round
       float part = 0.f;
       const int ri = S.sp_rows[i];
-      for (int uu = threadIdx.x; uu < U; uu += kThreads) {
+      uint32_t mask = 1u | (1u << ri);
+      for (int k = 0; k < i; ++k) mask |= 1u << S.sp_rows[k];
+      stream(mask, [&](int, bool valid, const auto& L) {
+        if (!valid) return;
         float r[VE];
-        spectr_target(uu, i, r);
+        spectr_target(L, i, r);
         float w[VE];
-        E::unit(srow(ri), uu, w);
+        L(ri, w);
 #pragma unroll
         for (int e = 0; e < VE; ++e) part += fmaxf(0.f, __fsub_rn(r[e], prob_of(w[e], S.M[ri], S.c[ri], S.invZ[ri])));
-      }
+      });
       part = warp_sum(part);
       const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
       if (lane == 0) S.red[warp] = part;
@@ -1981,23 +2268,26 @@ struct Kernel {
       __syncthreads();
     }
     float tot;
-    const int z = sample_cdf([&](int uu, float* r) { spectr_target(uu, nv, r); },
+    uint32_t mask = 1u;
+    for (int k = 0; k < nv; ++k) mask |= 1u << S.sp_rows[k];
+    const int z = sample_cdf(mask, [&](int, const auto& L, float* r) { spectr_target(L, nv, r); },
                              draw_uniform(p.seed, b, j, kDrawResidual), &tot);
     *Rd = tot;
     return z;
   }
 
   // running target after `rounds` rejected rounds, for one unit
-  __device__ __forceinline__ void spectr_target(int uu, int rounds, float* r) const {
+  template <class LD>
+  __device__ __forceinline__ void spectr_target(const LD& L, int rounds, float* r) const {
     float v[VE];
-    E::unit(srow(0), uu, v);
+    L(0, v);
 #pragma unroll
     for (int e = 0; e < VE; ++e) r[e] = prob_of(v[e], S.M[0], S.c[0], S.invZ[0]);
     for (int k = 0; k < rounds; ++k) {
       if (!(S.sp_invR[k] > 0.f)) continue;
       const int rk = S.sp_rows[k];
       float w[VE];
-      E::unit(srow(rk), uu, w);
+      L(rk, w);
 #pragma unroll
       for (int e = 0; e < VE; ++e)
         r[e] = __fmul_rn(fmaxf(0.f, __fsub_rn(r[e], prob_of(w[e], S.M[rk], S.c[rk], S.invZ[rk]))), S.sp_invR[k]);
@@ -2006,7 +2296,7 @@ struct Kernel {
 };
 
 template <int DT, int SCHEME>
-__global__ void __launch_bounds__(kThreads, SCHEME == MDS_IS ? 1 : 3) verify_kernel(const __grid_constant__ Params p) {
+__global__ void __launch_bounds__(kThreads, SCHEME == MDS_IS ? 1 : 2) verify_kernel(const __grid_constant__ Params p) {
   extern __shared__ __align__(128) char dsm[];
   __shared__ State S;
   Kernel<DT, SCHEME> k{p, S};
@@ -2014,24 +2304,36 @@ __global__ void __launch_bounds__(kThreads, SCHEME == MDS_IS ? 1 : 3) verify_ker
   k.cn = p.cn;
   k.tok0 = k.rank * p.slice;
   k.nvalid = max(0, min(p.slice, p.V - k.tok0));
-  k.U = p.slice / Kernel<DT, SCHEME>::VE;
-  k.nseg = (k.U + 31) / 32;
+  k.Uv = (k.nvalid + Kernel<DT, SCHEME>::VE - 1) / Kernel<DT, SCHEME>::VE;
+  k.nseg = (p.slice / Kernel<DT, SCHEME>::VE + 31) / 32;   // same in every CTA: peers map the same offsets
+  k.nsegv = (k.Uv + 31) / 32;                                // segments the residual pass writes
+  k.Uw = ((k.Uv + kWarps - 1) / kWarps + 31) & ~31;           // units per warp in a streaming pass
   k.bm_words = (p.slice + 31) / 32;
-  // dynamic shared memory: rows | segment sums | scheme region
+  // dynamic shared memory: ring | segment sums | scheme region
   //   IS : nodes t_n | weights W_r(n)
-  //   WIS: this CTA's candidate list | merged list, aliased later by the
-  //        special-token bitmap (the merged list is local; other CTAs only
-  //        ever read the CTA list)
-  k.rows = dsm;
-  k.segsum = reinterpret_cast<float*>(dsm + (size_t)p.rows_max * p.row_stride);
+  //   WIS: CTA list (two copies) | warp lists = staging list | merged list, the
+  //        last aliased later by the special-token bitmap (only the CTA list
+  //        is ever read by other CTAs)
+  k.ring = dsm;
+  k.segsum = reinterpret_cast<float*>(dsm + p.ring_bytes);
   {
     char* c = reinterpret_cast<char*>(k.segsum + ((k.nseg + 3) & ~3));
     k.isT = reinterpret_cast<float*>(c);
     k.isW = k.isT + kIsNodesMax;
-    k.cl_id = reinterpret_cast<int*>(c);
-    c += (size_t)p.cand_cap_cta * 4;
-    k.cl_e = reinterpret_cast<float*>(c);
-    c += (size_t)p.cand_cap_cta * p.rows_max * 4;
+    k.cl_base = c;
+    c += (size_t)2 * kListN * (1 + p.rows_max) * 4;
+    // the warps' set-aside lists and the staging list share one region: the
+    // lists are compacted into the CTA list before anything is staged
+    char* st = c;
+    k.ap_id = reinterpret_cast<int*>(st);
+    k.ap_l = reinterpret_cast<float*>(st + (size_t)kWarps * kWarpApp * 4);
+    k.cs_id = reinterpret_cast<int*>(c);
+    c += (size_t)p.cand_stage * 4;
+    k.cs_l = reinterpret_cast<float*>(c);
+    c += (size_t)p.cand_stage * p.rows_max * 4;
+    k.cs_x = reinterpret_cast<float*>(c);
+    c += (size_t)p.cand_stage * 4;
+    if (p.cand_cap > 0) c = st + max(c - st, (ptrdiff_t)kWarps * kWarpApp * 4 * (1 + p.rows_max));
     k.bitmap = reinterpret_cast<uint32_t*>(c);
     k.cm_id = reinterpret_cast<int*>(c);
     c += (size_t)p.cand_cap * 4;
@@ -2042,9 +2344,17 @@ __global__ void __launch_bounds__(kThreads, SCHEME == MDS_IS ? 1 : 3) verify_ker
     k.cm_sp = reinterpret_cast<int*>(c);
   }
   k.xbuf = 0;
-  k.mphase = 0u;
-  if (threadIdx.x == 0) mbar_init(&S.mbar);
+  k.clbuf = 0;
+  k.wphase = 0u;
+  if (threadIdx.x == 0) {
+    for (int w = 0; w < kWarps; ++w)
+      for (int i = 0; i < kWStages; ++i) mbar_init(&S.wbar[w][i]);
+    mbar_init_fence();
+  }
   __syncthreads();
+  // A peer's shared memory may be accessed only once every CTA of the
+  // cluster is running: one cluster barrier before the first remote store.
+  if (p.cn > 1) cluster_sync_all();
   for (;;) {
     if (k.rank == 0 && threadIdx.x == 0) {
       const int b = (int)(atomicAdd(p.queue, 1u) - p.ticket0);
@@ -2069,14 +2379,17 @@ __global__ void __launch_bounds__(kThreads, SCHEME == MDS_IS ? 1 : 3) verify_ker
 
 size_t smem_bytes(const Params& p) {
   const int VE = 16 / p.esize;
-  const int U = p.slice / VE;
-  const int nseg = (U + 31) / 32;
-  size_t bytes = (size_t)p.rows_max * p.row_stride + (size_t)((nseg + 3) & ~3) * 4;
+  const int nseg = (p.slice / VE + 31) / 32;
+  size_t bytes = (size_t)p.ring_bytes + (size_t)((nseg + 3) & ~3) * 4;
   if (p.scheme == MDS_IS) bytes += (size_t)kIsNodesMax * 4 * (1 + p.rows_max);
   if (p.scheme == MDS_WIS) {
     const size_t bm = (size_t)((p.slice + 31) / 32) * 4;
     const size_t cm = (size_t)p.cand_cap * 4 * (3 + p.rows_max);
-    bytes += (size_t)p.cand_cap_cta * 4 * (1 + p.rows_max) + (bm > cm ? bm : cm);
+    size_t stg = (size_t)p.cand_stage * 4 * (2 + p.rows_max);
+    const size_t app = (size_t)kWarps * kWarpApp * 4 * (1 + p.rows_max);
+    if (p.cand_cap > 0 && app > stg) stg = app;
+    bytes += (size_t)2 * kListN * 4 * (1 + p.rows_max) + stg +
+             (bm > cm ? bm : cm);
   }
   return bytes;
 }

@@ -142,3 +142,40 @@ def test_full_size_serving_sampled():
                          ("IS", [0, 1])):
         res = run_both(spec, scheme, seed=1, seqs=seqs)
         check(res, scheme)
+
+
+@pytest.mark.parametrize("cluster", [2, 4])
+def test_repeated_launches_are_identical(cluster):
+    # The result of a sequence may not depend on which cluster takes it, on
+    # the launch's cluster count or on what ran before: repeat the same
+    # verification with different batch capacities (so different grids) and
+    # interleaved launches of another configuration.
+    spec = small("llama2-32k", B=24, V=12007, K=4, model_ids=[0, 0, 1, 1], draft_sigma=[1.0, 0.6],
+                 t_draft=[1.2, 0.9])
+    w = make_workload(spec, device=DEV)
+    other = make_workload(small("tiny", B=8), device=DEV)
+    ref = {}
+    for rep, max_B in enumerate((24, 24, 64, 200, 24)):
+        v = mds.Verifier(max_B, spec.K, spec.L, spec.V, dtype=spec.dtype, cluster=cluster)
+        for scheme in ("WIS", "SpecTr", "IS"):
+            out, acc, diag = v.verify(w.target, w.draft_list(), w.model_ids, w.tokens, w.temps, scheme, 21,
+                                      diag=True)
+            torch.cuda.synchronize()
+            acc_h = acc.cpu().numpy().copy()
+            dg = diag.cpu().numpy().copy()
+            for b in range(spec.B):         # depths past the walk's end are not written
+                dg[b, acc_h[b] + 1:] = 0.0
+            got = (out.cpu().numpy().copy(), acc_h, dg)
+            if scheme not in ref:
+                ref[scheme] = got
+            else:
+                for name, a, b in zip(("tokens", "accept", "diag"), ref[scheme], got):
+                    bad = np.argwhere(~((a == b) | (np.isnan(a) & np.isnan(b)) if a.dtype.kind == "f" else a == b))
+                    assert bad.size == 0, (f"{scheme} launch {rep}: {name} differs at {bad[:4].tolist()}: "
+                                           f"{a[tuple(bad[0])]} vs {b[tuple(bad[0])]}")
+        assert v.status()[0] == 0
+        v.close()
+        t = mds.Verifier(8, other.spec.K, other.spec.L, other.spec.V, dtype=other.spec.dtype)
+        t.verify(other.target, other.draft_list(), other.model_ids, other.tokens, other.temps, "WIS", rep)
+        torch.cuda.synchronize()
+        t.close()
