@@ -27,6 +27,8 @@
 #include <cuda_bf16.h>
 #include <cooperative_groups.h>
 
+#include <type_traits>
+
 #include "mds_internal.h"
 
 namespace mds {
@@ -232,6 +234,7 @@ struct State {
   float red[kWarps * 3 * kMaxRows];
   float wthr[kWarps];        // per warp: bound on the target logits outside its list
   float wtau[kWarps];        // per warp: largest target logit dropped at a merge
+  int hcnt[2][kWarps];       // candidate-filter refresh: per-warp counts, double-buffered
   Cand wcand[kWarps * kTop];
   Cand blk[kTop];
   Cand fin[kTop];
@@ -242,7 +245,6 @@ struct State {
   float spec_val[kMaxSpecial];
   int om[MDS_MAX_S];
   float om_x[MDS_MAX_S], om_q[MDS_MAX_S], om_a[MDS_MAX_S], om_b[MDS_MAX_S];
-  float W[kMaxPairs];
   float lp_rs[kMaxPairs], lp_fl[kMaxPairs], lp_fh[kMaxPairs], lp_m[kMaxPairs];
   float A2, B2;
   // WIS candidate list bookkeeping
@@ -481,10 +483,29 @@ struct Kernel {
     }
   }
 
-  template <class FN>
-  __device__ void stream(uint32_t mask, FN&& fn) {
+  struct NoHook {
+    __device__ void operator()() const {}
+  };
+
+  // With a hook, every warp calls hook() (a block-wide step) after its 1st,
+  // 3rd, 7th, 15th and 31st group while that count is below the smallest
+  // group count of any warp, so all warps make the same calls.
+  template <class FN, class HOOK = NoHook>
+  __device__ void stream(uint32_t mask, FN&& fn, HOOK&& hook = HOOK{}) {
+    constexpr bool kHook = !std::is_same<std::decay_t<HOOK>, NoHook>::value;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int u0 = warp * Uw, u1 = min(u0 + Uw, Uv);
+    int gmin = 0, gi = 0;
+    if constexpr (kHook) {
+      gmin = 0x7fffffff;
+      for (int w = 0; w < kWarps; ++w) gmin = min(gmin, (max(0, min(Uw, Uv - w * Uw)) + 31) / 32);
+    }
+    auto after_group = [&]() {
+      if constexpr (kHook) {
+        ++gi;
+        if ((gi == 1 || gi == 7) && gi < gmin) hook();
+      }
+    };
     if (u0 >= u1) return;
     const int nrm = __popc(mask);
     const int su = stage_units(nrm);
@@ -492,6 +513,7 @@ struct Kernel {
       for (int g = u0; g < u1; g += 32) {
         const int gu = g + lane;
         fn(gu, gu < u1, GlobalLoad<DT>{S.gptr, tok0, p.V, gu, p.tma_ok != 0});
+        after_group();
       }
       return;
     }
@@ -516,6 +538,7 @@ struct Kernel {
       for (int g = cu0; g < cu1; g += 32) {
         const int gu = g + lane;
         fn(gu, gu < cu1, StageLoad<DT>{base, mask, su * 16, g - cu0 + lane});
+        after_group();
       }
       __syncwarp();
       if (lane == 0 && c + kWStages < nch) {
@@ -564,6 +587,20 @@ struct Kernel {
       if (__reduce_add_sync(0xffffffffu, cnt) >= kListN) t = c;
     }
     if (t != 0u) theta = fmaxf(theta, ord_val(t));
+    napp = drop_warp_list<R>(napp, theta, m, cr, pm, ps, wa_id, wa_l);
+#pragma unroll
+    for (int e = 0; e < VE; ++e)
+      if (!(v0[e] > theta)) aside &= ~(1u << e);
+    return napp;
+  }
+
+  // Warp-wide: drop the entries of the warp's list at or below `theta` (their
+  // exp values join the pruned sums) and compact the rest in order.
+  template <int R>
+  __device__ int drop_warp_list(int napp, float theta, const float (&m)[R], const float (&cr)[R], float (&pm)[R],
+                                float (&ps)[R], int* wa_id, float* wa_l) {
+    const int lane = threadIdx.x & 31;
+    constexpr int kPer = kWarpApp / 32;
 #pragma unroll
     for (int r = 0; r < R; ++r) {
       float wm = m[r];
@@ -610,9 +647,6 @@ struct Kernel {
     }
 #pragma unroll
     for (int r = 0; r < R; ++r) ps[r] = __fadd_rn(ps[r], warp_sum(add[r]));
-#pragma unroll
-    for (int e = 0; e < VE; ++e)
-      if (!(v0[e] > theta)) aside &= ~(1u << e);
     return outp;
   }
 
@@ -639,6 +673,7 @@ struct Kernel {
       cr[r] = S.c[r0 + r];
     }
     float theta = kNegInf;              // warp-uniform
+    bool first = true;                  // the warp's first group (warp-uniform)
     int napp = 0;                       // this warp's set-aside tokens (warp-uniform)
     float pm[R], ps[R];                 // pruned set-aside tokens: reference max and sum (warp-uniform)
 #pragma unroll
@@ -658,54 +693,30 @@ struct Kernel {
 #pragma unroll
         for (int e = 0; e < VE; ++e) v0[e] = kNegInf;
       }
+      const int t0 = tok0 + gu * VE;
       uint32_t aside = 0u;
       if constexpr (CAND) {
-        float mu = v0[0];
+        if (first) {
+          // the warp's first group: with every lane holding a whole unit, the
+          // 32 lanes' maxima are 32 tokens of the group at or above their
+          // minimum, so that minimum is at most the group's 32nd largest
+          // target logit
+          first = false;
+          float mx = v0[0];
 #pragma unroll
-        for (int e = 1; e < VE; ++e) mu = fmaxf(mu, v0[e]);
-        const int t0 = tok0 + gu * VE;
+          for (int e = 1; e < VE; ++e) mx = fmaxf(mx, v0[e]);
+          const bool whole = valid && t0 + VE <= p.V;
+          if (__all_sync(0xffffffffu, whole)) {
+#pragma unroll
+            for (int o = 16; o; o >>= 1) mx = fminf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+            theta = fmaxf(theta, mx);
+          }
+        }
 #pragma unroll
         for (int e = 0; e < VE; ++e)
           if (t0 + e < p.V && v0[e] > theta) aside |= 1u << e;
-        const int nadd = __reduce_add_sync(0xffffffffu, __popc(aside));
-        if (nadd) {
-          if (napp + nadd > kWarpApp) {
-            if (mu > m[0]) {   // keep the running maxima current for the pruned sums
-              sc[0] = (m[0] == kNegInf) ? 0.f : __fmul_rn(sc[0], ex2(__fmul_rn(__fsub_rn(m[0], mu), cr[0])));
-              m[0] = mu;
-            }
-            napp = prune_warp_list<R>(napp, theta, aside, v0, m, cr, pm, ps, wa_id, wa_l);
-          }
-          // append in lane order, each lane its flagged tokens in token order;
-          // the other rows' logits are re-read from the unit
-          int cnt = __popc(aside), incl = cnt;
-#pragma unroll
-          for (int o = 1; o < 32; o <<= 1) {
-            const int y = __shfl_up_sync(0xffffffffu, incl, o);
-            if (lane >= o) incl += y;
-          }
-          int pos = napp + incl - cnt;
-          if (aside) {
-            float vr[VE];
-#pragma unroll
-            for (int e = 0; e < VE; ++e)
-              if ((aside >> e) & 1u) {
-                wa_id[pos] = t0 + e;
-                wa_l[pos] = v0[e];
-                ++pos;
-              }
-#pragma unroll
-            for (int r = 1; r < R; ++r) {
-              L(r0 + r, vr);
-              int q = napp + incl - cnt;
-#pragma unroll
-              for (int e = 0; e < VE; ++e)
-                if ((aside >> e) & 1u) wa_l[r * kWarps * kWarpApp + q++] = vr[e];
-            }
-          }
-          napp += __shfl_sync(0xffffffffu, incl, 31);
-        }
       }
+      // sums of the tokens not set aside (one rescale per unit and row)
 #pragma unroll
       for (int r = 0; r < R; ++r) {
         float v[VE];
@@ -725,9 +736,103 @@ struct Kernel {
           sc[r] = (m[r] == kNegInf) ? 0.f : __fmul_rn(sc[r], ex2(__fmul_rn(__fsub_rn(m[r], mu), cr[r])));
           m[r] = mu;
         }
+        if (m[r] > kNegInf) {   // exp of -inf is 0; only -inf - -inf must be avoided
 #pragma unroll
-        for (int e = 0; e < VE; ++e)
-          if (!((aside >> e) & 1u) && v[e] > kNegInf) sc[r] = __fadd_rn(sc[r], ex2(__fmul_rn(__fsub_rn(v[e], m[r]), cr[r])));
+          for (int e = 0; e < VE; ++e) {
+            const float t = ex2(__fmul_rn(__fsub_rn(v[e], m[r]), cr[r]));
+            sc[r] = __fadd_rn(sc[r], ((aside >> e) & 1u) ? 0.f : t);
+          }
+        }
+      }
+      if constexpr (CAND) {
+        if (__any_sync(0xffffffffu, aside != 0u)) {
+          const int nadd = __reduce_add_sync(0xffffffffu, __popc(aside));
+          if (napp + nadd > kWarpApp) {
+            const uint32_t before = aside;
+            napp = prune_warp_list<R>(napp, theta, aside, v0, m, cr, pm, ps, wa_id, wa_l);
+            const uint32_t back = before & ~aside;   // unflagged by the raised theta: sum them now
+            if (back) {
+#pragma unroll
+              for (int r = 0; r < R; ++r) {
+                float v[VE];
+                if (r == 0) {
+#pragma unroll
+                  for (int e = 0; e < VE; ++e) v[e] = v0[e];
+                } else {
+                  L(r0 + r, v);
+                }
+#pragma unroll
+                for (int e = 0; e < VE; ++e)
+                  if (((back >> e) & 1u) && v[e] > kNegInf)
+                    sc[r] = __fadd_rn(sc[r], ex2(__fmul_rn(__fsub_rn(v[e], m[r]), cr[r])));
+              }
+            }
+          }
+          // append in lane order, each lane its flagged tokens in token order;
+          // the other rows' logits are re-read from the unit
+          const int cnt = __popc(aside);
+          int incl = cnt;
+#pragma unroll
+          for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += y;
+          }
+          if (aside) {
+            int pos = napp + incl - cnt;
+#pragma unroll
+            for (int e = 0; e < VE; ++e)
+              if ((aside >> e) & 1u) {
+                wa_id[pos] = t0 + e;
+                wa_l[pos] = v0[e];
+                ++pos;
+              }
+            float vr[VE];
+#pragma unroll
+            for (int r = 1; r < R; ++r) {
+              L(r0 + r, vr);
+              int q = napp + incl - cnt;
+#pragma unroll
+              for (int e = 0; e < VE; ++e)
+                if ((aside >> e) & 1u) wa_l[r * kWarps * kWarpApp + q++] = vr[e];
+            }
+          }
+          napp += __shfl_sync(0xffffffffu, incl, 31);
+        }
+      }
+    }, [&]() {
+      // CTA-wide refresh of the threshold: the kListN-th largest target
+      // logit among all warps' lists (bisection on order-preserving keys,
+      // one block barrier per step, counts double-buffered) is a lower bound
+      // of the CTA's; every warp raises theta to it and drops what fell below.
+      if constexpr (CAND) {
+        constexpr int kPer = kWarpApp / 32;
+        unsigned lk[kPer];
+#pragma unroll
+        for (int k = 0; k < kPer; ++k) lk[k] = (k * 32 + lane < napp) ? ord_key(wa_l[k * 32 + lane]) : 0u;
+        unsigned t = 0u;
+        int par = 0;
+#pragma unroll 1
+        for (int bit = 31; bit >= (DT == MDS_BF16 ? 16 : 0); --bit) {
+          const unsigned c = t | (1u << bit);
+          int cnt = 0;
+#pragma unroll
+          for (int k = 0; k < kPer; ++k) cnt += (lk[k] >= c) ? 1 : 0;
+          cnt = __reduce_add_sync(0xffffffffu, cnt);
+          if (lane == 0) S.hcnt[par][warp] = cnt;
+          __syncthreads();
+          int total = 0;
+#pragma unroll
+          for (int w = 0; w < kWarps; ++w) total += S.hcnt[par][w];
+          if (total >= kListN) t = c;
+          par ^= 1;
+        }
+        if (t != 0u) {
+          const float tc = ord_val(t);
+          if (tc > theta) {
+            theta = tc;
+            napp = drop_warp_list<R>(napp, theta, m, cr, pm, ps, wa_id, wa_l);
+          }
+        }
       }
     });
     if constexpr (CAND) {
@@ -1198,11 +1303,18 @@ struct Kernel {
       }
     }
     for (int it = 0; it < kLpMaxAugment; ++it) {
-      // adjacency (u -> v when pair {u,v} gives flow to u), sources, demands
+      // demands first: with none left (or, below, no supply left) no
+      // augmenting path exists
+      uint32_t dm = 0u;
+#pragma unroll
+      for (int t = 0; t < SM; ++t)
+        if (t < s && rd[t] > eps) dm |= 1u << t;
+      if (!dm) return;
+      // adjacency (u -> v when pair {u,v} gives flow to u), sources
       uint32_t adj[SM];
 #pragma unroll
       for (int t = 0; t < SM; ++t) adj[t] = 0u;
-      uint32_t srcm = 0u, dm = 0u, par = 0u;
+      uint32_t srcm = 0u, par = 0u;
       unsigned long long srcp = 0ull;
 #pragma unroll
       for (int i = 0; i < SM; ++i) {
@@ -1224,9 +1336,7 @@ struct Kernel {
           }
         }
       }
-#pragma unroll
-      for (int t = 0; t < SM; ++t)
-        if (t < s && rd[t] > eps) dm |= 1u << t;
+      if (!srcm) return;
       uint32_t visited = srcm, frontier = srcm, hit = srcm & dm;
       for (int level = 0; level < SM && !hit && frontier; ++level) {
         uint32_t nxt = 0u;
@@ -1310,9 +1420,8 @@ struct Kernel {
 
   // Solve one stage given Omega_1 in S.om (increasing token ids; entries
   // past s ignored) with q, a, b at those tokens in S.om_q / S.om_a / S.om_b
-  // and the Omega_2 masses: writes p_I on Omega_1 to S.om_x and the pair
-  // weights to S.W (layout of pidx(., ., SM)), and returns the stage output
-  // for the ordered inputs (A, B) and uniform u.  Single thread.
+  // and the Omega_2 masses: writes p_I on Omega_1 to S.om_x and returns the
+  // stage output for the ordered inputs (A, B) and uniform u.  Single thread.
   // Pair state: registers for SM = 5, the shared LP scratch for SM = 8.
   template <int SM>
   __device__ __forceinline__ int stage_solve_t(int s, float A2, float B2, int A, int Btok, float u) {
@@ -1353,31 +1462,53 @@ struct Kernel {
       }
     }
     lp_flow<SM>(s, rd, RS, FL, FH, eps);
+    // p_I on Omega_1: base + flow + half of the pair mass left over
 #pragma unroll
     for (int i = 0; i < SM; ++i) {
 #pragma unroll
       for (int j = i + 1; j < SM; ++j) {
         if (j >= s) continue;
         const int e = pidx(i, j, SM);
-        const float m = __fadd_rn(__fmul_rn(ak[i], bk[j]), __fmul_rn(ak[j], bk[i]));
         const float half = __fmul_rn(0.5f, RS[e]);
-        const float to_i = __fadd_rn(FL[e], half), to_j = __fadd_rn(FH[e], half);
-        x[i] = __fadd_rn(x[i], to_i);
-        x[j] = __fadd_rn(x[j], to_j);
-        S.W[e] = m > 0.f ? __fdiv_rn(to_i, m) : 0.5f;
+        x[i] = __fadd_rn(x[i], __fadd_rn(FL[e], half));
+        x[j] = __fadd_rn(x[j], __fadd_rn(FH[e], half));
       }
     }
 #pragma unroll
     for (int t = 0; t < SM; ++t) S.om_x[t] = x[t];
-    int pa = -1, pb = -1;
-    for (int t = 0; t < s; ++t) {
-      if (S.om[t] == A) pa = t;
-      if (S.om[t] == Btok) pb = t;
-    }
+    // the stage output for the ordered inputs (A, B): only the weight of
+    // the pair {A, B} is needed
     if (A == Btok) return A;
+    int pa = -1, pb = -1;
+#pragma unroll
+    for (int t = 0; t < SM; ++t) {
+      if (t < s && S.om[t] == A) pa = t;
+      if (t < s && S.om[t] == Btok) pb = t;
+    }
     if (pa >= 0 && pb >= 0) {
-      const int e = pidx(pa, pb, SM);
-      const float wa = (pa < pb) ? S.W[e] : __fsub_rn(1.f, S.W[e]);
+      const int lo = min(pa, pb), hi = max(pa, pb);
+      const int e = pidx(lo, hi, SM);
+      float fl = 0.f, rs = 0.f, alo = 0.f, ahi = 0.f, blo = 0.f, bhi = 0.f;
+#pragma unroll
+      for (int k = 0; k < SM * (SM - 1) / 2; ++k)
+        if (k == e) {
+          fl = FL[k];
+          rs = RS[k];
+        }
+#pragma unroll
+      for (int t = 0; t < SM; ++t) {
+        if (t == lo) {
+          alo = ak[t];
+          blo = bk[t];
+        }
+        if (t == hi) {
+          ahi = ak[t];
+          bhi = bk[t];
+        }
+      }
+      const float m = __fadd_rn(__fmul_rn(alo, bhi), __fmul_rn(ahi, blo));
+      const float wlo = m > 0.f ? __fdiv_rn(__fadd_rn(fl, __fmul_rn(0.5f, rs)), m) : 0.5f;
+      const float wa = (pa < pb) ? wlo : __fsub_rn(1.f, wlo);
       return (u < wa) ? A : Btok;
     }
     if (pa >= 0) return A;
@@ -1599,80 +1730,88 @@ struct Kernel {
     return S.Y;
   }
 
-  // One stage on the merged candidate list, by warp 0 of every CTA.
-  // Returns false (and changes nothing) if the list cannot certify Omega_1.
+  // One stage on the candidate list (at most 32 entries, by token id), by
+  // warp 0 of every CTA, one entry per lane.  Returns false (and changes
+  // nothing) if the list cannot certify Omega_1.
   __device__ bool wis_stage_fast(int A, int Btok, int rb, float u) {
+    static_assert(kListN <= 32, "one list entry per lane");
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int s = min(p.wis_s, p.V);
     const int n = S.ncand;
     if (warp == 0) {
-      Cand top[kTop];
-#pragma unroll
-      for (int t = 0; t < kTop; ++t) top[t] = CAND_NONE;
-      float suma = 0.f, sumb = 0.f;
       const float iz0 = S.invZ[0], izb = S.invZ[rb];
-      for (int i = lane; i < n; i += 32) {
-        const float q = __fmul_rn(cm_e[i], iz0);
-        float a;
-        if (cm_sp[i]) {
-          a = cm_a[i];
+      const bool have = lane < n;
+      float q = 0.f, a = 0.f, b = 0.f, key = kNegInf;
+      if (have) {
+        q = __fmul_rn(cm_e[lane], iz0);
+        if (cm_sp[lane]) {
+          a = cm_a[lane];
         } else {
-          a = 0.f;
           for (int r = 1; r < S.nrows; ++r)
-            if (S.gamma[r] != 0.f) a = __fmaf_rn(S.gamma[r], __fmul_rn(cm_e[r * p.cand_cap + i], S.invZ[r]), a);
+            if (S.gamma[r] != 0.f) a = __fmaf_rn(S.gamma[r], __fmul_rn(cm_e[r * p.cand_cap + lane], S.invZ[r]), a);
         }
-        const float b = __fmul_rn(cm_e[rb * p.cand_cap + i], izb);
-        cand_insert(top, Cand{__fmaf_rn(-a, b, q), i, a, b}, suma, sumb);   // id: list index (token order)
+        b = __fmul_rn(cm_e[rb * p.cand_cap + lane], izb);
+        key = __fadd_rn(__fmaf_rn(-a, b, q), 0.f);   // -0 -> +0: keys compare as floats
       }
-      float ra, rbs;
-      warp_merge(top, S.fin, s, ra, rbs);
-      suma = warp_sum(suma);
-      sumb = warp_sum(sumb);
-      if (lane == 0) {
-        // certification: s candidates, and the s-th key above every key
-        // outside the list (each such key is <= q < 2^-level / Z)
-        const float qout = __fmul_rn(__fmul_rn(S.cand_q, iz0), 1.0001f);
-        const bool ok = (n >= s) && (S.cand_all || S.fin[s - 1].key > qout);
-        S.fast_ok = ok ? 1 : 0;
-        if (ok) {
-          // Omega_2 masses: complement (generic law) + candidates outside Omega_1
+      // Omega_1: s rounds of a warp max over order-preserving keys, ties to
+      // the lower lane (the lower token id)
+      unsigned kk = have ? ord_key(key) : 0u;
+      uint32_t selm = 0u;
+      float kth = kNegInf;
+      for (int t = 0; t < s; ++t) {
+        const unsigned km = __reduce_max_sync(0xffffffffu, kk);
+        const uint32_t who = __ballot_sync(0xffffffffu, km != 0u && kk == km);
+        if (!who) break;
+        const int wl = __ffs(who) - 1;
+        selm |= 1u << wl;
+        if (lane == wl) kk = 0u;
+        kth = ord_val(km);
+      }
+      const bool sel = (selm >> lane) & 1u;
+      // certification: s entries, and the s-th key above every key outside
+      // the list (each such key is <= its q <= q(tau))
+      const float qout = __fmul_rn(__fmul_rn(S.cand_q, iz0), 1.0001f);
+      const bool ok = __popc(selm) == s && (S.cand_all || kth > qout);
+      const float ra = warp_sum((have && !sel) ? a : 0.f);
+      const float rbm = warp_sum((have && !sel) ? b : 0.f);
+      if (!ok) {
+        if (lane == 0) S.fast_ok = 0;
+      } else {
+        // Omega_1 by token id = the selected lanes in increasing order
+        const int rk = __popc(selm & ((1u << lane) - 1u));
+        if (lane >= s && lane < MDS_MAX_S) {   // slots past s are ignored by the solve; keep them defined
+          S.om[lane] = -1;
+          S.om_q[lane] = 0.f;
+          S.om_a[lane] = 0.f;
+          S.om_b[lane] = 0.f;
+        }
+        if (sel) {
+          S.om[rk] = cm_id[lane];
+          S.om_q[rk] = q;
+          S.om_a[rk] = a;
+          S.om_b[rk] = b;
+        }
+        __syncwarp();
+        if (lane == 0) {
+          // Omega_2 masses: complement (generic law) + list entries outside Omega_1
           float sa = 0.f;
           for (int r = 1; r < S.nrows; ++r)
             if (S.gamma[r] != 0.f) sa = __fmaf_rn(S.gamma[r], __fmul_rn(S.pc[r], S.invZ[r]), sa);
-          float sb = __fmul_rn(S.pc[rb], izb);
-          sa = __fadd_rn(sa, __fadd_rn(suma, ra));
-          sb = __fadd_rn(sb, __fadd_rn(sumb, rbs));
-          omega1_sorted(S.fin, s);   // list indices, increasing = token order
-          int oi[MDS_MAX_S];
-#pragma unroll
-          for (int t = 0; t < MDS_MAX_S; ++t) {
-            oi[t] = (t < s) ? S.om[t] : -1;
-            const int ii = (t < s) ? oi[t] : 0;
-            S.om[t] = (t < s) ? cm_id[ii] : -1;      // token ids for the solve
-            S.om_q[t] = (t < s) ? __fmul_rn(cm_e[ii], iz0) : 0.f;
-          }
+          const float sb = __fadd_rn(__fmul_rn(S.pc[rb], izb), rbm);
+          sa = __fadd_rn(sa, ra);
           S.Y = stage_solve(s, sa, sb, A, Btok, u);
-#pragma unroll
-          for (int t = 0; t < MDS_MAX_S; ++t) S.om[t] = oi[t];   // back to list indices
           S.A2 = sa;
           S.B2 = sb;
+          S.fast_ok = 1;
         }
-      }
-      __syncwarp();
-      if (S.fast_ok) {
-        // law update on the list: specials outside Omega_1, then Omega_1
+        __syncwarp();
+        // law update on the list: Omega_1 takes its x, other specials mix
         const float A2 = S.A2, B2 = S.B2;
-        for (int i = lane; i < n; i += 32) {
-          int t1 = -1;
-          for (int t = 0; t < s; ++t)
-            if (S.om[t] == i) t1 = t;
-          if (t1 >= 0) {
-            cm_a[i] = S.om_x[t1];
-            cm_sp[i] = 1;
-          } else if (cm_sp[i]) {
-            const float b = __fmul_rn(cm_e[rb * p.cand_cap + i], izb);
-            cm_a[i] = __fmul_rn(0.5f, __fadd_rn(__fmul_rn(cm_a[i], B2), __fmul_rn(b, A2)));
-          }
+        if (sel) {
+          cm_a[lane] = S.om_x[rk];
+          cm_sp[lane] = 1;
+        } else if (have && cm_sp[lane]) {
+          cm_a[lane] = __fmul_rn(0.5f, __fadd_rn(__fmul_rn(a, B2), __fmul_rn(b, A2)));
         }
         __syncwarp();
         if (lane == 0) gamma_update(rb, A2, B2);
