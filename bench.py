@@ -211,6 +211,29 @@ def agreement(g_tok, g_acc, outs):
     return {"sequences": len(outs), "identical": same, "band": band, "mismatch": bad}
 
 
+# ----------------------------------------------------------------- ranks
+
+
+def rank_seed(spec, rank):
+    """Data seed of a rank's own batch (weak scaling: every rank verifies
+    B sequences of its own, independent of the others)."""
+    return spec.data_seed + 7919 * rank
+
+
+def combine_ranks(rows, abytes, ms, world, device):
+    """Whole-job figures over ranks: visited rows and algorithmic bytes
+    summed, the time of the slowest rank."""
+    if world == 1:
+        return rows, abytes, ms
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(rows), float(abytes)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    m = torch.tensor([float(ms)], dtype=torch.float64, device=device)
+    dist.all_reduce(m, op=dist.ReduceOp.MAX)
+    return int(round(t[0].item())), int(round(t[1].item())), float(m[0].item())
+
+
 # ----------------------------------------------------------------- main
 
 
@@ -264,7 +287,7 @@ def main():
     dev = torch.device("cuda", local if world > 1 else 0)
     torch.cuda.set_device(dev)
     from paper_2410_18234_gb300 import mds
-    w = make_workload(spec, device=dev, seed=spec.data_seed + 7919 * rank)
+    w = make_workload(spec, device=dev, seed=rank_seed(spec, rank))
     v = mds.Verifier(spec.B, spec.K, spec.L, spec.V, dtype=spec.dtype, cluster=args.cluster, device=dev.index)
     drafts = w.draft_list()
     out_tokens = torch.empty(spec.B, spec.L + 1, dtype=torch.int32, device=dev)
@@ -303,18 +326,15 @@ def main():
         dist.barrier()
     clk = clocks.stop() if clocks else None
     times = [s.elapsed_time(e) for s, e in zip(starts, ends)]
-    ms = float(np.mean(times))
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms_own = float(np.mean(times))
 
     tok = w.tokens.cpu().numpy()
     o_tok = out_tokens.cpu().numpy()
     o_acc = out_acc.cpu().numpy()
     rows, abytes = walk_accounting(tok, w.model_ids, o_tok, o_acc, spec.V, es)
-    value = rows * world / (ms * 1e-3)
-    achieved = abytes / (ms * 1e-3) / 1e9
+    rows_all, _, ms = combine_ranks(rows, abytes, ms_own, world, dev)
+    value = rows_all / (ms * 1e-3)
+    achieved = abytes / (ms_own * 1e-3) / 1e9   # this rank's kernel against one GPU's peak
     peak, peak_kind = hbm_peak()
 
     # ------------------------------------------------------------- e2e through the host-buffer entry
@@ -339,7 +359,7 @@ def main():
         h2d = (h_target.numel() * h_target.element_size() + sum(d.numel() * d.element_size() for d in h_drafts)
                + h_tokens.numel() * 4 + h_temps.numel() * 4)
         d2h = h_out.numel() * 4 + h_acc.numel() * 4
-        e2e = {"value": rows * world / e2e_s, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+        e2e = {"value": rows_all / e2e_s, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
                "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_s * 1e3}
 
     # ------------------------------------------------------------- oracle agreement + cpu baseline
@@ -370,7 +390,7 @@ def main():
             "e2e": e2e,
             "gpu_launches": args.steps,
             "clocks": clk,
-            "vocab_rows_per_step": rows,
+            "vocab_rows_per_step": rows_all,
             "block_efficiency": float(np.mean(o_acc + 1)),
             "oracle_agreement": parity,
             "status_bits": bits,

@@ -429,6 +429,7 @@ struct Kernel {
   char* ring;          // streaming rings: kWarps x kWStages stages
   uint32_t* bitmap;    // special-token bits of this CTA's slice
   float* segsum;       // per-segment residual sums
+  float* chksum;       // per-chunk (32 segments) residual sums
   float* isW;          // IS: weights [rows][kIsNodesMax]
   float* isT;          // IS: nodes t_n
   char* cl_base;       // WIS: this CTA's buffered tokens and their logits per row,
@@ -1133,9 +1134,23 @@ struct Kernel {
       if (lane == 31) segsum[gu >> 5] = part;   // groups start at multiples of 32 units
     });
     __syncthreads();   // every warp's segment sums
+    // chunks of 32 segments: inclusive scans by the warps (their last value
+    // is the chunk's sum), chunks added in order by thread 0
+    const int nchk = (nsegv + 31) / 32;
+    for (int k = warp; k < nchk; k += kWarps) {
+      const int g = k * 32 + lane;
+      float v = g < nsegv ? segsum[g] : 0.f;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const float t = __shfl_up_sync(0xffffffffu, v, o);
+        if (lane >= o) v = __fadd_rn(v, t);
+      }
+      if (lane == 31) chksum[k] = v;
+    }
+    __syncthreads();
     if (threadIdx.x == 0) {
       float tot = 0.f;
-      for (int g = 0; g < nsegv; ++g) tot = __fadd_rn(tot, segsum[g]);
+      for (int k = 0; k < nchk; ++k) tot = __fadd_rn(tot, chksum[k]);
       S.xch[xbuf][0] = tot;
     }
     cluster_gather(S, 1, xbuf, cn);
@@ -1172,26 +1187,49 @@ struct Kernel {
     const int owner = S.owner;
     if (rank == owner) {
       if (threadIdx.x == 0) {
+        // chunk: the first whose running total exceeds T (else the last with mass)
         float run = S.run;
-        int g = -1, glast = -1;
-        float run_g = 0.f, run_last = 0.f;
-        for (int h = 0; h < nsegv; ++h) {
-          if (segsum[h] > 0.f) {
-            glast = h;
+        int k = -1, klast = -1;
+        float run_k = 0.f, run_last = 0.f;
+        for (int h = 0; h < nchk; ++h) {
+          if (chksum[h] > 0.f) {
+            klast = h;
             run_last = run;
           }
-          if (g < 0 && __fadd_rn(run, segsum[h]) > T) {
-            g = h;
-            run_g = run;
+          if (k < 0 && __fadd_rn(run, chksum[h]) > T) {
+            k = h;
+            run_k = run;
           }
-          run = __fadd_rn(run, segsum[h]);
+          run = __fadd_rn(run, chksum[h]);
         }
-        if (g < 0) {
-          g = glast;
-          run_g = run_last;
+        if (k < 0) {
+          k = klast;
+          run_k = run_last;
         }
-        S.seg = g;
-        S.run = run_g;
+        S.seg = k;
+        S.run = run_k;
+      }
+      __syncthreads();
+      if (warp == 0) {
+        // segment inside the chunk: the same scan as the chunk's sum
+        const int k = S.seg;
+        const float base = S.run;
+        const int g = k * 32 + lane;
+        const float sv = (k >= 0 && g < nsegv) ? segsum[g] : 0.f;
+        float v = sv;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const float t = __shfl_up_sync(0xffffffffu, v, o);
+          if (lane >= o) v = __fadd_rn(v, t);
+        }
+        const float vprev = __shfl_up_sync(0xffffffffu, v, 1);
+        const unsigned hit = __ballot_sync(0xffffffffu, __fadd_rn(base, v) > T);
+        const unsigned pos = __ballot_sync(0xffffffffu, sv > 0.f);
+        const int l = hit ? __ffs(hit) - 1 : (pos ? 31 - __clz(pos) : 0);
+        if (lane == l) {
+          S.seg = k * 32 + l;
+          S.run = (l > 0) ? __fadd_rn(base, vprev) : base;
+        }
       }
       __syncthreads();
       if (warp == 0) {
@@ -2448,15 +2486,16 @@ __global__ void __launch_bounds__(kThreads, SCHEME == MDS_IS ? 1 : 2) verify_ker
   k.nsegv = (k.Uv + 31) / 32;                                // segments the residual pass writes
   k.Uw = ((k.Uv + kWarps - 1) / kWarps + 31) & ~31;           // units per warp in a streaming pass
   k.bm_words = (p.slice + 31) / 32;
-  // dynamic shared memory: ring | segment sums | scheme region
+  // dynamic shared memory: ring | segment sums | chunk sums | scheme region
   //   IS : nodes t_n | weights W_r(n)
   //   WIS: CTA list (two copies) | warp lists = staging list | merged list, the
   //        last aliased later by the special-token bitmap (only the CTA list
   //        is ever read by other CTAs)
   k.ring = dsm;
   k.segsum = reinterpret_cast<float*>(dsm + p.ring_bytes);
+  k.chksum = k.segsum + ((k.nseg + 3) & ~3);
   {
-    char* c = reinterpret_cast<char*>(k.segsum + ((k.nseg + 3) & ~3));
+    char* c = reinterpret_cast<char*>(k.chksum + ((((k.nseg + 31) / 32) + 3) & ~3));
     k.isT = reinterpret_cast<float*>(c);
     k.isW = k.isT + kIsNodesMax;
     k.cl_base = c;
@@ -2519,7 +2558,7 @@ __global__ void __launch_bounds__(kThreads, SCHEME == MDS_IS ? 1 : 2) verify_ker
 size_t smem_bytes(const Params& p) {
   const int VE = 16 / p.esize;
   const int nseg = (p.slice / VE + 31) / 32;
-  size_t bytes = (size_t)p.ring_bytes + (size_t)((nseg + 3) & ~3) * 4;
+  size_t bytes = (size_t)p.ring_bytes + (size_t)((nseg + 3) & ~3) * 4 + (size_t)((((nseg + 31) / 32) + 3) & ~3) * 4;
   if (p.scheme == MDS_IS) bytes += (size_t)kIsNodesMax * 4 * (1 + p.rows_max);
   if (p.scheme == MDS_WIS) {
     const size_t bm = (size_t)((p.slice + 31) / 32) * 4;
