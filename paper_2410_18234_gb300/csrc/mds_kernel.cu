@@ -27,8 +27,6 @@
 #include <cuda_bf16.h>
 #include <cooperative_groups.h>
 
-#include <type_traits>
-
 #include "mds_internal.h"
 
 namespace mds {
@@ -46,6 +44,7 @@ constexpr long long kWaitLimit = 1ll << 24;
 constexpr int kFastRows = 4;            // WIS candidate path: target + up to 3 draft models
 constexpr int kWStages = 4;             // stages of each warp's streaming ring
 constexpr int kWarpApp = 128;           // candidate tokens one warp can hold during the stats pass
+constexpr int kSampleStride = 4;        // the candidate filter's starting threshold samples 1 unit in 4
 
 // Order-preserving map of floats (not NaN) to unsigned; every key is > 0.
 __device__ __forceinline__ unsigned ord_key(float f) {
@@ -160,6 +159,12 @@ struct Elt<MDS_F32> {
     v[2] = x.z;
     v[3] = x.w;
   }
+  __device__ static __forceinline__ void unpack(const uint4& x, float* v) {
+    v[0] = __uint_as_float(x.x);
+    v[1] = __uint_as_float(x.y);
+    v[2] = __uint_as_float(x.z);
+    v[3] = __uint_as_float(x.w);
+  }
 };
 template <>
 struct Elt<MDS_BF16> {
@@ -178,6 +183,16 @@ struct Elt<MDS_BF16> {
   __device__ static __forceinline__ float global(const char* row, int x) {
     return __uint_as_float((uint32_t)__ldg(reinterpret_cast<const unsigned short*>(row) + x) << 16);
   }
+  __device__ static __forceinline__ void unpack(const uint4& x, float* v) {
+    v[0] = __uint_as_float(x.x << 16);
+    v[1] = __uint_as_float(x.x & 0xffff0000u);
+    v[2] = __uint_as_float(x.y << 16);
+    v[3] = __uint_as_float(x.y & 0xffff0000u);
+    v[4] = __uint_as_float(x.z << 16);
+    v[5] = __uint_as_float(x.z & 0xffff0000u);
+    v[6] = __uint_as_float(x.w << 16);
+    v[7] = __uint_as_float(x.w & 0xffff0000u);
+  }
   __device__ static __forceinline__ void unit_global(const char* at, float* v) {
     const uint4 x = __ldg(reinterpret_cast<const uint4*>(at));
     v[0] = __uint_as_float(x.x << 16);
@@ -193,8 +208,11 @@ struct Elt<MDS_BF16> {
 
 // Probability of a logit under a row's statistics.  The same expression is
 // used for in-pass values and point lookups so both give identical bits.
+// Exponents: a term is 2^fma(l, c, -round(M c)) (one rounding, l c exact
+// inside the FMA); a partial sum moves from reference m to M by the factor
+// 2^(round(m c) - round(M c)), so every term of a row shares one reference.
 __device__ __forceinline__ float prob_of(float l, float M, float c, float invZ) {
-  return __fmul_rn(ex2(__fmul_rn(__fsub_rn(l, M), c)), invZ);
+  return __fmul_rn(ex2(__fmaf_rn(l, c, -__fmul_rn(M, c))), invZ);
 }
 
 // ------------------------------------------------------------------ shared state
@@ -234,7 +252,6 @@ struct State {
   float red[kWarps * 3 * kMaxRows];
   float wthr[kWarps];        // per warp: bound on the target logits outside its list
   float wtau[kWarps];        // per warp: largest target logit dropped at a merge
-  int hcnt[2][kWarps];       // candidate-filter refresh: per-warp counts, double-buffered
   Cand wcand[kWarps * kTop];
   Cand blk[kTop];
   Cand fin[kTop];
@@ -272,8 +289,8 @@ struct State {
 
 __device__ __forceinline__ void combine_ms(float& m, float& s, float m2, float s2, float c) {
   const float M = fmaxf(m, m2);
-  const float a = (m == kNegInf) ? 0.f : __fmul_rn(s, ex2(__fmul_rn(__fsub_rn(m, M), c)));
-  const float b = (m2 == kNegInf) ? 0.f : __fmul_rn(s2, ex2(__fmul_rn(__fsub_rn(m2, M), c)));
+  const float a = (m == kNegInf) ? 0.f : __fmul_rn(s, ex2(__fsub_rn(__fmul_rn(m, c), __fmul_rn(M, c))));
+  const float b = (m2 == kNegInf) ? 0.f : __fmul_rn(s2, ex2(__fsub_rn(__fmul_rn(m2, c), __fmul_rn(M, c))));
   m = M;
   s = __fadd_rn(a, b);
 }
@@ -484,29 +501,10 @@ struct Kernel {
     }
   }
 
-  struct NoHook {
-    __device__ void operator()() const {}
-  };
-
-  // With a hook, every warp calls hook() (a block-wide step) after its 1st,
-  // 3rd, 7th, 15th and 31st group while that count is below the smallest
-  // group count of any warp, so all warps make the same calls.
-  template <class FN, class HOOK = NoHook>
-  __device__ void stream(uint32_t mask, FN&& fn, HOOK&& hook = HOOK{}) {
-    constexpr bool kHook = !std::is_same<std::decay_t<HOOK>, NoHook>::value;
+  template <class FN>
+  __device__ void stream(uint32_t mask, FN&& fn) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int u0 = warp * Uw, u1 = min(u0 + Uw, Uv);
-    int gmin = 0, gi = 0;
-    if constexpr (kHook) {
-      gmin = 0x7fffffff;
-      for (int w = 0; w < kWarps; ++w) gmin = min(gmin, (max(0, min(Uw, Uv - w * Uw)) + 31) / 32);
-    }
-    auto after_group = [&]() {
-      if constexpr (kHook) {
-        ++gi;
-        if ((gi == 1 || gi == 7) && gi < gmin) hook();
-      }
-    };
     if (u0 >= u1) return;
     const int nrm = __popc(mask);
     const int su = stage_units(nrm);
@@ -514,7 +512,6 @@ struct Kernel {
       for (int g = u0; g < u1; g += 32) {
         const int gu = g + lane;
         fn(gu, gu < u1, GlobalLoad<DT>{S.gptr, tok0, p.V, gu, p.tma_ok != 0});
-        after_group();
       }
       return;
     }
@@ -539,7 +536,6 @@ struct Kernel {
       for (int g = cu0; g < cu1; g += 32) {
         const int gu = g + lane;
         fn(gu, gu < cu1, StageLoad<DT>{base, mask, su * 16, g - cu0 + lane});
-        after_group();
       }
       __syncwarp();
       if (lane == 0 && c + kWStages < nch) {
@@ -608,7 +604,7 @@ struct Kernel {
 #pragma unroll
       for (int o = 16; o; o >>= 1) wm = fmaxf(wm, __shfl_xor_sync(0xffffffffu, wm, o));
       if (wm > pm[r]) {
-        ps[r] = (pm[r] == kNegInf) ? 0.f : __fmul_rn(ps[r], ex2(__fmul_rn(__fsub_rn(pm[r], wm), cr[r])));
+        ps[r] = (pm[r] == kNegInf) ? 0.f : __fmul_rn(ps[r], ex2(__fsub_rn(__fmul_rn(pm[r], cr[r]), __fmul_rn(wm, cr[r]))));
         pm[r] = wm;
       }
     }
@@ -641,7 +637,7 @@ struct Kernel {
       } else if (present) {
 #pragma unroll
         for (int r = 0; r < R; ++r)
-          if (l[r] > kNegInf) add[r] = __fadd_rn(add[r], ex2(__fmul_rn(__fsub_rn(l[r], pm[r]), cr[r])));
+          if (l[r] > kNegInf) add[r] = __fadd_rn(add[r], ex2(__fmaf_rn(l[r], cr[r], -__fmul_rn(pm[r], cr[r]))));
       }
       outp += __popc(bal);
       __syncwarp();
@@ -655,9 +651,10 @@ struct Kernel {
   // sum of exp((l - m) c) per row, rescaled once per unit.  With CAND (WIS,
   // R = all rows) the pass also finds the kListN largest target logits of the
   // sequence (ties: smaller token id first), which are kept out of the sums:
-  // each warp sets aside every token above `theta`, the kListN-th largest
-  // target logit it kept so far, and prunes its list back to kListN when it
-  // fills; the CTA keeps the first kListN of its warps' lists and the
+  // each warp sets aside every token above `theta`, which starts at the
+  // kListN-th largest of the threads' target maxima over a sample and
+  // rises to the kListN-th largest target logit the warp holds whenever its
+  // list fills; the CTA keeps the first kListN of its warps' lists and the
   // cluster the first kListN of its CTAs' lists.  Every pruned or never
   // set-aside token has a target logit <= tau, the last kept one.  One
   // cluster exchange gives every CTA M and Z of each row, the candidate list
@@ -673,14 +670,66 @@ struct Kernel {
       sc[r] = 0.f;
       cr[r] = S.c[r0 + r];
     }
-    float theta = kNegInf;              // warp-uniform
-    bool first = true;                  // the warp's first group (warp-uniform)
     int napp = 0;                       // this warp's set-aside tokens (warp-uniform)
     float pm[R], ps[R];                 // pruned set-aside tokens: reference max and sum (warp-uniform)
 #pragma unroll
     for (int r = 0; r < R; ++r) {
       pm[r] = kNegInf;
       ps[r] = 0.f;
+    }
+    // The filter's starting threshold: the kListN-th largest of the threads'
+    // target maxima over a sample of the CTA's slice (every kSampleStride-th
+    // 16-byte unit, plain loads).  Those maxima are kThreads distinct
+    // tokens, so the threshold is at most the CTA's kListN-th largest target
+    // logit: every token at or below it can be in no list.
+    float theta = kNegInf;              // warp-uniform
+    if constexpr (CAND) {
+      float mx = kNegInf;
+      constexpr int kBatch = 16;        // loads in flight per thread
+      for (int u0 = threadIdx.x * kSampleStride; u0 < Uv; u0 += kThreads * kBatch * kSampleStride) {
+        if (p.tma_ok) {
+          // whole, 16-byte aligned units: raw loads first, then the maxima
+          uint4 raw[kBatch];
+#pragma unroll
+          for (int b = 0; b < kBatch; ++b) {
+            const int u = u0 + b * kThreads * kSampleStride;
+            raw[b] = (u < Uv) ? __ldg(reinterpret_cast<const uint4*>(S.gptr[r0] + ((size_t)tok0 + (size_t)u * VE) * p.esize))
+                              : make_uint4(0u, 0u, 0u, 0u);   // skipped below
+          }
+#pragma unroll
+          for (int b = 0; b < kBatch; ++b) {
+            if (u0 + b * kThreads * kSampleStride >= Uv) continue;
+            float v[VE];
+            E::unpack(raw[b], v);
+#pragma unroll
+            for (int e = 0; e < VE; ++e) mx = fmaxf(mx, v[e]);
+          }
+        } else {
+          for (int b = 0; b < kBatch; ++b) {
+            const int u = u0 + b * kThreads * kSampleStride;
+            if (u >= Uv) break;
+            float v[VE];
+            GlobalLoad<DT>{S.gptr, tok0, p.V, u, false}(r0, v);
+#pragma unroll
+            for (int e = 0; e < VE; ++e) mx = fmaxf(mx, v[e]);
+          }
+        }
+      }
+      static_assert(kWarps * 3 * kMaxRows >= kThreads, "scratch for the thread maxima");
+      S.red[threadIdx.x] = mx;
+      if (threadIdx.x == 0) S.wthr[0] = kNegInf;
+      __syncthreads();
+      if (mx > kNegInf) {
+        int rk = 0;   // rank among the threads' maxima (larger first, then lower thread)
+        for (int j = 0; j < kThreads; ++j) {
+          const float o = S.red[j];
+          rk += (o > mx || (o == mx && j < (int)threadIdx.x)) ? 1 : 0;
+        }
+        if (rk == kListN - 1) S.wthr[0] = mx;
+      }
+      __syncthreads();
+      theta = S.wthr[0];
+      __syncthreads();   // S.red and S.wthr are rewritten after the pass
     }
     int* wa_id = ap_id + warp * kWarpApp;
     float* wa_l = ap_l + warp * kWarpApp;   // row r at wa_l[r * kWarps * kWarpApp + i]
@@ -695,24 +744,9 @@ struct Kernel {
         for (int e = 0; e < VE; ++e) v0[e] = kNegInf;
       }
       const int t0 = tok0 + gu * VE;
+      (void)t0;
       uint32_t aside = 0u;
       if constexpr (CAND) {
-        if (first) {
-          // the warp's first group: with every lane holding a whole unit, the
-          // 32 lanes' maxima are 32 tokens of the group at or above their
-          // minimum, so that minimum is at most the group's 32nd largest
-          // target logit
-          first = false;
-          float mx = v0[0];
-#pragma unroll
-          for (int e = 1; e < VE; ++e) mx = fmaxf(mx, v0[e]);
-          const bool whole = valid && t0 + VE <= p.V;
-          if (__all_sync(0xffffffffu, whole)) {
-#pragma unroll
-            for (int o = 16; o; o >>= 1) mx = fminf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-            theta = fmaxf(theta, mx);
-          }
-        }
 #pragma unroll
         for (int e = 0; e < VE; ++e)
           if (t0 + e < p.V && v0[e] > theta) aside |= 1u << e;
@@ -734,13 +768,13 @@ struct Kernel {
 #pragma unroll
         for (int e = 1; e < VE; ++e) mu = fmaxf(mu, v[e]);
         if (mu > m[r]) {
-          sc[r] = (m[r] == kNegInf) ? 0.f : __fmul_rn(sc[r], ex2(__fmul_rn(__fsub_rn(m[r], mu), cr[r])));
+          sc[r] = (m[r] == kNegInf) ? 0.f : __fmul_rn(sc[r], ex2(__fsub_rn(__fmul_rn(m[r], cr[r]), __fmul_rn(mu, cr[r]))));
           m[r] = mu;
         }
         if (m[r] > kNegInf) {   // exp of -inf is 0; only -inf - -inf must be avoided
 #pragma unroll
           for (int e = 0; e < VE; ++e) {
-            const float t = ex2(__fmul_rn(__fsub_rn(v[e], m[r]), cr[r]));
+            const float t = ex2(__fmaf_rn(v[e], cr[r], -__fmul_rn(m[r], cr[r])));
             sc[r] = __fadd_rn(sc[r], ((aside >> e) & 1u) ? 0.f : t);
           }
         }
@@ -765,7 +799,7 @@ struct Kernel {
 #pragma unroll
                 for (int e = 0; e < VE; ++e)
                   if (((back >> e) & 1u) && v[e] > kNegInf)
-                    sc[r] = __fadd_rn(sc[r], ex2(__fmul_rn(__fsub_rn(v[e], m[r]), cr[r])));
+                    sc[r] = __fadd_rn(sc[r], ex2(__fmaf_rn(v[e], cr[r], -__fmul_rn(m[r], cr[r]))));
               }
             }
           }
@@ -798,41 +832,6 @@ struct Kernel {
             }
           }
           napp += __shfl_sync(0xffffffffu, incl, 31);
-        }
-      }
-    }, [&]() {
-      // CTA-wide refresh of the threshold: the kListN-th largest target
-      // logit among all warps' lists (bisection on order-preserving keys,
-      // one block barrier per step, counts double-buffered) is a lower bound
-      // of the CTA's; every warp raises theta to it and drops what fell below.
-      if constexpr (CAND) {
-        constexpr int kPer = kWarpApp / 32;
-        unsigned lk[kPer];
-#pragma unroll
-        for (int k = 0; k < kPer; ++k) lk[k] = (k * 32 + lane < napp) ? ord_key(wa_l[k * 32 + lane]) : 0u;
-        unsigned t = 0u;
-        int par = 0;
-#pragma unroll 1
-        for (int bit = 31; bit >= (DT == MDS_BF16 ? 16 : 0); --bit) {
-          const unsigned c = t | (1u << bit);
-          int cnt = 0;
-#pragma unroll
-          for (int k = 0; k < kPer; ++k) cnt += (lk[k] >= c) ? 1 : 0;
-          cnt = __reduce_add_sync(0xffffffffu, cnt);
-          if (lane == 0) S.hcnt[par][warp] = cnt;
-          __syncthreads();
-          int total = 0;
-#pragma unroll
-          for (int w = 0; w < kWarps; ++w) total += S.hcnt[par][w];
-          if (total >= kListN) t = c;
-          par ^= 1;
-        }
-        if (t != 0u) {
-          const float tc = ord_val(t);
-          if (tc > theta) {
-            theta = tc;
-            napp = drop_warp_list<R>(napp, theta, m, cr, pm, ps, wa_id, wa_l);
-          }
         }
       }
     });
@@ -907,7 +906,7 @@ struct Kernel {
 #pragma unroll
           for (int r = 0; r < R; ++r) {
             const float l = ap_l[r * kWarps * kWarpApp + i];
-            const float ev = (l > kNegInf) ? ex2(__fmul_rn(__fsub_rn(l, S.xch[xbuf][sx * r]), cr[r])) : 0.f;
+            const float ev = (l > kNegInf) ? ex2(__fmaf_rn(l, cr[r], -__fmul_rn(S.xch[xbuf][sx * r], cr[r]))) : 0.f;
             if (rk < kListN)
               kp_s[r] = ev;
             else
@@ -969,7 +968,7 @@ struct Kernel {
         for (int q = 0; q < cn; ++q) {
           const float mq = S.gat[q * nx + sx * r];
           if (!(mq > kNegInf)) continue;
-          const float f = ex2(__fmul_rn(__fsub_rn(mq, mm), cr[r]));
+          const float f = ex2(__fsub_rn(__fmul_rn(mq, cr[r]), __fmul_rn(mm, cr[r])));
           const float sq = S.gat[q * nx + sx * r + 1];
           ss = __fadd_rn(ss, __fmul_rn(sq, f));
           zz = __fadd_rn(zz, __fmul_rn(CAND ? __fadd_rn(sq, S.gat[q * nx + sx * r + 2]) : sq, f));
@@ -1036,7 +1035,7 @@ struct Kernel {
 #pragma unroll
           for (int r = 0; r < R; ++r) {
             const float l = cs_l[r * p.cand_stage + i];
-            cm_e[r * p.cand_cap + pos] = (l > kNegInf) ? ex2(__fmul_rn(__fsub_rn(l, S.M[r0 + r]), cr[r])) : 0.f;
+            cm_e[r * p.cand_cap + pos] = (l > kNegInf) ? ex2(__fmaf_rn(l, cr[r], -__fmul_rn(S.M[r0 + r], cr[r]))) : 0.f;
           }
           cm_sp[pos] = 0;
           cm_a[pos] = 0.f;
@@ -1045,7 +1044,7 @@ struct Kernel {
 #pragma unroll
           for (int r = 0; r < R; ++r) {
             const float l = cs_l[r * p.cand_stage + i];
-            if (l > kNegInf) add[r] = __fadd_rn(add[r], ex2(__fmul_rn(__fsub_rn(l, S.M[r0 + r]), cr[r])));
+            if (l > kNegInf) add[r] = __fadd_rn(add[r], ex2(__fmaf_rn(l, cr[r], -__fmul_rn(S.M[r0 + r], cr[r]))));
           }
         }
       }
@@ -1071,7 +1070,7 @@ struct Kernel {
         for (int w = 0; w < kWarps; ++w) tau = fmaxf(tau, S.wtau[w]);
         S.ncand = n;
         S.cand_all = (n == p.V) ? 1 : 0;
-        S.cand_q = (tau > kNegInf) ? ex2(__fmul_rn(__fsub_rn(tau, S.M[r0]), cr[0])) : 0.f;
+        S.cand_q = (tau > kNegInf) ? ex2(__fmaf_rn(tau, cr[0], -__fmul_rn(S.M[r0], cr[0]))) : 0.f;
       }
       clbuf ^= 1;
       __syncthreads();
