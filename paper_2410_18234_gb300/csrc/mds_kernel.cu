@@ -447,6 +447,7 @@ struct Kernel {
   uint32_t* bitmap;    // special-token bits of this CTA's slice
   float* segsum;       // per-segment residual sums
   float* chksum;       // per-chunk (32 segments) residual sums
+  float* segref;       // bonus draw: each segment sum's reference (round(max * c))
   float* isW;          // IS: weights [rows][kIsNodesMax]
   float* isT;          // IS: nodes t_n
   char* cl_base;       // WIS: this CTA's buffered tokens and their logits per row,
@@ -1116,7 +1117,7 @@ struct Kernel {
   // same sums.  Returns the token (cluster-uniform) and the total mass.
   template <class RF>
   __device__ int sample_cdf(uint32_t mask, const RF& rf, float u01, float* total) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
     stream(mask, [&](int gu, bool valid, const auto& L) {
       float part = 0.f;
       if (valid) {
@@ -1133,6 +1134,16 @@ struct Kernel {
       if (lane == 31) segsum[gu >> 5] = part;   // groups start at multiples of 32 units
     });
     __syncthreads();   // every warp's segment sums
+    return cdf_search(rf, u01, total);
+  }
+
+  // The search of an inverse-CDF draw once segsum[] holds every segment's
+  // weight (this CTA's slice, token order): the smallest token whose running
+  // sum exceeds u * (total over the cluster).  rf(gu, L, r) gives the
+  // weights of unit gu for the re-walk of the owning segment.
+  template <class RF>
+  __device__ int cdf_search(const RF& rf, float u01, float* total) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     // chunks of 32 segments: inclusive scans by the warps (their last value
     // is the chunk's sum), chunks added in order by thread 0
     const int nchk = (nsegv + 31) / 32;
@@ -1281,6 +1292,92 @@ struct Kernel {
     const int z = S.Zslot;
     __syncthreads();
     return z;
+  }
+
+  // Bonus draw (depth L): one pass over the target row gives its max, its
+  // sum and the segment sums of the inverse-CDF draw from q.  Each warp takes
+  // every exponent against its own running maximum (a warp-uniform
+  // reference), so the same values feed the lane sums and the segment
+  // sums; a segment sum keeps its reference and becomes q mass once M and Z
+  // are known.
+  __device__ int bonus_pass(float u01, float* total) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const float c = S.c[0];
+    float wmax = kNegInf, wref = kNegInf;   // warp-uniform; wref = round(wmax c)
+    float sc = 0.f;                         // this lane's sum, relative to wref
+    stream(1u, [&](int gu, bool valid, const auto& L) {
+      float v[VE];
+      if (valid) {
+        L(0, v);
+      } else {
+#pragma unroll
+        for (int e = 0; e < VE; ++e) v[e] = kNegInf;
+      }
+      float wm = v[0];
+#pragma unroll
+      for (int e = 1; e < VE; ++e) wm = fmaxf(wm, v[e]);
+#pragma unroll
+      for (int o = 16; o; o >>= 1) wm = fmaxf(wm, __shfl_xor_sync(0xffffffffu, wm, o));
+      if (wm > wmax) {
+        const float nref = __fmul_rn(wm, c);
+        sc = (wmax == kNegInf) ? 0.f : __fmul_rn(sc, ex2(__fsub_rn(wref, nref)));
+        wmax = wm;
+        wref = nref;
+      }
+      float part = 0.f;
+      if (wmax > kNegInf) {
+#pragma unroll
+        for (int e = 0; e < VE; ++e) part = __fadd_rn(part, ex2(__fmaf_rn(v[e], c, -wref)));
+      }
+      sc = __fadd_rn(sc, part);
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const float t = __shfl_up_sync(0xffffffffu, part, o);
+        if (lane >= o) part = __fadd_rn(part, t);
+      }
+      if (lane == 31) {
+        segsum[gu >> 5] = part;
+        segref[gu >> 5] = wref;
+      }
+    });
+    // M and Z: warps (one reference each), then the CTA, then the cluster
+    const float ss = warp_sum(sc);
+    if (lane == 0) {
+      S.red[warp * 2] = wmax;
+      S.red[warp * 2 + 1] = ss;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      float mm = kNegInf, zz = 0.f;
+      for (int w = 0; w < kWarps; ++w) combine_ms(mm, zz, S.red[w * 2], S.red[w * 2 + 1], c);
+      S.xch[xbuf][0] = mm;
+      S.xch[xbuf][1] = zz;
+    }
+    cluster_gather(S, 2, xbuf, cn);
+    if (threadIdx.x == 0) {
+      float mm = kNegInf, zz = 0.f;
+      for (int q = 0; q < cn; ++q) combine_ms(mm, zz, S.gat[2 * q], S.gat[2 * q + 1], c);
+      if (!(mm > kNegInf) || mm != mm) {
+        atomicOr(p.status, MDS_ST_NONFINITE);
+        mm = 0.f;
+      }
+      S.M[0] = mm;
+      finish_row(0, zz);
+    }
+    __syncthreads();
+    // segment sums -> q mass
+    const float mc = __fmul_rn(S.M[0], c), iz = S.invZ[0];
+    for (int g = threadIdx.x; g < nsegv; g += kThreads)
+      segsum[g] = (segref[g] > kNegInf) ? __fmul_rn(__fmul_rn(segsum[g], ex2(__fsub_rn(segref[g], mc))), iz) : 0.f;
+    __syncthreads();
+    return cdf_search(
+        [&](int, const auto& L, float* r) {
+          float v[VE];
+          L(0, v);
+#pragma unroll
+          for (int e = 0; e < VE; ++e) r[e] = prob_of(v[e], S.M[0], S.c[0], S.invZ[0]);
+        },
+        u01, total);
   }
 
   // ---------------------------------------------------------------- schemes
@@ -2190,21 +2287,13 @@ struct Kernel {
         S.R = 0.f;
       }
       __syncthreads();
-      depth_stats(SCHEME == MDS_WIS && !bonus && S.nv > 1);
+      if (!bonus) depth_stats(SCHEME == MDS_WIS && S.nv > 1);
       int Z;
       float qY = 0.f, pIY = 0.f, Rdiag = 0.f;
       int Ydiag = -1;
       if (bonus) {
         float tot;
-        Z = sample_cdf(
-            1u,
-            [&](int, const auto& L, float* r) {
-              float v[VE];
-              L(0, v);
-#pragma unroll
-              for (int e = 0; e < VE; ++e) r[e] = prob_of(v[e], S.M[0], S.c[0], S.invZ[0]);
-            },
-            draw_uniform(p.seed, b, j, kDrawBonus), &tot);
+        Z = bonus_pass(draw_uniform(p.seed, b, j, kDrawBonus), &tot);
         Rdiag = tot;
       } else if constexpr (SCHEME == MDS_SPECTR) {
         Z = spectr(b, j, &qY, &pIY, &Ydiag, &Rdiag);
@@ -2485,7 +2574,7 @@ __global__ void __launch_bounds__(kThreads, SCHEME == MDS_IS ? 1 : 2) verify_ker
   k.nsegv = (k.Uv + 31) / 32;                                // segments the residual pass writes
   k.Uw = ((k.Uv + kWarps - 1) / kWarps + 31) & ~31;           // units per warp in a streaming pass
   k.bm_words = (p.slice + 31) / 32;
-  // dynamic shared memory: ring | segment sums | chunk sums | scheme region
+  // dynamic shared memory: ring | segment sums | chunk sums | segment references | scheme region
   //   IS : nodes t_n | weights W_r(n)
   //   WIS: CTA list (two copies) | warp lists = staging list | merged list, the
   //        last aliased later by the special-token bitmap (only the CTA list
@@ -2493,8 +2582,9 @@ __global__ void __launch_bounds__(kThreads, SCHEME == MDS_IS ? 1 : 2) verify_ker
   k.ring = dsm;
   k.segsum = reinterpret_cast<float*>(dsm + p.ring_bytes);
   k.chksum = k.segsum + ((k.nseg + 3) & ~3);
+  k.segref = k.chksum + ((((k.nseg + 31) / 32) + 3) & ~3);
   {
-    char* c = reinterpret_cast<char*>(k.chksum + ((((k.nseg + 31) / 32) + 3) & ~3));
+    char* c = reinterpret_cast<char*>(k.segref + ((k.nseg + 3) & ~3));
     k.isT = reinterpret_cast<float*>(c);
     k.isW = k.isT + kIsNodesMax;
     k.cl_base = c;
@@ -2557,7 +2647,7 @@ __global__ void __launch_bounds__(kThreads, SCHEME == MDS_IS ? 1 : 2) verify_ker
 size_t smem_bytes(const Params& p) {
   const int VE = 16 / p.esize;
   const int nseg = (p.slice / VE + 31) / 32;
-  size_t bytes = (size_t)p.ring_bytes + (size_t)((nseg + 3) & ~3) * 4 + (size_t)((((nseg + 31) / 32) + 3) & ~3) * 4;
+  size_t bytes = (size_t)p.ring_bytes + (size_t)((nseg + 3) & ~3) * 4 * 2 + (size_t)((((nseg + 31) / 32) + 3) & ~3) * 4;
   if (p.scheme == MDS_IS) bytes += (size_t)kIsNodesMax * 4 * (1 + p.rows_max);
   if (p.scheme == MDS_WIS) {
     const size_t bm = (size_t)((p.slice + 31) / 32) * 4;
