@@ -28,7 +28,7 @@ struct mds_ctx {
 
 namespace {
 
-constexpr int kRingBytes = 64 * 1024;   // streaming rings: 8 warps x 4 stages of 2 KB
+constexpr int kRingBytes = 80 * 1024;   // streaming rings: 8 warps x 5 stages of 2 KB
 
 struct DeviceGuard {
   int prev = -1;

@@ -42,8 +42,8 @@ constexpr int kLpMaxAugment = 4096;
 constexpr float kLpEpsRel = 1e-6f;
 constexpr long long kWaitLimit = 1ll << 24;
 constexpr int kFastRows = 4;            // WIS candidate path: target + up to 3 draft models
-constexpr int kWStages = 4;             // stages of each warp's streaming ring
-constexpr int kWarpApp = 128;           // candidate tokens one warp can hold during the stats pass
+constexpr int kWStages = 5;             // stages of each warp's streaming ring
+constexpr int kWarpApp = 64;            // candidate tokens one warp can hold during the stats pass
 constexpr int kSampleStride = 4;        // the candidate filter's starting threshold samples 1 unit in 4
 
 // Order-preserving map of floats (not NaN) to unsigned; every key is > 0.
@@ -444,7 +444,7 @@ struct Kernel {
   const Params& p;
   State& S;
   char* ring;          // streaming rings: kWarps x kWStages stages
-  uint32_t* bitmap;    // special-token bits of this CTA's slice
+  uint32_t* bitmap;    // one bit per 16-byte unit of this CTA's slice that holds a special token
   float* segsum;       // per-segment residual sums
   float* chksum;       // per-chunk (32 segments) residual sums
   float* segref;       // bonus draw: each segment sum's reference (round(max * c))
@@ -746,37 +746,51 @@ struct Kernel {
       }
       const int t0 = tok0 + gu * VE;
       (void)t0;
+      float mu0 = v0[0];
+#pragma unroll
+      for (int e = 1; e < VE; ++e) mu0 = fmaxf(mu0, v0[e]);
       uint32_t aside = 0u;
       if constexpr (CAND) {
+        if (mu0 > theta) {   // only then can a token of the unit pass
 #pragma unroll
-        for (int e = 0; e < VE; ++e)
-          if (t0 + e < p.V && v0[e] > theta) aside |= 1u << e;
+          for (int e = 0; e < VE; ++e)
+            if (t0 + e < p.V && v0[e] > theta) aside |= 1u << e;
+        }
       }
       // sums of the tokens not set aside (one rescale per unit and row)
 #pragma unroll
       for (int r = 0; r < R; ++r) {
         float v[VE];
+        float mu = mu0;
         if (r == 0) {
 #pragma unroll
           for (int e = 0; e < VE; ++e) v[e] = v0[e];
-        } else if (valid) {
-          L(r0 + r, v);
         } else {
+          if (valid) {
+            L(r0 + r, v);
+          } else {
 #pragma unroll
-          for (int e = 0; e < VE; ++e) v[e] = kNegInf;
+            for (int e = 0; e < VE; ++e) v[e] = kNegInf;
+          }
+          mu = v[0];
+#pragma unroll
+          for (int e = 1; e < VE; ++e) mu = fmaxf(mu, v[e]);
         }
-        float mu = v[0];
-#pragma unroll
-        for (int e = 1; e < VE; ++e) mu = fmaxf(mu, v[e]);
         if (mu > m[r]) {
           sc[r] = (m[r] == kNegInf) ? 0.f : __fmul_rn(sc[r], ex2(__fsub_rn(__fmul_rn(m[r], cr[r]), __fmul_rn(mu, cr[r]))));
           m[r] = mu;
         }
         if (m[r] > kNegInf) {   // exp of -inf is 0; only -inf - -inf must be avoided
+          const float mc = __fmul_rn(m[r], cr[r]);
+          if (!aside) {
 #pragma unroll
-          for (int e = 0; e < VE; ++e) {
-            const float t = ex2(__fmaf_rn(v[e], cr[r], -__fmul_rn(m[r], cr[r])));
-            sc[r] = __fadd_rn(sc[r], ((aside >> e) & 1u) ? 0.f : t);
+            for (int e = 0; e < VE; ++e) sc[r] = __fadd_rn(sc[r], ex2(__fmaf_rn(v[e], cr[r], -mc)));
+          } else {
+#pragma unroll
+            for (int e = 0; e < VE; ++e) {
+              const float t = ex2(__fmaf_rn(v[e], cr[r], -mc));
+              sc[r] = __fadd_rn(sc[r], ((aside >> e) & 1u) ? 0.f : t);
+            }
           }
         }
       }
@@ -1741,11 +1755,9 @@ struct Kernel {
           if (r == rb) bb[e] = pr;
         }
       }
-      const uint32_t bits = (bitmap[(uu * VE) >> 5] >> ((uu * VE) & 31)) & ((1u << VE) - 1u);
-      if (bits) {
+      if ((bitmap[uu >> 5] >> (uu & 31)) & 1u) {   // the unit holds a special token
 #pragma unroll
-        for (int e = 0; e < VE; ++e)
-          if (bits >> e & 1u) a[e] = special_lookup(tbase + e, a[e]);
+        for (int e = 0; e < VE; ++e) a[e] = special_lookup(tbase + e, a[e]);
       }
 #pragma unroll
       for (int e = 0; e < VE; ++e) {
@@ -1858,7 +1870,7 @@ struct Kernel {
     __syncthreads();
     if (threadIdx.x < s) {
       const int loc = S.om[threadIdx.x] - tok0;
-      if (loc >= 0 && loc < p.slice) atomicOr(&bitmap[loc >> 5], 1u << (loc & 31));
+      if (loc >= 0 && loc < p.slice) atomicOr(&bitmap[(loc / VE) >> 5], 1u << ((loc / VE) & 31));
     }
     __syncthreads();
     return S.Y;
@@ -1973,7 +1985,7 @@ struct Kernel {
     __syncthreads();
     for (int i = threadIdx.x; i < S.nspec; i += kThreads) {
       const int loc = S.spec_id[i] - tok0;
-      if (loc >= 0 && loc < p.slice) atomicOr(&bitmap[loc >> 5], 1u << (loc & 31));
+      if (loc >= 0 && loc < p.slice) atomicOr(&bitmap[(loc / VE) >> 5], 1u << ((loc / VE) & 31));
     }
     __syncthreads();
   }
@@ -2428,11 +2440,9 @@ struct Kernel {
 #pragma unroll
       for (int e = 0; e < VE; ++e) a[e] = __fmaf_rn(g, prob_of(v[e], S.M[rr], S.c[rr], S.invZ[rr]), a[e]);
     }
-    const uint32_t bits = (bitmap[(gu * VE) >> 5] >> ((gu * VE) & 31)) & ((1u << VE) - 1u);
-    if (bits) {
+    if ((bitmap[gu >> 5] >> (gu & 31)) & 1u) {   // the unit holds a special token
 #pragma unroll
-      for (int e = 0; e < VE; ++e)
-        if (bits >> e & 1u) a[e] = special_lookup(tbase + e, a[e]);
+      for (int e = 0; e < VE; ++e) a[e] = special_lookup(tbase + e, a[e]);
     }
 #pragma unroll
     for (int e = 0; e < VE; ++e) r[e] = fmaxf(0.f, __fsub_rn(q[e], a[e]));
@@ -2573,7 +2583,7 @@ __global__ void __launch_bounds__(kThreads, SCHEME == MDS_IS ? 1 : 2) verify_ker
   k.nseg = (p.slice / Kernel<DT, SCHEME>::VE + 31) / 32;   // same in every CTA: peers map the same offsets
   k.nsegv = (k.Uv + 31) / 32;                                // segments the residual pass writes
   k.Uw = ((k.Uv + kWarps - 1) / kWarps + 31) & ~31;           // units per warp in a streaming pass
-  k.bm_words = (p.slice + 31) / 32;
+  k.bm_words = (p.slice / Kernel<DT, SCHEME>::VE + 31) / 32;   // one bit per 16-byte unit
   // dynamic shared memory: ring | segment sums | chunk sums | segment references | scheme region
   //   IS : nodes t_n | weights W_r(n)
   //   WIS: CTA list (two copies) | warp lists = staging list | merged list, the
@@ -2650,7 +2660,7 @@ size_t smem_bytes(const Params& p) {
   size_t bytes = (size_t)p.ring_bytes + (size_t)((nseg + 3) & ~3) * 4 * 2 + (size_t)((((nseg + 31) / 32) + 3) & ~3) * 4;
   if (p.scheme == MDS_IS) bytes += (size_t)kIsNodesMax * 4 * (1 + p.rows_max);
   if (p.scheme == MDS_WIS) {
-    const size_t bm = (size_t)((p.slice + 31) / 32) * 4;
+    const size_t bm = (size_t)((p.slice / VE + 31) / 32) * 4;
     const size_t cm = (size_t)p.cand_cap * 4 * (3 + p.rows_max);
     size_t stg = (size_t)p.cand_stage * 4 * (2 + p.rows_max);
     const size_t app = (size_t)kWarps * kWarpApp * 4 * (1 + p.rows_max);
