@@ -679,27 +679,30 @@ struct Kernel {
       ps[r] = 0.f;
     }
     // The filter's starting threshold: the kListN-th largest of the threads'
-    // target maxima over a sample of the CTA's slice (every kSampleStride-th
-    // 16-byte unit, plain loads).  Those maxima are kThreads distinct
+    // target maxima over a sample of the CTA's slice (one 128-byte line in
+    // kSampleStride, plain loads).  Those maxima are kThreads distinct
     // tokens, so the threshold is at most the CTA's kListN-th largest target
     // logit: every token at or below it can be in no list.
     float theta = kNegInf;              // warp-uniform
     if constexpr (CAND) {
       float mx = kNegInf;
       constexpr int kBatch = 16;        // loads in flight per thread
-      for (int u0 = threadIdx.x * kSampleStride; u0 < Uv; u0 += kThreads * kBatch * kSampleStride) {
+      // sample: 8 consecutive units (one 128-byte line) out of every
+      // 8 * kSampleStride, so the sample touches only its own lines
+      auto sample_unit = [&](int i) { return (i >> 3) * (8 * kSampleStride) + (i & 7); };
+      for (int i0 = threadIdx.x * 8; sample_unit(i0) < Uv; i0 += kThreads * kBatch) {
         if (p.tma_ok) {
           // whole, 16-byte aligned units: raw loads first, then the maxima
           uint4 raw[kBatch];
 #pragma unroll
           for (int b = 0; b < kBatch; ++b) {
-            const int u = u0 + b * kThreads * kSampleStride;
+            const int u = sample_unit(i0 + (b & 7) + (b >> 3) * kThreads * 8);
             raw[b] = (u < Uv) ? __ldg(reinterpret_cast<const uint4*>(S.gptr[r0] + ((size_t)tok0 + (size_t)u * VE) * p.esize))
                               : make_uint4(0u, 0u, 0u, 0u);   // skipped below
           }
 #pragma unroll
           for (int b = 0; b < kBatch; ++b) {
-            if (u0 + b * kThreads * kSampleStride >= Uv) continue;
+            if (sample_unit(i0 + (b & 7) + (b >> 3) * kThreads * 8) >= Uv) continue;
             float v[VE];
             E::unpack(raw[b], v);
 #pragma unroll
@@ -707,8 +710,8 @@ struct Kernel {
           }
         } else {
           for (int b = 0; b < kBatch; ++b) {
-            const int u = u0 + b * kThreads * kSampleStride;
-            if (u >= Uv) break;
+            const int u = sample_unit(i0 + (b & 7) + (b >> 3) * kThreads * 8);
+            if (u >= Uv) continue;
             float v[VE];
             GlobalLoad<DT>{S.gptr, tok0, p.V, u, false}(r0, v);
 #pragma unroll
