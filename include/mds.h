@@ -123,10 +123,14 @@ int mds_verify(mds_ctx* ctx, const void* target_logits, const void* const* draft
                int scheme, uint64_t philox_seed, int32_t* out_tokens, int32_t* out_accept_len,
                float* out_diag, int B, void* stream);
 
-/* Same as mds_verify with every buffer in HOST memory (pinned memory gives
- * the fastest copies).  The context stages the inputs into device buffers it
- * owns (allocated on first use, grown as needed), runs the verification and
- * copies the outputs back, all on `stream`, and synchronises the stream
+/* Same as mds_verify with every buffer in HOST memory.  When the target and
+ * every draft logits buffer are page-locked host memory mapped into the
+ * device's address space (cudaHostAlloc / cudaHostRegister with mapping,
+ * e.g. torch pin_memory()), the kernel reads the logits in place with plain
+ * loads, so only the rows the walk visits cross the host link; otherwise the
+ * context first copies them into device buffers it owns (allocated on first
+ * use, grown as needed).  Tokens and temperatures are always staged, and the
+ * outputs copied back, all on `stream`; the call synchronises the stream
  * before returning. */
 int mds_verify_host(mds_ctx* ctx, const void* target_logits, const void* const* draft_logits,
                     const int32_t* draft_model_id, const int32_t* draft_tokens, const float* temperatures,

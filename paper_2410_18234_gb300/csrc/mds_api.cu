@@ -131,6 +131,17 @@ int clusters_for(mds_ctx* ctx, const mds::Params& p) {
 
 bool aligned(const void* ptr, size_t a) { return ((uintptr_t)ptr % a) == 0; }
 
+// Page-locked host memory mapped into the device's address space: the
+// pointer the device reads it through; null for any other memory.
+const void* mapped_host(const void* h) {
+  cudaPointerAttributes a{};
+  if (cudaPointerGetAttributes(&a, h) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  return (a.type == cudaMemoryTypeHost) ? a.devicePointer : nullptr;
+}
+
 }  // namespace
 
 extern "C" {
@@ -182,10 +193,12 @@ int mds_create(mds_ctx** out, const mds_config* cfg, int device) {
   return MDS_OK;
 }
 
-int mds_verify(mds_ctx* ctx, const void* target_logits, const void* const* draft_logits,
-               const int32_t* draft_model_id, const int32_t* draft_tokens, const float* temperatures,
-               int scheme, uint64_t philox_seed, int32_t* out_tokens, int32_t* out_accept_len,
-               float* out_diag, int B, void* stream) {
+// mds_verify with the choice of reading rows by bulk copies (device memory)
+// or by plain loads only (rows in mapped host memory).
+static int verify_impl(mds_ctx* ctx, const void* target_logits, const void* const* draft_logits,
+                       const int32_t* draft_model_id, const int32_t* draft_tokens, const float* temperatures,
+                       int scheme, uint64_t philox_seed, int32_t* out_tokens, int32_t* out_accept_len,
+                       float* out_diag, int B, void* stream, bool bulk_ok) {
   if (!ctx) return MDS_EINVAL;
   const mds_config& c = ctx->cfg;
   if (scheme < MDS_SINGLE || scheme > MDS_SPECTR) return MDS_EINVAL;
@@ -233,6 +246,7 @@ int mds_verify(mds_ctx* ctx, const void* target_logits, const void* const* draft
   p.is_h = c.is_h;
   p.n_models = n_models;
   p.tma_ok = tma_ok ? 1 : 0;
+  p.bulk_ok = bulk_ok ? 1 : 0;
   DeviceGuard g(ctx->device);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   int clusters = clusters_for(ctx, p);
@@ -246,6 +260,14 @@ int mds_verify(mds_ctx* ctx, const void* target_logits, const void* const* draft
   ctx->tickets += (unsigned)(B + clusters);
   ctx->last_cn = p.cn;
   return MDS_OK;
+}
+
+int mds_verify(mds_ctx* ctx, const void* target_logits, const void* const* draft_logits,
+               const int32_t* draft_model_id, const int32_t* draft_tokens, const float* temperatures,
+               int scheme, uint64_t philox_seed, int32_t* out_tokens, int32_t* out_accept_len,
+               float* out_diag, int B, void* stream) {
+  return verify_impl(ctx, target_logits, draft_logits, draft_model_id, draft_tokens, temperatures, scheme,
+                     philox_seed, out_tokens, out_accept_len, out_diag, B, stream, true);
 }
 
 int mds_verify_host(mds_ctx* ctx, const void* target_logits, const void* const* draft_logits,
@@ -262,8 +284,18 @@ int mds_verify_host(mds_ctx* ctx, const void* target_logits, const void* const* 
   for (int k = 0; k < c.K; ++k)
     if (!draft_logits[k]) return MDS_EINVAL;
   const size_t es = (size_t)esize_of(c.dtype);
-  const size_t n_tgt = round_up((size_t)B * c.K * (c.L + 1) * c.V * es, 256);
-  const size_t n_drf = round_up((size_t)B * c.L * c.V * es, 256);
+  DeviceGuard g0(ctx->device);
+  // Logits in mapped page-locked host memory are read in place: only the
+  // rows the walk visits cross the host link (plain loads, no bulk copies).
+  const void* z_tgt = mapped_host(target_logits);
+  const void* z_drf[MDS_MAX_K];
+  bool zero_copy = z_tgt != nullptr;
+  for (int k = 0; k < c.K; ++k) {
+    z_drf[k] = zero_copy ? mapped_host(draft_logits[k]) : nullptr;
+    zero_copy = zero_copy && z_drf[k] != nullptr;
+  }
+  const size_t n_tgt = zero_copy ? 0 : round_up((size_t)B * c.K * (c.L + 1) * c.V * es, 256);
+  const size_t n_drf = zero_copy ? 0 : round_up((size_t)B * c.L * c.V * es, 256);
   const size_t n_tok = round_up((size_t)B * c.K * c.L * 4, 256);
   const size_t n_tmp = round_up((size_t)B * (1 + c.K) * 4, 256);
   const size_t n_out = round_up((size_t)B * (c.L + 1) * 4, 256);
@@ -291,12 +323,19 @@ int mds_verify_host(mds_ctx* ctx, const void* target_logits, const void* const* 
   char* d_dg = d_acc + n_acc;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const void* dptr[MDS_MAX_K];
-  bool ok = cudaMemcpyAsync(d_tgt, target_logits, (size_t)B * c.K * (c.L + 1) * c.V * es, cudaMemcpyHostToDevice,
-                            st) == cudaSuccess;
-  for (int k = 0; k < c.K && ok; ++k) {
-    dptr[k] = d_drf + k * n_drf;
-    ok = cudaMemcpyAsync(d_drf + k * n_drf, draft_logits[k], (size_t)B * c.L * c.V * es, cudaMemcpyHostToDevice,
+  const void* tptr = z_tgt;
+  bool ok = true;
+  if (zero_copy) {
+    for (int k = 0; k < c.K; ++k) dptr[k] = z_drf[k];
+  } else {
+    tptr = d_tgt;
+    ok = cudaMemcpyAsync(d_tgt, target_logits, (size_t)B * c.K * (c.L + 1) * c.V * es, cudaMemcpyHostToDevice,
                          st) == cudaSuccess;
+    for (int k = 0; k < c.K && ok; ++k) {
+      dptr[k] = d_drf + k * n_drf;
+      ok = cudaMemcpyAsync(d_drf + k * n_drf, draft_logits[k], (size_t)B * c.L * c.V * es, cudaMemcpyHostToDevice,
+                           st) == cudaSuccess;
+    }
   }
   ok = ok && cudaMemcpyAsync(d_tok, draft_tokens, (size_t)B * c.K * c.L * 4, cudaMemcpyHostToDevice, st) == cudaSuccess;
   ok = ok && cudaMemcpyAsync(d_tmp, temperatures, (size_t)B * (1 + c.K) * 4, cudaMemcpyHostToDevice, st) == cudaSuccess;
@@ -304,9 +343,10 @@ int mds_verify_host(mds_ctx* ctx, const void* target_logits, const void* const* 
     cudaGetLastError();
     return MDS_ECUDA;
   }
-  int rc = mds_verify(ctx, d_tgt, dptr, draft_model_id, reinterpret_cast<const int32_t*>(d_tok),
-                      reinterpret_cast<const float*>(d_tmp), scheme, philox_seed, reinterpret_cast<int32_t*>(d_out),
-                      reinterpret_cast<int32_t*>(d_acc), out_diag ? reinterpret_cast<float*>(d_dg) : nullptr, B, stream);
+  int rc = verify_impl(ctx, tptr, dptr, draft_model_id, reinterpret_cast<const int32_t*>(d_tok),
+                       reinterpret_cast<const float*>(d_tmp), scheme, philox_seed, reinterpret_cast<int32_t*>(d_out),
+                       reinterpret_cast<int32_t*>(d_acc), out_diag ? reinterpret_cast<float*>(d_dg) : nullptr, B,
+                       stream, !zero_copy);
   if (rc != MDS_OK) {
     cudaStreamSynchronize(st);
     return rc;

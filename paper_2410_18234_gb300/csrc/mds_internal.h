@@ -41,6 +41,7 @@ struct Params {
   int rows_max;                        // rows per depth at most (1 + distinct models)
   int n_models;                        // distinct draft models (ids are 0..n_models-1 after remap)
   int tma_ok;                          // rows are 16-byte aligned with 16-byte-multiple length
+  int bulk_ok;                         // rows may be read with bulk copies (device memory, not mapped host memory)
   int cand_cap;                        // WIS candidate list capacity (kListN; 0: no candidate path)
   int cand_stage;                      // WIS staging capacity (every CTA's list: cn * kListN)
   int8_t model_of[MDS_MAX_K];          // remapped model id per branch

@@ -478,8 +478,9 @@ struct Kernel {
   // unit gu of row r.  With 16-byte aligned rows the rows of `mask` flow
   // through the warp's own ring of kWStages stages (cp.async.bulk issued by
   // lane 0 up to kWStages stages ahead, completion counted on the stage's
-  // mbarrier); otherwise, or when a stage could not hold a group of every
-  // row, units are loaded straight from global memory.  No block barrier is
+  // mbarrier); otherwise (rows not 16-byte aligned, rows in mapped host
+  // memory, or a stage too small for a group of every row), units are loaded
+  // straight from global memory.  No block barrier is
   // taken inside a pass, nor at its end: a caller synchronises the block
   // before reading what other warps wrote.  Every wait is bounded.
   __device__ __forceinline__ int stage_units(int nrm) const {
@@ -509,7 +510,7 @@ struct Kernel {
     if (u0 >= u1) return;
     const int nrm = __popc(mask);
     const int su = stage_units(nrm);
-    if (!p.tma_ok || su < 32) {
+    if (!p.tma_ok || !p.bulk_ok || su < 32) {
       for (int g = u0; g < u1; g += 32) {
         const int gu = g + lane;
         fn(gu, gu < u1, GlobalLoad<DT>{S.gptr, tok0, p.V, gu, p.tma_ok != 0});

@@ -109,6 +109,7 @@ extern "C" int mds_verify_noalloc(const mds_config* cfg_in, int device, const vo
     p.V = c.V;
     p.wis_s = c.wis_s;
     p.is_h = c.is_h;
+    p.bulk_ok = 1;
     p.n_models = n_models;
     p.tma_ok = tma_ok ? 1 : 0;
     int clusters = mds::max_active_clusters(p);

@@ -179,3 +179,28 @@ def test_repeated_launches_are_identical(cluster):
         t.verify(other.target, other.draft_list(), other.model_ids, other.tokens, other.temps, "WIS", rep)
         torch.cuda.synchronize()
         t.close()
+
+
+def test_host_entry_point_reads_pinned_logits_in_place():
+    # mds_verify_host: pinned logits are read in place (plain loads over the
+    # host link), pageable ones are copied first; both must give exactly the
+    # device entry point's result
+    spec = small("two-models-50k", B=8, V=6000)
+    w = make_workload(spec, device=DEV)
+    v = mds.Verifier(spec.B, spec.K, spec.L, spec.V, dtype=spec.dtype)
+    out, acc, diag = v.verify(w.target, w.draft_list(), w.model_ids, w.tokens, w.temps, "WIS", 3, diag=True)
+    torch.cuda.synchronize()
+    ref = (out.cpu().numpy(), acc.cpu().numpy())
+    for pinned in (True, False):
+        def host(t):
+            t = t.cpu()
+            return t.pin_memory() if pinned else t
+        h_out = torch.empty(spec.B, spec.L + 1, dtype=torch.int32)
+        h_acc = torch.empty(spec.B, dtype=torch.int32)
+        h_out, h_acc = (h_out.pin_memory(), h_acc.pin_memory()) if pinned else (h_out, h_acc)
+        mds.mds_verify_host(v.ctx, host(w.target), [host(d) for d in w.draft_list()], w.model_ids, host(w.tokens),
+                            host(w.temps), "WIS", 3, h_out, h_acc)
+        assert np.array_equal(h_out.numpy(), ref[0]), f"pinned={pinned}"
+        assert np.array_equal(h_acc.numpy(), ref[1]), f"pinned={pinned}"
+    assert v.status()[0] == 0
+    v.close()
