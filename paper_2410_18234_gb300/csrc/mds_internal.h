@@ -37,10 +37,10 @@ struct Params {
   float is_h;
   int cn;                              // CTAs per cluster
   int slice;                           // tokens per CTA (multiple of 8)
-  int ring_bytes;                      // streaming ring (kStages stages)
+  int ring_bytes;                      // streaming rings of all warps (each warp: 5 stages)
   int rows_max;                        // rows per depth at most (1 + distinct models)
   int n_models;                        // distinct draft models (ids are 0..n_models-1 after remap)
-  int tma_ok;                          // rows are 16-byte aligned with 16-byte-multiple length
+  int tma_ok;                          // rows are 16-byte aligned with a 16-byte-multiple length
   int bulk_ok;                         // rows may be read with bulk copies (device memory, not mapped host memory)
   int cand_cap;                        // WIS candidate list capacity (kListN; 0: no candidate path)
   int cand_stage;                      // WIS staging capacity (every CTA's list: cn * kListN)
@@ -60,7 +60,7 @@ int max_active_clusters(const Params& p);
 // Launch the persistent verification kernel with `clusters` clusters.
 cudaError_t launch(const Params& p, int clusters, cudaStream_t stream);
 
-// Launch geometry (cluster size, slice, row stride, list capacities) that
+// Launch geometry (cluster size, slice, ring and list capacities) that
 // mds_verify would use for this configuration; MDS_OK or MDS_EVOCAB.
 int launch_geometry(const mds_config& cfg, int device, int scheme, int n_models, Params& p);
 

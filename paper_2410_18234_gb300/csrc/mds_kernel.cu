@@ -233,15 +233,14 @@ struct State {
   int model_row[MDS_MAX_K];   // row index of each (remapped) draft model, -1 if not loaded
   const char* gptr[kMaxRows];
   float M[kMaxRows], c[kMaxRows], invZ[kMaxRows];
-  int tma_bytes;
   // walk
   int nv;                     // valid branches
   int vbr[MDS_MAX_K];         // valid branch ids, ascending
   int X[MDS_MAX_K];           // their tokens at this depth
   int vrow[MDS_MAX_K];        // row of each valid branch's draft model
   // outcome of the depth
-  int Y, Z, accepted, flags;
-  float qY, pIY, R;
+  int Y, accepted;
+  float qY, pIY;
   int next_b;
   int Zslot;
   int tok_j[32];
@@ -262,10 +261,9 @@ struct State {
   float spec_val[kMaxSpecial];
   int om[MDS_MAX_S];
   float om_x[MDS_MAX_S], om_q[MDS_MAX_S], om_a[MDS_MAX_S], om_b[MDS_MAX_S];
-  float lp_rs[kMaxPairs], lp_fl[kMaxPairs], lp_fh[kMaxPairs], lp_m[kMaxPairs];
+  float lp_rs[kMaxPairs], lp_fl[kMaxPairs], lp_fh[kMaxPairs];
   float A2, B2;
   // WIS candidate list bookkeeping
-  int wcnt[kWarps];
   float pc[kMaxRows];        // complement exp mass per row
   int ncand, cand_all, fast_ok;
   float cand_q;
@@ -275,10 +273,9 @@ struct State {
   // IS: quadrature grid
   int is_mlo, is_n;
   int is_cnt[kMaxRows];
-  float rho_min, rho_max;
   // CDF search
   int owner, seg;
-  float run, T;
+  float run;
   // streaming: one ring per warp, one mbarrier per stage
   uint64_t wbar[kWarps][kWStages];
   int wapp[kWarps];          // tokens each warp set aside (may exceed kWarpApp: overflow)
@@ -2067,8 +2064,6 @@ struct Kernel {
       if (mhi - mlo + 1 > kIsNodesMax) mhi = mlo + kIsNodesMax - 1;
       S.is_mlo = mlo;
       S.is_n = mhi - mlo + 1;
-      S.rho_min = rlo;
-      S.rho_max = rhi;
     }
     __syncthreads();
     const int nn = S.is_n;
@@ -2299,8 +2294,6 @@ struct Kernel {
         }
         S.c[0] = __fdiv_rn(kLog2e, tq);
         S.nrows = nr;
-        S.flags = 0;
-        S.R = 0.f;
       }
       __syncthreads();
       if (!bonus) depth_stats(SCHEME == MDS_WIS && S.nv > 1);
