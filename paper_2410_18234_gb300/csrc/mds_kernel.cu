@@ -458,7 +458,7 @@ struct Kernel {
   float* cm_e;         //      ... exp values per row [rows][cap]
   float* cm_a;         //      ... current law value of special tokens
   int* cm_sp;          //      ... special flag
-  int rank, cn, tok0, nvalid, Uv, Uw, nseg, nsegv, bm_words;   // nseg: layout (slice); nsegv: written (valid units)
+  int rank, cn, tok0, nvalid, Uv, nseg, nsegv, bm_words;   // nseg: layout (slice); nsegv: written (valid units)
   int xbuf;
   int clbuf;           // which copy of the CTA list the next candidate pass publishes
   uint32_t wphase;     // parity of each stage of this warp's ring
@@ -468,8 +468,9 @@ struct Kernel {
   }
 
   // ---------------------------------------------------------------- streaming engine
-  // Warp w owns units [w*Uw, min((w+1)*Uw, Uv)) of the CTA's slice (Uw a
-  // multiple of 32) and walks them in groups of 32, one unit per lane:
+  // The CTA's slice is cut into chunks of su units (a multiple of 32, one
+  // ring stage) taken round-robin by the warps (warp w: chunks w, w + kWarps,
+  // ...), each walked in groups of 32, one unit per lane:
   // fn(gu, valid, L) is called by all 32 lanes together, gu the unit's index
   // in the slice (a group starts at a multiple of 32) and L(r, v) loading
   // unit gu of row r.  With 16-byte aligned rows the rows of `mask` flow
@@ -484,12 +485,13 @@ struct Kernel {
     return ((p.ring_bytes / kWarps / kWStages) / (16 * nrm)) & ~31;
   }
 
-  __device__ __forceinline__ void issue_stage(int c, uint32_t mask, int su, int u0, int u1) {
+  // Issue this warp's k-th stage: chunk c = warp + k * kWarps of su units.
+  __device__ __forceinline__ void issue_stage(int k, uint32_t mask, int su) {
     const int warp = threadIdx.x >> 5;
-    const int stage = c % kWStages;
+    const int stage = k % kWStages;
     char* dst = ring + (size_t)(warp * kWStages + stage) * (p.ring_bytes / kWarps / kWStages);
-    const int cu0 = u0 + c * su;
-    const int bytes = (min(cu0 + su, u1) - cu0) * 16;
+    const int cu0 = (warp + k * kWarps) * su;
+    const int bytes = (min(cu0 + su, Uv) - cu0) * 16;
     mbar_expect_tx(&S.wbar[warp][stage], (uint32_t)(bytes * __popc(mask)));
     int pos = 0;
     for (int r = 0; r < S.nrows; ++r) {
@@ -503,25 +505,25 @@ struct Kernel {
   template <class FN>
   __device__ void stream(uint32_t mask, FN&& fn) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int u0 = warp * Uw, u1 = min(u0 + Uw, Uv);
-    if (u0 >= u1) return;
     const int nrm = __popc(mask);
     const int su = stage_units(nrm);
     if (!p.tma_ok || !p.bulk_ok || su < 32) {
-      for (int g = u0; g < u1; g += 32) {
+      for (int g = warp * 32; g < Uv; g += kWarps * 32) {
         const int gu = g + lane;
-        fn(gu, gu < u1, GlobalLoad<DT>{S.gptr, tok0, p.V, gu, p.tma_ok != 0});
+        fn(gu, gu < Uv, GlobalLoad<DT>{S.gptr, tok0, p.V, gu, p.tma_ok != 0});
       }
       return;
     }
-    const int nch = (u1 - u0 + su - 1) / su;
+    const int nchunk = (Uv + su - 1) / su;
+    const int nk = (nchunk - warp + kWarps - 1) / kWarps;   // this warp's chunks: warp, warp + kWarps, ...
+    if (nk <= 0) return;
     if (lane == 0) {
       fence_proxy_async();
-      for (int c = 0; c < nch && c < kWStages; ++c) issue_stage(c, mask, su, u0, u1);
+      for (int k = 0; k < nk && k < kWStages; ++k) issue_stage(k, mask, su);
     }
     __syncwarp();
-    for (int c = 0; c < nch; ++c) {
-      const int stage = c % kWStages;
+    for (int k = 0; k < nk; ++k) {
+      const int stage = k % kWStages;
       const char* base = ring + (size_t)(warp * kWStages + stage) * (p.ring_bytes / kWarps / kWStages);
       long long spins = 0;
       while (!mbar_try_wait(&S.wbar[warp][stage], (wphase >> stage) & 1u)) {
@@ -531,15 +533,15 @@ struct Kernel {
         }
       }
       wphase ^= 1u << stage;
-      const int cu0 = u0 + c * su, cu1 = min(cu0 + su, u1);
+      const int cu0 = (warp + k * kWarps) * su, cu1 = min(cu0 + su, Uv);
       for (int g = cu0; g < cu1; g += 32) {
         const int gu = g + lane;
         fn(gu, gu < cu1, StageLoad<DT>{base, mask, su * 16, g - cu0 + lane});
       }
       __syncwarp();
-      if (lane == 0 && c + kWStages < nch) {
+      if (lane == 0 && k + kWStages < nk) {
         fence_proxy_async();
-        issue_stage(c + kWStages, mask, su, u0, u1);
+        issue_stage(k + kWStages, mask, su);
       }
       __syncwarp();
     }
@@ -2579,7 +2581,6 @@ __global__ void __launch_bounds__(kThreads, SCHEME == MDS_IS ? 1 : 2) verify_ker
   k.Uv = (k.nvalid + Kernel<DT, SCHEME>::VE - 1) / Kernel<DT, SCHEME>::VE;
   k.nseg = (p.slice / Kernel<DT, SCHEME>::VE + 31) / 32;   // same in every CTA: peers map the same offsets
   k.nsegv = (k.Uv + 31) / 32;                                // segments the residual pass writes
-  k.Uw = ((k.Uv + kWarps - 1) / kWarps + 31) & ~31;           // units per warp in a streaming pass
   k.bm_words = (p.slice / Kernel<DT, SCHEME>::VE + 31) / 32;   // one bit per 16-byte unit
   // dynamic shared memory: ring | segment sums | chunk sums | segment references | scheme region
   //   IS : nodes t_n | weights W_r(n)
