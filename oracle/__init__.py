@@ -19,6 +19,8 @@ theory   brute-force linear programs and closed forms used as pins
          the truncation bound of Section 4).
 enum     exhaustive enumeration of selection rules over Omega^K (tiny
          vocabularies), used to pin the induced distribution p_I.
+truncated  the truncated-alphabet scheme (Section 4) and top-k / top-p
+         preprocessing (Section 5), with the enumerated law that pins it.
 
 Parity status: every function here is pinned by a ``-m "not gpu"`` test
 (see tests/test_oracle_*.py) except the SpecTr-style sequential-rejection

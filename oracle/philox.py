@@ -18,6 +18,8 @@ multiple of 2^-24 in [0, 1).  Draw ids:
             sequential-rejection baseline's round i uses 16 + i)
     32      residual resample
     33      bonus token after L accepted positions
+    34      truncated alphabet: keep the token drawn on Omega_0
+    35      truncated alphabet: replacement drawn outside Omega_0
 """
 import numpy as np
 

@@ -37,6 +37,12 @@ WIS      the paper's weighted importance sampling with the variant truncated
          (module ``wis``).
 SpecTr   sequential-rejection baseline (reading: Algorithm 1 applied to the
          valid drafts in turn against the running residual target).
+WIS0     WIS on the truncated alphabet Omega_0 = the ``omega0`` most probable
+         target tokens, followed by the keep / replace step that restores the
+         target (Section 4, "truncated alphabet"; module ``truncated``).
+
+Optional top-k / top-p preprocessing (Section 5) replaces the target and
+draft rows by their filtered, renormalised versions before any scheme runs.
 
 Each depth also records the margins of its discrete decisions; a depth whose
 margin is below the band thresholds is flagged ``band`` (GPU and oracle may
@@ -48,8 +54,9 @@ from . import philox
 from .philox import DRAW_ACCEPT, DRAW_BONUS, DRAW_RESIDUAL, DRAW_SELECT
 from . import wis as wis_mod
 from . import is_laplace
+from . import truncated
 
-SCHEMES = {"single": 0, "IS": 1, "WIS": 2, "SpecTr": 3}
+SCHEMES = {"single": 0, "IS": 1, "WIS": 2, "SpecTr": 3, "WIS0": 4}
 
 # Band thresholds (absolute, on quantities in [0, 1] or scaled as stated).
 BAND_ACCEPT = 1e-6   # |u - min(1, q(Y)/p_I(Y))|
@@ -161,10 +168,16 @@ def _spectr_step(rec, q, dists, X, seed, b, j):
 
 
 def verify_sequence(b, target_logits, draft_logits, draft_model_id, draft_tokens, temperatures,
-                    scheme, seed, wis_s=5, is_h=0.25, draw_id=None):
+                    scheme, seed, wis_s=5, is_h=0.25, draw_id=None, omega0=40, top_k=0, top_p=1.0):
     """Walk the sequence stored at index b of the arrays; its Philox draws use
     sequence id ``draw_id`` (default b).  Returns (tokens [L+1] with -1
     padding, accept_len, list of DepthRecord)."""
+    filt = top_k > 0 or top_p < 1.0
+
+    def dist(logits, temperature, rec):
+        d = softmax_t(logits, temperature)
+        return truncated.top_filter(d, top_k, top_p, rec.note) if filt else d
+
     sid = b if draw_id is None else int(draw_id)
     K = target_logits.shape[1]
     L = draft_tokens.shape[2]
@@ -175,13 +188,13 @@ def verify_sequence(b, target_logits, draft_logits, draft_model_id, draft_tokens
         rec = DepthRecord(j)
         records.append(rec)
         kstar = valid[0]
-        q = softmax_t(target_logits[b, kstar, j], temperatures[b, 0])
+        q = dist(target_logits[b, kstar, j], temperatures[b, 0], rec)
         # one row per distinct draft model, read from its lowest valid branch
         rows = {}
         for k in valid:
             d = int(draft_model_id[k])
             if d not in rows:
-                rows[d] = softmax_t(draft_logits[k][b, j], temperatures[b, 1 + k])
+                rows[d] = dist(draft_logits[k][b, j], temperatures[b, 1 + k], rec)
         X = [int(draft_tokens[b, k, j]) for k in valid]
         dists = [rows[int(draft_model_id[k])] for k in valid]
         if scheme == "single":
@@ -200,6 +213,8 @@ def verify_sequence(b, target_logits, draft_logits, draft_model_id, draft_tokens
                                   philox.uniform(seed, sid, j, DRAW_RESIDUAL))
         elif scheme == "SpecTr":
             Z = _spectr_step(rec, q, dists, X, seed, sid, j)
+        elif scheme == "WIS0":
+            Z = truncated.truncated_step(rec, q, dists, X, seed, sid, j, omega0, wis_s)
         else:
             raise ValueError(f"unknown scheme {scheme!r}")
         rec.Z = int(Z)
@@ -212,7 +227,7 @@ def verify_sequence(b, target_logits, draft_logits, draft_model_id, draft_tokens
     # all L positions accepted: bonus token from the target row at depth L
     rec = DepthRecord(L)
     records.append(rec)
-    q = softmax_t(target_logits[b, valid[0], L], temperatures[b, 0])
+    q = dist(target_logits[b, valid[0], L], temperatures[b, 0], rec)
     z, m = inverse_cdf(q, philox.uniform(seed, sid, L, DRAW_BONUS))
     rec.note("cdf", m, BAND_CDF)
     rec.Z = int(z)
@@ -221,7 +236,7 @@ def verify_sequence(b, target_logits, draft_logits, draft_model_id, draft_tokens
 
 
 def oracle_verify(target_logits, draft_logits, draft_model_id, draft_tokens, temperatures,
-                  scheme, seed, wis_s=5, is_h=0.25, seqs=None, seq_ids=None):
+                  scheme, seed, wis_s=5, is_h=0.25, seqs=None, seq_ids=None, omega0=40, top_k=0, top_p=1.0):
     """Oracle over a batch.
 
     target_logits  [B, K, L+1, V] (any real dtype; upcast exactly to fp64)
@@ -233,6 +248,8 @@ def oracle_verify(target_logits, draft_logits, draft_model_id, draft_tokens, tem
     seq_ids        optional global sequence ids of the B stored sequences (a
                    sample of a larger batch); Philox draws use these ids and
                    the results are keyed by them
+    omega0         |Omega_0| of the truncated-alphabet scheme WIS0
+    top_k, top_p   preprocessing of every row (0 / 1.0: off)
 
     Returns (out_tokens, accept_len, records {id: [DepthRecord]}).  Without
     seq_ids the arrays are [B, L+1] and [B] and rows of sequences not in
@@ -248,12 +265,13 @@ def oracle_verify(target_logits, draft_logits, draft_model_id, draft_tokens, tem
         out_d, acc_d = {}, {}
         for i, sid in enumerate(seq_ids):
             o, a, r = verify_sequence(i, target_logits, draft_logits, draft_model_id, draft_tokens, temps,
-                                      scheme, seed, wis_s, is_h, draw_id=sid)
+                                      scheme, seed, wis_s, is_h, draw_id=sid, omega0=omega0,
+                                      top_k=top_k, top_p=top_p)
             out_d[int(sid)], acc_d[int(sid)], recs[int(sid)] = o, a, r
         return out_d, acc_d, recs
     for b in (range(B) if seqs is None else seqs):
         o, a, r = verify_sequence(b, target_logits, draft_logits, draft_model_id, draft_tokens,
-                                  temps, scheme, seed, wis_s, is_h)
+                                  temps, scheme, seed, wis_s, is_h, omega0=omega0, top_k=top_k, top_p=top_p)
         out[b] = o
         acc[b] = a
         recs[b] = r
