@@ -5,10 +5,15 @@ TEST INFRASTRUCTURE ONLY (see ``oracle/__init__``).  Plain fp64 numpy.
 Truncated alphabet (Section 4, "truncated alphabet" scheme; the non-iid
 appendix's closing remark on applying it to distinct drafts)
 ------------------------------------------------------------------------
-Omega_0 is a high-probability subset of the vocabulary under the target q:
-here the M tokens with the largest q (ties: lower token id first; with one
-temperature per row this is the same order as the target logits).  With
-p_a = q(Omega_0) and the renormalised target q~ = q 1[Omega_0] / p_a:
+Omega_0 is a high-probability subset of the vocabulary under the target q.
+Reading of "a subset of size M": the tokens whose probability is strictly
+above the (M+1)-th largest probability (counted with multiplicity), so at
+most M tokens; tokens tied at the cut are all left out, which makes Omega_0
+a function of the distribution alone, not of the token numbering.  With one
+temperature per row this is the same as comparing target logits.  If
+M >= V, Omega_0 is the whole vocabulary.  The scheme below returns target
+tokens for any choice of Omega_0; the choice only moves the acceptance
+rate.  With p_a = q(Omega_0) and q~ = q 1[Omega_0] / p_a:
 
 1. The multi-draft scheme is run on the alphabet Omega_0 with target q~ and
    produces Y' ~ q~.  Reading of the two passages together: only the input
@@ -27,7 +32,8 @@ p_a = q(Omega_0) and the renormalised target q~ = q 1[Omega_0] / p_a:
    from Omega \\ Omega_0 in proportion to q (draw 35, inverse CDF in token-id
    order).  Then Pr(Z = x) = p_a q~(x) = q(x) on Omega_0 and
    (1 - p_a) q(x) / (1 - p_a) = q(x) outside it.
-If Omega \\ Omega_0 carries no target mass (M >= V), Y' is always kept.
+If Omega \\ Omega_0 carries no target mass (M >= V), Y' is always kept; if
+Omega_0 is empty (ties at the top), the output is drawn from q (draw 35).
 
 Top-k / top-p preprocessing (Section 5: top-p with p = 0.95 on both models;
 top-k with k = 5 or 10 on both models)
@@ -80,9 +86,13 @@ def top_filter(dist, top_k=0, top_p=1.0, note=None):
 
 
 def omega0(q, M):
-    """Omega_0: the M most probable target tokens, ties to the lower id;
-    returned in increasing token-id order."""
-    return np.sort(top_order(q)[:min(int(M), len(q))])
+    """Omega_0: the tokens with probability above the (M+1)-th largest one
+    (every token if M >= V), in increasing token-id order."""
+    q = np.asarray(q, dtype=np.float64)
+    if int(M) >= len(q):
+        return np.arange(len(q))
+    cut = np.sort(q)[::-1][int(M)]
+    return np.flatnonzero(q > cut)
 
 
 def truncate(dist, om):
@@ -101,6 +111,12 @@ def truncated_step(rec, q, dists, X, seed, sid, j, M, s):
     (Y, q~(Y), p_I(Y), ratio in Omega_0 terms, Y as a vocabulary id)."""
     from .verify import BAND_CDF, _speculative_step, inverse_cdf
     om = omega0(q, M)
+    rest = np.asarray(q, dtype=np.float64).copy()
+    rest[om] = 0.0
+    if len(om) == 0:
+        z, m = inverse_cdf(rest, philox.uniform(seed, sid, j, DRAW_OUTSIDE))
+        rec.note("cdf", m, BAND_CDF)
+        return int(z)
     where = {int(t): i for i, t in enumerate(om)}
     pa = float(q[om].sum())
     qt = q[om] / pa
@@ -120,8 +136,6 @@ def truncated_step(rec, q, dists, X, seed, sid, j, M, s):
         y = _speculative_step(rec, qt, pI, Y, philox.uniform(seed, sid, j, philox.DRAW_ACCEPT),
                               philox.uniform(seed, sid, j, philox.DRAW_RESIDUAL))
         rec.Y = int(om[Y])
-    rest = np.asarray(q, dtype=np.float64).copy()
-    rest[om] = 0.0
     if rest.sum() <= 0.0:
         return int(om[y])
     u_keep = philox.uniform(seed, sid, j, DRAW_KEEP)
@@ -143,6 +157,8 @@ def output_law(q, dists, M, s):
     q = np.asarray(q, dtype=np.float64)
     V = len(q)
     om = omega0(q, M)
+    if len(om) == 0:
+        return q.copy()
     where = {int(t): i for i, t in enumerate(om)}
     pa = float(q[om].sum())
     qt = q[om] / pa

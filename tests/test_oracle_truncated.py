@@ -57,13 +57,38 @@ def test_output_law_with_sparse_rows():
     np.testing.assert_allclose(truncated.output_law(q3, [p, p, off], 3, 2), q3, atol=1e-12)
 
 
-def test_omega0_order_and_ties():
+def test_omega0_cut_and_ties():
+    """At most M tokens, all strictly above the (M+1)-th largest probability;
+    tokens tied at the cut are left out together."""
     q = np.array([0.1, 0.3, 0.1, 0.3, 0.2])
-    assert truncated.omega0(q, 1).tolist() == [1]
+    assert truncated.omega0(q, 1).tolist() == []          # 0.3 twice: tied at the cut
     assert truncated.omega0(q, 2).tolist() == [1, 3]
     assert truncated.omega0(q, 3).tolist() == [1, 3, 4]
-    assert truncated.omega0(q, 4).tolist() == [0, 1, 3, 4]
+    assert truncated.omega0(q, 4).tolist() == [1, 3, 4]   # 0.1 twice: tied at the cut
+    assert truncated.omega0(q, 5).tolist() == [0, 1, 2, 3, 4]
     assert truncated.omega0(q, 9).tolist() == [0, 1, 2, 3, 4]
+    for _ in range(30):
+        d = np.round(_dir(12, 0.5), 2)
+        M = int(RNG.integers(0, 13))
+        om = truncated.omega0(d, M)
+        assert len(om) <= M
+        inside = np.zeros(12, dtype=bool)
+        inside[om] = True
+        if inside.any() and (~inside).any():
+            assert d[inside].min() > d[~inside].max()
+        # the cut is the (M+1)-th largest value: one more token would need a tie break
+        if M < 12:
+            assert np.sum(d >= np.sort(d)[::-1][M]) >= M + 1
+
+
+def test_empty_omega0_samples_the_target():
+    """All tokens tied: Omega_0 is empty and the output is drawn from q."""
+    q = np.full(4, 0.25)
+    p = _dir(4)
+    np.testing.assert_allclose(truncated.output_law(q, [p, p], 2, 2), q, atol=1e-15)
+    rec = DepthRecord(0)
+    z = truncated.truncated_step(rec, q, [p, p], [0, 1], 3, 0, 0, 2, 2)
+    assert 0 <= z < 4
 
 
 def _sample_z(q, dists, X, M, s, n, seed):
