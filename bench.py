@@ -46,6 +46,7 @@ def parse():
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--scheme", default=None)
     ap.add_argument("--cluster", type=int, default=0)
+    ap.add_argument("--omega0", type=int, default=20, help="|Omega_0| of the truncated-alphabet scheme WIS0")
     ap.add_argument("--B", type=int, default=0, help="override the batch (profiling on a small case)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
@@ -168,7 +169,7 @@ def recorded_traffic(workload, scheme):
 # ----------------------------------------------------------------- oracle leg
 
 
-def oracle_rate(w, scheme, seconds, seqs=None):
+def oracle_rate(w, scheme, seconds, seqs=None, omega0=20):
     """The oracle, as it stands, over a bounded prefix of the workload's
     sequences (host cores).  Returns (vocab_rows/s, sample description,
     outputs) for the sequences it finished."""
@@ -182,7 +183,7 @@ def oracle_rate(w, scheme, seconds, seqs=None):
     for b in order:
         host = host_copy(w, [b])
         t0 = time.perf_counter()
-        o, a, recs = oracle_verify(*host, scheme, spec.verify_seed, seq_ids=[b])
+        o, a, recs = oracle_verify(*host, scheme, spec.verify_seed, seq_ids=[b], omega0=omega0)
         t_total += time.perf_counter() - t0
         out = np.asarray(o[b])[None]
         r, _ = walk_accounting(host[3], w.model_ids, out, np.array([a[b]]), spec.V, es)
@@ -258,12 +259,12 @@ def main():
         # each step: the oracle over a bounded sample of the workload
         per_step = max(2.0, args.cpu_seconds / max(1, args.steps + args.warmup))
         for _ in range(args.warmup):
-            oracle_rate(w, scheme, per_step / 4)
+            oracle_rate(w, scheme, per_step / 4, omega0=args.omega0)
         rates = []
         desc = ""
         t0 = time.perf_counter()
         for _ in range(args.steps):
-            r, desc, _ = oracle_rate(w, scheme, per_step)
+            r, desc, _ = oracle_rate(w, scheme, per_step, omega0=args.omega0)
             rates.append(r)
         wall = time.perf_counter() - t0
         value = float(np.mean(rates))
@@ -272,7 +273,8 @@ def main():
                 "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
                 "data": "synthetic",
                 "config": {"workload": spec.name, "B": spec.B, "K": spec.K, "L": spec.L, "V": spec.V,
-                           "logits": spec.dtype, "scheme": scheme},
+                           "logits": spec.dtype, "scheme": scheme,
+                           **({"omega0": args.omega0} if scheme == "WIS0" else {})},
                 "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
                                  "sample": f"per step {desc}"},
                 "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -288,7 +290,8 @@ def main():
     torch.cuda.set_device(dev)
     from paper_2410_18234_gb300 import mds
     w = make_workload(spec, device=dev, seed=rank_seed(spec, rank))
-    v = mds.Verifier(spec.B, spec.K, spec.L, spec.V, dtype=spec.dtype, cluster=args.cluster, device=dev.index)
+    v = mds.Verifier(spec.B, spec.K, spec.L, spec.V, dtype=spec.dtype, cluster=args.cluster, device=dev.index,
+                     omega0=args.omega0)
     drafts = w.draft_list()
     out_tokens = torch.empty(spec.B, spec.L + 1, dtype=torch.int32, device=dev)
     out_acc = torch.empty(spec.B, dtype=torch.int32, device=dev)
@@ -369,7 +372,7 @@ def main():
     cpu = None
     parity = None
     if rank == 0 and world == 1 and not (args.no_cpu_baseline and args.no_parity):
-        rate, desc, outs = oracle_rate(w, scheme, args.cpu_seconds)
+        rate, desc, outs = oracle_rate(w, scheme, args.cpu_seconds, omega0=args.omega0)
         parity = agreement(o_tok, o_acc, outs)
         if not args.no_cpu_baseline:
             cpu = {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc}
@@ -384,6 +387,7 @@ def main():
             "vs_baseline": None, "dtype": "f32", "data": "synthetic",
             "config": {"workload": spec.name, "B": spec.B, "K": spec.K, "L": spec.L, "V": spec.V,
                        "logits": spec.dtype, "scheme": scheme, "cluster": cn, "l2_flush": True,
+                       **({"omega0": args.omega0} if scheme == "WIS0" else {}),
                        "parallelism": f"sequence-sharded x{world}", "seed": spec.verify_seed},
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "peak_kind": peak_kind,

@@ -22,7 +22,8 @@
  * (b, j, draw, 0) and key (seed low 32 bits, seed high 32 bits); the uniform
  * is (word0 >> 8) * 2^-24.  Draw ids: 0..15 importance-step selection (stage
  * m of the pairwise stages uses m), 16..31 accept (the sequential-rejection
- * baseline's round i uses 16 + i), 32 residual, 33 bonus.
+ * baseline's round i uses 16 + i), 32 residual, 33 bonus, 34 truncated
+ * alphabet keep test, 35 truncated alphabet replacement.
  *
  * Threading: a context may be used from one host thread at a time and its
  * calls must not overlap on the GPU (they share a work counter and a status
@@ -54,12 +55,18 @@ extern "C" {
 #define MDS_ST_TIMEOUT 8u     /* a bounded wait on a bulk copy gave up         */
 #define MDS_ST_LP_CAP 16u     /* the stage LP hit its augmentation cap         */
 #define MDS_ST_BADTOKEN 32u   /* a draft token was outside [0, V) (token 0 used) */
+#define MDS_ST_OMEGA0 64u     /* MDS_WIS0: the candidate list could not certify the
+                                 cut of Omega_0 (ties around its last entries); the
+                                 tokens above the certified bound formed Omega_0.
+                                 The output still follows the target; only the
+                                 acceptance rate can differ from the exact cut. */
 
 /* ---- limits ------------------------------------------------------------ */
 #define MDS_MAX_K 16      /* draft branches per sequence                    */
 #define MDS_MAX_L 64      /* draft positions per branch                     */
 #define MDS_MAX_S 8       /* LP truncation threshold s (|Omega_1|)          */
 #define MDS_MAX_IS_MODELS 4  /* distinct draft models for plain IS          */
+#define MDS_MAX_OMEGA0 30 /* |Omega_0| of the truncated alphabet, MDS_WIS0  */
 
 typedef struct mds_ctx mds_ctx;
 
@@ -70,8 +77,18 @@ typedef struct mds_ctx mds_ctx;
  * "Variant of Truncated LP", Eq. heur2), pairwise stages for K > 2
  * (Remark 4) and the non-iid key q - p_1 p_2 (non-iid appendix).
  * MDS_SPECTR: sequential-rejection baseline (Algorithm 1 applied to the
- * valid drafts in turn against the running residual target). */
-typedef enum { MDS_SINGLE = 0, MDS_IS = 1, MDS_WIS = 2, MDS_SPECTR = 3 } mds_scheme;
+ * valid drafts in turn against the running residual target).
+ * MDS_WIS0: the truncated-alphabet scheme (Section 4) around MDS_WIS.
+ * Omega_0 is the set of target tokens whose logit is above the (M+1)-th
+ * largest target logit, M = omega0 (at most M tokens; tokens tied at the cut
+ * are all left out).  With p_a = q(Omega_0), the WIS stages run on the
+ * alphabet Omega_0 against q / p_a, using only the valid draft tokens that
+ * lie in Omega_0 with their draft laws restricted to Omega_0 and
+ * renormalised (the non-iid appendix's remark); Algorithm 1 against q / p_a
+ * gives Y' (drawn from q / p_a directly when no draft token lies in
+ * Omega_0).  Y' is kept with probability p_a (draw 34), otherwise the output
+ * is drawn from the tokens outside Omega_0 in proportion to q (draw 35). */
+typedef enum { MDS_SINGLE = 0, MDS_IS = 1, MDS_WIS = 2, MDS_SPECTR = 3, MDS_WIS0 = 4 } mds_scheme;
 
 /* Storage type of the logits. */
 typedef enum { MDS_F32 = 0, MDS_BF16 = 1 } mds_dtype;
@@ -86,6 +103,9 @@ typedef struct {
                       of the paper's experiments, Section 5)                  */
   float is_h;      /* trapezoid step in ln t for plain IS (0: 0.25)           */
   int cluster;     /* CTAs per sequence: 1, 2, 4, 8 or 16 (0: chosen from max_B and the device) */
+  int omega0;      /* |Omega_0| for MDS_WIS0, 1..MDS_MAX_OMEGA0 (0: 20; the paper's
+                      runs use 10 to 50, Section 5, Table "Effect of LP
+                      Truncation and Alphabet Truncation")                    */
 } mds_config;
 
 /* Create a context on CUDA device `device`.  Allocates the context's device
@@ -115,7 +135,8 @@ int mds_create(mds_ctx** out, const mds_config* cfg, int device);
  * Pointers must be aligned to the element size; rows whose byte length is a
  * multiple of 16 at 16-byte-aligned bases are fetched with bulk copies.
  * Plain IS supports at most MDS_MAX_IS_MODELS distinct draft models
- * (MDS_EUNSUP otherwise).  Returns MDS_OK after the launch was issued, or a
+ * (MDS_EUNSUP otherwise).  For MDS_WIS0, out_diag holds q(Y)/p_a and p_I(Y)
+ * of the inner step on Omega_0 (Y = -1 when no draft token lies in it).  Returns MDS_OK after the launch was issued, or a
  * negative code with nothing launched.  Data-dependent anomalies are reported
  * through the status word (mds_status). */
 int mds_verify(mds_ctx* ctx, const void* target_logits, const void* const* draft_logits,

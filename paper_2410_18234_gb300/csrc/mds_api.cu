@@ -87,7 +87,9 @@ int geometry(const mds_ctx* ctx, int scheme, int n_models, mds::Params& p) {
   p.rows_max = 1 + n_models;
   p.scheme = scheme;
   p.ring_bytes = kRingBytes;
-  const bool lists = scheme == MDS_WIS && p.rows_max <= 4;
+  // candidate lists: WIS with at most three draft models in the stats pass;
+  // the truncated alphabet always (its Omega_0 comes from the list)
+  const bool lists = (scheme == MDS_WIS && p.rows_max <= 4) || scheme == MDS_WIS0;
   auto fill = [&](int cn) {
     p.cn = cn;
     p.slice = (int)round_up((size_t)((c.V + cn - 1) / cn), 8);
@@ -164,6 +166,8 @@ int mds_create(mds_ctx** out, const mds_config* cfg, int device) {
   mds_config c = *cfg;
   if (c.wis_s == 0) c.wis_s = 5;
   if (c.is_h == 0.f) c.is_h = 0.25f;
+  if (c.omega0 == 0) c.omega0 = 20;
+  if (c.omega0 < 1 || c.omega0 > MDS_MAX_OMEGA0) return MDS_EINVAL;
   if (c.max_B < 1 || c.K < 1 || c.K > MDS_MAX_K || c.L < 1 || c.L > MDS_MAX_L || c.V < 1 || c.V > (1 << 24))
     return MDS_ESHAPE;
   if (c.dtype != MDS_F32 && c.dtype != MDS_BF16) return MDS_EINVAL;
@@ -201,7 +205,7 @@ static int verify_impl(mds_ctx* ctx, const void* target_logits, const void* cons
                        float* out_diag, int B, void* stream, bool bulk_ok) {
   if (!ctx) return MDS_EINVAL;
   const mds_config& c = ctx->cfg;
-  if (scheme < MDS_SINGLE || scheme > MDS_SPECTR) return MDS_EINVAL;
+  if (scheme < MDS_SINGLE || scheme > MDS_WIS0) return MDS_EINVAL;
   if (B < 0 || B > c.max_B) return MDS_ESHAPE;
   if (B == 0) return MDS_OK;
   if (!target_logits || !draft_logits || !draft_model_id || !draft_tokens || !temperatures || !out_tokens ||
@@ -243,6 +247,7 @@ static int verify_impl(mds_ctx* ctx, const void* target_logits, const void* cons
   p.L = c.L;
   p.V = c.V;
   p.wis_s = c.wis_s;
+  p.omega0 = c.omega0;
   p.is_h = c.is_h;
   p.n_models = n_models;
   p.tma_ok = tma_ok ? 1 : 0;
@@ -374,7 +379,8 @@ int mds_status(mds_ctx* ctx, const char** msg) {
     return MDS_ECUDA;
   }
   if (msg) {
-    if (st & MDS_ST_BADTOKEN) *msg = "draft token outside [0, V); token 0 used";
+    if (st & MDS_ST_OMEGA0) *msg = "Omega_0 cut not certified by the candidate list; certified subset used";
+    else if (st & MDS_ST_BADTOKEN) *msg = "draft token outside [0, V); token 0 used";
     else if (st & MDS_ST_LP_CAP) *msg = "stage LP reached its augmentation cap";
     else if (st & MDS_ST_TIMEOUT) *msg = "a bounded wait on a bulk copy gave up";
     else if (st & MDS_ST_ZERO_RESID) *msg = "zero residual mass after a rejection; target row sampled";

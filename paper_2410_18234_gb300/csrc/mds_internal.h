@@ -34,6 +34,7 @@ struct Params {
   int dtype;                           // MDS_F32 / MDS_BF16
   int esize;                           // bytes per logit
   int wis_s;
+  int omega0;                          // |Omega_0| bound M of MDS_WIS0
   float is_h;
   int cn;                              // CTAs per cluster
   int slice;                           // tokens per CTA (multiple of 8)

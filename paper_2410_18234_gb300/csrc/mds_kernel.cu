@@ -134,6 +134,7 @@ __device__ __forceinline__ float draw_uniform(unsigned long long seed, int b, in
   return (float)(w >> 8) * 0x1p-24f;
 }
 constexpr int kDrawSelect = 0, kDrawAccept = 16, kDrawResidual = 32, kDrawBonus = 33;
+constexpr int kDrawKeep = 34, kDrawOutside = 35;   // truncated alphabet: keep Y', replace it
 
 // ------------------------------------------------------------------ element IO
 
@@ -267,6 +268,11 @@ struct State {
   float pc[kMaxRows];        // complement exp mass per row
   int ncand, cand_all, fast_ok;
   float cand_q;
+  float cand_tau;            // every target logit outside the list is <= cand_tau
+  // truncated alphabet: kept inputs (list lane, row) and the depth's outcome
+  int k_lane[MDS_MAX_K], k_row[MDS_MAX_K];
+  int o0_n, o0_all, o0_Yp;
+  float o0_cut, o0_pa, o0_R;
   // SpecTr: inverse residual masses of rejected rounds
   float sp_invR[MDS_MAX_K];
   int sp_rows[MDS_MAX_K];
@@ -1089,6 +1095,7 @@ struct Kernel {
         S.ncand = n;
         S.cand_all = (n == p.V) ? 1 : 0;
         S.cand_q = (tau > kNegInf) ? ex2(__fmaf_rn(tau, cr[0], -__fmul_rn(S.M[r0], cr[0]))) : 0.f;
+        S.cand_tau = tau;
       }
       clbuf ^= 1;
       __syncthreads();
@@ -1103,15 +1110,33 @@ struct Kernel {
     S.invZ[r] = __frcp_rn(Z);
   }
 
-  // Statistics of every row loaded at this depth (candidates for WIS).
+  // Statistics of every row loaded at this depth (candidates for WIS and the
+  // truncated alphabet).
   __device__ void depth_stats(bool cand) {
     const int nr = S.nrows;
     if (cand && nr <= kFastRows && p.cand_cap > 0) {
       switch (nr) {
+        case 1: if constexpr (SCHEME == MDS_WIS0) { stats_pass<1, true>(0); return; } break;
         case 2: stats_pass<2, true>(0); return;
         case 3: stats_pass<3, true>(0); return;
         case 4: stats_pass<4, true>(0); return;
         default: break;
+      }
+    }
+    if constexpr (SCHEME == MDS_WIS0) {
+      if (p.cand_cap > 0) {
+        // more draft rows than one pass holds: the draft rows first (a pass
+        // without a list clears it), then the target with its list
+        for (int r0 = 1; r0 < nr; r0 += 4) {
+          switch (min(4, nr - r0)) {
+            case 1: stats_pass<1, false>(r0); break;
+            case 2: stats_pass<2, false>(r0); break;
+            case 3: stats_pass<3, false>(r0); break;
+            default: stats_pass<4, false>(r0); break;
+          }
+        }
+        stats_pass<1, true>(0);
+        return;
       }
     }
     for (int r0 = 0; r0 < nr; r0 += 4) {
@@ -2244,6 +2269,207 @@ struct Kernel {
   }
 
   // ---------------------------------------------------------------- one sequence
+  // ---------------------------------------------------------------- truncated alphabet
+  // Warp-wide inverse CDF over one weight per lane (lane order is the list's
+  // token-id order): the smallest lane whose running sum exceeds u * total,
+  // the last lane with positive weight if rounding leaves none, -1 if the
+  // total is not positive.
+  __device__ __forceinline__ int lane_cdf(float w, float u01, float* total) const {
+    const int lane = threadIdx.x & 31;
+    float c = w;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const float t = __shfl_up_sync(0xffffffffu, c, o);
+      if (lane >= o) c = __fadd_rn(c, t);
+    }
+    const float tot = __shfl_sync(0xffffffffu, c, 31);
+    *total = tot;
+    if (!(tot > 0.f)) return -1;
+    const unsigned who = __ballot_sync(0xffffffffu, c > __fmul_rn(u01, tot));
+    if (who) return __ffs(who) - 1;
+    return 31 - __clz(__ballot_sync(0xffffffffu, w > 0.f));
+  }
+
+  // One depth of the truncated-alphabet scheme (Section 4, read together with
+  // the non-iid appendix's remark on keeping only the inputs in Omega_0).
+  // Omega_0 = the target tokens above the (M+1)-th largest target logit.  The
+  // candidate list holds every token above cand_tau, so the cut is exact when
+  // the list's (M+1)-th entry is >= cand_tau (or the list holds the whole
+  // vocabulary, or every token outside it is -inf); otherwise the tokens above
+  // cand_tau form Omega_0 and the status says so.  Warp 0 runs the WIS stages
+  // on Omega_0, one list entry per lane, against q~ = q / p_a with the kept
+  // inputs' draft laws restricted to Omega_0 and renormalised, then
+  // Algorithm 1 against q~ (a lane-level inverse CDF for the residual).  The
+  // result Y' is kept with probability p_a; otherwise a streaming draw over
+  // the tokens outside Omega_0 in proportion to q replaces it.  Every CTA of
+  // the cluster computes the same warp-0 result from the same list.
+  __device__ int wis0_step(int b, int j, float* qYo, float* pIYo, int* Yo, float* Ro) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    if (warp == 0) {
+      const unsigned FULL = 0xffffffffu;
+      const int n = max(0, S.ncand);
+      const bool have = lane < n;
+      const int id = have ? cm_id[lane] : 0;
+      const float l = have ? E::global(S.gptr[0], id) : kNegInf;
+      int rk = 0;   // rank in the list by (larger logit, then lower id)
+      for (int t = 0; t < 32; ++t) {
+        const float lt = __shfl_sync(FULL, l, t);
+        const int it = __shfl_sync(FULL, id, t);
+        rk += (t < n && cand_before(lt, it, l, id)) ? 1 : 0;
+      }
+      const int M = p.omega0;
+      const bool all0 = M >= p.V;
+      float cut = kNegInf;
+      bool cert;
+      if (all0) {
+        cert = S.cand_all != 0;
+      } else {
+        const unsigned who = __ballot_sync(FULL, have && rk == M);
+        if (who) cut = __shfl_sync(FULL, l, __ffs(who) - 1);
+        const float tau = S.cand_tau;
+        cert = S.cand_all || (who ? cut >= tau : !(tau > kNegInf));
+        if (!cert) cut = fmaxf(cut, tau);
+      }
+      const bool in0 = have && (all0 || l > cut);
+      const int n0 = __popc(__ballot_sync(FULL, in0));
+      const float q = in0 ? prob_of(l, S.M[0], S.c[0], S.invZ[0]) : 0.f;
+      const float pa = warp_sum(q);
+      const float qt = (in0 && pa > 0.f) ? __fdiv_rn(q, pa) : 0.f;
+      // draft laws of this depth's rows restricted to Omega_0, renormalised
+      for (int r = 1; r < S.nrows; ++r) {
+        const float pr = in0 ? prob_row(r, id) : 0.f;
+        const float P = warp_sum(pr);
+        cm_e[r * p.cand_cap + lane] = (P > 0.f) ? __fdiv_rn(pr, P) : 0.f;
+      }
+      __syncwarp();
+      // kept inputs: valid branches (branch order) whose token lies in Omega_0
+      int nk = 0;
+      for (int i = 0; i < S.nv; ++i) {
+        const unsigned w = __ballot_sync(FULL, in0 && id == S.X[i]);
+        if (!w) continue;
+        const int li = __ffs(w) - 1;
+        if (!(cm_e[S.vrow[i] * p.cand_cap + li] > 0.f)) continue;   // impossible draw: dropped
+        if (lane == 0) {
+          S.k_lane[nk] = li;
+          S.k_row[nk] = S.vrow[i];
+        }
+        ++nk;
+      }
+      __syncwarp();
+      int yl = -1, Yl = -1;
+      float qY = 0.f, pIY = 0.f, R = 0.f;
+      if (n0 > 0 && nk == 0) {
+        float t;
+        yl = lane_cdf(qt, draw_uniform(p.seed, b, j, kDrawResidual), &t);
+      } else if (n0 > 0) {
+        float a = cm_e[S.k_row[0] * p.cand_cap + lane];
+        int A = S.k_lane[0];
+        const int s = min(p.wis_s, n0);
+        for (int m = 1; m < nk; ++m) {
+          const int Bl = S.k_lane[m];
+          const float bb = cm_e[S.k_row[m] * p.cand_cap + lane];
+          const float u = draw_uniform(p.seed, b, j, kDrawSelect + m - 1);
+          // Omega_1: the s largest keys q~ - a b in Omega_0, ties to the lower id
+          unsigned kk = in0 ? ord_key(__fadd_rn(__fmaf_rn(-a, bb, qt), 0.f)) : 0u;
+          uint32_t selm = 0u;
+          for (int t = 0; t < s; ++t) {
+            const unsigned km = __reduce_max_sync(FULL, kk);
+            const uint32_t who = __ballot_sync(FULL, km != 0u && kk == km);
+            if (!who) break;
+            const int wl = __ffs(who) - 1;
+            selm |= 1u << wl;
+            if (lane == wl) kk = 0u;
+          }
+          const bool sel = (selm >> lane) & 1u;
+          const int sn = __popc(selm);
+          const float A2 = warp_sum((in0 && !sel) ? a : 0.f);
+          const float B2 = warp_sum((in0 && !sel) ? bb : 0.f);
+          const int rk1 = __popc(selm & ((1u << lane) - 1u));
+          if (lane >= sn && lane < MDS_MAX_S) {
+            S.om[lane] = -1;
+            S.om_q[lane] = 0.f;
+            S.om_a[lane] = 0.f;
+            S.om_b[lane] = 0.f;
+          }
+          if (sel) {
+            S.om[rk1] = id;
+            S.om_q[rk1] = qt;
+            S.om_a[rk1] = a;
+            S.om_b[rk1] = bb;
+          }
+          __syncwarp();
+          if (lane == 0) S.Y = stage_solve(sn, A2, B2, cm_id[A], cm_id[Bl], u);
+          __syncwarp();
+          const int Yt = S.Y;
+          A = max(0, __ffs(__ballot_sync(FULL, in0 && id == Yt)) - 1);   // Yt is A's or B's token
+          a = sel ? S.om_x[rk1] : (in0 ? __fmul_rn(0.5f, __fadd_rn(__fmul_rn(a, B2), __fmul_rn(bb, A2))) : 0.f);
+          __syncwarp();
+        }
+        Yl = A;
+        qY = __shfl_sync(FULL, qt, A);
+        pIY = __shfl_sync(FULL, a, A);
+        const float ratio = pIY > 0.f ? __fdiv_rn(qY, pIY) : kPosInf;
+        if (draw_uniform(p.seed, b, j, kDrawAccept) < fminf(1.f, ratio)) {
+          yl = A;
+        } else {
+          const float ures = draw_uniform(p.seed, b, j, kDrawResidual);
+          yl = lane_cdf(in0 ? fmaxf(0.f, __fsub_rn(qt, a)) : 0.f, ures, &R);
+          if (yl < 0) {   // only by rounding: sample q~
+            if (lane == 0 && rank == 0) atomicOr(p.status, MDS_ST_ZERO_RESID);
+            float t;
+            yl = lane_cdf(qt, ures, &t);
+          }
+        }
+      }
+      if (lane == 0) {
+        if (!cert && rank == 0) atomicOr(p.status, MDS_ST_OMEGA0);
+        S.o0_n = n0;
+        S.o0_all = (all0 && S.cand_all) ? 1 : 0;
+        S.o0_cut = cut;
+        S.o0_pa = pa;
+        S.o0_R = R;
+        S.o0_Yp = (yl >= 0) ? cm_id[yl] : -1;
+        S.Y = (Yl >= 0) ? cm_id[Yl] : -1;
+        S.qY = qY;
+        S.pIY = pIY;
+      }
+    }
+    __syncthreads();
+    *Yo = S.Y;
+    *qYo = S.qY;
+    *pIYo = S.pIY;
+    *Ro = S.o0_R;
+    const int Yp = S.o0_Yp;
+    if (S.o0_n > 0 && (S.o0_all || draw_uniform(p.seed, b, j, kDrawKeep) < S.o0_pa)) return Yp;
+    // replace: a draw over the tokens outside Omega_0 in proportion to q
+    const float cut = S.o0_cut;
+    const bool all0 = S.o0_all != 0;
+    float tot;
+    int Z = sample_cdf(
+        1u,
+        [&](int, const auto& L, float* r) {
+          float v[VE];
+          L(0, v);
+#pragma unroll
+          for (int e = 0; e < VE; ++e) r[e] = (all0 || v[e] > cut) ? 0.f : prob_of(v[e], S.M[0], S.c[0], S.invZ[0]);
+        },
+        draw_uniform(p.seed, b, j, kDrawOutside), &tot);
+    if (Z < 0) {   // no target mass outside Omega_0
+      if (Yp >= 0) return Yp;
+      if (threadIdx.x == 0 && rank == 0) atomicOr(p.status, MDS_ST_ZERO_RESID);
+      Z = sample_cdf(
+          1u,
+          [&](int, const auto& L, float* r) {
+            float v[VE];
+            L(0, v);
+#pragma unroll
+            for (int e = 0; e < VE; ++e) r[e] = prob_of(v[e], S.M[0], S.c[0], S.invZ[0]);
+          },
+          draw_uniform(p.seed, b, j, kDrawOutside), &tot);
+    }
+    return Z;
+  }
+
   __device__ __forceinline__ void run_sequence(int b) {
     const int K = p.K, L = p.L, V = p.V;
     const int tid = threadIdx.x;
@@ -2298,7 +2524,7 @@ struct Kernel {
         S.nrows = nr;
       }
       __syncthreads();
-      if (!bonus) depth_stats(SCHEME == MDS_WIS && S.nv > 1);
+      if (!bonus) depth_stats((SCHEME == MDS_WIS && S.nv > 1) || SCHEME == MDS_WIS0);
       int Z;
       float qY = 0.f, pIY = 0.f, Rdiag = 0.f;
       int Ydiag = -1;
@@ -2308,6 +2534,8 @@ struct Kernel {
         Rdiag = tot;
       } else if constexpr (SCHEME == MDS_SPECTR) {
         Z = spectr(b, j, &qY, &pIY, &Ydiag, &Rdiag);
+      } else if constexpr (SCHEME == MDS_WIS0) {
+        Z = wis0_step(b, j, &qY, &pIY, &Ydiag, &Rdiag);
       } else {
         // importance step -> Y and the law p_I (kept in S for the residual)
         int Y;
@@ -2657,7 +2885,7 @@ size_t smem_bytes(const Params& p) {
   const int nseg = (p.slice / VE + 31) / 32;
   size_t bytes = (size_t)p.ring_bytes + (size_t)((nseg + 3) & ~3) * 4 * 2 + (size_t)((((nseg + 31) / 32) + 3) & ~3) * 4;
   if (p.scheme == MDS_IS) bytes += (size_t)kIsNodesMax * 4 * (1 + p.rows_max);
-  if (p.scheme == MDS_WIS) {
+  if (p.scheme == MDS_WIS || p.scheme == MDS_WIS0) {
     const size_t bm = (size_t)((p.slice / VE + 31) / 32) * 4;
     const size_t cm = (size_t)p.cand_cap * 4 * (3 + p.rows_max);
     size_t stg = (size_t)p.cand_stage * 4 * (2 + p.rows_max);
@@ -2677,6 +2905,7 @@ static KernelFn kernel_for(int dtype, int scheme) {
       case MDS_IS: return verify_kernel<MDS_F32, MDS_IS>;
       case MDS_WIS: return verify_kernel<MDS_F32, MDS_WIS>;
       case MDS_SPECTR: return verify_kernel<MDS_F32, MDS_SPECTR>;
+      case MDS_WIS0: return verify_kernel<MDS_F32, MDS_WIS0>;
       default: return verify_kernel<MDS_F32, MDS_SINGLE>;
     }
   }
@@ -2684,6 +2913,7 @@ static KernelFn kernel_for(int dtype, int scheme) {
     case MDS_IS: return verify_kernel<MDS_BF16, MDS_IS>;
     case MDS_WIS: return verify_kernel<MDS_BF16, MDS_WIS>;
     case MDS_SPECTR: return verify_kernel<MDS_BF16, MDS_SPECTR>;
+    case MDS_WIS0: return verify_kernel<MDS_BF16, MDS_WIS0>;
     default: return verify_kernel<MDS_BF16, MDS_SINGLE>;
   }
 }
@@ -2692,7 +2922,7 @@ cudaError_t configure_kernel(int dtype) {
   int dev = 0, optin = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
-  for (int scheme = MDS_SINGLE; scheme <= MDS_SPECTR; ++scheme) {
+  for (int scheme = MDS_SINGLE; scheme <= MDS_WIS0; ++scheme) {
     const void* fn = (const void*)kernel_for(dtype, scheme);
     cudaFuncAttributes fa;
     cudaError_t e = cudaFuncGetAttributes(&fa, fn);

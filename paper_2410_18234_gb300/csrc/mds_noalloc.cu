@@ -46,13 +46,15 @@ extern "C" int mds_verify_noalloc(const mds_config* cfg_in, int device, const vo
   mds_config c = *cfg_in;
   if (c.wis_s == 0) c.wis_s = 5;
   if (c.is_h == 0.f) c.is_h = 0.25f;
+  if (c.omega0 == 0) c.omega0 = 20;
+  if (c.omega0 < 1 || c.omega0 > MDS_MAX_OMEGA0) return MDS_EINVAL;
   if (c.max_B < 1 || c.K < 1 || c.K > MDS_MAX_K || c.L < 1 || c.L > MDS_MAX_L || c.V < 1 || c.V > (1 << 24))
     return MDS_ESHAPE;
   if (c.dtype != MDS_F32 && c.dtype != MDS_BF16) return MDS_EINVAL;
   if (c.wis_s < 1 || c.wis_s > MDS_MAX_S || !(c.is_h > 0.f) || c.is_h > 4.f) return MDS_EINVAL;
   if (c.cluster != 0 && c.cluster != 1 && c.cluster != 2 && c.cluster != 4 && c.cluster != 8 && c.cluster != 16)
     return MDS_EINVAL;
-  if (scheme < MDS_SINGLE || scheme > MDS_SPECTR) return MDS_EINVAL;
+  if (scheme < MDS_SINGLE || scheme > MDS_WIS0) return MDS_EINVAL;
   if (B < 0 || B > c.max_B) return MDS_ESHAPE;
   // the scratch this launch needs (it does not grow with B, K, L or V)
   if (kScratchNeeded > MDS_NOALLOC_SCRATCH_BYTES) return MDS_ESHAPE;
@@ -108,6 +110,7 @@ extern "C" int mds_verify_noalloc(const mds_config* cfg_in, int device, const vo
     p.L = c.L;
     p.V = c.V;
     p.wis_s = c.wis_s;
+    p.omega0 = c.omega0;
     p.is_h = c.is_h;
     p.bulk_ok = 1;
     p.n_models = n_models;

@@ -17,8 +17,8 @@ import torch
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "_lib", "libmds.so")
 
-MDS_SINGLE, MDS_IS, MDS_WIS, MDS_SPECTR = 0, 1, 2, 3
-SCHEMES = {"single": MDS_SINGLE, "IS": MDS_IS, "WIS": MDS_WIS, "SpecTr": MDS_SPECTR}
+MDS_SINGLE, MDS_IS, MDS_WIS, MDS_SPECTR, MDS_WIS0 = 0, 1, 2, 3, 4
+SCHEMES = {"single": MDS_SINGLE, "IS": MDS_IS, "WIS": MDS_WIS, "SpecTr": MDS_SPECTR, "WIS0": MDS_WIS0}
 MDS_F32, MDS_BF16 = 0, 1
 DTYPES = {"f32": MDS_F32, "bf16": MDS_BF16}
 TORCH_DTYPES = {MDS_F32: torch.float32, MDS_BF16: torch.bfloat16}
@@ -26,7 +26,9 @@ TORCH_DTYPES = {MDS_F32: torch.float32, MDS_BF16: torch.bfloat16}
 MDS_OK, MDS_EINVAL, MDS_ESHAPE, MDS_EVOCAB, MDS_ECUDA, MDS_EUNSUP = 0, -1, -2, -3, -4, -5
 MDS_ST_NONFINITE, MDS_ST_BADTEMP, MDS_ST_ZERO_RESID, MDS_ST_TIMEOUT, MDS_ST_LP_CAP, MDS_ST_BADTOKEN = \
     1, 2, 4, 8, 16, 32
+MDS_ST_OMEGA0 = 64
 MDS_MAX_K = 16
+MDS_MAX_OMEGA0 = 30
 
 # every symbol include/mds.h declares
 EXPORTS = ("mds_create", "mds_verify", "mds_verify_host", "mds_verify_noalloc", "mds_status",
@@ -36,7 +38,7 @@ EXPORTS = ("mds_create", "mds_verify", "mds_verify_host", "mds_verify_noalloc", 
 class MdsConfig(ctypes.Structure):
     _fields_ = [("max_B", ctypes.c_int), ("K", ctypes.c_int), ("L", ctypes.c_int), ("V", ctypes.c_int),
                 ("dtype", ctypes.c_int), ("wis_s", ctypes.c_int), ("is_h", ctypes.c_float),
-                ("cluster", ctypes.c_int)]
+                ("cluster", ctypes.c_int), ("omega0", ctypes.c_int)]
 
 
 class MdsError(RuntimeError):
@@ -83,9 +85,9 @@ def error_string(code):
 # ----------------------------------------------------------- C entry points
 
 
-def mds_create(max_B, K, L, V, dtype="bf16", wis_s=5, is_h=0.25, cluster=0, device=0):
+def mds_create(max_B, K, L, V, dtype="bf16", wis_s=5, is_h=0.25, cluster=0, device=0, omega0=0):
     cfg = MdsConfig(int(max_B), int(K), int(L), int(V), DTYPES[dtype] if isinstance(dtype, str) else int(dtype),
-                    int(wis_s), float(is_h), int(cluster))
+                    int(wis_s), float(is_h), int(cluster), int(omega0))
     h = ctypes.c_void_p()
     rc = _lib.mds_create(ctypes.byref(h), ctypes.byref(cfg), int(device))
     if rc != MDS_OK:
@@ -151,12 +153,12 @@ def mds_verify_host(ctx, target, drafts, model_ids, tokens, temps, scheme, seed,
 
 def mds_verify_noalloc(max_B, K, L, V, target, drafts, model_ids, tokens, temps, scheme, seed, out_tokens,
                        out_accept, out_diag=None, stream=None, dtype="bf16", wis_s=5, is_h=0.25, cluster=0,
-                       device=0):
+                       device=0, omega0=0):
     """Context-free entry point for callers that cannot allocate device
     memory (see include/mds.h): the configuration is passed directly and the
     kernel's scratch is a static device array inside the library."""
     cfg = MdsConfig(int(max_B), int(K), int(L), int(V), DTYPES[dtype] if isinstance(dtype, str) else int(dtype),
-                    int(wis_s), float(is_h), int(cluster))
+                    int(wis_s), float(is_h), int(cluster), int(omega0))
     Kn = len(model_ids)
     B = int(tokens.shape[0])
     if stream is None:
@@ -195,11 +197,11 @@ def mds_destroy(ctx):
 class Verifier:
     """Owns one context; allocates outputs with torch on the context's device."""
 
-    def __init__(self, max_B, K, L, V, dtype="bf16", wis_s=5, is_h=0.25, cluster=0, device=0):
+    def __init__(self, max_B, K, L, V, dtype="bf16", wis_s=5, is_h=0.25, cluster=0, device=0, omega0=0):
         self.max_B, self.K, self.L, self.V = int(max_B), int(K), int(L), int(V)
         self.dtype = dtype
         self.device = torch.device("cuda", device)
-        self.ctx = mds_create(max_B, K, L, V, dtype, wis_s, is_h, cluster, device)
+        self.ctx = mds_create(max_B, K, L, V, dtype, wis_s, is_h, cluster, device, omega0)
 
     def verify(self, target, drafts, model_ids, tokens, temps, scheme, seed, diag=False, out=None, stream=None):
         B = int(tokens.shape[0])

@@ -59,7 +59,8 @@ def test_create_rejects_bad_config_before_touching_a_device():
         with pytest.raises(mds.MdsError) as e:
             mds.mds_create(**c)
         assert e.value.code == mds.MDS_ESHAPE
-    for c in (dict(wis_s=9), dict(is_h=-1.0), dict(cluster=3), dict(dtype=7)):
+    for c in (dict(wis_s=9), dict(is_h=-1.0), dict(cluster=3), dict(dtype=7), dict(omega0=-2),
+              dict(omega0=mds.MDS_MAX_OMEGA0 + 1)):
         with pytest.raises(mds.MdsError) as e:
             mds.mds_create(4, 2, 4, 100, **c)
         assert e.value.code == mds.MDS_EINVAL
@@ -72,3 +73,20 @@ def test_verify_rejects_null_context(lib):
     lib.mds_status.restype = ctypes.c_int
     assert lib.mds_status(None, None) == -1
     lib.mds_destroy(None)
+
+
+def test_binding_config_matches_the_header():
+    """The ctypes mirror of mds_config has the header's fields in order, and
+    the scheme ids and limits agree."""
+    from paper_2410_18234_gb300 import mds
+    text = open(HEADER).read()
+    body = re.search(r"typedef struct \{(.*?)\} mds_config;", text, flags=re.S).group(1)
+    body = re.sub(r"/\*.*?\*/", "", body, flags=re.S)
+    fields = re.findall(r"\b(\w+)\s*;", body)
+    assert [f[0] for f in mds.MdsConfig._fields_] == fields
+    enum = re.search(r"typedef enum \{([^}]*)\} mds_scheme;", text).group(1)
+    ids = dict((k, int(v)) for k, v in re.findall(r"(MDS_\w+)\s*=\s*(\d+)", enum))
+    for name, sid in mds.SCHEMES.items():
+        assert ids["MDS_" + name.upper()] == sid
+    assert int(re.search(r"#define MDS_MAX_OMEGA0 (\d+)", text).group(1)) == mds.MDS_MAX_OMEGA0
+    assert int(re.search(r"#define MDS_ST_OMEGA0 (\d+)u", text).group(1)) == mds.MDS_ST_OMEGA0

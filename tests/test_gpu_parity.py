@@ -24,18 +24,19 @@ from parity import compare, check  # noqa: E402
 DEV = "cuda:0"
 
 
-def run_both(spec, scheme, seed, cluster=0, seqs=None, wis_s=5):
+def run_both(spec, scheme, seed, cluster=0, seqs=None, wis_s=5, omega0=20):
     w = make_workload(spec, device=DEV)
-    v = mds.Verifier(spec.B, spec.K, spec.L, spec.V, dtype=spec.dtype, wis_s=wis_s, cluster=cluster)
+    v = mds.Verifier(spec.B, spec.K, spec.L, spec.V, dtype=spec.dtype, wis_s=wis_s, cluster=cluster, omega0=omega0)
     out, acc, diag = v.verify(w.target, w.draft_list(), w.model_ids, w.tokens, w.temps, scheme, seed, diag=True)
     torch.cuda.synchronize()
     bits, msg = v.status()
     cn = v.cluster_size
     v.close()
     if seqs is None:
-        o_out, o_acc, recs = oracle_verify(*host_copy(w), scheme, seed, wis_s=wis_s)
+        o_out, o_acc, recs = oracle_verify(*host_copy(w), scheme, seed, wis_s=wis_s, omega0=omega0)
     else:
-        o_out, o_acc, recs = oracle_verify(*host_copy(w, seqs), scheme, seed, wis_s=wis_s, seq_ids=seqs)
+        o_out, o_acc, recs = oracle_verify(*host_copy(w, seqs), scheme, seed, wis_s=wis_s, seq_ids=seqs,
+                                           omega0=omega0)
     res = compare(out.cpu().numpy(), acc.cpu().numpy(), o_out, o_acc, recs, g_diag=diag.cpu().numpy(),
                   scheme=scheme)
     res["status"] = bits
