@@ -21,6 +21,8 @@ enum     exhaustive enumeration of selection rules over Omega^K (tiny
          vocabularies), used to pin the induced distribution p_I.
 truncated  the truncated-alphabet scheme (Section 4) and top-k / top-p
          preprocessing (Section 5), with the enumerated law that pins it.
+sorted_lp  the truncated LP with the sorted rule on Omega_2 (Section 4 Eq.
+         heur, Algorithm 2, App. I): no device counterpart yet.
 
 Parity status: every function here is pinned by a ``-m "not gpu"`` test
 (see tests/test_oracle_*.py) except the SpecTr-style sequential-rejection

@@ -37,6 +37,8 @@ WIS      the paper's weighted importance sampling with the variant truncated
          (module ``wis``).
 SpecTr   sequential-rejection baseline (reading: Algorithm 1 applied to the
          valid drafts in turn against the running residual target).
+WISsort  the truncated LP with the sorted rule on Omega_2 (Section 4 Eq. heur,
+         Algorithm 2; module ``sorted_lp``), pairwise stages for K > 2.
 WIS0     WIS on the truncated alphabet Omega_0 = the ``omega0`` most probable
          target tokens, followed by the keep / replace step that restores the
          target (Section 4, "truncated alphabet"; module ``truncated``).
@@ -55,8 +57,10 @@ from .philox import DRAW_ACCEPT, DRAW_BONUS, DRAW_RESIDUAL, DRAW_SELECT
 from . import wis as wis_mod
 from . import is_laplace
 from . import truncated
+from . import sorted_lp
 
-SCHEMES = {"single": 0, "IS": 1, "WIS": 2, "SpecTr": 3, "WIS0": 4}
+SCHEMES = {"single": 0, "IS": 1, "WIS": 2, "SpecTr": 3, "WIS0": 4,
+           "WISsort": None}   # None: no device scheme id (the oracle alone has it)
 
 # Band thresholds (absolute, on quantities in [0, 1] or scaled as stated).
 BAND_ACCEPT = 1e-6   # |u - min(1, q(Y)/p_I(Y))|
@@ -213,6 +217,11 @@ def verify_sequence(b, target_logits, draft_logits, draft_model_id, draft_tokens
                                   philox.uniform(seed, sid, j, DRAW_RESIDUAL))
         elif scheme == "SpecTr":
             Z = _spectr_step(rec, q, dists, X, seed, sid, j)
+        elif scheme == "WISsort":
+            us = [philox.uniform(seed, sid, j, DRAW_SELECT + m) for m in range(max(0, len(X) - 1))]
+            Y, pI = sorted_lp.sorted_select(rec, q, dists, X, us, wis_s)
+            Z = _speculative_step(rec, q, pI, Y, philox.uniform(seed, sid, j, DRAW_ACCEPT),
+                                  philox.uniform(seed, sid, j, DRAW_RESIDUAL))
         elif scheme == "WIS0":
             Z = truncated.truncated_step(rec, q, dists, X, seed, sid, j, omega0, wis_s)
         else:
