@@ -59,24 +59,32 @@ def parse():
 # ----------------------------------------------------------------- accounting
 
 
-def walk_accounting(tokens, model_ids, out_tokens, acc, V, esize):
+def walk_accounting(tokens, model_ids, out_tokens, acc, V, esize, scheme="WIS", omega0=20):
     """Rows the walk consumed per sequence, replayed from the outputs:
-    returns (vocab_rows, algorithmic_bytes) summed over the batch."""
+    returns (vocab_rows, algorithmic_bytes) summed over the batch.  A depth
+    verifies its target row and one row per distinct draft model (vocab-rows);
+    the truncated alphabet reads only the target row in full and each draft
+    row at the at most omega0 tokens of Omega_0, which is what its bytes count."""
     B, K, L = tokens.shape
     mids = np.asarray(model_ids)
     rows = 0
+    point = 0      # WIS0: draft logits read at Omega_0
     for b in range(B):
         valid = np.arange(K)
         for j in range(int(acc[b]) + 1):
             if j == L:
                 rows += 1
                 break
-            rows += 1 + len(np.unique(mids[valid]))
+            d = len(np.unique(mids[valid]))
+            rows += 1 + d
+            point += d
             z = out_tokens[b, j]
             valid = valid[tokens[b, valid, j] == z]
             if len(valid) == 0:
                 break
     per_seq_io = 4 * (K * L + (1 + K) + (L + 1) + 1)
+    if scheme == "WIS0":
+        return rows, (rows - point) * V * esize + point * min(omega0, V) * esize + B * per_seq_io
     return rows, rows * V * esize + B * per_seq_io
 
 
@@ -186,7 +194,7 @@ def oracle_rate(w, scheme, seconds, seqs=None, omega0=20):
         o, a, recs = oracle_verify(*host, scheme, spec.verify_seed, seq_ids=[b], omega0=omega0)
         t_total += time.perf_counter() - t0
         out = np.asarray(o[b])[None]
-        r, _ = walk_accounting(host[3], w.model_ids, out, np.array([a[b]]), spec.V, es)
+        r, _ = walk_accounting(host[3], w.model_ids, out, np.array([a[b]]), spec.V, es, scheme, omega0)
         rows += r
         done.append(b)
         outs[b] = (o[b], a[b], recs[b])
@@ -334,7 +342,7 @@ def main():
     tok = w.tokens.cpu().numpy()
     o_tok = out_tokens.cpu().numpy()
     o_acc = out_acc.cpu().numpy()
-    rows, abytes = walk_accounting(tok, w.model_ids, o_tok, o_acc, spec.V, es)
+    rows, abytes = walk_accounting(tok, w.model_ids, o_tok, o_acc, spec.V, es, scheme, args.omega0)
     rows_all, _, ms = combine_ranks(rows, abytes, ms_own, world, dev)
     value = rows_all / (ms * 1e-3)
     achieved = abytes / (ms_own * 1e-3) / 1e9   # this rank's kernel against one GPU's peak

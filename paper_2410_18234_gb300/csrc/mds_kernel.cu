@@ -1114,29 +1114,20 @@ struct Kernel {
   // truncated alphabet).
   __device__ void depth_stats(bool cand) {
     const int nr = S.nrows;
+    if constexpr (SCHEME == MDS_WIS0) {
+      // the truncated draft laws p_d 1[Omega_0] / p_d(Omega_0) do not involve
+      // the draft rows' normalisers: only the target row is streamed
+      if (p.cand_cap > 0) {
+        stats_pass<1, true>(0);
+        return;
+      }
+    }
     if (cand && nr <= kFastRows && p.cand_cap > 0) {
       switch (nr) {
-        case 1: if constexpr (SCHEME == MDS_WIS0) { stats_pass<1, true>(0); return; } break;
         case 2: stats_pass<2, true>(0); return;
         case 3: stats_pass<3, true>(0); return;
         case 4: stats_pass<4, true>(0); return;
         default: break;
-      }
-    }
-    if constexpr (SCHEME == MDS_WIS0) {
-      if (p.cand_cap > 0) {
-        // more draft rows than one pass holds: the draft rows first (a pass
-        // without a list clears it), then the target with its list
-        for (int r0 = 1; r0 < nr; r0 += 4) {
-          switch (min(4, nr - r0)) {
-            case 1: stats_pass<1, false>(r0); break;
-            case 2: stats_pass<2, false>(r0); break;
-            case 3: stats_pass<3, false>(r0); break;
-            default: stats_pass<4, false>(r0); break;
-          }
-        }
-        stats_pass<1, true>(0);
-        return;
       }
     }
     for (int r0 = 0; r0 < nr; r0 += 4) {
@@ -2335,11 +2326,19 @@ struct Kernel {
       const float q = in0 ? prob_of(l, S.M[0], S.c[0], S.invZ[0]) : 0.f;
       const float pa = warp_sum(q);
       const float qt = (in0 && pa > 0.f) ? __fdiv_rn(q, pa) : 0.f;
-      // draft laws of this depth's rows restricted to Omega_0, renormalised
+      // draft laws of this depth's rows restricted to Omega_0, renormalised:
+      // point loads of the draft logits at Omega_0, exponents against their
+      // own maximum (the rows' full normalisers cancel)
       for (int r = 1; r < S.nrows; ++r) {
-        const float pr = in0 ? prob_row(r, id) : 0.f;
-        const float P = warp_sum(pr);
-        cm_e[r * p.cand_cap + lane] = (P > 0.f) ? __fdiv_rn(pr, P) : 0.f;
+        const float lr = in0 ? E::global(S.gptr[r], id) : kNegInf;
+        float ref = lr;
+#pragma unroll
+        for (int o = 16; o; o >>= 1) ref = fmaxf(ref, __shfl_xor_sync(FULL, ref, o));
+        const float cr = S.c[r];
+        const float e = (in0 && ref > kNegInf) ? ex2(__fmaf_rn(lr, cr, -__fmul_rn(ref, cr))) : 0.f;
+        const float P = warp_sum(e);
+        if (lane == 0 && rank == 0 && P != P) atomicOr(p.status, MDS_ST_NONFINITE);
+        cm_e[r * p.cand_cap + lane] = (P > 0.f) ? __fdiv_rn(e, P) : 0.f;
       }
       __syncwarp();
       // kept inputs: valid branches (branch order) whose token lies in Omega_0
