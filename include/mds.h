@@ -106,6 +106,13 @@ typedef struct {
   int omega0;      /* |Omega_0| for MDS_WIS0, 1..MDS_MAX_OMEGA0 (0: 20; the paper's
                       runs use 10 to 50, Section 5, Table "Effect of LP
                       Truncation and Alphabet Truncation")                    */
+  int acc_prob;    /* 1: out_diag[b][j][2] holds the residual mass R = sum_k
+                      max(0, q_k - p_I(k)) at every visited depth below L, so
+                      that 1 - R = sum_k min(q_k, p_I(k)) is the depth's
+                      acceptance probability (Theorem 1's objective for the
+                      depth's draft laws); costs one more pass over the rows
+                      at accepted depths.  0: R only after a rejection (0 when
+                      accepted).  Used by MDS_SINGLE, MDS_IS and MDS_WIS.     */
 } mds_config;
 
 /* Create a context on CUDA device `device`.  Allocates the context's device
@@ -131,7 +138,8 @@ int mds_create(mds_ctx** out, const mds_config* cfg, int device);
  *                  correction or bonus token), -1 after them
  *   out_accept_len [B] int32 in [0, L]: accepted draft positions
  *   out_diag       optional [B][L+1][4] float32: per depth q(Y), p_I(Y), the
- *                  residual mass (0 if accepted) and Y; NULL to skip
+ *                  residual mass (0 if accepted, unless acc_prob) and Y; NULL
+ *                  to skip
  * Pointers must be aligned to the element size; rows whose byte length is a
  * multiple of 16 at 16-byte-aligned bases are fetched with bulk copies.
  * Plain IS supports at most MDS_MAX_IS_MODELS distinct draft models

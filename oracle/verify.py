@@ -95,7 +95,7 @@ def inverse_cdf(r, u):
 class DepthRecord:
     """Per-(sequence, depth) diagnostics."""
 
-    __slots__ = ("j", "Y", "Z", "ratio", "u_acc", "accepted", "margins", "band", "qY", "pIY", "in_S")
+    __slots__ = ("j", "Y", "Z", "ratio", "u_acc", "accepted", "margins", "band", "qY", "pIY", "in_S", "R")
 
     def __init__(self, j):
         self.j = j
@@ -109,6 +109,7 @@ class DepthRecord:
         self.qY = float("nan")
         self.pIY = float("nan")
         self.in_S = False
+        self.R = float("nan")   # residual mass sum max(0, q - p_I); 1 - R = sum min(q, p_I)
 
     def note(self, name, value, threshold):
         prev = self.margins.get(name, np.inf)
@@ -125,6 +126,8 @@ def _speculative_step(rec, q, pI, Y, u_acc, u_res):
     rec.pIY = float(pI[Y])
     rec.ratio = float(ratio)
     rec.u_acc = float(u_acc)
+    # Theorem 1: the step accepts with probability sum_k min(q_k, p_I(k)) = 1 - R
+    rec.R = float(np.maximum(0.0, q - pI).sum())
     acc_prob = min(1.0, ratio)
     rec.note("accept", abs(u_acc - acc_prob), BAND_ACCEPT)
     if u_acc < acc_prob:

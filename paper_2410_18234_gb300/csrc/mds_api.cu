@@ -168,6 +168,7 @@ int mds_create(mds_ctx** out, const mds_config* cfg, int device) {
   if (c.is_h == 0.f) c.is_h = 0.25f;
   if (c.omega0 == 0) c.omega0 = 20;
   if (c.omega0 < 1 || c.omega0 > MDS_MAX_OMEGA0) return MDS_EINVAL;
+  if (c.acc_prob != 0 && c.acc_prob != 1) return MDS_EINVAL;
   if (c.max_B < 1 || c.K < 1 || c.K > MDS_MAX_K || c.L < 1 || c.L > MDS_MAX_L || c.V < 1 || c.V > (1 << 24))
     return MDS_ESHAPE;
   if (c.dtype != MDS_F32 && c.dtype != MDS_BF16) return MDS_EINVAL;
@@ -248,6 +249,7 @@ static int verify_impl(mds_ctx* ctx, const void* target_logits, const void* cons
   p.V = c.V;
   p.wis_s = c.wis_s;
   p.omega0 = c.omega0;
+  p.acc_prob = c.acc_prob;
   p.is_h = c.is_h;
   p.n_models = n_models;
   p.tma_ok = tma_ok ? 1 : 0;

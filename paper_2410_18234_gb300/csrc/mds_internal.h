@@ -35,6 +35,7 @@ struct Params {
   int esize;                           // bytes per logit
   int wis_s;
   int omega0;                          // |Omega_0| bound M of MDS_WIS0
+  int acc_prob;                        // 1: residual mass R at accepted depths too
   float is_h;
   int cn;                              // CTAs per cluster
   int slice;                           // tokens per CTA (multiple of 8)

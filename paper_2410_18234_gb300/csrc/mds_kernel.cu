@@ -2559,10 +2559,14 @@ struct Kernel {
         // Algorithm 1 on Y
         const float uacc = draw_uniform(p.seed, b, j, kDrawAccept);
         const float ratio = pIY > 0.f ? __fdiv_rn(qY, pIY) : kPosInf;
-        if (uacc < fminf(1.f, ratio)) {
+        const bool acc = uacc < fminf(1.f, ratio);
+        if (acc && !p.acc_prob) {
           Z = Y;
         } else {
-          const float ures = draw_uniform(p.seed, b, j, kDrawResidual);
+          // the residual mass R = sum max(0, q - p_I) and, after a rejection,
+          // the draw from it; with acc_prob an accepted depth computes R too
+          // (1 - R = sum min(q, p_I), the depth's acceptance probability)
+          const float ures = acc ? 0.f : draw_uniform(p.seed, b, j, kDrawResidual);
           float tot;
           bool done = false;
           if constexpr (SCHEME == MDS_WIS) {
@@ -2599,7 +2603,9 @@ struct Kernel {
                 ures, &tot);
           }
           Rdiag = tot;
-          if (Z < 0) {
+          if (acc) {
+            Z = Y;
+          } else if (Z < 0) {
             if (tid == 0) atomicOr(p.status, MDS_ST_ZERO_RESID);
             Z = sample_cdf(
                 1u,

@@ -48,6 +48,7 @@ extern "C" int mds_verify_noalloc(const mds_config* cfg_in, int device, const vo
   if (c.is_h == 0.f) c.is_h = 0.25f;
   if (c.omega0 == 0) c.omega0 = 20;
   if (c.omega0 < 1 || c.omega0 > MDS_MAX_OMEGA0) return MDS_EINVAL;
+  if (c.acc_prob != 0 && c.acc_prob != 1) return MDS_EINVAL;
   if (c.max_B < 1 || c.K < 1 || c.K > MDS_MAX_K || c.L < 1 || c.L > MDS_MAX_L || c.V < 1 || c.V > (1 << 24))
     return MDS_ESHAPE;
   if (c.dtype != MDS_F32 && c.dtype != MDS_BF16) return MDS_EINVAL;
@@ -111,6 +112,7 @@ extern "C" int mds_verify_noalloc(const mds_config* cfg_in, int device, const vo
     p.V = c.V;
     p.wis_s = c.wis_s;
     p.omega0 = c.omega0;
+    p.acc_prob = c.acc_prob;
     p.is_h = c.is_h;
     p.bulk_ok = 1;
     p.n_models = n_models;

@@ -38,7 +38,7 @@ EXPORTS = ("mds_create", "mds_verify", "mds_verify_host", "mds_verify_noalloc", 
 class MdsConfig(ctypes.Structure):
     _fields_ = [("max_B", ctypes.c_int), ("K", ctypes.c_int), ("L", ctypes.c_int), ("V", ctypes.c_int),
                 ("dtype", ctypes.c_int), ("wis_s", ctypes.c_int), ("is_h", ctypes.c_float),
-                ("cluster", ctypes.c_int), ("omega0", ctypes.c_int)]
+                ("cluster", ctypes.c_int), ("omega0", ctypes.c_int), ("acc_prob", ctypes.c_int)]
 
 
 class MdsError(RuntimeError):
@@ -85,9 +85,9 @@ def error_string(code):
 # ----------------------------------------------------------- C entry points
 
 
-def mds_create(max_B, K, L, V, dtype="bf16", wis_s=5, is_h=0.25, cluster=0, device=0, omega0=0):
+def mds_create(max_B, K, L, V, dtype="bf16", wis_s=5, is_h=0.25, cluster=0, device=0, omega0=0, acc_prob=0):
     cfg = MdsConfig(int(max_B), int(K), int(L), int(V), DTYPES[dtype] if isinstance(dtype, str) else int(dtype),
-                    int(wis_s), float(is_h), int(cluster), int(omega0))
+                    int(wis_s), float(is_h), int(cluster), int(omega0), int(acc_prob))
     h = ctypes.c_void_p()
     rc = _lib.mds_create(ctypes.byref(h), ctypes.byref(cfg), int(device))
     if rc != MDS_OK:
@@ -153,12 +153,12 @@ def mds_verify_host(ctx, target, drafts, model_ids, tokens, temps, scheme, seed,
 
 def mds_verify_noalloc(max_B, K, L, V, target, drafts, model_ids, tokens, temps, scheme, seed, out_tokens,
                        out_accept, out_diag=None, stream=None, dtype="bf16", wis_s=5, is_h=0.25, cluster=0,
-                       device=0, omega0=0):
+                       device=0, omega0=0, acc_prob=0):
     """Context-free entry point for callers that cannot allocate device
     memory (see include/mds.h): the configuration is passed directly and the
     kernel's scratch is a static device array inside the library."""
     cfg = MdsConfig(int(max_B), int(K), int(L), int(V), DTYPES[dtype] if isinstance(dtype, str) else int(dtype),
-                    int(wis_s), float(is_h), int(cluster), int(omega0))
+                    int(wis_s), float(is_h), int(cluster), int(omega0), int(acc_prob))
     Kn = len(model_ids)
     B = int(tokens.shape[0])
     if stream is None:
@@ -197,11 +197,12 @@ def mds_destroy(ctx):
 class Verifier:
     """Owns one context; allocates outputs with torch on the context's device."""
 
-    def __init__(self, max_B, K, L, V, dtype="bf16", wis_s=5, is_h=0.25, cluster=0, device=0, omega0=0):
+    def __init__(self, max_B, K, L, V, dtype="bf16", wis_s=5, is_h=0.25, cluster=0, device=0, omega0=0,
+                 acc_prob=0):
         self.max_B, self.K, self.L, self.V = int(max_B), int(K), int(L), int(V)
         self.dtype = dtype
         self.device = torch.device("cuda", device)
-        self.ctx = mds_create(max_B, K, L, V, dtype, wis_s, is_h, cluster, device, omega0)
+        self.ctx = mds_create(max_B, K, L, V, dtype, wis_s, is_h, cluster, device, omega0, acc_prob)
 
     def verify(self, target, drafts, model_ids, tokens, temps, scheme, seed, diag=False, out=None, stream=None):
         B = int(tokens.shape[0])

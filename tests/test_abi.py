@@ -60,7 +60,7 @@ def test_create_rejects_bad_config_before_touching_a_device():
             mds.mds_create(**c)
         assert e.value.code == mds.MDS_ESHAPE
     for c in (dict(wis_s=9), dict(is_h=-1.0), dict(cluster=3), dict(dtype=7), dict(omega0=-2),
-              dict(omega0=mds.MDS_MAX_OMEGA0 + 1)):
+              dict(omega0=mds.MDS_MAX_OMEGA0 + 1), dict(acc_prob=2), dict(acc_prob=-1)):
         with pytest.raises(mds.MdsError) as e:
             mds.mds_create(4, 2, 4, 100, **c)
         assert e.value.code == mds.MDS_EINVAL

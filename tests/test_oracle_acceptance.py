@@ -1,0 +1,60 @@
+"""Pins for the per-depth acceptance probability the oracle records.
+
+Theorem 1: the two-step scheme accepts the intermediate token with
+probability sum_k min(q_k, p_I(k)) = 1 - R, R = sum_k max(0, q_k - p_I(k)).
+Checked against the single-draft closed form 1 - TV(p, q) (App. A), against
+Theorem 3's optimum for K = 2 i.i.d. drafts when the WIS LP is not truncated
+(s = |Omega|), and against the empirical accept rate of the sampler.
+"""
+import numpy as np
+import pytest
+
+from oracle import theory
+from oracle.verify import oracle_verify
+
+
+def _rows(V, B, K, L, seed, sigma=1.0):
+    rng = np.random.default_rng(seed)
+    row = rng.normal(0.0, 1.5, size=V)
+    tl = np.broadcast_to(row, (B, K, L + 1, V)).copy()
+    drow = row + rng.normal(0.0, sigma, size=V)
+    drafts = [np.broadcast_to(drow, (B, L, V)).copy() for _ in range(K)]
+    pd = np.exp(drow - drow.max())
+    pd /= pd.sum()
+    q = np.exp(row - row.max())
+    q /= q.sum()
+    tokens = rng.choice(V, size=(B, K, L), p=pd)
+    return tl, drafts, np.zeros(K, dtype=int), tokens, np.ones((B, 1 + K)), q, pd
+
+
+def test_single_draft_is_one_minus_tv():
+    tl, dr, mids, tok, temps, q, p = _rows(7, 4, 1, 1, seed=1)
+    _, _, recs = oracle_verify(tl, dr, mids, tok, temps, "single", seed=3)
+    for b in recs:
+        assert 1.0 - recs[b][0].R == pytest.approx(np.minimum(p, q).sum(), abs=1e-14)
+
+
+def test_untruncated_wis_attains_theorem3():
+    for seed in range(4):
+        V = 5
+        tl, dr, mids, tok, temps, q, p = _rows(V, 3, 2, 1, seed=seed)
+        _, _, recs = oracle_verify(tl, dr, mids, tok, temps, "WIS", seed=1, wis_s=V)
+        for b in recs:
+            if tok[b, 0, 0] == tok[b, 1, 0]:
+                continue    # one valid token value: the step is Algorithm 1 on p
+            assert 1.0 - recs[b][0].R == pytest.approx(theory.thm3_pstar(p, q), abs=1e-6)
+
+
+@pytest.mark.parametrize("scheme", ["WIS", "IS"])
+def test_accept_rate_matches(scheme):
+    """Same rows for every sequence, independent draws: the fraction of
+    accepted depth-0 steps estimates 1 - R (binomial 4 sigma)."""
+    V, B = 6, 4000
+    tl, dr, mids, tok, temps, q, p = _rows(V, B, 3, 1, seed=9)
+    _, _, recs = oracle_verify(tl, dr, mids, tok, temps, scheme, seed=17)
+    acc = np.array([recs[b][0].accepted for b in range(B)], dtype=float)
+    pacc = np.array([1.0 - recs[b][0].R for b in range(B)])
+    # p_I, hence R, depends on which draft values were drawn; the mean of the
+    # per-sequence acceptance probabilities is the expected rate
+    m = pacc.mean()
+    assert abs(acc.mean() - m) < 4.0 * np.sqrt(m * (1 - m) / B)
