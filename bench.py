@@ -48,6 +48,8 @@ def parse():
     ap.add_argument("--cluster", type=int, default=0)
     ap.add_argument("--omega0", type=int, default=20, help="|Omega_0| of the truncated-alphabet scheme WIS0")
     ap.add_argument("--B", type=int, default=0, help="override the batch (profiling on a small case)")
+    ap.add_argument("--K", type=int, default=0, help="override the branch count, keeping the first K branches' "
+                                                    "draft models (profiling on a small case)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-parity", action="store_true")
@@ -256,6 +258,8 @@ def main():
     spec = WORKLOADS[args.workload]
     if args.B:
         spec = spec.with_(B=args.B)
+    if args.K:
+        spec = spec.with_(K=args.K, model_ids=list(spec.model_ids)[:args.K])
     scheme = args.scheme or spec.schemes[0]
     es = 4 if spec.dtype == "f32" else 2
 
