@@ -403,7 +403,7 @@ def main():
                        "parallelism": f"sequence-sharded x{world}", "seed": spec.verify_seed},
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "peak_kind": peak_kind,
-                         "traffic": recorded_traffic(spec.name, scheme),
+                         "traffic": None if (args.B or args.K) else recorded_traffic(spec.name, scheme),
                          "algorithmic_bytes_per_launch": int(abytes), "kernel": "verify_kernel"},
             "cpu_baseline": cpu,
             "e2e": e2e,
