@@ -21,6 +21,7 @@ the value is the sum over ranks divided by the slowest rank's time.
 import argparse
 import hashlib
 import json
+import re
 import os
 import subprocess
 import sys
@@ -155,10 +156,16 @@ def hbm_peak():
 
 
 def kernel_source_hash():
+    """Hash of the library's code with comments and blank lines removed, so
+    that recorded counters survive edits to comments only."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2410_18234_gb300", "csrc")
     for name in sorted(os.listdir(csrc)):
-        h.update(open(os.path.join(csrc, name), "rb").read())
+        text = open(os.path.join(csrc, name), encoding="utf-8").read()
+        text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+        text = re.sub(r"//[^\n]*", "", text)
+        lines = [ln.rstrip() for ln in text.splitlines() if ln.strip()]
+        h.update(name.encode() + b"\0" + "\n".join(lines).encode())
     return h.hexdigest()[:16]
 
 

@@ -7,11 +7,14 @@
 //   1. streams its slice of the target row and of one row per distinct draft
 //      model through a small shared-memory ring (cp.async.bulk with mbarrier
 //      completion), computing the temperature-softmax statistics online and,
-//      for the weighted scheme, collecting the candidate tokens; one exchange
-//      over distributed shared memory combines the cluster,
+//      for the weighted schemes, collecting the candidate tokens; one exchange
+//      over distributed shared memory combines the cluster (the truncated
+//      alphabet streams the target row only: its draft laws on Omega_0 need
+//      no draft normaliser),
 //   2. runs the importance step of the selected scheme (Definition 1 /
 //      Theorem 1) -- for the weighted scheme on the candidate list alone
-//      whenever that list provably holds every stage's Omega_1,
+//      whenever that list provably holds every stage's Omega_1, for the
+//      truncated alphabet on Omega_0 read off the same list (Section 4),
 //   3. applies Algorithm 1 (accept with probability min(1, q(Y)/p_I(Y)), else
 //      an inverse-CDF draw from max(0, q - p_I) in token order, streaming the
 //      rows again, typically from L2), and
