@@ -31,7 +31,7 @@ def _softmax64(logits, t):
     return e / e.sum()
 
 
-def _case(V, model_ids, seed):
+def _case(V, model_ids, seed, n=N):
     K, L = len(model_ids), 1
     g = torch.Generator(device="cpu").manual_seed(seed)
     row = (3.0 * torch.randn(V, generator=g)).to(torch.bfloat16)
@@ -41,14 +41,14 @@ def _case(V, model_ids, seed):
     t_target, t_draft = 1.0, [1.1, 0.8, 1.3][:n_models]
     temps = torch.tensor([t_target] + [t_draft[m] for m in model_ids], dtype=torch.float32)
     # each branch draws its token from its own model's law, independently per sequence
-    tokens = torch.empty(N, K, L, dtype=torch.int32)
+    tokens = torch.empty(n, K, L, dtype=torch.int32)
     for k, m in enumerate(model_ids):
         p = torch.from_numpy(_softmax64(drows[m].float().numpy(), t_draft[m]))
-        tokens[:, k, 0] = torch.multinomial(p, N, replacement=True, generator=g).to(torch.int32)
-    target = row.to(DEV).view(1, 1, 1, V).expand(N, K, L + 1, V).contiguous()
-    drafts = [drows[m].to(DEV).view(1, 1, V).expand(N, L, V).contiguous() for m in model_ids]
+        tokens[:, k, 0] = torch.multinomial(p, n, replacement=True, generator=g).to(torch.int32)
+    target = row.to(DEV).view(1, 1, 1, V).expand(n, K, L + 1, V).contiguous()
+    drafts = [drows[m].to(DEV).view(1, 1, V).expand(n, L, V).contiguous() for m in model_ids]
     q = _softmax64(row.float().numpy(), t_target)
-    return target, drafts, tokens.to(DEV), temps.to(DEV).view(1, -1).expand(N, -1).contiguous(), q
+    return target, drafts, tokens.to(DEV), temps.to(DEV).view(1, -1).expand(n, -1).contiguous(), q
 
 
 def _coarse_tv(z, q):
@@ -71,5 +71,21 @@ def test_first_token_follows_the_target(V):
         assert z.min() >= 0 and z.max() < V
         tv = _coarse_tv(z, q)
         assert tv < 4.0 / np.sqrt(N), (scheme, tv)
+    assert v.status()[0] == 0
+    v.close()
+
+
+def test_first_token_follows_the_target_at_a_million_draws():
+    """N = 2^20 draws (threshold 4/sqrt(N) = 0.0039) for the two weighted
+    schemes on V = 257."""
+    n = 1 << 20
+    model_ids = [0, 0, 1, 1]
+    target, drafts, tokens, temps, q = _case(257, model_ids, seed=11, n=n)
+    v = mds.Verifier(n, len(model_ids), 1, 257, dtype="bf16", omega0=5)
+    for scheme in ("WIS", "WIS0"):
+        out, acc, _ = v.verify(target, drafts, model_ids, tokens, temps, scheme, seed=99)
+        torch.cuda.synchronize()
+        tv = _coarse_tv(out[:, 0].cpu().numpy().astype(np.int64), q)
+        assert tv < 4.0 / np.sqrt(n), (scheme, tv)
     assert v.status()[0] == 0
     v.close()
