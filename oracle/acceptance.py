@@ -1,0 +1,98 @@
+"""Oracle: acceptance probability of each scheme on one row (analytic).
+
+TEST INFRASTRUCTURE ONLY (see ``oracle/__init__``).  Plain fp64 numpy.
+
+For a target law q and the valid branches' draft laws, the probability that
+a depth accepts one of the draft tokens:
+
+single, IS, WIS   Theorem 1: sum_k min(q_k, p_I(k)) with p_I the law of the
+                  intermediate token (the draft law itself; the Laplace
+                  identity of ``is_laplace``; the pairwise stage chain of
+                  ``wis``).
+SpecTr            the sequential-rejection reading: 1 - prod_i R_i, R_i the
+                  residual mass left after round i.
+optimal           Theorem 3 for K = 2 i.i.d. drafts and Remark 2's
+                  conjectured form for K > 2 (``theory.pstar_sorted``), the
+                  ceiling of any token-level selection rule.
+
+Running the module prints these for depth 0 of a few sequences of every
+named synthetic workload (the counterpart of the paper's Table 2 on the
+stand-in rows):  python -m oracle.acceptance
+"""
+import numpy as np
+
+from . import enum, is_laplace, theory
+
+
+def scheme_acceptance(q, dists, mids, scheme, s=5, is_h=0.25):
+    """Acceptance probability of ``scheme`` for target q and the valid
+    branches' draft laws ``dists`` (model ids ``mids``)."""
+    q = np.asarray(q, dtype=np.float64)
+    if scheme == "single" or len(dists) == 1:
+        return float(np.minimum(q, dists[0]).sum())
+    if scheme == "WIS":
+        pI = enum.wis_stages(q, dists, s)[-1].pI
+        return float(np.minimum(q, pI).sum())
+    if scheme == "IS":
+        rows, counts = {}, {}
+        for d, m in zip(dists, mids):
+            rows[m] = d
+            counts[m] = counts.get(m, 0) + 1
+        return float(np.minimum(q, is_laplace.is_law(q, rows, counts, is_h)).sum())
+    if scheme == "SpecTr":
+        qi, reject = q.copy(), 1.0
+        for p in dists:
+            r = np.maximum(0.0, qi - p)
+            R = float(r.sum())
+            reject *= R
+            if R > 0:
+                qi = r / R
+        return 1.0 - reject
+    raise ValueError(scheme)
+
+
+def optimal_acceptance(q, p, K):
+    """Theorem 3 (K = 2) / Remark 2's conjecture (K > 2) for i.i.d. drafts."""
+    return theory.pstar_sorted(p, q, K)
+
+
+def _softmax(x, t):
+    z = np.asarray(x, dtype=np.float64) / t
+    e = np.exp(z - z.max())
+    return e / e.sum()
+
+
+def table(names=None, seqs=(0, 1, 2, 3)):
+    """Rows of (workload, sequence, K, single, IS, WIS, SpecTr, optimal) at
+    depth 0; IS is skipped above 60000 tokens (its quadrature costs V x T)."""
+    from synth import WORKLOADS, make_workload
+    out = []
+    for name in names or list(WORKLOADS):
+        spec = WORKLOADS[name].with_(B=max(seqs) + 1)
+        w = make_workload(spec, device="cpu")
+        for b in seqs:
+            temps = w.temps[b].double().numpy()
+            q = _softmax(w.target[b, 0, 0].float().numpy(), temps[0])
+            dists = [_softmax(w.drafts[k, b, 0].float().numpy(), temps[1 + k]) for k in range(spec.K)]
+            mids = list(spec.model_ids)
+            row = {"workload": name, "b": b, "K": spec.K}
+            for sch in ("single", "IS", "WIS", "SpecTr"):
+                if sch == "IS" and spec.V > 60000:
+                    row[sch] = None
+                    continue
+                row[sch] = scheme_acceptance(q, dists, mids, sch)
+            iid = len(set(mids)) == 1
+            row["optimal"] = optimal_acceptance(q, dists[0], spec.K) if iid else None
+            out.append(row)
+    return out
+
+
+if __name__ == "__main__":
+    import sys
+    rows = table(sys.argv[1:] or None)
+    print("| workload | b | K | single | IS | WIS (s = 5) | SpecTr reading | optimal (Thm 3 / Remark 2) |")
+    print("|---|---|---|---|---|---|---|---|")
+    f = lambda v: "—" if v is None else f"{v:.4f}"   # noqa: E731
+    for r in rows:
+        print(f"| {r['workload']} | {r['b']} | {r['K']} | {f(r['single'])} | {f(r['IS'])} | {f(r['WIS'])} | "
+              f"{f(r['SpecTr'])} | {f(r['optimal'])} |")

@@ -115,6 +115,29 @@ def remark2_pstar(p, q, K=2):
     return best
 
 
+def pstar_sorted(p, q, K=2):
+    """Theorem 3 / Remark 2 on any vocabulary size: the minimum over S of
+    sum_S q - (sum_S p)^K + 1 (for K = 2 the optimum of Theorem 3; for K > 2
+    Remark 2's conjectured form), by a scan over V + 1 sets.
+
+    Why a scan suffices: t^K is convex, so -t^K = min_l [(K-1) l^K - K l^(K-1) t]
+    (its tangent lines), and the minimum over S and l can be taken in either
+    order.  For a fixed l the inner minimum of sum_{s in S} (q_s - K l^(K-1) p_s)
+    takes exactly the tokens with q_s / p_s below K l^(K-1) (ties contribute
+    0), so some optimal S is a prefix of the tokens sorted by the ratio
+    q_s / p_s (tokens with p_s = 0 last).  This is a derivation from the
+    paper's closed form, not an algorithm the paper states; it is pinned
+    against the 2^V-subset minimum."""
+    p = np.asarray(p, dtype=np.float64)
+    q = np.asarray(q, dtype=np.float64)
+    with np.errstate(divide="ignore", invalid="ignore"):
+        ratio = np.where(p > 0, q / np.where(p > 0, p, 1.0), np.inf)
+    order = np.argsort(ratio, kind="stable")
+    Q = np.concatenate([[0.0], np.cumsum(q[order])])
+    P = np.concatenate([[0.0], np.cumsum(p[order])])
+    return float(np.min(Q - P ** K) + 1.0)
+
+
 def thm2_condition(p, q, tol=0.0):
     """Theorem 2, Eq. (conj): sum_S q >= (sum_S p)^2 for every subset S.
     S = Omega holds with equality (1 >= 1) and is skipped so that rounding of

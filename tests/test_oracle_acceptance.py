@@ -58,3 +58,35 @@ def test_accept_rate_matches(scheme):
     # per-sequence acceptance probabilities is the expected rate
     m = pacc.mean()
     assert abs(acc.mean() - m) < 4.0 * np.sqrt(m * (1 - m) / B)
+
+
+def test_analytic_evaluator_matches_the_walk_and_the_ceiling():
+    """oracle.acceptance: single / IS / WIS equal 1 - R of the walk's depth 0;
+    every scheme stays below Theorem 3's optimum for K = 2 i.i.d. drafts (the
+    optimum over all token-level selection rules)."""
+    from oracle import acceptance
+    for seed in range(5):
+        V, B = 6, 2
+        tl, dr, mids, tok, temps, q, p = _rows(V, B, 2, 1, seed=40 + seed)
+        best = theory.thm3_pstar(p, q)
+        assert acceptance.optimal_acceptance(q, p, 2) == pytest.approx(best, abs=1e-12)
+        for scheme in ("single", "IS", "WIS", "SpecTr"):
+            val = acceptance.scheme_acceptance(q, [p, p], [0, 0], scheme)
+            assert val <= best + 1e-9, (scheme, val, best)
+            if scheme == "SpecTr":
+                continue
+            _, _, recs = oracle_verify(tl, dr, mids, tok, temps, scheme, seed=1)
+            for b in recs:
+                if scheme != "single" and tok[b, 0, 0] == tok[b, 1, 0]:
+                    continue   # one distinct token: the walk's step is Algorithm 1 on p
+                assert 1.0 - recs[b][0].R == pytest.approx(val, abs=1e-9), (scheme, b)
+
+
+def test_spectr_evaluator_matches_its_sampler():
+    from oracle import acceptance
+    V, B = 5, 4000
+    tl, dr, mids, tok, temps, q, p = _rows(V, B, 3, 1, seed=3)
+    _, _, recs = oracle_verify(tl, dr, mids, tok, temps, "SpecTr", seed=8)
+    rate = np.mean([recs[b][0].accepted for b in range(B)])
+    want = acceptance.scheme_acceptance(q, [p, p, p], [0, 0, 0], "SpecTr")
+    assert abs(rate - want) < 4.0 * np.sqrt(want * (1 - want) / B)

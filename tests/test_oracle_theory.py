@@ -120,3 +120,39 @@ def test_figure2_optimal_curves_reach_one_on_the_predicted_range():
                 assert pstar == pytest.approx(1.0, abs=1e-12)
             elif q2 < lo - 1e-9 or q2 > hi + 1e-9:
                 assert pstar < 1 - 1e-9
+
+
+def test_sorted_scan_equals_subset_minimum():
+    """The ratio-sorted prefix scan gives Theorem 3's subset minimum (K = 2)
+    and Remark 2's conjectured form (K = 3, 4) exactly, on random rows with
+    zeros in p and in q."""
+    rng = np.random.default_rng(31)
+    for _ in range(60):
+        V = int(rng.integers(1, 10))
+        p = rng.dirichlet(np.full(V, 0.6))
+        q = rng.dirichlet(np.full(V, 0.6))
+        if V > 2:
+            p[rng.integers(0, V)] = 0.0
+            q[rng.integers(0, V)] = 0.0
+            p /= p.sum()
+            q /= q.sum()
+        assert theory.pstar_sorted(p, q) == pytest.approx(theory.thm3_pstar(p, q), abs=1e-12)
+        for K in (3, 4):
+            assert theory.pstar_sorted(p, q, K) == pytest.approx(theory.remark2_pstar(p, q, K), abs=1e-12)
+
+
+def test_sorted_scan_example1_and_large_rows():
+    """Example 1's interval (P* = 1 on [0.25, 0.75]) and, on a 50000-token
+    row, the sandwich 1 - TV(p, q) <= P*(K=2) <= 1 (two drafts do no worse
+    than one)."""
+    p = np.array([0.5, 0.5])
+    for q1, want_one in ((0.2, False), (0.25, True), (0.5, True), (0.75, True), (0.8, False)):
+        v = theory.pstar_sorted(p, np.array([q1, 1 - q1]))
+        assert (abs(v - 1.0) < 1e-12) == want_one
+    rng = np.random.default_rng(2)
+    lq = 4.0 * rng.standard_normal(50000)
+    lp = lq + rng.standard_normal(50000)
+    q = np.exp(lq - lq.max()); q /= q.sum()
+    p = np.exp(lp - lp.max()); p /= p.sum()
+    v = theory.pstar_sorted(p, q)
+    assert np.minimum(p, q).sum() - 1e-12 <= v <= 1.0 + 1e-12
