@@ -11,6 +11,10 @@ single, IS, WIS   Theorem 1: sum_k min(q_k, p_I(k)) with p_I the law of the
                   ``wis``).
 SpecTr            the sequential-rejection reading: 1 - prod_i R_i, R_i the
                   residual mass left after round i.
+WIS0              the truncated alphabet (Section 4): p_a = q(Omega_0) times
+                  the expectation, over which branches land in Omega_0, of
+                  the inner WIS acceptance sum_{Omega_0} min(q~, p_I) of the
+                  kept inputs (their draft laws truncated to Omega_0).
 optimal           Theorem 3 for K = 2 i.i.d. drafts and Remark 2's
                   conjectured form for K > 2 (``theory.pstar_sorted``), the
                   ceiling of any token-level selection rule.
@@ -19,9 +23,11 @@ Running the module prints these for depth 0 of a few sequences of every
 named synthetic workload (the counterpart of the paper's Table 2 on the
 stand-in rows):  python -m oracle.acceptance
 """
+import itertools
+
 import numpy as np
 
-from . import enum, is_laplace, theory
+from . import enum, is_laplace, theory, truncated
 
 
 def scheme_acceptance(q, dists, mids, scheme, s=5, is_h=0.25):
@@ -49,6 +55,34 @@ def scheme_acceptance(q, dists, mids, scheme, s=5, is_h=0.25):
                 qi = r / R
         return 1.0 - reject
     raise ValueError(scheme)
+
+
+def truncated_acceptance(q, dists, M, s=5):
+    """Probability that a truncated-alphabet depth outputs an accepted draft
+    token (kept by the p_a test), for target q and the valid branches' draft
+    laws ``dists`` in branch order."""
+    q = np.asarray(q, dtype=np.float64)
+    om = truncated.omega0(q, M)
+    if len(om) == 0:
+        return 0.0
+    pa = float(q[om].sum())
+    qt = q[om] / pa
+    inside = [float(np.asarray(d, dtype=np.float64)[om].sum()) for d in dists]
+    laws = [truncated.truncate(d, om) for d in dists]
+    total = 0.0
+    for pattern in itertools.product((0, 1), repeat=len(dists)):
+        pr = 1.0
+        for hit, pin in zip(pattern, inside):
+            pr *= pin if hit else 1.0 - pin
+        kept = [i for i, hit in enumerate(pattern) if hit and laws[i] is not None]
+        if pr == 0.0 or not kept:
+            continue
+        if len(kept) == 1:
+            pI = laws[kept[0]]
+        else:
+            pI = enum.wis_stages(qt, [laws[i] for i in kept], s)[-1].pI
+        total += pr * float(np.minimum(qt, pI).sum())
+    return pa * total
 
 
 def optimal_acceptance(q, p, K):
@@ -81,6 +115,7 @@ def table(names=None, seqs=(0, 1, 2, 3)):
                     row[sch] = None
                     continue
                 row[sch] = scheme_acceptance(q, dists, mids, sch)
+            row["WIS0"] = truncated_acceptance(q, dists, 20)
             iid = len(set(mids)) == 1
             row["optimal"] = optimal_acceptance(q, dists[0], spec.K) if iid else None
             out.append(row)
@@ -90,9 +125,9 @@ def table(names=None, seqs=(0, 1, 2, 3)):
 if __name__ == "__main__":
     import sys
     rows = table(sys.argv[1:] or None)
-    print("| workload | b | K | single | IS | WIS (s = 5) | SpecTr reading | optimal (Thm 3 / Remark 2) |")
-    print("|---|---|---|---|---|---|---|---|")
+    print("| workload | b | K | single | IS | WIS (s = 5) | WIS0 (M = 20) | SpecTr reading | optimal (Thm 3 / Remark 2) |")
+    print("|---|---|---|---|---|---|---|---|---|")
     f = lambda v: "—" if v is None else f"{v:.4f}"   # noqa: E731
     for r in rows:
         print(f"| {r['workload']} | {r['b']} | {r['K']} | {f(r['single'])} | {f(r['IS'])} | {f(r['WIS'])} | "
-              f"{f(r['SpecTr'])} | {f(r['optimal'])} |")
+              f"{f(r['WIS0'])} | {f(r['SpecTr'])} | {f(r['optimal'])} |")

@@ -90,3 +90,35 @@ def test_spectr_evaluator_matches_its_sampler():
     rate = np.mean([recs[b][0].accepted for b in range(B)])
     want = acceptance.scheme_acceptance(q, [p, p, p], [0, 0, 0], "SpecTr")
     assert abs(rate - want) < 4.0 * np.sqrt(want * (1 - want) / B)
+
+
+def test_truncated_evaluator_matches_enumeration():
+    """WIS0's acceptance by its membership-pattern formula equals a direct
+    enumeration of the draft tuple: for each tuple, the kept inputs' stage
+    chain selects Y with law beta(. | tuple), Algorithm 1 against q~ accepts
+    with min(1, q~(Y)/p_I(Y)), and the p_a test keeps it."""
+    from oracle import acceptance, enum, truncated
+    rng = np.random.default_rng(12)
+    for V, K, M in ((5, 2, 3), (5, 3, 2), (6, 3, 4), (4, 2, 4)):
+        q = rng.dirichlet(np.full(V, 0.7))
+        rows = [rng.dirichlet(np.full(V, 0.7)) for _ in range(2)]
+        dists = [rows[k % 2] for k in range(K)]
+        om = truncated.omega0(q, M)
+        where = {int(t): i for i, t in enumerate(om)}
+        pa = q[om].sum()
+        qt = q[om] / pa
+        laws = [truncated.truncate(d, om) for d in dists]
+        want = 0.0
+        for x, pr in enum._tuples(dists):
+            kept = [i for i in range(K) if int(x[i]) in where]
+            if pr == 0.0 or not kept:
+                continue
+            xs = [where[int(x[i])] for i in kept]
+            if len(kept) == 1:
+                beta, pI = {xs[0]: 1.0}, laws[kept[0]]
+            else:
+                stages = enum.wis_stages(qt, [laws[i] for i in kept], 2)
+                beta, pI = enum.wis_beta(stages, xs), stages[-1].pI
+            want += pr * sum(by * min(1.0, qt[y] / pI[y]) for y, by in beta.items())
+        got = acceptance.truncated_acceptance(q, dists, M, s=2)
+        assert got == pytest.approx(pa * want, abs=1e-12)
