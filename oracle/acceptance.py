@@ -21,7 +21,7 @@ optimal           Theorem 3 for K = 2 i.i.d. drafts and Remark 2's
 
 Running the module prints these for depth 0 of a few sequences of every
 named synthetic workload (the counterpart of the paper's Table 2 on the
-stand-in rows):  python -m oracle.acceptance
+stand-in rows):  python -m oracle.acceptance [--top-p=0.95] [workload ...]
 """
 import itertools
 
@@ -96,9 +96,10 @@ def _softmax(x, t):
     return e / e.sum()
 
 
-def table(names=None, seqs=(0, 1, 2, 3)):
-    """Rows of (workload, sequence, K, single, IS, WIS, SpecTr, optimal) at
-    depth 0; IS is skipped above 60000 tokens (its quadrature costs V x T)."""
+def table(names=None, seqs=(0, 1, 2, 3), top_p=1.0):
+    """Rows of (workload, sequence, K, single, IS, WIS, WIS0, SpecTr,
+    optimal) at depth 0, every row top-p filtered first when top_p < 1
+    (Section 5); IS is skipped above 60000 tokens (its quadrature costs V x T)."""
     from synth import WORKLOADS, make_workload
     out = []
     for name in names or list(WORKLOADS):
@@ -108,6 +109,9 @@ def table(names=None, seqs=(0, 1, 2, 3)):
             temps = w.temps[b].double().numpy()
             q = _softmax(w.target[b, 0, 0].float().numpy(), temps[0])
             dists = [_softmax(w.drafts[k, b, 0].float().numpy(), temps[1 + k]) for k in range(spec.K)]
+            if top_p < 1.0:
+                q = truncated.top_filter(q, top_p=top_p)
+                dists = [truncated.top_filter(d, top_p=top_p) for d in dists]
             mids = list(spec.model_ids)
             row = {"workload": name, "b": b, "K": spec.K}
             for sch in ("single", "IS", "WIS", "SpecTr"):
@@ -124,7 +128,11 @@ def table(names=None, seqs=(0, 1, 2, 3)):
 
 if __name__ == "__main__":
     import sys
-    rows = table(sys.argv[1:] or None)
+    args = sys.argv[1:]
+    tp = 1.0
+    if args and args[0].startswith("--top-p="):
+        tp = float(args.pop(0).split("=", 1)[1])
+    rows = table(args or None, top_p=tp)
     print("| workload | b | K | single | IS | WIS (s = 5) | WIS0 (M = 20) | SpecTr reading | optimal (Thm 3 / Remark 2) |")
     print("|---|---|---|---|---|---|---|---|---|")
     f = lambda v: "—" if v is None else f"{v:.4f}"   # noqa: E731
