@@ -24,7 +24,8 @@ truncated  the truncated-alphabet scheme (Section 4) and top-k / top-p
 sorted_lp  the truncated LP with the sorted rule on Omega_2 (Section 4 Eq.
          heur, Algorithm 2, App. I): no device counterpart yet.
 acceptance  analytic acceptance probability of each scheme on one row, and the
-         optimum of Theorem 3 / Remark 2 for any vocabulary size.
+         optimum of Theorem 3 (K = 2; Remark 2's conjectured form for K > 2)
+         for any vocabulary size.
 
 Parity status: every function here is pinned by a ``-m "not gpu"`` test
 (see tests/test_oracle_*.py) except the SpecTr-style sequential-rejection
