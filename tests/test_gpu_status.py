@@ -6,7 +6,6 @@ the outputs stay valid tokens.  B above the context's max_B and an unknown
 scheme id are rejected before any launch.  None of these faults the GPU:
 each anomaly is checked by the kernel before the value is used.
 """
-import numpy as np
 import pytest
 import torch
 

@@ -5,7 +5,6 @@ than Omega_0 (Omega_0 = the whole vocabulary), more draft models than one
 statistics pass holds, every cluster size, rows fetched with plain loads,
 peaked targets, and sampled sequences of the full-size workloads.
 """
-import numpy as np
 import pytest
 import torch
 
