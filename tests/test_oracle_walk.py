@@ -83,14 +83,16 @@ def _tv(counts, q):
     return 0.5 * np.abs(counts / n - q).sum(), n
 
 
-@pytest.mark.parametrize("scheme,N", [("single", 12000), ("WIS", 12000), ("SpecTr", 12000), ("IS", 2500)])
+@pytest.mark.parametrize("scheme,N", [("single", 12000), ("WIS", 12000), ("SpecTr", 12000), ("IS", 2500),
+                                      ("WIS0", 12000), ("WISsort", 12000)])
 def test_walk_emits_target_model_samples(scheme, N):
     """Z_0 ~ q(root); given a continued walk through z, Z_1 ~ q(z); after two
     accepted positions the bonus ~ q(z0, z1).  TV below 4/sqrt(n) per law."""
     V, K, L = 3, 2, 2
     rng = np.random.default_rng(5 + len(scheme))
     target, drafts, mids, tokens, temps, row_t = _tree_inputs(N, V, K, L, rng)
-    out, acc, _ = oracle_verify(target, drafts, mids, tokens, temps, scheme, seed=99, wis_s=2)
+    # WIS0 with |Omega_0| = 2 < V: a two-token inner stage and the keep / replace step at every depth
+    out, acc, _ = oracle_verify(target, drafts, mids, tokens, temps, scheme, seed=99, wis_s=2, omega0=2)
 
     def q_of(prefix):
         x = row_t(prefix)
