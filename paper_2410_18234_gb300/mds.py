@@ -113,6 +113,34 @@ def _ids(model_ids, K):
     return arr
 
 
+def check_buffers(K, L, V, dtype, target, drafts, model_ids, tokens, temps, out_tokens, out_accept,
+                  out_diag=None, placement=None):
+    """Shapes, element types, contiguity and placement ("cuda", "cpu" or None
+    to skip) of one call's tensors.  The C ABI takes bare pointers and the
+    sizes from its configuration, so a tensor of the wrong shape would be read
+    or written out of bounds: the binding rejects it first (MdsError with
+    MDS_ESHAPE or MDS_EINVAL)."""
+    st = TORCH_DTYPES[DTYPES[dtype] if isinstance(dtype, str) else int(dtype)]
+    if len(model_ids) != K or len(drafts) < K:
+        raise MdsError(MDS_EINVAL, f"{len(model_ids)} model ids and {len(drafts)} draft buffers for K = {K}")
+    B = int(tokens.shape[0]) if tokens.dim() >= 1 else -1
+    want = [("target", target, (B, K, L + 1, V), st), ("tokens", tokens, (B, K, L), torch.int32),
+            ("temperatures", temps, (B, 1 + K), torch.float32),
+            ("out_tokens", out_tokens, (B, L + 1), torch.int32), ("out_accept_len", out_accept, (B,), torch.int32)]
+    want += [(f"draft_logits[{k}]", drafts[k], (B, L, V), st) for k in range(K)]
+    if out_diag is not None:
+        want.append(("out_diag", out_diag, (B, L + 1, 4), torch.float32))
+    for name, t, shape, dt in want:
+        if tuple(t.shape) != shape:
+            raise MdsError(MDS_ESHAPE, f"{name} has shape {tuple(t.shape)}, expected {shape}")
+        if t.dtype != dt:
+            raise MdsError(MDS_EINVAL, f"{name} has type {t.dtype}, expected {dt}")
+        if not t.is_contiguous():
+            raise MdsError(MDS_EINVAL, f"{name} is not contiguous")
+        if placement is not None and (t.device.type == "cuda") != (placement == "cuda"):
+            raise MdsError(MDS_EINVAL, f"{name} is on {t.device}, expected {placement} memory")
+
+
 def mds_verify(ctx, target, drafts, model_ids, tokens, temps, scheme, seed, out_tokens, out_accept,
                out_diag=None, stream=None):
     """Device-buffer entry point.  ``drafts`` is a sequence of K device
@@ -157,6 +185,8 @@ def mds_verify_noalloc(max_B, K, L, V, target, drafts, model_ids, tokens, temps,
     """Context-free entry point for callers that cannot allocate device
     memory (see include/mds.h): the configuration is passed directly and the
     kernel's scratch is a static device array inside the library."""
+    check_buffers(int(K), int(L), int(V), dtype, target, drafts, model_ids, tokens, temps, out_tokens, out_accept,
+                  out_diag, "cuda")
     cfg = MdsConfig(int(max_B), int(K), int(L), int(V), DTYPES[dtype] if isinstance(dtype, str) else int(dtype),
                     int(wis_s), float(is_h), int(cluster), int(omega0), int(acc_prob))
     Kn = len(model_ids)
@@ -212,6 +242,8 @@ class Verifier:
             out_diag = torch.empty(B, self.L + 1, 4, dtype=torch.float32, device=self.device) if diag else None
         else:
             out_tokens, out_accept, out_diag = out
+        check_buffers(self.K, self.L, self.V, self.dtype, target, drafts, model_ids, tokens, temps, out_tokens,
+                      out_accept, out_diag, "cuda")
         mds_verify(self.ctx, target, drafts, model_ids, tokens, temps, scheme, seed, out_tokens, out_accept,
                    out_diag, stream)
         return out_tokens, out_accept, out_diag
@@ -224,6 +256,8 @@ class Verifier:
             out_diag = None
         else:
             out_tokens, out_accept, out_diag = out
+        check_buffers(self.K, self.L, self.V, self.dtype, target, drafts, model_ids, tokens, temps, out_tokens,
+                      out_accept, out_diag, "cpu")
         mds_verify_host(self.ctx, target, drafts, model_ids, tokens, temps, scheme, seed, out_tokens, out_accept,
                         out_diag, stream)
         return out_tokens, out_accept, out_diag
