@@ -90,3 +90,25 @@ def test_binding_config_matches_the_header():
         assert ids["MDS_" + name.upper()] == sid
     assert int(re.search(r"#define MDS_MAX_OMEGA0 (\d+)", text).group(1)) == mds.MDS_MAX_OMEGA0
     assert int(re.search(r"#define MDS_ST_OMEGA0 (\d+)u", text).group(1)) == mds.MDS_ST_OMEGA0
+
+
+def test_header_compiles_as_c_and_matches_the_binding_layout(tmp_path):
+    """include/mds.h is plain C (C99), and mds_config's size and field
+    offsets as a C compiler lays them out equal the ctypes mirror's."""
+    import shutil
+    import subprocess
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("no C compiler")
+    from paper_2410_18234_gb300 import mds
+    fields = [f[0] for f in mds.MdsConfig._fields_]
+    prints = "".join(f'printf("%zu\\n", offsetof(mds_config, {f}));' for f in fields)
+    src = tmp_path / "layout.c"
+    src.write_text('#include <stddef.h>\n#include <stdio.h>\n#include "mds.h"\n'
+                   'int main(void) { printf("%zu\\n", sizeof(mds_config)); ' + prints + " return 0; }\n")
+    exe = tmp_path / "layout"
+    subprocess.run([gcc, "-std=c99", "-Wall", "-Werror", "-I", os.path.join(ROOT, "include"), str(src), "-o",
+                    str(exe)], check=True)
+    got = [int(x) for x in subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout.split()]
+    assert got[0] == ctypes.sizeof(mds.MdsConfig)
+    assert got[1:] == [getattr(mds.MdsConfig, f).offset for f in fields]
