@@ -171,18 +171,23 @@ int mds_verify_host(mds_ctx* ctx, const void* target_logits, const void* const* 
  * serving loop whose memory is fixed at start-up, or under an allocator that
  * forbids growth after warm-up) and so cannot create a context.  It takes
  * the configuration directly and the same buffers as mds_verify (caller-
- * owned device memory; same layouts, alignment rules and return codes).  It
- * allocates nothing: the kernel's scratch (status word and work counter, 8
- * bytes) lives in a file-scope device array of MDS_NOALLOC_SCRATCH_BYTES that
- * every GPU loading the library holds until the process exits; a need beyond
- * that size is rejected with MDS_ESHAPE (the need does not grow with B, K, L
- * or V).  The first call on a device looks up that array's device address
- * and sets kernel attributes, so make it before any stream capture.  Every
- * call clears the scratch on `stream` and then launches; all calls share the
- * one array, so calls that overlap on the GPU race.  The status word is not
- * reported (use a context for mds_status).  The paper has no counterpart to
- * this entry point: it exists only for callers that cannot allocate. */
-#define MDS_NOALLOC_SCRATCH_BYTES 256
+ * owned device memory; same layouts, alignment rules and return codes) and
+ * runs the same kernel as mds_verify would for that configuration, so its
+ * outputs are the same.  It allocates nothing: the kernels' scratch (a status
+ * word, and for single, WIS and WIS0 the slice engine's control words, task
+ * ring, per-sequence state and slice records, which grow with B and with the
+ * number of slices per row, about V / 8192) lives in a file-scope device
+ * array of MDS_NOALLOC_SCRATCH_BYTES (8 MiB) that every GPU loading the
+ * library holds until the process exits; a call whose scratch exceeds it
+ * (for llama3-like rows, beyond roughly 900 sequences per call) is rejected
+ * with MDS_ESHAPE before any launch.  The first call on a device looks up
+ * that array's device address and sets kernel attributes, so make it before
+ * any stream capture.  Every call clears the parts of the scratch that must
+ * start at zero on `stream`, then launches; all calls share the one array,
+ * so calls that overlap on the GPU race.  The status word is not reported
+ * (use a context for mds_status).  The paper has no counterpart to this entry
+ * point: it exists only for callers that cannot allocate. */
+#define MDS_NOALLOC_SCRATCH_BYTES (8u << 20)
 int mds_verify_noalloc(const mds_config* cfg, int device, const void* target_logits,
                        const void* const* draft_logits, const int32_t* draft_model_id,
                        const int32_t* draft_tokens, const float* temperatures, int scheme,
@@ -194,8 +199,17 @@ int mds_verify_noalloc(const mds_config* cfg, int device, const void* target_log
  * static description of the highest set bit. */
 int mds_status(mds_ctx* ctx, const char** msg);
 
-/* Number of CTAs per sequence the context launches with (for reporting). */
+/* CTAs per sequence of the context's last launch (for reporting): the
+ * cluster size of the per-sequence engine, or 0 when the call ran on the
+ * slice-dataflow engine, where every CTA works on every sequence's slices. */
 int mds_cluster_size(const mds_ctx* ctx);
+
+/* Diagnostics of an instrumented build (compiled with MDS_PHASE_TIMERS; the
+ * default build returns MDS_EUNSUP): synchronises device `device`, copies
+ * up to n phase counters of the slice-dataflow engine (SM cycles summed over
+ * CTAs, and task and decision counts, in the order the library's source
+ * lists them) to cycles, clears them and returns how many counters exist. */
+int mds_phase_timers(int device, unsigned long long* cycles, int n);
 
 /* Static text for a return code. */
 const char* mds_error_string(int code);

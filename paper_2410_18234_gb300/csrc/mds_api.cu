@@ -5,6 +5,7 @@
 #include <mutex>
 #include <vector>
 
+#include "mds_flow.h"
 #include "mds_internal.h"
 
 struct mds_ctx {
@@ -24,6 +25,13 @@ struct mds_ctx {
   // staging buffers of mds_verify_host
   void* h_buf;
   size_t h_bytes;
+  // slice-dataflow engine: workspace (control words, task ring, per-sequence
+  // state and slice records; grown on demand, zero between launches) and the
+  // launch counter that tags the ring's entries
+  void* f_buf;
+  size_t f_bytes;
+  unsigned epoch;
+  int f_grid;
 };
 
 namespace {
@@ -57,15 +65,24 @@ int cuda_fail(cudaError_t e, const char* where) {
   return MDS_ECUDA;
 }
 
-bool configured[2] = {false, false};
+// Kernel attributes (dynamic shared memory limit, non-portable cluster size)
+// belong to a device's context: set once per (device, logit type), on the
+// current device.
+constexpr int kMaxDevices = 64;
+bool configured[kMaxDevices][2] = {};
 std::mutex config_mu;
 
 int ensure_configured(int dtype) {
+  int dev = 0;
+  const cudaError_t ge = cudaGetDevice(&dev);
+  if (ge != cudaSuccess) return cuda_fail(ge, "cudaGetDevice");
+  if (dev < 0 || dev >= kMaxDevices) return cuda_fail(cudaErrorInvalidDevice, "kernel configuration");
   std::lock_guard<std::mutex> lk(config_mu);
-  if (!configured[dtype]) {
-    const cudaError_t e = mds::configure_kernel(dtype);
+  if (!configured[dev][dtype]) {
+    cudaError_t e = mds::configure_kernel(dtype);
+    if (e == cudaSuccess) e = mds::flow::configure(dtype);
     if (e != cudaSuccess) return cuda_fail(e, "kernel configuration");
-    configured[dtype] = true;
+    configured[dev][dtype] = true;
   }
   return MDS_OK;
 }
@@ -188,6 +205,10 @@ int mds_create(mds_ctx** out, const mds_config* cfg, int device) {
   ctx->tickets = 0u;
   ctx->h_buf = nullptr;
   ctx->h_bytes = 0;
+  ctx->f_buf = nullptr;
+  ctx->f_bytes = 0;
+  ctx->epoch = 0u;
+  ctx->f_grid = mds::flow::grid_size(device);
   cudaError_t me = cudaMalloc(&ctx->work, 256);
   if (me == cudaSuccess) me = cudaMemset(ctx->work, 0, 256);
   if (me != cudaSuccess) {
@@ -195,6 +216,47 @@ int mds_create(mds_ctx** out, const mds_config* cfg, int device) {
     return cuda_fail(me, "workspace allocation");
   }
   *out = ctx;
+  return MDS_OK;
+}
+
+// The slice-dataflow engine serves single, WIS and WIS0 where its slice
+// geometry fits (every configuration of the benchmarks); the per-sequence
+// engine serves the rest.  Grows the context's workspace (zeroed) as needed.
+int flow_verify(mds_ctx* ctx, const void* target_logits, const void* const* draft_logits, const int8_t* model_of,
+                int n_models, const int32_t* draft_tokens, const float* temperatures, int scheme,
+                uint64_t philox_seed, int32_t* out_tokens, int32_t* out_accept_len, float* out_diag, int B,
+                void* stream, bool bulk_ok, bool aligned16) {
+  const mds_config& c = ctx->cfg;
+  mds::flow::Params p{};
+  if (!mds::flow_params(c, ctx->f_grid, scheme, model_of, n_models, bulk_ok, aligned16, p)) return mds::kNotServed;
+  const size_t total = mds::flow::workspace_bytes(p, c.max_B, ctx->f_grid);
+  DeviceGuard g(ctx->device);
+  if (total > ctx->f_bytes) {
+    // the previous buffer may still be in use by an earlier launch
+    if (ctx->f_buf) {
+      cudaDeviceSynchronize();
+      cudaFree(ctx->f_buf);
+    }
+    ctx->f_buf = nullptr;
+    ctx->f_bytes = 0;
+    cudaError_t e = cudaMalloc(&ctx->f_buf, total);
+    if (e == cudaSuccess) e = cudaMemset(ctx->f_buf, 0, total);
+    if (e != cudaSuccess) {
+      if (ctx->f_buf) cudaFree(ctx->f_buf);
+      ctx->f_buf = nullptr;
+      return cuda_fail(e, "dataflow workspace allocation");
+    }
+    ctx->f_bytes = total;
+  }
+  mds::flow::carve_workspace(p, static_cast<char*>(ctx->f_buf), c.max_B, ctx->f_grid);
+  mds::flow_buffers(p, target_logits, draft_logits, draft_tokens, temperatures, out_tokens, out_accept_len, out_diag,
+                    B, philox_seed);
+  p.status = ctx->work;
+  ctx->epoch = (ctx->epoch + 1u == 0u) ? 1u : ctx->epoch + 1u;
+  p.epoch = ctx->epoch;
+  const cudaError_t le = mds::flow::launch(p, ctx->f_grid, static_cast<cudaStream_t>(stream));
+  if (le != cudaSuccess) return cuda_fail(le, "dataflow kernel launch");
+  ctx->last_cn = 0;
   return MDS_OK;
 }
 
@@ -231,6 +293,11 @@ static int verify_impl(mds_ctx* ctx, const void* target_logits, const void* cons
     p.drafts[k] = static_cast<const char*>(draft_logits[k]);
   }
   if (scheme == MDS_IS && n_models > MDS_MAX_IS_MODELS) return MDS_EUNSUP;
+  {
+    const int frc = flow_verify(ctx, target_logits, draft_logits, p.model_of, n_models, draft_tokens, temperatures,
+                                scheme, philox_seed, out_tokens, out_accept_len, out_diag, B, stream, bulk_ok, tma_ok);
+    if (frc != mds::kNotServed) return frc;
+  }
   p.dtype = c.dtype;
   int rc = geometry(ctx, scheme, n_models, p);
   if (rc != MDS_OK) return rc;
@@ -395,10 +462,20 @@ int mds_status(mds_ctx* ctx, const char** msg) {
 
 int mds_cluster_size(const mds_ctx* ctx) { return ctx ? ctx->last_cn : 0; }
 
+int mds_phase_timers(int device, unsigned long long* cycles, int n) {
+  if (!cycles || n < 0) return MDS_EINVAL;
+  DeviceGuard g(device);
+  const int r = mds::flow::read_phase_timers(cycles, n);
+  if (r == -2) return MDS_EUNSUP;
+  if (r < 0) return cuda_fail(cudaGetLastError(), "mds_phase_timers");
+  return r;
+}
+
 void mds_destroy(mds_ctx* ctx) {
   if (!ctx) return;
   DeviceGuard g(ctx->device);
   if (ctx->h_buf) cudaFree(ctx->h_buf);
+  if (ctx->f_buf) cudaFree(ctx->f_buf);
   if (ctx->work) cudaFree(ctx->work);
   delete ctx;
 }
@@ -414,4 +491,42 @@ int launch_geometry(const mds_config& cfg, int device, int scheme, int n_models,
   return geometry(&view, scheme, n_models, p);
 }
 int prepare_kernels(int dtype) { return ensure_configured(dtype); }
+int record_cuda_error(cudaError_t e, const char* where) { return cuda_fail(e, where); }
+
+bool flow_params(const mds_config& c, int grid, int scheme, const int8_t* model_of, int n_models, bool bulk_ok,
+                 bool aligned16, flow::Params& p) {
+  if (scheme != MDS_SINGLE && scheme != MDS_WIS && scheme != MDS_WIS0) return false;
+  if (grid <= 0 || c.cluster != 0 || c.max_B > 65535) return false;   // ring entries hold 16-bit ids
+  p = flow::Params{};
+  p.scheme = scheme;
+  p.dtype = c.dtype;
+  p.esize = esize_of(c.dtype);
+  p.K = c.K;
+  p.L = c.L;
+  p.V = c.V;
+  p.B = c.max_B;
+  p.wis_s = c.wis_s;
+  p.omega0 = c.omega0;
+  p.acc_prob = c.acc_prob;
+  p.n_models = n_models;
+  for (int k = 0; k < c.K; ++k) p.model_of[k] = model_of[k];
+  if (!flow::plan_geometry(p, grid)) return false;
+  p.aligned = aligned16 ? 1 : 0;
+  p.bulk = (bulk_ok && aligned16) ? 1 : 0;
+  return true;
+}
+
+void flow_buffers(flow::Params& p, const void* target_logits, const void* const* draft_logits,
+                  const int32_t* draft_tokens, const float* temperatures, int32_t* out_tokens,
+                  int32_t* out_accept_len, float* out_diag, int B, uint64_t seed) {
+  p.target = static_cast<const char*>(target_logits);
+  for (int k = 0; k < p.K; ++k) p.drafts[k] = static_cast<const char*>(draft_logits[k]);
+  p.tokens = draft_tokens;
+  p.temps = temperatures;
+  p.out_tokens = out_tokens;
+  p.out_accept = out_accept_len;
+  p.out_diag = out_diag;
+  p.B = B;
+  p.seed = seed;
+}
 }  // namespace mds

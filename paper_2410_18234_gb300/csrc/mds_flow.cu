@@ -1,0 +1,2386 @@
+// Slice-dataflow engine for batched multi-draft speculative verification on
+// GB300 (sm_103a): schemes single, weighted importance sampling (WIS) and the
+// truncated alphabet (WIS0).
+//
+// Every row the walk visits (the target row and one row per distinct draft
+// model at a depth, the target row at the bonus depth) is cut into slices of
+// T tokens.  One pass of one sequence is ns slice tasks over the same rows.
+// The grid is persistent (every CTA of the launch resident): in each CTA one
+// scheduler warp takes task numbers from a global counter, waits for the
+// task's publication in a ring in global memory, reads the sequence's pass
+// descriptor and bulk-copies the task's slice of every row of the pass into
+// one of two shared-memory buffers (cp.async.bulk, mbarrier completion).  The
+// eight compute warps reduce the slice to a record in global memory:
+//   stats    row maxima and exp sums (2^fma(l, c, -round(m c)) against the
+//            slice maximum m) and, for the weighted schemes, the slice's
+//            largest target logits (the candidate list) with every row's logit
+//            there; the sums leave the list out, so every later mass is a sum
+//            of positive terms;
+//   resid    the residual mass sum max(0, q - p_I) of Algorithm 1;
+//   replace  the target mass outside Omega_0 (truncated alphabet);
+//   full     a full-vocabulary stage of the weighted scheme: the slice's top-s
+//            keys q - a b with a and b, and the Omega_2 masses of the rest;
+//   bonus    the target row's maximum and sum at depth L.
+// The CTA whose task completes a pass (a per-sequence counter) runs the
+// decision for that sequence: it combines the records in slice order, runs the
+// importance step (the WIS stages on the merged candidate list, Omega_1 by
+// the keys q - a b, the stage LP, Remark 4's pairwise stages), Algorithm 1's
+// accept test, and the inverse-CDF search of a residual draw (slice by the
+// records, token by one re-read of that slice), then advances the walk and
+// publishes the sequence's next pass.  Decisions depend only on the data and
+// the Philox draws, never on which CTA takes a task, so results are
+// bit-reproducible.  Every wait is bounded in time; a wait that gives up sets
+// MDS_ST_TIMEOUT and an abort flag on which every CTA leaves, after waiting
+// for its own copies in flight.
+#include <cuda_bf16.h>
+
+#include "mds_device.cuh"
+#include "mds_flow.h"
+
+namespace mds {
+namespace flow {
+namespace {
+
+using namespace mds::dev;
+
+constexpr int kCW = 8;                 // compute warps
+constexpr int kCT = kCW * 32;          // compute threads
+constexpr int kBlock = kCT + 32;       // + the scheduler warp
+constexpr int kNBuf = 2;               // slice buffers per CTA
+constexpr int kCandCap = 1024;         // candidate tokens one slice may set aside
+constexpr int kListMax = 64;           // candidate list length at most
+constexpr int kHdr = 2 * kMaxRows + 2; // record: (max, sum) per row, tau, list length
+constexpr int kTopF = 8;               // per-thread candidates of a full stage (>= MDS_MAX_S)
+constexpr int kTopW = 8;               // thread maxima each warp offers to the slice's threshold
+constexpr unsigned long long kWaitNs = 2000000000ull;   // 2 s bound on every wait
+constexpr unsigned FULLM = 0xffffffffu;
+static_assert(kHdr % 4 == 0, "record header keeps 16-byte alignment");
+static_assert(kTopF >= MDS_MAX_S, "full-stage candidates");
+
+enum : int { kNone = 0, kStats = 1, kResid = 2, kBonus = 3, kFull = 4, kReplace = 5 };
+
+// Phase-timer slots (SM cycles summed over CTAs, or counts).
+enum : int {
+  kPhKernel = 0,        // time in the kernel (per CTA, summed)
+  kPhWaitFull,          // compute warps waiting for a loaded slice
+  kPhTaskList,          // stats tasks with the candidate list
+  kPhTaskStats,         // stats tasks without it (and the bonus row)
+  kPhTaskResid,         // residual and replace tasks
+  kPhTaskFull,          // full-vocabulary stage tasks
+  kPhDecStats,          // stats decisions (all of it)
+  kPhDecCombine,        //   of which: combining records and the list merge
+  kPhDecStages,         //   of which: the WIS stages on the list
+  kPhDecResid,          // residual and replace decisions (with the search)
+  kPhDecFull,           // full-stage decisions
+  kPhDecBonus,          // bonus decisions
+  kPhPush,              // publishing the next pass
+  kPhSchedPoll,         // scheduler waiting for a published task
+  kPhSchedEmpty,        // scheduler waiting for a free buffer
+  kPhTasks,             // count: slice tasks
+  kPhDecisions,         // count: decisions
+  kPhaseN
+};
+
+// ------------------------------------------------------------------ state
+
+struct FRow {
+  const char* ptr;     // row start (token 0)
+  float c;             // log2(e) / temperature
+  float M, invZ;       // row maximum and inverse normaliser (after the stats decision)
+  float gamma;         // WIS: coefficient of this draft row in the generic law
+};
+struct __align__(16) FPass {   // what the slice tasks of a pass read
+  int kind, j, nrows, nstream;
+  int list, rb, nspec, all0;
+  float cut;
+  int pad0, pad1, pad2;
+  FRow row[kMaxRows];          // target, then one row per distinct draft model of the valid branches
+  int spec_id[kMaxSpecial];    // WIS: tokens with an explicit law value (every Omega_1 so far)
+  float spec_val[kMaxSpecial];
+  int pad3[2];
+};
+static_assert(sizeof(FPass) % 16 == 0, "pass descriptor copies in 16-byte chunks");
+struct __align__(16) FWalk {   // decision state of a sequence between passes
+  unsigned valid;              // valid branches at the current depth
+  int stage, A;                // WIS full stages: next stage, current stage input
+  int Y;                       // intermediate token
+  float qY, pIY;
+  int acc;                     // accept test passed
+  float ures;                  // uniform of the pending inverse-CDF draw
+  float R;                     // residual mass (diagnostics)
+  int Yp;                      // WIS0: output of the inner step on Omega_0 (-1: none)
+  int Ydiag;
+  int zres;                    // the pending draw is the zero-residual fallback (sample q)
+  int pad[4];
+};
+static_assert(sizeof(FWalk) % 16 == 0, "walk state copies in 16-byte chunks");
+struct __align__(16) FSeq {
+  FPass P;
+  FWalk W;
+};
+
+struct FDesc {
+  FPass P;
+  int b, slice, exit, pad;
+};
+
+struct Cand {  // full-stage candidate: larger key first, then smaller token id
+  float key;
+  int id;
+  float a, b;
+};
+#define CAND_NONE Cand{kNegInf, 0x7fffffff, 0.f, 0.f}
+__device__ __forceinline__ bool better(float ka, int ia, float kb, int ib) {
+  return ka > kb || (ka == kb && ia < ib);
+}
+
+struct DState {                // the decision's working state (shared memory)
+  FPass P;
+  FWalk W;
+  int nv;
+  int vbr[MDS_MAX_K], X[MDS_MAX_K], vrow[MDS_MAX_K];
+  // candidate list (token-id order)
+  int n, cand_all;
+  float cand_q, cand_tau;
+  int cm_id[kListMax];
+  float cm_l0[kListMax];
+  float cm_e[kListRowsMax][kListMax];
+  float cm_a[kListMax];
+  int cm_sp[kListMax];
+  float pc[kListRowsMax];
+  int ksl[kMaxSlicesList];
+  int fin_s[kListMax], fin_i[kListMax];
+  // stage
+  int om[MDS_MAX_S];
+  float om_q[MDS_MAX_S], om_a[MDS_MAX_S], om_b[MDS_MAX_S], om_x[MDS_MAX_S];
+  float A2, B2;
+  int Y, fast_ok;
+  Cand fin[kTopF];
+  // search
+  int seg, cross, lastp, tok;
+  float run;
+  // truncated alphabet
+  int k_lane[MDS_MAX_K], k_row[MDS_MAX_K];
+  int o0_n, o0_all, o0_Yp;
+  float o0_cut, o0_pa, o0_R;
+  float rtot;
+  unsigned tbase;
+};
+
+struct FShared {
+  uint64_t full[kNBuf], empty[kNBuf];
+  FDesc desc[kNBuf];
+  float red[kCW * 2 * kMaxRows];
+  float mrow[kMaxRows];
+  float wth[kCW];
+  int ncand, last, issued, consumed;
+  float theta, addtau;
+  unsigned tkey[kCW * 8];       // the warps' largest thread maxima (order-preserving keys)
+  float add[kMaxRows];
+  uint32_t bitmap[64];         // one bit per 16-byte unit of a slice holding a special token
+  Cand wcand[kCW * kTopF];
+  Cand blk[kTopF];
+  float Rs[kMaxSlices];        // slice masses of a search
+  float hm[kMaxSlices];        // slice maxima of the bonus draw
+  int flag_ok, flag_ab;
+#ifdef MDS_PHASE_TIMERS
+  unsigned long long tm[kPhaseN];
+#endif
+  DState D;
+};
+
+// ------------------------------------------------------------------ memory helpers
+
+__device__ __forceinline__ unsigned long long ld_acquire(const unsigned long long* a) {
+  unsigned long long v;
+  asm volatile("ld.acquire.gpu.u64 %0, [%1];" : "=l"(v) : "l"(a) : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_release(unsigned long long* a, unsigned long long v) {
+  asm volatile("st.release.gpu.u64 [%0], %1;" ::"l"(a), "l"(v) : "memory");
+}
+__device__ __forceinline__ unsigned ld_relaxed(const unsigned* a) {
+  unsigned v;
+  asm volatile("ld.relaxed.gpu.u32 %0, [%1];" : "=r"(v) : "l"(a) : "memory");
+  return v;
+}
+__device__ __forceinline__ unsigned long long now_ns() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+__device__ __forceinline__ void cbar() { asm volatile("bar.sync 1, %0;" ::"n"(kCT) : "memory"); }
+
+// 16-byte chunk copies of state between global (L2, coherent) and shared memory.
+__device__ __forceinline__ void copy_in(void* dst, const void* src, int bytes, int t, int nt) {
+  const int4* s = reinterpret_cast<const int4*>(src);
+  int4* d = reinterpret_cast<int4*>(dst);
+  for (int i = t; i < bytes / 16; i += nt) d[i] = __ldcg(s + i);
+}
+__device__ __forceinline__ void copy_out(void* dst, const void* src, int bytes, int t, int nt) {
+  const int4* s = reinterpret_cast<const int4*>(src);
+  int4* d = reinterpret_cast<int4*>(dst);
+  for (int i = t; i < bytes / 16; i += nt) __stcg(d + i, s[i]);
+}
+
+// ------------------------------------------------------------------ phase timers
+// Built with -DMDS_PHASE_TIMERS, every CTA accumulates SM cycles per phase
+// (thread 0 of the compute warps, lane 0 of the scheduler warp) and adds them
+// to g_phase when it leaves; mds_phase_timers() reads and clears them.
+// Without it the macros vanish.
+#ifdef MDS_PHASE_TIMERS
+__device__ unsigned long long g_phase[kPhaseN];
+#define PT_T0(v) const long long v = clock64()
+#define PT_ADD(i, v)                                             \
+  do {                                                           \
+    if ((threadIdx.x & 0xff) == 0) S.tm[i] += (unsigned long long)(clock64() - (v)); \
+  } while (0)
+#define PT_CNT(i)                                 \
+  do {                                            \
+    if ((threadIdx.x & 0xff) == 0) S.tm[i] += 1ull; \
+  } while (0)
+#else
+#define PT_T0(v)
+#define PT_ADD(i, v)
+#define PT_CNT(i)
+#endif
+
+// ------------------------------------------------------------------ the engine
+
+template <int DT>
+struct Eng {
+  using E = Elt<DT>;
+  static constexpr int VE = E::VE;
+
+  const Params& p;
+  FShared& S;
+  char* bufs;     // kNBuf x kBufBytes
+  int* cid;       // candidate ids
+  float* cl;      // candidate target logits
+  int* crank;     // candidate ranks
+  int* cord;      // candidates ranked past the list, in rank order
+
+  __device__ __forceinline__ unsigned long long tag_of(unsigned t) const {
+    return ((unsigned long long)p.epoch << 32) | (unsigned long long)(t + 1u);
+  }
+  __device__ __forceinline__ bool aborted() const { return ld_relaxed(&p.ctl[kCtlAbort]) != 0u; }
+  __device__ __forceinline__ void set_abort(unsigned bits) const {
+    atomicOr(p.status, bits);
+    atomicExch(&p.ctl[kCtlAbort], 1u);
+  }
+  __device__ __forceinline__ char* buf(int bi) const { return bufs + (size_t)bi * kBufBytes; }
+  __device__ __forceinline__ const char* srow(const char* b, int r) const { return b + (size_t)r * p.T * p.esize; }
+  __device__ __forceinline__ uint4 raw(const char* b, int r, int u) const {
+    return *reinterpret_cast<const uint4*>(srow(b, r) + 16 * u);
+  }
+  __device__ __forceinline__ float prob_row(const FPass& P, int r, int x) const {
+    return prob_of(E::global(P.row[r].ptr, x), P.row[r].M, P.row[r].c, P.row[r].invZ);
+  }
+  __device__ __forceinline__ float spec_lookup(const FPass& P, int tok, float fallback) const {
+    for (int i = 0; i < P.nspec; ++i)
+      if (P.spec_id[i] == tok) return P.spec_val[i];
+    return fallback;
+  }
+  // Point value of the current law p_I (WIS): explicit value of a special
+  // token, else sum_r gamma_r p_r(x) in row order.
+  __device__ float law_at(const FPass& P, int x) const {
+    float a = 0.f;
+    for (int r = 1; r < P.nrows; ++r)
+      if (P.row[r].gamma != 0.f) a = __fmaf_rn(P.row[r].gamma, prob_row(P, r, x), a);
+    return spec_lookup(P, x, a);
+  }
+
+  // -------------------------------------------------------------- planning
+  // Rows of depth j for the valid branches (the lowest valid branch's target
+  // row, then one row per distinct draft model in branch order) into *P (if
+  // given) and, if X is given, the valid branches, their tokens and rows.
+  // One thread.
+  __device__ void plan_rows(int b, int j, unsigned valid, bool bonus, FPass* P, int* nv, int* vbr, int* X,
+                            int* vrow) const {
+    const int K = p.K, L = p.L, V = p.V;
+    const int kstar = __ffs(valid) - 1;
+    if (P) {
+      P->row[0].ptr = p.target + ((((size_t)b * K + kstar) * (L + 1) + j) * (size_t)V) * p.esize;
+      float tq = p.temps[(size_t)b * (1 + K)];
+      if (!(tq > 0.f) || !(tq < kPosInf)) {
+        atomicOr(p.status, MDS_ST_BADTEMP);
+        tq = 1.f;
+      }
+      P->row[0].c = __fdiv_rn(kLog2e, tq);
+    }
+    int mrow[MDS_MAX_K];
+    for (int m = 0; m < MDS_MAX_K; ++m) mrow[m] = -1;
+    int nr = 1, n = 0;
+    if (!bonus) {
+      for (int k = 0; k < K; ++k) {
+        if (!(valid >> k & 1u)) continue;
+        const int m = p.model_of[k];
+        if (mrow[m] < 0) {
+          mrow[m] = nr;
+          if (P) {
+            P->row[nr].ptr = p.drafts[k] + (((size_t)b * L + j) * (size_t)V) * p.esize;
+            float td = p.temps[(size_t)b * (1 + K) + 1 + k];
+            if (!(td > 0.f) || !(td < kPosInf)) {
+              atomicOr(p.status, MDS_ST_BADTEMP);
+              td = 1.f;
+            }
+            P->row[nr].c = __fdiv_rn(kLog2e, td);
+          }
+          ++nr;
+        }
+        if (X) {
+          int x = p.tokens[((size_t)b * K + k) * L + j];
+          if (x < 0 || x >= V) {
+            atomicOr(p.status, MDS_ST_BADTOKEN);
+            x = 0;
+          }
+          vbr[n] = k;
+          X[n] = x;
+          vrow[n] = mrow[m];
+        }
+        ++n;
+      }
+    }
+    if (nv) *nv = n;
+    if (!P) return;
+    for (int r = 0; r < nr; ++r) {
+      P->row[r].M = 0.f;
+      P->row[r].invZ = 0.f;
+      P->row[r].gamma = 0.f;
+    }
+    P->nrows = nr;
+    P->j = j;
+    P->nspec = 0;
+    P->rb = 0;
+    P->cut = 0.f;
+    P->all0 = 0;
+    if (bonus) {
+      P->kind = kBonus;
+      P->nstream = 1;
+      P->list = 0;
+    } else {
+      P->kind = kStats;
+      if (p.scheme == MDS_WIS0) {
+        P->nstream = 1;
+        P->list = 1;
+      } else if (p.scheme == MDS_WIS) {
+        P->nstream = nr;
+        P->list = (n > 1 && nr <= kListRowsMax && p.ln > 0) ? 1 : 0;
+      } else {
+        P->nstream = min(2, nr);
+        P->list = 0;
+      }
+    }
+  }
+
+  // -------------------------------------------------------------- scheduler warp
+  __device__ bool wait_mbar(uint64_t* bar, uint32_t parity) const {
+    const unsigned long long t0 = now_ns();
+    for (int it = 0;; ++it) {
+      if (mbar_try_wait(bar, parity)) return true;
+      if ((it & 63) == 63 && now_ns() - t0 > kWaitNs) return false;
+    }
+  }
+
+  __device__ void scheduler() {
+    const int lane = threadIdx.x & 31;
+    const unsigned N0 = (unsigned)p.B * (unsigned)p.ns;
+    for (int k = 0;; ++k) {
+      const int bi = k % kNBuf;
+      FDesc& D = S.desc[bi];
+      // the compute warps released this buffer (lane 0 waits; bounded)
+      int ok = 1;
+      PT_T0(t_empty);
+      if (lane == 0 && k >= kNBuf) ok = wait_mbar(&S.empty[bi], ((k / kNBuf) - 1) & 1) ? 1 : 0;
+      PT_ADD(kPhSchedEmpty, t_empty);
+      ok = __shfl_sync(FULLM, ok, 0);
+      if (!ok) {
+        // the compute warps still hold the buffer: leave it untouched
+        if (lane == 0) set_abort(MDS_ST_TIMEOUT);
+        return;
+      }
+      unsigned t = 0;
+      int have = 0, b = 0, s = 0;
+      if (lane == 0 && !aborted()) {
+        t = atomicAdd(&p.ctl[kCtlHead], 1u);
+        if (t < N0) {
+          b = (int)(t / (unsigned)p.ns);
+          s = (int)(t % (unsigned)p.ns);
+          st_release(&p.ring_rtag[t % (unsigned)p.ring_cap], tag_of(t));
+          plan_rows(b, 0, (p.K >= 32) ? FULLM : ((1u << p.K) - 1u), false, &D.P, nullptr, nullptr, nullptr, nullptr);
+          have = 1;
+        } else {
+          const unsigned slot = t % (unsigned)p.ring_cap;
+          const unsigned long long want = tag_of(t);
+          const unsigned long long t0 = now_ns();
+          PT_T0(t_poll);
+          for (int it = 0;; ++it) {
+            if (ld_acquire(&p.ring_tag[slot]) == want) {
+              const unsigned pay = __ldcg(&p.ring_pay[slot]);
+              b = (int)(pay >> 16);
+              s = (int)(pay & 0xffffu);
+              st_release(&p.ring_rtag[slot], want);
+              have = 2;
+              break;
+            }
+            if (ld_relaxed(&p.ctl[kCtlDone]) >= (unsigned)p.B || aborted()) break;
+            if ((it & 15) == 15 && now_ns() - t0 > kWaitNs) {
+              set_abort(MDS_ST_TIMEOUT);
+              break;
+            }
+            __nanosleep(it < 16 ? 32 : 256);
+          }
+          PT_ADD(kPhSchedPoll, t_poll);
+        }
+      }
+      have = __shfl_sync(FULLM, have, 0);
+      b = __shfl_sync(FULLM, b, 0);
+      s = __shfl_sync(FULLM, s, 0);
+      if (have == 2) copy_in(&D.P, &reinterpret_cast<const FSeq*>(p.seq)[b].P, (int)sizeof(FPass), lane, 32);
+      if (lane == 0) {
+        D.b = b;
+        D.slice = s;
+        D.exit = have ? 0 : 1;
+      }
+      __syncwarp();
+      if (lane == 0) {
+        if (have && p.bulk) {
+          const int tok0 = s * p.T;
+          const int n = min(p.T, p.V - tok0);
+          const uint32_t bytes = (uint32_t)n * (uint32_t)p.esize;
+          fence_proxy_async();
+          mbar_expect_tx(&S.full[bi], bytes * (uint32_t)D.P.nstream);
+          for (int r = 0; r < D.P.nstream; ++r)
+            bulk_copy(buf(bi) + (size_t)r * p.T * p.esize, D.P.row[r].ptr + (size_t)tok0 * p.esize, bytes, &S.full[bi]);
+        } else {
+          mbar_arrive(&S.full[bi]);
+        }
+        S.issued = k + 1;
+      }
+      __syncwarp();
+      if (!have) return;
+    }
+  }
+
+  // -------------------------------------------------------------- slice loading (plain loads)
+  // Rows [0, R) of the slice [tok0, tok0 + n) into shared memory; units past
+  // n read -inf.  Used where bulk copies are not (mapped host memory, rows
+  // not 16-byte aligned) and by the search's re-read of one slice.
+  __device__ void load_plain(const FPass& P, int R, char* b, int tok0, int n) const {
+    const int U = (n + VE - 1) / VE;
+    for (int r = 0; r < R; ++r) {
+      const char* src = P.row[r].ptr + (size_t)tok0 * p.esize;
+      char* dst = b + (size_t)r * p.T * p.esize;
+      for (int u = threadIdx.x; u < U; u += kCT) {
+        uint4 x;
+        if (p.aligned) {
+          x = __ldg(reinterpret_cast<const uint4*>(src + 16 * (size_t)u));
+        } else {
+          uint32_t w[4];
+          if constexpr (DT == MDS_BF16) {
+            const unsigned short* s16 = reinterpret_cast<const unsigned short*>(src);
+#pragma unroll
+            for (int h = 0; h < 4; ++h) {
+              const int t0 = u * VE + 2 * h;
+              const uint32_t lo = (t0 < n) ? (uint32_t)__ldg(s16 + t0) : 0xff80u;
+              const uint32_t hi = (t0 + 1 < n) ? (uint32_t)__ldg(s16 + t0 + 1) : 0xff80u;
+              w[h] = lo | (hi << 16);
+            }
+          } else {
+            const float* s32 = reinterpret_cast<const float*>(src);
+#pragma unroll
+            for (int h = 0; h < 4; ++h) {
+              const int t0 = u * VE + h;
+              w[h] = (t0 < n) ? __float_as_uint(__ldg(s32 + t0)) : 0xff800000u;
+            }
+          }
+          x = make_uint4(w[0], w[1], w[2], w[3]);
+        }
+        *reinterpret_cast<uint4*>(dst + 16 * (size_t)u) = x;
+      }
+    }
+    cbar();
+  }
+
+  // One bit per 16-byte unit of the slice that holds a special token.
+  __device__ void build_bitmap(const FPass& P, int tok0, int n) const {
+    const int words = ((n + VE - 1) / VE + 31) / 32;
+    for (int i = threadIdx.x; i < words; i += kCT) S.bitmap[i] = 0u;
+    cbar();
+    for (int i = threadIdx.x; i < P.nspec; i += kCT) {
+      const int loc = P.spec_id[i] - tok0;
+      if (loc >= 0 && loc < n) atomicOr(&S.bitmap[(loc / VE) >> 5], 1u << ((loc / VE) & 31));
+    }
+    cbar();
+  }
+
+  // -------------------------------------------------------------- block reductions (fixed order)
+  // Sum over the compute threads: warp trees, then warps in order.  Every
+  // compute thread gets the result.
+  __device__ float block_sum(float v, float* scratch) const {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    v = warp_sum(v);
+    cbar();
+    if (lane == 0) scratch[warp] = v;
+    cbar();
+    float t = 0.f;
+#pragma unroll
+    for (int w = 0; w < kCW; ++w) t = __fadd_rn(t, scratch[w]);
+    return t;
+  }
+  __device__ float block_max(float v, float* scratch) const {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    v = warp_max(v);
+    cbar();
+    if (lane == 0) scratch[warp] = v;
+    cbar();
+    float t = kNegInf;
+#pragma unroll
+    for (int w = 0; w < kCW; ++w) t = fmaxf(t, scratch[w]);
+    return t;
+  }
+
+  // -------------------------------------------------------------- stats task
+  // R rows (compile time, at most kListRowsMax) with or without the candidate
+  // list.  Record: (max, sum) per row, tau (largest target logit of the slice
+  // outside its list), list length, then the list (larger target logit
+  // first, ties to the smaller id): ids, then each row's logits.
+  template <int R, bool LIST>
+  __device__ void stats_small(const FPass& P, const char* b, int tok0, int n, float* rec) {
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int U = (n + VE - 1) / VE;
+    const int LN = p.ln;
+    float c[R];
+#pragma unroll
+    for (int r = 0; r < R; ++r) c[r] = P.row[r].c;
+    // phase A: maxima
+    float tmax = kNegInf;
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      float mx = kNegInf;
+      for (int u = tid; u < U; u += kCT) mx = fmaxf(mx, E::unit_max(raw(b, r, u)));
+      if (r == 0) tmax = mx;
+      mx = warp_max(mx);
+      if (lane == 0) S.red[warp * kMaxRows + r] = mx;
+    }
+    if constexpr (LIST) {
+      // each warp's kTopW largest thread maxima (distinct tokens) ...
+      unsigned key = (tmax > kNegInf) ? ord_key(__fadd_rn(tmax, 0.f)) : 0u;
+      for (int t = 0; t < kTopW; ++t) {
+        const unsigned km = __reduce_max_sync(FULLM, key);
+        const unsigned who = __ballot_sync(FULLM, km != 0u && key == km);
+        if (lane == 0) S.tkey[warp * kTopW + t] = km;
+        if (who && lane == __ffs(who) - 1) key = 0u;
+      }
+    }
+    if (tid == 0) S.ncand = 0;
+    cbar();
+    if constexpr (LIST) {
+      // ... and theta = the LN-th largest of them: at least LN tokens of the
+      // slice are >= theta (-inf if fewer than LN thread maxima are finite)
+      if (warp == 0) {
+        unsigned k2[kTopW * kCW / 32];
+        int rk2[kTopW * kCW / 32];
+#pragma unroll
+        for (int i = 0; i < kTopW * kCW / 32; ++i) {
+          k2[i] = S.tkey[lane + 32 * i];
+          rk2[i] = 0;
+        }
+        for (int q = 0; q < kTopW * kCW; ++q) {
+          const unsigned kq = S.tkey[q];
+#pragma unroll
+          for (int i = 0; i < kTopW * kCW / 32; ++i)
+            rk2[i] += (kq > k2[i] || (kq == k2[i] && q < lane + 32 * i)) ? 1 : 0;
+        }
+#pragma unroll
+        for (int i = 0; i < kTopW * kCW / 32; ++i)
+          if (rk2[i] == LN - 1) S.theta = (k2[i] != 0u) ? ord_val(k2[i]) : kNegInf;
+      }
+      cbar();
+    }
+    float m[R];
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      float t = kNegInf;
+#pragma unroll
+      for (int w = 0; w < kCW; ++w) t = fmaxf(t, S.red[w * kMaxRows + r]);
+      m[r] = t;
+    }
+    float theta = kNegInf;
+    if constexpr (LIST) theta = S.theta;
+    float sm[R], tau;
+    int nc = 0;
+    for (int attempt = 0; attempt < 2; ++attempt) {
+      // phase B: sums of the tokens outside the candidates; candidates set aside
+#pragma unroll
+      for (int r = 0; r < R; ++r) sm[r] = 0.f;
+      tau = kNegInf;
+      for (int u = tid; u < U; u += kCT) {
+        const uint4 x0 = raw(b, 0, u);
+        float v0[VE];
+        E::unpack(x0, v0);
+        uint32_t cm = 0u;
+        if constexpr (LIST) {
+          const float um = E::unit_max(x0);
+          if (um > theta) {
+#pragma unroll
+            for (int e = 0; e < VE; ++e) {
+              if (v0[e] > theta)
+                cm |= 1u << e;
+              else
+                tau = fmaxf(tau, v0[e]);
+            }
+#pragma unroll
+            for (int e = 0; e < VE; ++e)
+              if (cm >> e & 1u) {
+                const int pos = atomicAdd(&S.ncand, 1);
+                if (pos < kCandCap) {
+                  cid[pos] = tok0 + u * VE + e;
+                  cl[pos] = v0[e];
+                }
+              }
+          } else {
+            tau = fmaxf(tau, um);
+          }
+        }
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+          float v[VE];
+          if (r == 0) {
+#pragma unroll
+            for (int e = 0; e < VE; ++e) v[e] = v0[e];
+          } else {
+            E::unpack(raw(b, r, u), v);
+          }
+          if (m[r] > kNegInf) {
+            const float mc = __fmul_rn(m[r], c[r]);
+            if (!cm) {
+#pragma unroll
+              for (int e = 0; e < VE; ++e) sm[r] = __fadd_rn(sm[r], ex2(__fmaf_rn(v[e], c[r], -mc)));
+            } else {
+#pragma unroll
+              for (int e = 0; e < VE; ++e) {
+                const float t = ex2(__fmaf_rn(v[e], c[r], -mc));
+                sm[r] = __fadd_rn(sm[r], (cm >> e & 1u) ? 0.f : t);
+              }
+            }
+          }
+        }
+      }
+      cbar();
+      nc = S.ncand;
+      if (!LIST || nc <= kCandCap) break;
+      // too many tokens above the threshold (ties or adversarial orderings):
+      // raise it to the kCandCap-th largest target logit by bisection on
+      // order-preserving keys, then redo the pass
+      unsigned t = 0u;
+      for (int bit = 31; bit >= 0; --bit) {   // keys of negative logits use every bit
+        const unsigned cand = t | (1u << bit);
+        int cnt = 0;
+        for (int u = tid; u < U; u += kCT) {
+          float v[VE];
+          E::unpack(raw(b, 0, u), v);
+#pragma unroll
+          for (int e = 0; e < VE; ++e) cnt += (v[e] == v[e] && ord_key(__fadd_rn(v[e], 0.f)) >= cand) ? 1 : 0;
+        }
+        cnt = __reduce_add_sync(FULLM, cnt);
+        cbar();
+        if (lane == 0) S.red[warp] = __int_as_float(cnt);
+        cbar();
+        int tot = 0;
+#pragma unroll
+        for (int w = 0; w < kCW; ++w) tot += __float_as_int(S.red[w]);
+        if (tot >= kCandCap) t = cand;
+      }
+      theta = fmaxf(theta, ord_val(t));
+      cbar();
+      if (tid == 0) S.ncand = 0;
+      cbar();
+    }
+    nc = min(nc, kCandCap);   // the bisection leaves fewer than kCandCap; never read past the arrays
+    // block sums of the rows (fixed order)
+    float tot[R];
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      const float v = warp_sum(sm[r]);
+      if (lane == 0) S.red[warp * kMaxRows + r] = v;
+    }
+    if constexpr (LIST) {
+      tau = warp_max(tau);
+      if (lane == 0) S.wth[warp] = tau;
+    }
+    cbar();
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      float t = 0.f;
+#pragma unroll
+      for (int w = 0; w < kCW; ++w) t = __fadd_rn(t, S.red[w * kMaxRows + r]);
+      tot[r] = t;
+    }
+    if constexpr (LIST) {
+      tau = kNegInf;
+#pragma unroll
+      for (int w = 0; w < kCW; ++w) tau = fmaxf(tau, S.wth[w]);
+      // phase C: ranks; the first LN go to the record, the rest back to the sums
+      for (int i = tid; i < nc; i += kCT) {
+        const float li = cl[i];
+        const int ii = cid[i];
+        int rk = 0;
+        for (int q = 0; q < nc; ++q) rk += better(cl[q], cid[q], li, ii) ? 1 : 0;
+        crank[i] = rk;
+      }
+      cbar();
+      int* rid = reinterpret_cast<int*>(rec + kHdr);
+      for (int i = tid; i < nc; i += kCT) {
+        const int rk = crank[i];
+        if (rk < LN) {
+          const int id = cid[i];
+          __stcg(rid + rk, id);
+          __stcg(rec + kHdr + LN + rk, cl[i]);
+#pragma unroll
+          for (int r = 1; r < R; ++r) {
+            float v[VE];
+            const int loc = id - tok0;
+            E::unpack(raw(b, r, loc / VE), v);
+            float l = v[0];
+#pragma unroll
+            for (int e = 1; e < VE; ++e)
+              if (e == loc % VE) l = v[e];
+            __stcg(rec + kHdr + LN * (1 + r) + rk, l);
+          }
+        } else {
+          cord[rk - LN] = i;
+        }
+      }
+      cbar();
+      const int nd = nc - LN;
+      if (nd > 0 && warp == 0) {
+        float add[R];
+#pragma unroll
+        for (int r = 0; r < R; ++r) add[r] = 0.f;
+        float at = kNegInf;
+        for (int t = lane; t < nd; t += 32) {
+          const int i = cord[t];
+          const int id = cid[i];
+          const int loc = id - tok0;
+          at = fmaxf(at, cl[i]);
+#pragma unroll
+          for (int r = 0; r < R; ++r) {
+            float v[VE];
+            E::unpack(raw(b, r, loc / VE), v);
+            float l = v[0];
+#pragma unroll
+            for (int e = 1; e < VE; ++e)
+              if (e == loc % VE) l = v[e];
+            if (m[r] > kNegInf) add[r] = __fadd_rn(add[r], ex2(__fmaf_rn(l, c[r], -__fmul_rn(m[r], c[r]))));
+          }
+        }
+#pragma unroll
+        for (int r = 0; r < R; ++r) add[r] = warp_sum(add[r]);
+        at = warp_max(at);
+        if (lane == 0) {
+#pragma unroll
+          for (int r = 0; r < R; ++r) S.add[r] = add[r];
+          S.addtau = at;
+        }
+      }
+      cbar();
+      if (nd > 0) {
+#pragma unroll
+        for (int r = 0; r < R; ++r) tot[r] = __fadd_rn(tot[r], S.add[r]);
+        tau = fmaxf(tau, S.addtau);
+      }
+    }
+    if (tid == 0) {
+#pragma unroll
+      for (int r = 0; r < R; ++r) {
+        __stcg(rec + 2 * r, m[r]);
+        __stcg(rec + 2 * r + 1, tot[r]);
+      }
+      __stcg(rec + 2 * kMaxRows, tau);
+      __stcg(reinterpret_cast<int*>(rec) + 2 * kMaxRows + 1, LIST ? min(nc, LN) : 0);
+    }
+  }
+
+  // Stats of any number of rows, one row at a time, no candidate list.
+  __device__ void stats_rows(const FPass& P, const char* b, int n, float* rec) {
+    const int tid = threadIdx.x;
+    const int U = (n + VE - 1) / VE;
+    for (int r = 0; r < P.nstream; ++r) {
+      float mx = kNegInf;
+      for (int u = tid; u < U; u += kCT) mx = fmaxf(mx, E::unit_max(raw(b, r, u)));
+      mx = block_max(mx, S.red);
+      const float c = P.row[r].c;
+      float sm = 0.f;
+      if (mx > kNegInf) {
+        const float mc = __fmul_rn(mx, c);
+        for (int u = tid; u < U; u += kCT) {
+          float v[VE];
+          E::unpack(raw(b, r, u), v);
+#pragma unroll
+          for (int e = 0; e < VE; ++e) sm = __fadd_rn(sm, ex2(__fmaf_rn(v[e], c, -mc)));
+        }
+      }
+      sm = block_sum(sm, S.red + kCW);
+      if (tid == 0) {
+        __stcg(rec + 2 * r, mx);
+        __stcg(rec + 2 * r + 1, sm);
+      }
+    }
+  }
+
+  // -------------------------------------------------------------- weights of the inverse-CDF draws
+  // Residual max(0, q - p_I) (kResid; p_I = sum_r gamma_r p_r with the
+  // special tokens' explicit values), or the target mass outside Omega_0
+  // (kReplace: tokens with a logit above `cut` weigh 0 unless all0 says
+  // Omega_0 is empty of them), or the target mass (kBonus).
+  __device__ __forceinline__ void weights(const FPass& P, const char* b, int u, int tok0, float* w) const {
+    float v0[VE];
+    E::unpack(raw(b, 0, u), v0);
+    const float M0 = P.row[0].M, c0 = P.row[0].c, iz0 = P.row[0].invZ;
+    if (P.kind == kResid) {
+      float a[VE];
+#pragma unroll
+      for (int e = 0; e < VE; ++e) a[e] = 0.f;
+      for (int r = 1; r < P.nstream; ++r) {
+        const float g = P.row[r].gamma;
+        if (g == 0.f) continue;
+        float v[VE];
+        E::unpack(raw(b, r, u), v);
+        const float M = P.row[r].M, c = P.row[r].c, iz = P.row[r].invZ;
+#pragma unroll
+        for (int e = 0; e < VE; ++e) a[e] = __fmaf_rn(g, prob_of(v[e], M, c, iz), a[e]);
+      }
+      if (P.nspec > 0 && ((S.bitmap[u >> 5] >> (u & 31)) & 1u)) {
+#pragma unroll
+        for (int e = 0; e < VE; ++e) a[e] = spec_lookup(P, tok0 + u * VE + e, a[e]);
+      }
+#pragma unroll
+      for (int e = 0; e < VE; ++e) w[e] = fmaxf(0.f, __fsub_rn(prob_of(v0[e], M0, c0, iz0), a[e]));
+    } else if (P.kind == kReplace) {
+#pragma unroll
+      for (int e = 0; e < VE; ++e) w[e] = (P.all0 || v0[e] > P.cut) ? 0.f : prob_of(v0[e], M0, c0, iz0);
+    } else {
+#pragma unroll
+      for (int e = 0; e < VE; ++e) w[e] = prob_of(v0[e], M0, c0, iz0);
+    }
+  }
+
+  __device__ void resid_task(const FPass& P, const char* b, int tok0, int n, float* rec) {
+    if (P.kind == kResid && P.nspec > 0) build_bitmap(P, tok0, n);
+    const int U = (n + VE - 1) / VE;
+    float part = 0.f;
+    for (int u = threadIdx.x; u < U; u += kCT) {
+      float w[VE];
+      weights(P, b, u, tok0, w);
+#pragma unroll
+      for (int e = 0; e < VE; ++e) part = __fadd_rn(part, w[e]);
+    }
+    part = block_sum(part, S.red);
+    if (threadIdx.x == 0) __stcg(rec, part);
+  }
+
+  // -------------------------------------------------------------- full-vocabulary stage task
+  __device__ __forceinline__ static void cand_insert(Cand (&top)[kTopF], const Cand& c, float& ra, float& rb) {
+    if (better(c.key, c.id, top[kTopF - 1].key, top[kTopF - 1].id)) {
+      ra = __fadd_rn(ra, top[kTopF - 1].a);
+      rb = __fadd_rn(rb, top[kTopF - 1].b);
+      top[kTopF - 1] = c;
+#pragma unroll
+      for (int t = kTopF - 1; t > 0; --t) {
+        if (better(top[t].key, top[t].id, top[t - 1].key, top[t - 1].id)) {
+          const Cand x = top[t];
+          top[t] = top[t - 1];
+          top[t - 1] = x;
+        }
+      }
+    } else {
+      ra = __fadd_rn(ra, c.a);
+      rb = __fadd_rn(rb, c.b);
+    }
+  }
+
+  // Warp-wide merge of per-lane sorted lists (best first): lane 0 writes the
+  // warp's best `rounds` entries to out[0..rounds) and CAND_NONE after them;
+  // every entry not popped adds its a and b (fixed order) to rest_a / rest_b.
+  __device__ static void warp_merge(Cand (&top)[kTopF], Cand* out, int rounds, float& rest_a, float& rest_b) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll 1
+    for (int t = 0; t < kTopF; ++t) {
+      if (t >= rounds) {
+        if (lane == 0) out[t] = CAND_NONE;
+        continue;
+      }
+      float bk = top[0].key;
+      int bid = top[0].id;
+#pragma unroll
+      for (int o = 16; o; o >>= 1) {
+        const float ok = __shfl_xor_sync(FULLM, bk, o);
+        const int oid = __shfl_xor_sync(FULLM, bid, o);
+        if (better(ok, oid, bk, bid)) {
+          bk = ok;
+          bid = oid;
+        }
+      }
+      const bool mine = (top[0].id == bid && top[0].key == bk && bid != 0x7fffffff);
+      const unsigned who = __ballot_sync(FULLM, mine);
+      const int src = who ? __ffs(who) - 1 : 0;
+      const float wa = __shfl_sync(FULLM, top[0].a, src);
+      const float wb = __shfl_sync(FULLM, top[0].b, src);
+      if (mine) {
+#pragma unroll
+        for (int i = 0; i < kTopF - 1; ++i) top[i] = top[i + 1];
+        top[kTopF - 1] = CAND_NONE;
+      }
+      if (lane == 0) out[t] = who ? Cand{bk, bid, wa, wb} : CAND_NONE;
+    }
+    float ra = 0.f, rb = 0.f;
+#pragma unroll
+    for (int i = 0; i < kTopF; ++i) {
+      ra = __fadd_rn(ra, top[i].a);
+      rb = __fadd_rn(rb, top[i].b);
+    }
+    rest_a = warp_sum(ra);
+    rest_b = warp_sum(rb);
+  }
+
+  // Record: [0] a-mass and [1] b-mass of the slice outside its top s, [4..)
+  // the top s (key, id, a, b) as four arrays of kTopF.
+  __device__ void full_task(const FPass& P, const char* b, int tok0, int n, float* rec) {
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int s = min(p.wis_s, p.V);
+    const int rb = P.rb;
+    if (P.nspec > 0) build_bitmap(P, tok0, n);
+    Cand top[kTopF];
+#pragma unroll
+    for (int t = 0; t < kTopF; ++t) top[t] = CAND_NONE;
+    float suma = 0.f, sumb = 0.f;
+    const int U = (n + VE - 1) / VE;
+    const float M0 = P.row[0].M, c0 = P.row[0].c, iz0 = P.row[0].invZ;
+    for (int u = tid; u < U; u += kCT) {
+      float v0[VE], a[VE], bb[VE];
+      E::unpack(raw(b, 0, u), v0);
+#pragma unroll
+      for (int e = 0; e < VE; ++e) {
+        a[e] = 0.f;
+        bb[e] = 0.f;
+      }
+      for (int r = 1; r < P.nstream; ++r) {
+        const float g = P.row[r].gamma;
+        if (g == 0.f && r != rb) continue;
+        float v[VE];
+        E::unpack(raw(b, r, u), v);
+        const float M = P.row[r].M, c = P.row[r].c, iz = P.row[r].invZ;
+#pragma unroll
+        for (int e = 0; e < VE; ++e) {
+          const float pr = prob_of(v[e], M, c, iz);
+          if (g != 0.f) a[e] = __fmaf_rn(g, pr, a[e]);
+          if (r == rb) bb[e] = pr;
+        }
+      }
+      if (P.nspec > 0 && ((S.bitmap[u >> 5] >> (u & 31)) & 1u)) {
+#pragma unroll
+        for (int e = 0; e < VE; ++e) a[e] = spec_lookup(P, tok0 + u * VE + e, a[e]);
+      }
+#pragma unroll
+      for (int e = 0; e < VE; ++e) {
+        if (u * VE + e >= n) break;
+        const float q = prob_of(v0[e], M0, c0, iz0);
+        cand_insert(top, Cand{__fmaf_rn(-a[e], bb[e], q), tok0 + u * VE + e, a[e], bb[e]}, suma, sumb);
+      }
+    }
+    {
+      float ra, rbs;
+      warp_merge(top, S.wcand + warp * kTopF, s, ra, rbs);
+      suma = warp_sum(suma);
+      sumb = warp_sum(sumb);
+      if (lane == 0) {
+        S.red[warp * 2] = __fadd_rn(suma, ra);
+        S.red[warp * 2 + 1] = __fadd_rn(sumb, rbs);
+      }
+    }
+    cbar();
+    if (warp == 0) {
+#pragma unroll
+      for (int t = 0; t < kTopF; ++t) top[t] = (lane < kCW) ? S.wcand[lane * kTopF + t] : CAND_NONE;
+      float ra, rbs;
+      warp_merge(top, S.blk, s, ra, rbs);
+      __syncwarp();
+      if (lane == 0) {
+        float sa = ra, sb = rbs;
+        for (int w = 0; w < kCW; ++w) {
+          sa = __fadd_rn(sa, S.red[w * 2]);
+          sb = __fadd_rn(sb, S.red[w * 2 + 1]);
+        }
+        __stcg(rec + 0, sa);
+        __stcg(rec + 1, sb);
+      }
+      if (lane < kTopF) {
+        __stcg(rec + 4 + lane, S.blk[lane].key);
+        __stcg(reinterpret_cast<int*>(rec) + 4 + kTopF + lane, S.blk[lane].id);
+        __stcg(rec + 4 + 2 * kTopF + lane, S.blk[lane].a);
+        __stcg(rec + 4 + 3 * kTopF + lane, S.blk[lane].b);
+      }
+    }
+  }
+
+  // -------------------------------------------------------------- compute warps
+  __device__ void process(int bi) {
+    FDesc& Dd = S.desc[bi];
+    char* b = buf(bi);
+    const int s = Dd.slice, seqb = Dd.b;
+    const int tok0 = s * p.T, n = min(p.T, p.V - tok0);
+    const FPass& P = Dd.P;
+    if (!p.bulk) load_plain(P, P.nstream, b, tok0, n);
+    float* rec = p.rec + ((size_t)seqb * p.ns + s) * p.rec_floats;
+    PT_T0(t_task);
+    PT_CNT(kPhTasks);
+    switch (P.kind) {
+      case kStats:
+      case kBonus:
+        if (P.list) {
+          switch (P.nstream) {
+            case 1: stats_small<1, true>(P, b, tok0, n, rec); break;
+            case 2: stats_small<2, true>(P, b, tok0, n, rec); break;
+            case 3: stats_small<3, true>(P, b, tok0, n, rec); break;
+            default: stats_small<4, true>(P, b, tok0, n, rec); break;
+          }
+        } else {
+          switch (P.nstream) {
+            case 1: stats_small<1, false>(P, b, tok0, n, rec); break;
+            case 2: stats_small<2, false>(P, b, tok0, n, rec); break;
+            default: stats_rows(P, b, n, rec); break;
+          }
+        }
+        break;
+      case kResid:
+      case kReplace: resid_task(P, b, tok0, n, rec); break;
+      case kFull: full_task(P, b, tok0, n, rec); break;
+      default: break;
+    }
+    PT_ADD(P.kind == kStats ? (P.list ? kPhTaskList : kPhTaskStats)
+                            : (P.kind == kBonus ? kPhTaskStats : (P.kind == kFull ? kPhTaskFull : kPhTaskResid)),
+           t_task);
+    if (P.kind == kStats && P.j == 0 && s == 0) {
+      // the sequence's outputs start as -1 (the decisions overwrite them)
+      for (int j = threadIdx.x; j <= p.L; j += kCT) __stcg(p.out_tokens + (size_t)seqb * (p.L + 1) + j, -1);
+      if (threadIdx.x == 0) __stcg(p.out_accept + seqb, -1);
+    }
+    __threadfence();
+    cbar();
+    if (threadIdx.x == 0) S.last = (atomicAdd(&p.cnt[seqb], 1u) == (unsigned)(p.ns - 1)) ? 1 : 0;
+    cbar();
+    if (S.last) {
+      __threadfence();
+      decide(Dd, b);
+    }
+  }
+
+  __device__ void compute() {
+    for (int k = 0;; ++k) {
+      const int bi = k % kNBuf;
+      const uint32_t par = (k / kNBuf) & 1;
+      // thread 0 waits (bounded); the others then see the completed phase
+      PT_T0(t_wait);
+      if (threadIdx.x == 0) {
+        const bool ok = wait_mbar(&S.full[bi], par);
+        if (!ok) set_abort(MDS_ST_TIMEOUT);
+        S.flag_ok = ok ? 1 : 0;
+        S.flag_ab = aborted() ? 1 : 0;
+      }
+      cbar();
+      PT_ADD(kPhWaitFull, t_wait);
+      if (!S.flag_ok) break;
+      while (!mbar_try_wait(&S.full[bi], par)) {
+      }
+      if (S.desc[bi].exit) break;
+      if (!S.flag_ab) process(bi);
+      // generic accesses of this buffer before the next bulk copy into it
+      fence_proxy_async();
+      cbar();
+      if (threadIdx.x == 0) {
+        S.consumed = k + 1;
+        mbar_arrive(&S.empty[bi]);
+      }
+    }
+  }
+
+  // ============================================================== decisions
+  // Run by the compute warps of the CTA that completed a pass of sequence b.
+
+  __device__ void push(int b, int kind) {
+    DState& D = S.D;
+    const int tid = threadIdx.x;
+    PT_T0(t_push);
+    if (tid == 0) D.P.kind = kind;
+    cbar();
+    FSeq* g = &reinterpret_cast<FSeq*>(p.seq)[b];
+    copy_out(&g->P, &D.P, (int)sizeof(FPass), tid, kCT);
+    copy_out(&g->W, &D.W, (int)sizeof(FWalk), tid, kCT);
+    if (tid == 0) __stcg(p.cnt + b, 0u);
+    __threadfence();
+    cbar();
+    if (tid == 0) D.tbase = (unsigned)p.B * (unsigned)p.ns + atomicAdd(&p.ctl[kCtlTail], (unsigned)p.ns);
+    cbar();
+    for (int i = tid; i < p.ns; i += kCT) {
+      const unsigned t = D.tbase + (unsigned)i;
+      const unsigned slot = t % (unsigned)p.ring_cap;
+      if (t >= (unsigned)p.ring_cap) {
+        // the slot's previous task must have been taken
+        const unsigned long long prev = tag_of(t - (unsigned)p.ring_cap);
+        const unsigned long long t0 = now_ns();
+        for (int it = 0; ld_acquire(&p.ring_rtag[slot]) != prev; ++it) {
+          if (aborted()) break;
+          if ((it & 15) == 15 && now_ns() - t0 > kWaitNs) {
+            set_abort(MDS_ST_TIMEOUT);
+            break;
+          }
+          __nanosleep(64);
+        }
+      }
+      __stcg(p.ring_pay + slot, ((unsigned)b << 16) | (unsigned)i);
+      st_release(&p.ring_tag[slot], tag_of(t));
+    }
+    PT_ADD(kPhPush, t_push);
+  }
+
+  __device__ void finish(int b, int acc_len) {
+    if (threadIdx.x == 0) {
+      __stcg(p.out_accept + b, acc_len);
+      __stcg(p.cnt + b, 0u);
+      __threadfence();
+      atomicAdd(&p.ctl[kCtlDone], 1u);
+    }
+  }
+
+  // Z decided at the current depth: outputs, then the next depth's pass,
+  // the bonus pass, or the end of the sequence.
+  __device__ void walk(int b, int Z, float R, float qY, float pIY, int Ydiag) {
+    DState& D = S.D;
+    const int j = D.P.j;
+    cbar();   // every thread has read the depth before thread 0 re-plans
+    if (threadIdx.x == 0) {
+      __stcg(p.out_tokens + (size_t)b * (p.L + 1) + j, Z);
+      if (p.out_diag) {
+        float* dg = p.out_diag + ((size_t)b * (p.L + 1) + j) * 4;
+        __stcg(dg + 0, qY);
+        __stcg(dg + 1, pIY);
+        __stcg(dg + 2, R);
+        __stcg(dg + 3, (float)Ydiag);
+      }
+      unsigned nv = 0u;
+      for (int i = 0; i < D.nv; ++i)
+        if (D.X[i] == Z) nv |= 1u << D.vbr[i];
+      D.W.valid = nv;
+      D.tok = nv ? ((j + 1 == p.L) ? kBonus : kStats) : kNone;
+      if (nv) {
+        D.W.stage = 0;
+        D.W.zres = 0;
+        plan_rows(b, j + 1, nv, j + 1 == p.L, &D.P, &D.nv, D.vbr, D.X, D.vrow);
+      }
+    }
+    cbar();
+    const int next = D.tok;
+    if (next == kNone)
+      finish(b, j);
+    else
+      push(b, next);
+  }
+
+  // Combine the records of a stats pass: every row's M and 1/Z, and with
+  // candidate lists the sequence's list (the first LN of the slices' lists
+  // by (logit, id)), its complement masses and tau.
+  __device__ void combine_stats(const FDesc& Dd, int b, char* scratch) {
+    DState& D = S.D;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int ns = p.ns, R = Dd.P.nstream, LN = p.ln;
+    const bool list = Dd.P.list != 0;
+    const float* recb = p.rec + (size_t)b * ns * p.rec_floats;
+    float* hm = reinterpret_cast<float*>(scratch);        // [R][ns] slice maxima
+    float* hs = hm + R * ns;                              // [R][ns] slice sums
+    float* htau = hs + R * ns;                            // [ns]
+    int* hnl = reinterpret_cast<int*>(htau + ns);         // [ns]
+    int* eid = hnl + ns;                                  // [ns][LN]
+    float* el = reinterpret_cast<float*>(eid + ns * LN);  // [R][ns][LN]
+    for (int i = tid; i < R * ns; i += kCT) {
+      const int r = i / ns, s = i - r * ns;
+      hm[i] = __ldcg(recb + (size_t)s * p.rec_floats + 2 * r);
+      hs[i] = __ldcg(recb + (size_t)s * p.rec_floats + 2 * r + 1);
+    }
+    if (list) {
+      for (int s = tid; s < ns; s += kCT) {
+        htau[s] = __ldcg(recb + (size_t)s * p.rec_floats + 2 * kMaxRows);
+        hnl[s] = __ldcg(reinterpret_cast<const int*>(recb + (size_t)s * p.rec_floats) + 2 * kMaxRows + 1);
+      }
+      for (int i = tid; i < ns * LN * (1 + R); i += kCT) {
+        const int f = i / (ns * LN), rest = i - f * ns * LN;
+        const int s = rest / LN, q = rest - s * LN;
+        const float v = __ldcg(recb + (size_t)s * p.rec_floats + kHdr + f * LN + q);
+        if (f == 0)
+          eid[rest] = __float_as_int(v);
+        else
+          el[(f - 1) * ns * LN + rest] = v;
+      }
+    }
+    cbar();
+    // row maxima
+    if (tid < R) {
+      float M = kNegInf;
+      for (int s = 0; s < ns; ++s) M = fmaxf(M, hm[tid * ns + s]);
+      if (!(M > kNegInf) || M != M) {
+        atomicOr(p.status, MDS_ST_NONFINITE);
+        M = 0.f;
+      }
+      D.P.row[tid].M = M;
+    }
+    cbar();
+    if (!list) {
+      if (tid < R) {
+        const float M = D.P.row[tid].M, c = D.P.row[tid].c;
+        float Z = 0.f;
+        for (int s = 0; s < ns; ++s) {
+          const float ms = hm[tid * ns + s];
+          if (ms > kNegInf) Z = __fadd_rn(Z, __fmul_rn(hs[tid * ns + s], ref_shift(ms, M, c)));
+        }
+        finish_row(tid, Z);
+      }
+      cbar();
+      return;
+    }
+    // merge of the slices' lists (warp 0): lane s holds slice s's head; ties
+    // of the logit go to the lower slice, which holds the lower token ids
+    if (warp == 0) {
+      const int nl = (lane < ns) ? hnl[lane] : 0;
+      int h = 0;
+      unsigned key = (h < nl) ? ord_key(__fadd_rn(el[lane * LN], 0.f)) : 0u;
+      int nf = 0;
+      for (int t = 0; t < LN; ++t) {
+        const unsigned km = __reduce_max_sync(FULLM, key);
+        if (!km) break;
+        const unsigned who = __ballot_sync(FULLM, key == km);
+        if (lane == __ffs(who) - 1) {
+          D.fin_s[t] = lane;
+          D.fin_i[t] = h;
+          ++h;
+          key = (h < nl) ? ord_key(__fadd_rn(el[lane * LN + h], 0.f)) : 0u;
+        }
+        nf = t + 1;
+      }
+      if (lane < ns) D.ksl[lane] = h;
+      // tau: the largest target logit left out (slices' own and dropped entries)
+      float tau = (lane < ns) ? htau[lane] : kNegInf;
+      for (int q = h; q < nl; ++q) tau = fmaxf(tau, el[lane * LN + q]);
+      tau = warp_max(tau);
+      if (lane == 0) {
+        D.n = nf;
+        D.cand_tau = tau;
+        D.cand_all = (nf == p.V) ? 1 : 0;
+      }
+    }
+    cbar();
+    const int nf = D.n;
+    // dropped entries' masses per row (warp r, fixed order) and the slices' sums
+    if (warp < R) {
+      const int r = warp;
+      const float M = D.P.row[r].M, c = D.P.row[r].c;
+      float add = 0.f;
+      for (int i = lane; i < ns * LN; i += 32) {
+        const int s = i / LN, q = i - s * LN;
+        if (q >= D.ksl[s] && q < hnl[s]) add = __fadd_rn(add, exp_term(el[r * ns * LN + i], M, c));
+      }
+      add = warp_sum(add);
+      if (lane == 0) {
+        float C = 0.f;
+        for (int s = 0; s < ns; ++s) {
+          const float ms = hm[r * ns + s];
+          if (ms > kNegInf) C = __fadd_rn(C, __fmul_rn(hs[r * ns + s], ref_shift(ms, M, c)));
+        }
+        D.pc[r] = __fadd_rn(C, add);
+      }
+    }
+    // the list by token id (positions by counting)
+    if (warp == 0) {
+      for (int t = lane; t < nf; t += 32) {
+        const int idx = D.fin_s[t] * LN + D.fin_i[t];
+        const int id = eid[idx];
+        int pos = 0;
+        for (int q = 0; q < nf; ++q) pos += (eid[D.fin_s[q] * LN + D.fin_i[q]] < id) ? 1 : 0;
+        D.cm_id[pos] = id;
+        D.cm_l0[pos] = el[idx];
+        for (int r = 0; r < R; ++r) D.cm_e[r][pos] = exp_term(el[r * ns * LN + idx], D.P.row[r].M, D.P.row[r].c);
+        D.cm_sp[pos] = 0;
+        D.cm_a[pos] = 0.f;
+      }
+    }
+    cbar();
+    if (warp < R) {
+      const int r = warp;
+      float z = 0.f;
+      for (int t = lane; t < nf; t += 32) z = __fadd_rn(z, D.cm_e[r][t]);
+      z = warp_sum(z);
+      if (lane == 0) finish_row(r, __fadd_rn(D.pc[r], z));
+    }
+    cbar();
+    if (tid == 0) {
+      const float tau = D.cand_tau;
+      D.cand_q = (tau > kNegInf) ? exp_term(tau, D.P.row[0].M, D.P.row[0].c) : 0.f;
+    }
+    cbar();
+  }
+
+  __device__ void finish_row(int r, float Z) {
+    if (!(Z > 0.f) || !(Z < kPosInf) || Z != Z) {
+      atomicOr(p.status, MDS_ST_NONFINITE);
+      Z = 1.f;
+    }
+    S.D.P.row[r].invZ = __frcp_rn(Z);
+  }
+
+  // -------------------------------------------------------------- WIS stage on the candidate list
+  // Warp 0, one list entry per lane.  Returns false (changing nothing) if
+  // the list cannot certify Omega_1: fewer than s entries, or the s-th key
+  // not above every key outside the list (each such key is <= its q <= q(tau)).
+  __device__ bool wis_stage_list(int A, int Btok, int rb, float u) {
+    DState& D = S.D;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int s = min(p.wis_s, p.V);
+    const int n = D.n;
+    if (warp == 0) {
+      const float iz0 = D.P.row[0].invZ, izb = D.P.row[rb].invZ;
+      const bool have = lane < n;
+      float q = 0.f, a = 0.f, bq = 0.f, key = kNegInf;
+      if (have) {
+        q = __fmul_rn(D.cm_e[0][lane], iz0);
+        if (D.cm_sp[lane]) {
+          a = D.cm_a[lane];
+        } else {
+          for (int r = 1; r < D.P.nrows; ++r)
+            if (D.P.row[r].gamma != 0.f) a = __fmaf_rn(D.P.row[r].gamma, __fmul_rn(D.cm_e[r][lane], D.P.row[r].invZ), a);
+        }
+        bq = __fmul_rn(D.cm_e[rb][lane], izb);
+        key = __fadd_rn(__fmaf_rn(-a, bq, q), 0.f);   // -0 -> +0: keys compare as floats
+      }
+      unsigned kk = have ? ord_key(key) : 0u;
+      uint32_t selm = 0u;
+      float kth = kNegInf;
+      for (int t = 0; t < s; ++t) {
+        const unsigned km = __reduce_max_sync(FULLM, kk);
+        const uint32_t who = __ballot_sync(FULLM, km != 0u && kk == km);
+        if (!who) break;
+        const int wl = __ffs(who) - 1;
+        selm |= 1u << wl;
+        if (lane == wl) kk = 0u;
+        kth = ord_val(km);
+      }
+      const bool sel = (selm >> lane) & 1u;
+      const float qout = __fmul_rn(__fmul_rn(D.cand_q, iz0), 1.0001f);
+      const bool ok = __popc(selm) == s && (D.cand_all || kth > qout);
+      const float ra = warp_sum((have && !sel) ? a : 0.f);
+      const float rbm = warp_sum((have && !sel) ? bq : 0.f);
+      if (!ok) {
+        if (lane == 0) D.fast_ok = 0;
+      } else {
+        const int rk = __popc(selm & ((1u << lane) - 1u));
+        if (lane >= s && lane < MDS_MAX_S) {
+          D.om[lane] = -1;
+          D.om_q[lane] = 0.f;
+          D.om_a[lane] = 0.f;
+          D.om_b[lane] = 0.f;
+        }
+        if (sel) {
+          D.om[rk] = D.cm_id[lane];
+          D.om_q[rk] = q;
+          D.om_a[rk] = a;
+          D.om_b[rk] = bq;
+        }
+        __syncwarp();
+        if (lane == 0) {
+          // Omega_2 masses: complement (generic law) + list entries outside Omega_1
+          float sa = 0.f;
+          for (int r = 1; r < D.P.nrows; ++r)
+            if (D.P.row[r].gamma != 0.f) sa = __fmaf_rn(D.P.row[r].gamma, __fmul_rn(D.pc[r], D.P.row[r].invZ), sa);
+          const float sb = __fadd_rn(__fmul_rn(D.pc[rb], izb), rbm);
+          sa = __fadd_rn(sa, ra);
+          D.Y = solve(s, sa, sb, A, Btok, u);
+          D.A2 = sa;
+          D.B2 = sb;
+          D.fast_ok = 1;
+        }
+        __syncwarp();
+        const float A2 = D.A2, B2 = D.B2;
+        if (sel) {
+          D.cm_a[lane] = D.om_x[rk];
+          D.cm_sp[lane] = 1;
+        } else if (have && D.cm_sp[lane]) {
+          D.cm_a[lane] = __fmul_rn(0.5f, __fadd_rn(__fmul_rn(a, B2), __fmul_rn(bq, A2)));
+        }
+        __syncwarp();
+        if (lane == 0) gamma_update(rb, A2, B2);
+      }
+    }
+    cbar();
+    return D.fast_ok != 0;
+  }
+
+  __device__ int solve(int s, float A2, float B2, int A, int Btok, float u) {
+    DState& D = S.D;
+    bool capped = false;
+    const int y = (s <= 5) ? stage_solve<5>(s, A2, B2, A, Btok, u, D.om, D.om_q, D.om_a, D.om_b, D.om_x, &capped)
+                           : stage_solve<MDS_MAX_S>(s, A2, B2, A, Btok, u, D.om, D.om_q, D.om_a, D.om_b, D.om_x,
+                                                    &capped);
+    if (capped) atomicOr(p.status, MDS_ST_LP_CAP);
+    return y;
+  }
+
+  // Generic law after a stage: gamma <- (B2/2) gamma + (A2/2) e_rb.  One thread.
+  __device__ void gamma_update(int rb, float A2, float B2) {
+    DState& D = S.D;
+    const float hB = __fmul_rn(0.5f, B2), hA = __fmul_rn(0.5f, A2);
+    for (int r = 1; r < D.P.nrows; ++r) D.P.row[r].gamma = __fmul_rn(hB, D.P.row[r].gamma);
+    D.P.row[rb].gamma = __fadd_rn(D.P.row[rb].gamma, hA);
+  }
+
+  // The list's special tokens into the table form used by the residual and
+  // the point lookups.  One thread.
+  __device__ void list_to_table() {
+    DState& D = S.D;
+    int k = 0;
+    for (int i = 0; i < D.n && k < kMaxSpecial; ++i)
+      if (D.cm_sp[i]) {
+        D.P.spec_id[k] = D.cm_id[i];
+        D.P.spec_val[k] = D.cm_a[i];
+        ++k;
+      }
+    D.P.nspec = k;
+  }
+
+  // -------------------------------------------------------------- decisions per pass kind
+  __device__ void accept_step(int b) {
+    DState& D = S.D;
+    if (threadIdx.x == 0) {
+      const int j = D.P.j;
+      const float u = draw_uniform(p.seed, b, j, kDrawAccept);
+      const float ratio = D.W.pIY > 0.f ? __fdiv_rn(D.W.qY, D.W.pIY) : kPosInf;
+      const bool acc = u < fminf(1.f, ratio);
+      D.W.acc = acc ? 1 : 0;
+      D.W.Ydiag = D.W.Y;
+      D.tok = (acc && !p.acc_prob) ? 1 : 0;
+      if (!D.tok) {
+        D.W.ures = acc ? 0.f : draw_uniform(p.seed, b, j, kDrawResidual);
+        if (p.scheme == MDS_SINGLE || D.nv == 1 || p.scheme != MDS_WIS) {
+          // residual against one draft law: rows 0 and the first valid branch's
+          for (int r = 0; r < D.P.nrows; ++r) D.P.row[r].gamma = 0.f;
+          D.P.row[D.vrow[0]].gamma = 1.f;
+          D.P.nspec = 0;
+          D.P.nstream = max(2, D.vrow[0] + 1);
+        } else {
+          D.P.nstream = D.P.nrows;
+        }
+      }
+    }
+    cbar();
+    if (D.tok)
+      walk(b, D.W.Y, 0.f, D.W.qY, D.W.pIY, D.W.Y);
+    else
+      push(b, kResid);
+  }
+
+  __device__ void decide_stats(const FDesc& Dd, int b, char* scratch) {
+    DState& D = S.D;
+    const int tid = threadIdx.x;
+    const int j = Dd.P.j;
+    if (tid == 0) {
+      if (j == 0) {
+        D.W = FWalk{};
+        D.W.valid = (p.K >= 32) ? FULLM : ((1u << p.K) - 1u);
+        D.W.Yp = -1;
+      }
+      plan_rows(b, j, D.W.valid, false, &D.P, &D.nv, D.vbr, D.X, D.vrow);
+    }
+    cbar();
+    PT_T0(t_comb);
+    combine_stats(Dd, b, scratch);
+    PT_ADD(kPhDecCombine, t_comb);
+    if (p.scheme == MDS_WIS0) {
+      wis0_decide(b);
+      return;
+    }
+    if (p.scheme == MDS_SINGLE || D.nv == 1) {
+      if (tid == 0) {
+        const int Y = D.X[0];
+        D.W.Y = Y;
+        D.W.qY = prob_row(D.P, 0, Y);
+        D.W.pIY = prob_row(D.P, D.vrow[0], Y);
+      }
+      cbar();
+      accept_step(b);
+      return;
+    }
+    // WIS: the pairwise stages (Remark 4) on the candidate list while it
+    // certifies Omega_1; from the first stage it cannot, full-vocabulary passes
+    if (tid == 0) {
+      for (int r = 0; r < D.P.nrows; ++r) D.P.row[r].gamma = 0.f;
+      D.P.row[D.vrow[0]].gamma = 1.f;
+      D.P.nspec = 0;
+    }
+    cbar();
+    int A = D.X[0];
+    bool fast = Dd.P.list != 0;
+    int m = 1;
+    PT_T0(t_stg);
+    if (fast) {
+      for (; m < D.nv; ++m) {
+        const float u = draw_uniform(p.seed, b, j, kDrawSelect + m - 1);
+        if (!wis_stage_list(A, D.X[m], D.vrow[m], u)) break;
+        A = D.Y;
+      }
+      if (tid == 0) list_to_table();
+      cbar();
+    }
+    PT_ADD(kPhDecStages, t_stg);
+    if (m < D.nv) {
+      if (tid == 0) {
+        D.W.stage = m;
+        D.W.A = A;
+        D.P.rb = D.vrow[m];
+        D.P.nstream = D.P.nrows;
+      }
+      cbar();
+      push(b, kFull);
+      return;
+    }
+    if (tid == 0) {
+      D.W.Y = A;
+      D.W.qY = prob_row(D.P, 0, A);
+      D.W.pIY = law_at(D.P, A);
+    }
+    cbar();
+    accept_step(b);
+  }
+
+  __device__ void decide_full(const FDesc& Dd, int b) {
+    DState& D = S.D;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int j = D.P.j, ns = p.ns;
+    if (tid == 0) plan_rows(b, j, D.W.valid, false, nullptr, &D.nv, D.vbr, D.X, D.vrow);
+    cbar();
+    const int m = D.W.stage;
+    const int A = D.W.A, Btok = D.X[m], rb = D.vrow[m];
+    const float u = draw_uniform(p.seed, b, j, kDrawSelect + m - 1);
+    const int s = min(p.wis_s, p.V);
+    const float* recb = p.rec + (size_t)b * ns * p.rec_floats;
+    // Omega_1: the top s of every slice's top s (s rounds of a block argmax)
+    float ra = 0.f, rbs = 0.f;
+    for (int r = 0; r < s; ++r) {
+      float bk = kNegInf;
+      int bid = 0x7fffffff, bi = -1;
+      for (int i = tid; i < ns * kTopF; i += kCT) {
+        const int sl = i / kTopF, t = i - sl * kTopF;
+        if (t >= s) continue;
+        const float* rc = recb + (size_t)sl * p.rec_floats;
+        const int id = __ldcg(reinterpret_cast<const int*>(rc) + 4 + kTopF + t);
+        bool taken = false;
+        for (int q = 0; q < r; ++q) taken |= (D.fin[q].id == id);
+        if (taken) continue;
+        const float key = __ldcg(rc + 4 + t);
+        if (id != 0x7fffffff && better(key, id, bk, bid)) {
+          bk = key;
+          bid = id;
+          bi = i;
+        }
+      }
+#pragma unroll
+      for (int o = 16; o; o >>= 1) {
+        const float ok = __shfl_xor_sync(FULLM, bk, o);
+        const int oid = __shfl_xor_sync(FULLM, bid, o);
+        const int oi = __shfl_xor_sync(FULLM, bi, o);
+        if (better(ok, oid, bk, bid)) {
+          bk = ok;
+          bid = oid;
+          bi = oi;
+        }
+      }
+      cbar();
+      if (lane == 0) {
+        S.red[warp * 3] = bk;
+        S.red[warp * 3 + 1] = __int_as_float(bid);
+        S.red[warp * 3 + 2] = __int_as_float(bi);
+      }
+      cbar();
+      if (tid == 0) {
+        float k2 = kNegInf;
+        int id2 = 0x7fffffff, i2 = -1;
+        for (int w = 0; w < kCW; ++w) {
+          const float kw = S.red[w * 3];
+          const int iw = __float_as_int(S.red[w * 3 + 1]);
+          if (better(kw, iw, k2, id2)) {
+            k2 = kw;
+            id2 = iw;
+            i2 = __float_as_int(S.red[w * 3 + 2]);
+          }
+        }
+        Cand c = CAND_NONE;
+        if (i2 >= 0) {
+          const float* rc = recb + (size_t)(i2 / kTopF) * p.rec_floats;
+          const int t = i2 % kTopF;
+          c = Cand{k2, id2, __ldcg(rc + 4 + 2 * kTopF + t), __ldcg(rc + 4 + 3 * kTopF + t)};
+        }
+        D.fin[r] = c;
+      }
+      cbar();
+    }
+    // Omega_2 masses: the slices' rests plus their top-s entries not taken
+    {
+      float sa = 0.f, sb = 0.f;
+      for (int i = tid; i < ns * kTopF; i += kCT) {
+        const int sl = i / kTopF, t = i - sl * kTopF;
+        const float* rc = recb + (size_t)sl * p.rec_floats;
+        if (t == 0) {
+          sa = __fadd_rn(sa, __ldcg(rc + 0));
+          sb = __fadd_rn(sb, __ldcg(rc + 1));
+        }
+        if (t >= s) continue;
+        const int id = __ldcg(reinterpret_cast<const int*>(rc) + 4 + kTopF + t);
+        if (id == 0x7fffffff) continue;
+        bool taken = false;
+        for (int q = 0; q < s; ++q) taken |= (D.fin[q].id == id);
+        if (taken) continue;
+        sa = __fadd_rn(sa, __ldcg(rc + 4 + 2 * kTopF + t));
+        sb = __fadd_rn(sb, __ldcg(rc + 4 + 3 * kTopF + t));
+      }
+      ra = block_sum(sa, S.red);
+      rbs = block_sum(sb, S.red + kCW);
+    }
+    if (warp == 0) {
+      if (lane < s) {
+        int id = D.fin[lane].id;
+        if (id < 0 || id >= p.V) id = 0;   // only with non-finite keys (status already set)
+        D.fin[lane].id = id;
+        D.om_q[lane] = prob_row(D.P, 0, id);
+      }
+      __syncwarp();
+      if (lane == 0) {
+        // Omega_1 by token id; q follows its token
+        int om[MDS_MAX_S];
+        float ak[MDS_MAX_S], bk[MDS_MAX_S], qk[MDS_MAX_S];
+        for (int t = 0; t < MDS_MAX_S; ++t) {
+          om[t] = (t < s) ? D.fin[t].id : 0x7fffffff;
+          ak[t] = (t < s) ? D.fin[t].a : 0.f;
+          bk[t] = (t < s) ? D.fin[t].b : 0.f;
+          qk[t] = (t < s) ? D.om_q[t] : 0.f;
+        }
+        for (int x = 1; x < MDS_MAX_S; ++x)   // insertion sort by id (at most 8 entries)
+          for (int y = x; y > 0 && om[y] < om[y - 1]; --y) {
+            const int ti = om[y];
+            om[y] = om[y - 1];
+            om[y - 1] = ti;
+            float tf = ak[y];
+            ak[y] = ak[y - 1];
+            ak[y - 1] = tf;
+            tf = bk[y];
+            bk[y] = bk[y - 1];
+            bk[y - 1] = tf;
+            tf = qk[y];
+            qk[y] = qk[y - 1];
+            qk[y - 1] = tf;
+          }
+        for (int t = 0; t < MDS_MAX_S; ++t) {
+          D.om[t] = om[t];
+          D.om_a[t] = ak[t];
+          D.om_b[t] = bk[t];
+          D.om_q[t] = qk[t];
+        }
+        D.Y = solve(s, ra, rbs, A, Btok, u);
+        D.A2 = ra;
+        D.B2 = rbs;
+      }
+      __syncwarp();
+      // law update: special tokens outside Omega_1, gamma, Omega_1 values
+      const float A2 = D.A2, B2 = D.B2;
+      for (int i = lane; i < D.P.nspec; i += 32) {
+        const int tokn = D.P.spec_id[i];
+        bool in1 = false;
+        for (int t = 0; t < s; ++t) in1 |= (D.om[t] == tokn);
+        if (!in1)
+          D.P.spec_val[i] =
+              __fmul_rn(0.5f, __fadd_rn(__fmul_rn(D.P.spec_val[i], B2), __fmul_rn(prob_row(D.P, rb, tokn), A2)));
+      }
+      __syncwarp();
+      if (lane == 0) {
+        gamma_update(rb, A2, B2);
+        for (int t = 0; t < s; ++t) {
+          int i = 0;
+          while (i < D.P.nspec && D.P.spec_id[i] != D.om[t]) ++i;
+          if (i == D.P.nspec && D.P.nspec < kMaxSpecial) {
+            D.P.spec_id[i] = D.om[t];
+            ++D.P.nspec;
+          }
+          if (i < kMaxSpecial) D.P.spec_val[i] = D.om_x[t];
+        }
+        D.W.A = D.Y;
+        D.W.stage = m + 1;
+        if (m + 1 < D.nv) D.P.rb = D.vrow[m + 1];
+      }
+    }
+    cbar();
+    if (m + 1 < D.nv) {
+      push(b, kFull);
+      return;
+    }
+    if (tid == 0) {
+      const int Y = D.W.A;
+      D.W.Y = Y;
+      D.W.qY = prob_row(D.P, 0, Y);
+      D.W.pIY = law_at(D.P, Y);
+    }
+    cbar();
+    accept_step(b);
+  }
+
+  // Inverse-CDF search over the weights of pass kind P.kind: the slice by
+  // the per-slice masses Rs[0..ns) (slice order), the token by one re-read of
+  // that slice in token order (contiguous runs per thread, a fixed-order
+  // exclusive scan, then the owning run).  Returns the smallest token whose
+  // running mass exceeds T, else the last token with positive weight.
+  __device__ int search(FPass& P, const float* Rs, float T, char* scratch) {
+    DState& D = S.D;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    if (tid == 0) {
+      float run = 0.f, run_last = 0.f, run_hit = 0.f;
+      int hit = -1, last = -1;
+      for (int s = 0; s < p.ns; ++s) {
+        const float v = Rs[s];
+        if (v > 0.f) {
+          last = s;
+          run_last = run;
+        }
+        if (hit < 0 && __fadd_rn(run, v) > T) {
+          hit = s;
+          run_hit = run;
+        }
+        run = __fadd_rn(run, v);
+      }
+      if (hit < 0) {
+        hit = max(last, 0);
+        run_hit = run_last;
+      }
+      D.seg = hit;
+      D.run = run_hit;
+      D.cross = kCT;
+      D.lastp = -1;
+    }
+    cbar();
+    const int s = D.seg;
+    const float base = D.run;
+    const int tok0 = s * p.T, n = min(p.T, p.V - tok0);
+    const int nst = (P.kind == kResid) ? P.nstream : 1;
+    load_plain(P, nst, scratch, tok0, n);
+    if (P.kind == kResid && P.nspec > 0) build_bitmap(P, tok0, n);
+    const int U = (n + VE - 1) / VE;
+    const int upt = (U + kCT - 1) / kCT;
+    const int u0 = min(U, tid * upt), u1 = min(U, u0 + upt);
+    float part = 0.f;
+    for (int u = u0; u < u1; ++u) {
+      float w[VE];
+      weights(P, scratch, u, tok0, w);
+#pragma unroll
+      for (int e = 0; e < VE; ++e) part = __fadd_rn(part, w[e]);
+    }
+    // exclusive scan over the threads (warp scans, then warps in order)
+    float incl = part;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const float t = __shfl_up_sync(FULLM, incl, o);
+      if (lane >= o) incl = __fadd_rn(incl, t);
+    }
+    if (lane == 31) S.red[warp] = incl;
+    cbar();
+    float wbase = base;
+    for (int w = 0; w < warp; ++w) wbase = __fadd_rn(wbase, S.red[w]);
+    const float excl = __fadd_rn(wbase, __fsub_rn(incl, part));
+    const float end = __fadd_rn(wbase, incl);
+    if (end > T && part > 0.f) atomicMin(&D.cross, tid);
+    if (part > 0.f) atomicMax(&D.lastp, tid);
+    cbar();
+    // the first run whose end passes T; if rounding left the slice short, the
+    // last run with mass (its last positive token); -1: no mass at all
+    const int owner = (D.cross < kCT) ? D.cross : D.lastp;
+    if (tid == (owner < 0 ? 0 : owner)) {
+      int tok = -1, last = -1;
+      float acc = excl;
+      if (owner >= 0) {
+        for (int u = u0; u < u1 && tok < 0; ++u) {
+          float w[VE];
+          weights(P, scratch, u, tok0, w);
+#pragma unroll
+          for (int e = 0; e < VE; ++e) {
+            if (w[e] > 0.f) last = tok0 + u * VE + e;
+            acc = __fadd_rn(acc, w[e]);
+            if (tok < 0 && acc > T && w[e] > 0.f) tok = tok0 + u * VE + e;
+          }
+        }
+      }
+      if (tok < 0) tok = last;
+      if (tok < 0) tok = tok0;
+      D.tok = min(tok, p.V - 1);
+    }
+    cbar();
+    return D.tok;
+  }
+
+  // Slice masses of pass `kind` from the records (Rs in shared memory) and
+  // their total in slice order.
+  __device__ float slice_masses(int b, float* Rs) {
+    const float* recb = p.rec + (size_t)b * p.ns * p.rec_floats;
+    for (int s = threadIdx.x; s < p.ns; s += kCT) Rs[s] = __ldcg(recb + (size_t)s * p.rec_floats);
+    cbar();
+    if (threadIdx.x == 0) {
+      float R = 0.f;
+      for (int s = 0; s < p.ns; ++s) R = __fadd_rn(R, Rs[s]);
+      S.D.rtot = R;
+    }
+    cbar();
+    return S.D.rtot;
+  }
+
+  __device__ void decide_resid(int b, char* scratch) {
+    DState& D = S.D;
+    const int tid = threadIdx.x;
+    if (tid == 0) plan_rows(b, D.P.j, D.W.valid, false, nullptr, &D.nv, D.vbr, D.X, D.vrow);
+    float* Rs = S.Rs;
+    const float R = slice_masses(b, Rs);
+    int Z = D.W.Y;
+    if (!D.W.acc) {
+      if (R > 0.f) {
+        Z = search(D.P, Rs, __fmul_rn(D.W.ures, R), scratch);
+      } else {
+        // zero residual mass (only by rounding): sample the target row
+        if (tid == 0) {
+          atomicOr(p.status, MDS_ST_ZERO_RESID);
+          D.W.zres = 1;
+          D.W.R = R;
+          D.P.cut = kPosInf;
+          D.P.all0 = 0;
+          D.P.nstream = 1;
+        }
+        cbar();
+        push(b, kReplace);
+        return;
+      }
+    }
+    walk(b, Z, R, D.W.qY, D.W.pIY, D.W.Ydiag);
+  }
+
+  __device__ void decide_replace(int b, char* scratch) {
+    DState& D = S.D;
+    const int tid = threadIdx.x;
+    if (tid == 0) plan_rows(b, D.P.j, D.W.valid, false, nullptr, &D.nv, D.vbr, D.X, D.vrow);
+    float* Rs = S.Rs;
+    const float R = slice_masses(b, Rs);
+    int Z;
+    if (R > 0.f) {
+      Z = search(D.P, Rs, __fmul_rn(D.W.ures, R), scratch);
+    } else if (!D.W.zres && D.W.Yp >= 0) {
+      Z = D.W.Yp;   // no target mass outside Omega_0
+    } else if (!D.W.zres) {
+      if (tid == 0) {
+        atomicOr(p.status, MDS_ST_ZERO_RESID);
+        D.W.zres = 1;
+        D.P.cut = kPosInf;
+        D.P.all0 = 0;
+      }
+      cbar();
+      push(b, kReplace);
+      return;
+    } else {
+      if (tid == 0) atomicOr(p.status, MDS_ST_NONFINITE);
+      Z = 0;
+    }
+    const float Rd = (p.scheme == MDS_WIS0) ? D.W.R : (D.W.zres ? D.W.R : R);
+    walk(b, Z, Rd, D.W.qY, D.W.pIY, D.W.Ydiag);
+  }
+
+  __device__ void decide_bonus(const FDesc& Dd, int b, char* scratch) {
+    DState& D = S.D;
+    const int tid = threadIdx.x;
+    const float* recb = p.rec + (size_t)b * p.ns * p.rec_floats;
+    float* hm = S.hm;
+    float* Rs = S.Rs;
+    for (int s = tid; s < p.ns; s += kCT) {
+      hm[s] = __ldcg(recb + (size_t)s * p.rec_floats);
+      Rs[s] = __ldcg(recb + (size_t)s * p.rec_floats + 1);
+    }
+    cbar();
+    if (tid == 0) {
+      float M = kNegInf;
+      for (int s = 0; s < p.ns; ++s) M = fmaxf(M, hm[s]);
+      if (!(M > kNegInf) || M != M) {
+        atomicOr(p.status, MDS_ST_NONFINITE);
+        M = 0.f;
+      }
+      const float c = D.P.row[0].c;
+      float Z = 0.f;
+      for (int s = 0; s < p.ns; ++s)
+        if (hm[s] > kNegInf) Z = __fadd_rn(Z, __fmul_rn(Rs[s], ref_shift(hm[s], M, c)));
+      D.P.row[0].M = M;
+      finish_row(0, Z);
+    }
+    cbar();
+    const float M = D.P.row[0].M, c = D.P.row[0].c, iz = D.P.row[0].invZ;
+    for (int s = tid; s < p.ns; s += kCT)
+      Rs[s] = (hm[s] > kNegInf) ? __fmul_rn(__fmul_rn(Rs[s], ref_shift(hm[s], M, c)), iz) : 0.f;
+    cbar();
+    if (tid == 0) {
+      float Q = 0.f;
+      for (int s = 0; s < p.ns; ++s) Q = __fadd_rn(Q, Rs[s]);
+      D.rtot = Q;
+    }
+    cbar();
+    const float Q = D.rtot;
+    const int Z = search(D.P, Rs, __fmul_rn(draw_uniform(p.seed, b, p.L, kDrawBonus), Q), scratch);
+    if (tid == 0) {
+      __stcg(p.out_tokens + (size_t)b * (p.L + 1) + p.L, Z);
+      if (p.out_diag) {
+        float* dg = p.out_diag + ((size_t)b * (p.L + 1) + p.L) * 4;
+        __stcg(dg + 0, 0.f);
+        __stcg(dg + 1, 0.f);
+        __stcg(dg + 2, Q);
+        __stcg(dg + 3, -1.f);
+      }
+    }
+    finish(b, p.L);
+  }
+
+  // -------------------------------------------------------------- truncated alphabet
+  // Warp-wide inverse CDF over one weight per lane (lane order = token-id
+  // order of the list): the smallest lane whose running sum exceeds
+  // u * total, the last lane with positive weight if rounding leaves none,
+  // -1 if the total is not positive.
+  __device__ __forceinline__ static int lane_cdf(float w, float u01, float* total) {
+    const int lane = threadIdx.x & 31;
+    float c = w;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const float t = __shfl_up_sync(FULLM, c, o);
+      if (lane >= o) c = __fadd_rn(c, t);
+    }
+    const float tot = __shfl_sync(FULLM, c, 31);
+    *total = tot;
+    if (!(tot > 0.f)) return -1;
+    const unsigned who = __ballot_sync(FULLM, c > __fmul_rn(u01, tot));
+    if (who) return __ffs(who) - 1;
+    return 31 - __clz(__ballot_sync(FULLM, w > 0.f));
+  }
+
+  // One depth of the truncated-alphabet scheme (Section 4, read with the
+  // non-iid appendix's remark on keeping only the inputs in Omega_0).
+  // Omega_0 = the target tokens above the (M+1)-th largest target logit, read
+  // off the candidate list (exact when the list's (M+1)-th entry is >= tau,
+  // the list holds the whole vocabulary, or every token outside it is -inf;
+  // otherwise the tokens above tau, with MDS_ST_OMEGA0).  Warp 0 runs the
+  // WIS stages on Omega_0 against q~ = q / p_a with the kept inputs' draft
+  // laws restricted to Omega_0 and renormalised (point loads of the draft
+  // logits there), then Algorithm 1 against q~.  Y' is kept with probability
+  // p_a, else a replace pass draws from the tokens outside Omega_0 by q.
+  __device__ void wis0_decide(int b) {
+    DState& D = S.D;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int j = D.P.j;
+    if (warp == 0) {
+      const int n = D.n;
+      const bool have = lane < n;
+      const int id = have ? D.cm_id[lane] : 0;
+      const float l = have ? D.cm_l0[lane] : kNegInf;
+      int rk = 0;   // rank in the list by (larger logit, then lower id)
+      for (int t = 0; t < 32; ++t) {
+        const float lt = __shfl_sync(FULLM, l, t);
+        const int it = __shfl_sync(FULLM, id, t);
+        rk += (t < n && better(lt, it, l, id)) ? 1 : 0;
+      }
+      const int M = p.omega0;
+      const bool all0 = M >= p.V;
+      float cut = kNegInf;
+      bool cert;
+      if (all0) {
+        cert = D.cand_all != 0;
+      } else {
+        const unsigned who = __ballot_sync(FULLM, have && rk == M);
+        if (who) cut = __shfl_sync(FULLM, l, __ffs(who) - 1);
+        const float tau = D.cand_tau;
+        cert = D.cand_all || (who ? cut >= tau : !(tau > kNegInf));
+        if (!cert) cut = fmaxf(cut, tau);
+      }
+      const bool in0 = have && (all0 || l > cut);
+      const int n0 = __popc(__ballot_sync(FULLM, in0));
+      const float q = in0 ? prob_of(l, D.P.row[0].M, D.P.row[0].c, D.P.row[0].invZ) : 0.f;
+      const float pa = warp_sum(q);
+      const float qt = (in0 && pa > 0.f) ? __fdiv_rn(q, pa) : 0.f;
+      // draft laws restricted to Omega_0 (exponents against their own maximum
+      // there; the rows' full normalisers cancel)
+      float ew[MDS_MAX_K];
+#pragma unroll
+      for (int k = 0; k < MDS_MAX_K; ++k) ew[k] = 0.f;
+      for (int r = 1; r < D.P.nrows; ++r) {
+        const float lr = in0 ? E::global(D.P.row[r].ptr, id) : kNegInf;
+        const float ref = warp_max(lr);
+        const float cr = D.P.row[r].c;
+        const float e = (in0 && ref > kNegInf) ? exp_term(lr, ref, cr) : 0.f;
+        const float Pm = warp_sum(e);
+        if (lane == 0 && Pm != Pm) atomicOr(p.status, MDS_ST_NONFINITE);
+        const float lw = (Pm > 0.f) ? __fdiv_rn(e, Pm) : 0.f;
+#pragma unroll
+        for (int k = 0; k < MDS_MAX_K; ++k)
+          if (k == r - 1) ew[k] = lw;
+      }
+      auto law = [&](int r) -> float {
+        float v = 0.f;
+#pragma unroll
+        for (int k = 0; k < MDS_MAX_K; ++k)
+          if (k == r - 1) v = ew[k];
+        return v;
+      };
+      // kept inputs: valid branches (branch order) whose token lies in Omega_0
+      int nk = 0;
+      for (int i = 0; i < D.nv; ++i) {
+        const unsigned w = __ballot_sync(FULLM, in0 && id == D.X[i]);
+        if (!w) continue;
+        const int li = __ffs(w) - 1;
+        const float lv = __shfl_sync(FULLM, law(D.vrow[i]), li);
+        if (!(lv > 0.f)) continue;   // impossible draw: dropped
+        if (lane == 0) {
+          D.k_lane[nk] = li;
+          D.k_row[nk] = D.vrow[i];
+        }
+        ++nk;
+      }
+      __syncwarp();
+      int yl = -1, Yl = -1;
+      float qY = 0.f, pIY = 0.f, R = 0.f;
+      if (n0 > 0 && nk == 0) {
+        float t;
+        yl = lane_cdf(qt, draw_uniform(p.seed, b, j, kDrawResidual), &t);
+      } else if (n0 > 0) {
+        float a = law(D.k_row[0]);
+        int A = D.k_lane[0];
+        const int s = min(p.wis_s, n0);
+        for (int m = 1; m < nk; ++m) {
+          const int Bl = D.k_lane[m];
+          const float bb = law(D.k_row[m]);
+          const float u = draw_uniform(p.seed, b, j, kDrawSelect + m - 1);
+          unsigned kk = in0 ? ord_key(__fadd_rn(__fmaf_rn(-a, bb, qt), 0.f)) : 0u;
+          uint32_t selm = 0u;
+          for (int t = 0; t < s; ++t) {
+            const unsigned km = __reduce_max_sync(FULLM, kk);
+            const uint32_t who = __ballot_sync(FULLM, km != 0u && kk == km);
+            if (!who) break;
+            const int wl = __ffs(who) - 1;
+            selm |= 1u << wl;
+            if (lane == wl) kk = 0u;
+          }
+          const bool sel = (selm >> lane) & 1u;
+          const int sn = __popc(selm);
+          const float A2 = warp_sum((in0 && !sel) ? a : 0.f);
+          const float B2 = warp_sum((in0 && !sel) ? bb : 0.f);
+          const int rk1 = __popc(selm & ((1u << lane) - 1u));
+          if (lane >= sn && lane < MDS_MAX_S) {
+            D.om[lane] = -1;
+            D.om_q[lane] = 0.f;
+            D.om_a[lane] = 0.f;
+            D.om_b[lane] = 0.f;
+          }
+          if (sel) {
+            D.om[rk1] = id;
+            D.om_q[rk1] = qt;
+            D.om_a[rk1] = a;
+            D.om_b[rk1] = bb;
+          }
+          __syncwarp();
+          if (lane == 0) D.Y = solve(sn, A2, B2, D.cm_id[A], D.cm_id[Bl], u);
+          __syncwarp();
+          const int Yt = D.Y;
+          A = max(0, __ffs(__ballot_sync(FULLM, in0 && id == Yt)) - 1);
+          a = sel ? D.om_x[rk1] : (in0 ? __fmul_rn(0.5f, __fadd_rn(__fmul_rn(a, B2), __fmul_rn(bb, A2))) : 0.f);
+          __syncwarp();
+        }
+        Yl = A;
+        qY = __shfl_sync(FULLM, qt, A);
+        pIY = __shfl_sync(FULLM, a, A);
+        const float ratio = pIY > 0.f ? __fdiv_rn(qY, pIY) : kPosInf;
+        if (draw_uniform(p.seed, b, j, kDrawAccept) < fminf(1.f, ratio)) {
+          yl = A;
+        } else {
+          const float ures = draw_uniform(p.seed, b, j, kDrawResidual);
+          yl = lane_cdf(in0 ? fmaxf(0.f, __fsub_rn(qt, a)) : 0.f, ures, &R);
+          if (yl < 0) {   // only by rounding: sample q~
+            if (lane == 0) atomicOr(p.status, MDS_ST_ZERO_RESID);
+            float t;
+            yl = lane_cdf(qt, ures, &t);
+          }
+        }
+      }
+      if (lane == 0) {
+        if (!cert) atomicOr(p.status, MDS_ST_OMEGA0);
+        D.o0_n = n0;
+        D.o0_all = (all0 && D.cand_all) ? 1 : 0;
+        D.o0_cut = cut;
+        D.o0_pa = pa;
+        D.W.R = R;
+        D.W.Yp = (yl >= 0) ? D.cm_id[yl] : -1;
+        D.W.Ydiag = (Yl >= 0) ? D.cm_id[Yl] : -1;
+        D.W.qY = qY;
+        D.W.pIY = pIY;
+        D.W.zres = 0;
+        const bool keep = D.o0_n > 0 && (D.o0_all || draw_uniform(p.seed, b, j, kDrawKeep) < D.o0_pa);
+        D.tok = keep ? 1 : 0;
+        if (!keep) {
+          D.W.ures = draw_uniform(p.seed, b, j, kDrawOutside);
+          D.P.cut = cut;
+          D.P.all0 = D.o0_all;
+          D.P.nstream = 1;
+        }
+      }
+    }
+    cbar();
+    if (D.tok)
+      walk(b, D.W.Yp, D.W.R, D.W.qY, D.W.pIY, D.W.Ydiag);
+    else
+      push(b, kReplace);
+  }
+
+  __device__ void decide(const FDesc& Dd, char* scratch) {
+    DState& D = S.D;
+    const int b = Dd.b;
+    const int kind = Dd.P.kind;
+    if (!(kind == kStats && Dd.P.j == 0)) {
+      const FSeq* g = &reinterpret_cast<const FSeq*>(p.seq)[b];
+      copy_in(&D.P, &g->P, (int)sizeof(FPass), threadIdx.x, kCT);
+      copy_in(&D.W, &g->W, (int)sizeof(FWalk), threadIdx.x, kCT);
+      cbar();
+    }
+    PT_T0(t_dec);
+    PT_CNT(kPhDecisions);
+    switch (kind) {
+      case kStats: decide_stats(Dd, b, scratch); break;
+      case kResid: decide_resid(b, scratch); break;
+      case kReplace: decide_replace(b, scratch); break;
+      case kFull: decide_full(Dd, b); break;
+      case kBonus: decide_bonus(Dd, b, scratch); break;
+      default: break;
+    }
+    cbar();
+    PT_ADD(kind == kStats ? kPhDecStats
+                          : (kind == kFull ? kPhDecFull : (kind == kBonus ? kPhDecBonus : kPhDecResid)),
+           t_dec);
+  }
+};
+
+template <int DT>
+__global__ void __launch_bounds__(kBlock, 2) flow_kernel(const __grid_constant__ Params p) {
+  extern __shared__ __align__(128) char dsm[];
+  __shared__ FShared S;
+  Eng<DT> e{p, S};
+  e.bufs = dsm;
+  char* c = dsm + (size_t)kNBuf * kBufBytes;
+  e.cid = reinterpret_cast<int*>(c);
+  e.cl = reinterpret_cast<float*>(c + kCandCap * 4);
+  e.crank = reinterpret_cast<int*>(c + 2 * kCandCap * 4);
+  e.cord = reinterpret_cast<int*>(c + 3 * kCandCap * 4);
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < kNBuf; ++i) {
+      mbar_init(&S.full[i], 1);
+      mbar_init(&S.empty[i], 1);
+    }
+    S.issued = 0;
+    S.consumed = 0;
+#ifdef MDS_PHASE_TIMERS
+    for (int i = 0; i < kPhaseN; ++i) S.tm[i] = 0ull;
+#endif
+    mbar_init_fence();
+  }
+  __syncthreads();
+  PT_T0(t_kernel);
+  if (threadIdx.x >= kCT)
+    e.scheduler();
+  else
+    e.compute();
+  __syncthreads();
+  // copies issued but never consumed (only after an abort): wait for them
+  if (threadIdx.x == kCT) {
+    for (int k = S.consumed; k < S.issued; ++k) (void)e.wait_mbar(&S.full[k % kNBuf], (k / kNBuf) & 1);
+  }
+  __syncthreads();
+#ifdef MDS_PHASE_TIMERS
+  if (threadIdx.x == 0) S.tm[kPhKernel] += (unsigned long long)(clock64() - t_kernel);
+  __syncthreads();
+  if (threadIdx.x < kPhaseN) atomicAdd(&g_phase[threadIdx.x], S.tm[threadIdx.x]);
+#endif
+  if (threadIdx.x == 0) {
+    __threadfence();
+    const unsigned out = atomicAdd(&p.ctl[kCtlExit], 1u);
+    if (out == gridDim.x - 1) {
+      // every CTA has left: reset for the next launch
+      if (ld_relaxed(&p.ctl[kCtlAbort]))
+        for (int b = 0; b < p.B; ++b) p.cnt[b] = 0u;
+      p.ctl[kCtlHead] = 0u;
+      p.ctl[kCtlTail] = 0u;
+      p.ctl[kCtlDone] = 0u;
+      p.ctl[kCtlAbort] = 0u;
+      __threadfence();
+      p.ctl[kCtlExit] = 0u;
+    }
+  }
+}
+
+size_t dyn_smem() { return (size_t)kNBuf * kBufBytes + 4 * (size_t)kCandCap * 4; }
+
+}  // namespace
+
+size_t seq_bytes() { return sizeof(FSeq); }
+
+namespace {
+size_t up256(size_t x) { return (x + 255) / 256 * 256; }
+struct Layout {
+  size_t ctl, tag, pay, cnt, seq, rec;
+  size_t cap;
+};
+Layout layout(const Params& p, int nseq, int grid) {
+  Layout L;
+  L.cap = (size_t)nseq * p.ns + (size_t)grid + 64;
+  L.ctl = 256;
+  L.tag = up256(L.cap * 8);
+  L.pay = up256(L.cap * 4);
+  L.cnt = up256((size_t)nseq * 4);
+  L.seq = up256((size_t)nseq * sizeof(FSeq));
+  L.rec = up256((size_t)nseq * p.ns * p.rec_floats * 4);
+  return L;
+}
+}  // namespace
+
+size_t workspace_bytes(const Params& p, int nseq, int grid) {
+  const Layout L = layout(p, nseq, grid);
+  return L.ctl + 2 * L.tag + L.pay + L.cnt + L.seq + L.rec;
+}
+
+size_t clear_bytes(const Params& p, int nseq, int grid) {
+  const Layout L = layout(p, nseq, grid);
+  return L.ctl + 2 * L.tag + L.pay + L.cnt;
+}
+
+void carve_workspace(Params& p, char* w, int nseq, int grid) {
+  const Layout L = layout(p, nseq, grid);
+  p.ctl = reinterpret_cast<unsigned*>(w);
+  w += L.ctl;
+  p.ring_tag = reinterpret_cast<unsigned long long*>(w);
+  w += L.tag;
+  p.ring_rtag = reinterpret_cast<unsigned long long*>(w);
+  w += L.tag;
+  p.ring_pay = reinterpret_cast<unsigned*>(w);
+  w += L.pay;
+  p.cnt = reinterpret_cast<unsigned*>(w);
+  w += L.cnt;
+  p.seq = w;
+  w += L.seq;
+  p.rec = reinterpret_cast<float*>(w);
+  p.ring_cap = (int)L.cap;
+}
+
+bool plan_geometry(Params& p, int grid) {
+  const int es = p.esize;
+  int nstream;
+  int list = 0;
+  if (p.scheme == MDS_WIS0) {
+    nstream = 1;
+    list = 1;
+  } else if (p.scheme == MDS_WIS) {
+    nstream = 1 + p.n_models;
+    list = (p.K > 1 && nstream <= kListRowsMax) ? 1 : 0;
+  } else if (p.scheme == MDS_SINGLE) {
+    nstream = 2;
+  } else {
+    return false;
+  }
+  if (nstream > kMaxRows) return false;
+  int Tmax = kBufBytes / (nstream * es);
+  Tmax = (Tmax / kSliceQuantum) * kSliceQuantum;
+  if (Tmax < kSliceQuantum) return false;
+  const int cap = list ? kMaxSlicesList : kMaxSlices;
+  int ns = (p.V + Tmax - 1) / Tmax;
+  if (ns > cap) return false;
+  // enough tasks for the grid: at least two per CTA at depth 0 where the
+  // vocabulary allows
+  const long want = (2L * grid + p.B - 1) / p.B;
+  if (ns < want) {
+    const int nsw = (int)(want < cap ? want : cap);
+    int T = (p.V + nsw - 1) / nsw;
+    T = ((T + kSliceQuantum - 1) / kSliceQuantum) * kSliceQuantum;
+    if (T < kSliceQuantum) T = kSliceQuantum;
+    if (T < Tmax) Tmax = T;
+    ns = (p.V + Tmax - 1) / Tmax;
+  }
+  p.T = Tmax;
+  p.ns = ns;
+  p.ln = list ? ((p.scheme == MDS_WIS0 && p.omega0 >= 32) ? 64 : 32) : 0;
+  if (p.ln > kListMax) return false;
+  const int lrows = list ? nstream : 0;
+  int rf = kHdr + p.ln * (1 + lrows);
+  if (rf < 4 + 4 * kTopF) rf = 4 + 4 * kTopF;
+  p.rec_floats = (rf + 3) & ~3;
+  p.hdr_floats = kHdr;
+  // the decision stages one stats pass's records in one slice buffer
+  const size_t stage = (size_t)(2 * nstream * ns + 2 * ns + ns * p.ln * (1 + lrows)) * 4;
+  if (stage > (size_t)kBufBytes) return false;
+  return true;
+}
+
+int grid_size(int device) {
+  int sms = 0;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device) != cudaSuccess) return 0;
+  int per = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, flow_kernel<MDS_BF16>, kBlock, dyn_smem()) != cudaSuccess)
+    return 0;
+  int per32 = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per32, flow_kernel<MDS_F32>, kBlock, dyn_smem()) != cudaSuccess)
+    return 0;
+  if (per32 < per) per = per32;
+  return per * sms;
+}
+
+cudaError_t configure(int) {
+  // both logit types: the grid size is taken over both
+  cudaError_t e = cudaFuncSetAttribute((const void*)flow_kernel<MDS_F32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)dyn_smem());
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute((const void*)flow_kernel<MDS_BF16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)dyn_smem());
+  return e;
+}
+
+int read_phase_timers(unsigned long long* out, int n) {
+#ifdef MDS_PHASE_TIMERS
+  unsigned long long h[kPhaseN];
+  if (cudaDeviceSynchronize() != cudaSuccess) return -1;
+  if (cudaMemcpyFromSymbol(h, g_phase, sizeof(h)) != cudaSuccess) return -1;
+  const unsigned long long z[kPhaseN] = {};
+  if (cudaMemcpyToSymbol(g_phase, z, sizeof(z)) != cudaSuccess) return -1;
+  const int m = n < kPhaseN ? n : kPhaseN;
+  for (int i = 0; i < m; ++i) out[i] = h[i];
+  return kPhaseN;
+#else
+  (void)out;
+  (void)n;
+  return -2;
+#endif
+}
+
+cudaError_t launch(const Params& p, int grid, cudaStream_t stream) {
+  const size_t smem = dyn_smem();
+  if (p.dtype == MDS_F32) {
+    flow_kernel<MDS_F32><<<grid, kBlock, smem, stream>>>(p);
+  } else {
+    flow_kernel<MDS_BF16><<<grid, kBlock, smem, stream>>>(p);
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace flow
+}  // namespace mds

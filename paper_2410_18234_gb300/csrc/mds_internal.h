@@ -66,7 +66,26 @@ cudaError_t launch(const Params& p, int clusters, cudaStream_t stream);
 // mds_verify would use for this configuration; MDS_OK or MDS_EVOCAB.
 int launch_geometry(const mds_config& cfg, int device, int scheme, int n_models, Params& p);
 
-// One-time kernel attribute set-up for a logit type; MDS_OK or MDS_ECUDA.
+// One-time kernel attribute set-up for a logit type on the current device;
+// MDS_OK or MDS_ECUDA.
 int prepare_kernels(int dtype);
+
+// Record the CUDA error behind an MDS_ECUDA return (the detail mds_error_string
+// reports for this host thread); returns MDS_ECUDA.
+int record_cuda_error(cudaError_t e, const char* where);
+
+namespace flow {
+struct Params;
+}
+constexpr int kNotServed = 1;   // a configuration left to the per-sequence engine
+
+// Slice-dataflow engine parameters of a call with configuration c on a grid
+// of `grid` CTAs (geometry sized for c.max_B sequences): false if the engine
+// does not serve the call.  Buffers are filled in by flow_buffers.
+bool flow_params(const mds_config& c, int grid, int scheme, const int8_t* model_of, int n_models, bool bulk_ok,
+                 bool aligned16, flow::Params& p);
+void flow_buffers(flow::Params& p, const void* target_logits, const void* const* draft_logits,
+                  const int32_t* draft_tokens, const float* temperatures, int32_t* out_tokens,
+                  int32_t* out_accept_len, float* out_diag, int B, uint64_t seed);
 
 }  // namespace mds

@@ -1,38 +1,57 @@
 // mds_verify_noalloc: the verification entry point for callers that cannot
 // allocate device memory.  See include/mds.h for the contract.
+//
+// The call takes the same engine as mds_verify for the same configuration:
+// the slice-dataflow engine (single, WIS, WIS0) with its workspace carved out
+// of the static array, or the per-sequence engine, whose scratch is the first
+// two words of the array.
 #include <mutex>
 
+#include "mds_flow.h"
 #include "mds_internal.h"
 
 namespace {
 
-// The kernel's scratch: word 0 the status word, word 1 the work counter.
-// Every GPU that loads the library holds this array until the process exits.
-static __device__ __align__(256) unsigned g_noalloc_scratch[MDS_NOALLOC_SCRATCH_BYTES / sizeof(unsigned)];
+// The kernels' scratch.  Bytes [0, 256): word 0 the status word, word 1 the
+// per-sequence engine's work counter.  Bytes [256, end): the dataflow
+// engine's workspace (control words, task ring, per-sequence state, slice
+// records).  Every GPU that loads the library holds this array until the
+// process exits.
+static __device__ __align__(256) unsigned char g_noalloc_scratch[MDS_NOALLOC_SCRATCH_BYTES];
 
+constexpr size_t kHead = 256;
 constexpr size_t kScratchNeeded = 2 * sizeof(unsigned);
 constexpr int kMaxDevices = 64;
 
 std::mutex g_mu;
-unsigned* g_scratch_ptr[kMaxDevices] = {};
+unsigned char* g_scratch_ptr[kMaxDevices] = {};
+int g_grid[kMaxDevices] = {};
+unsigned g_epoch[kMaxDevices] = {};
 
 bool aligned_to(const void* ptr, size_t a) { return ((uintptr_t)ptr % a) == 0; }
 
-// Device address of the scratch on the current device.  In host code the
-// array's name is only a host-side stand-in; the kernel must get the address
-// cudaGetSymbolAddress returns with the device current.
-int scratch_for(int device, unsigned** out) {
+// Device address of the scratch on the current device, and the dataflow
+// engine's grid there.  In host code the array's name is only a host-side
+// stand-in; the kernels must get the address cudaGetSymbolAddress returns
+// with the device current.
+int scratch_for(int device, unsigned char** out, int* grid) {
   std::lock_guard<std::mutex> lk(g_mu);
   if (!g_scratch_ptr[device]) {
     void* ptr = nullptr;
-    if (cudaGetSymbolAddress(&ptr, g_noalloc_scratch) != cudaSuccess || !ptr) {
-      cudaGetLastError();
-      return MDS_ECUDA;
-    }
-    g_scratch_ptr[device] = static_cast<unsigned*>(ptr);
+    const cudaError_t e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch);
+    if (e != cudaSuccess || !ptr) return mds::record_cuda_error(e, "cudaGetSymbolAddress");
+    g_scratch_ptr[device] = static_cast<unsigned char*>(ptr);
+    g_grid[device] = mds::flow::grid_size(device);
   }
   *out = g_scratch_ptr[device];
+  *grid = g_grid[device];
   return MDS_OK;
+}
+
+unsigned next_epoch(int device) {
+  std::lock_guard<std::mutex> lk(g_mu);
+  g_epoch[device] = (g_epoch[device] + 1u == 0u) ? 1u : g_epoch[device] + 1u;
+  return g_epoch[device];
 }
 
 }  // namespace
@@ -57,8 +76,6 @@ extern "C" int mds_verify_noalloc(const mds_config* cfg_in, int device, const vo
     return MDS_EINVAL;
   if (scheme < MDS_SINGLE || scheme > MDS_WIS0) return MDS_EINVAL;
   if (B < 0 || B > c.max_B) return MDS_ESHAPE;
-  // the scratch this launch needs (it does not grow with B, K, L or V)
-  if (kScratchNeeded > MDS_NOALLOC_SCRATCH_BYTES) return MDS_ESHAPE;
   if (device < 0 || device >= kMaxDevices) return MDS_EINVAL;
   if (B == 0) return MDS_OK;
   if (!target_logits || !draft_logits || !draft_model_id || !draft_tokens || !temperatures || !out_tokens ||
@@ -86,13 +103,37 @@ extern "C" int mds_verify_noalloc(const mds_config* cfg_in, int device, const vo
 
   int prev = -1;
   cudaGetDevice(&prev);
-  if (prev != device && cudaSetDevice(device) != cudaSuccess) {
-    cudaGetLastError();
-    return MDS_ECUDA;
+  if (prev != device) {
+    const cudaError_t se = cudaSetDevice(device);
+    if (se != cudaSuccess) return mds::record_cuda_error(se, "cudaSetDevice");
   }
   int rc = mds::prepare_kernels(c.dtype);
-  unsigned* scratch = nullptr;
-  if (rc == MDS_OK) rc = scratch_for(device, &scratch);
+  unsigned char* scratch = nullptr;
+  int grid = 0;
+  if (rc == MDS_OK) rc = scratch_for(device, &scratch, &grid);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (rc == MDS_OK) {
+    // the dataflow engine where mds_verify takes it (same geometry: same results)
+    mds::flow::Params fp{};
+    if (mds::flow_params(c, grid, scheme, p.model_of, n_models, true, tma_ok, fp)) {
+      const size_t need = mds::flow::workspace_bytes(fp, B, grid);
+      if (kHead + need > MDS_NOALLOC_SCRATCH_BYTES) {
+        rc = MDS_ESHAPE;
+      } else {
+        mds::flow::carve_workspace(fp, reinterpret_cast<char*>(scratch + kHead), B, grid);
+        mds::flow_buffers(fp, target_logits, draft_logits, draft_tokens, temperatures, out_tokens, out_accept_len,
+                          out_diag, B, philox_seed);
+        fp.status = reinterpret_cast<unsigned*>(scratch);
+        fp.epoch = next_epoch(device);
+        cudaError_t e = cudaMemsetAsync(scratch, 0, kHead, st);
+        if (e == cudaSuccess) e = cudaMemsetAsync(scratch + kHead, 0, mds::flow::clear_bytes(fp, B, grid), st);
+        if (e == cudaSuccess) e = mds::flow::launch(fp, grid, st);
+        if (e != cudaSuccess) rc = mds::record_cuda_error(e, "mds_verify_noalloc launch");
+      }
+      if (prev >= 0 && prev != device) cudaSetDevice(prev);
+      return rc;
+    }
+  }
   p.dtype = c.dtype;
   if (rc == MDS_OK) rc = mds::launch_geometry(c, device, scheme, n_models, p);
   if (rc == MDS_OK) {
@@ -102,8 +143,8 @@ extern "C" int mds_verify_noalloc(const mds_config* cfg_in, int device, const vo
     p.out_tokens = out_tokens;
     p.out_accept = out_accept_len;
     p.out_diag = out_diag;
-    p.status = scratch;
-    p.queue = scratch + 1;
+    p.status = reinterpret_cast<unsigned*>(scratch);
+    p.queue = reinterpret_cast<unsigned*>(scratch) + 1;
     p.ticket0 = 0u;   // the counter is cleared below for every call
     p.seed = philox_seed;
     p.B = B;
@@ -120,12 +161,9 @@ extern "C" int mds_verify_noalloc(const mds_config* cfg_in, int device, const vo
     int clusters = mds::max_active_clusters(p);
     if (clusters < 1) clusters = 1;
     if (clusters > B) clusters = B;
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
-    if (cudaMemsetAsync(scratch, 0, kScratchNeeded, st) != cudaSuccess ||
-        mds::launch(p, clusters, st) != cudaSuccess) {
-      cudaGetLastError();
-      rc = MDS_ECUDA;
-    }
+    cudaError_t e = cudaMemsetAsync(scratch, 0, kScratchNeeded, st);
+    if (e == cudaSuccess) e = mds::launch(p, clusters, st);
+    if (e != cudaSuccess) rc = mds::record_cuda_error(e, "mds_verify_noalloc launch");
   }
   if (prev >= 0 && prev != device) cudaSetDevice(prev);
   return rc;

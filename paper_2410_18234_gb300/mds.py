@@ -15,7 +15,9 @@ import os
 import torch
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(_HERE, "_lib", "libmds.so")
+# MDS_LIBRARY may name another build of the same library (the instrumented
+# libmds_timers.so); the default is the in-tree libmds.so.
+LIB_PATH = os.environ.get("MDS_LIBRARY") or os.path.join(_HERE, "_lib", "libmds.so")
 
 MDS_SINGLE, MDS_IS, MDS_WIS, MDS_SPECTR, MDS_WIS0 = 0, 1, 2, 3, 4
 SCHEMES = {"single": MDS_SINGLE, "IS": MDS_IS, "WIS": MDS_WIS, "SpecTr": MDS_SPECTR, "WIS0": MDS_WIS0}
@@ -32,7 +34,7 @@ MDS_MAX_OMEGA0 = 30
 
 # every symbol include/mds.h declares
 EXPORTS = ("mds_create", "mds_verify", "mds_verify_host", "mds_verify_noalloc", "mds_status",
-           "mds_cluster_size", "mds_error_string", "mds_destroy")
+           "mds_cluster_size", "mds_phase_timers", "mds_error_string", "mds_destroy")
 
 
 class MdsConfig(ctypes.Structure):
@@ -68,6 +70,8 @@ def load_library(path=LIB_PATH):
     lib.mds_status.restype = ctypes.c_int
     lib.mds_cluster_size.argtypes = [vp]
     lib.mds_cluster_size.restype = ctypes.c_int
+    lib.mds_phase_timers.argtypes = [ctypes.c_int, ctypes.POINTER(ctypes.c_uint64), ctypes.c_int]
+    lib.mds_phase_timers.restype = ctypes.c_int
     lib.mds_error_string.argtypes = [ctypes.c_int]
     lib.mds_error_string.restype = ctypes.c_char_p
     lib.mds_destroy.argtypes = [vp]
@@ -114,11 +118,13 @@ def _ids(model_ids, K):
 
 
 def check_buffers(K, L, V, dtype, target, drafts, model_ids, tokens, temps, out_tokens, out_accept,
-                  out_diag=None, placement=None):
+                  out_diag=None, placement=None, device=None):
     """Shapes, element types, contiguity and placement ("cuda", "cpu" or None
-    to skip) of one call's tensors.  The C ABI takes bare pointers and the
-    sizes from its configuration, so a tensor of the wrong shape would be read
-    or written out of bounds: the binding rejects it first (MdsError with
+    to skip; with ``device``, the CUDA device index every tensor must be on)
+    of one call's tensors.  The C ABI takes bare pointers and the sizes from
+    its configuration, so a tensor of the wrong shape would be read or written
+    out of bounds, and a tensor on another GPU would be dereferenced by a
+    kernel running elsewhere: the binding rejects both first (MdsError with
     MDS_ESHAPE or MDS_EINVAL)."""
     st = TORCH_DTYPES[DTYPES[dtype] if isinstance(dtype, str) else int(dtype)]
     if len(model_ids) != K or len(drafts) < K:
@@ -139,6 +145,8 @@ def check_buffers(K, L, V, dtype, target, drafts, model_ids, tokens, temps, out_
             raise MdsError(MDS_EINVAL, f"{name} is not contiguous")
         if placement is not None and (t.device.type == "cuda") != (placement == "cuda"):
             raise MdsError(MDS_EINVAL, f"{name} is on {t.device}, expected {placement} memory")
+        if device is not None and t.device.type == "cuda" and t.device.index != int(device):
+            raise MdsError(MDS_EINVAL, f"{name} is on {t.device}, expected cuda:{int(device)}")
 
 
 def mds_verify(ctx, target, drafts, model_ids, tokens, temps, scheme, seed, out_tokens, out_accept,
@@ -186,13 +194,13 @@ def mds_verify_noalloc(max_B, K, L, V, target, drafts, model_ids, tokens, temps,
     memory (see include/mds.h): the configuration is passed directly and the
     kernel's scratch is a static device array inside the library."""
     check_buffers(int(K), int(L), int(V), dtype, target, drafts, model_ids, tokens, temps, out_tokens, out_accept,
-                  out_diag, "cuda")
+                  out_diag, "cuda", device=int(device))
     cfg = MdsConfig(int(max_B), int(K), int(L), int(V), DTYPES[dtype] if isinstance(dtype, str) else int(dtype),
                     int(wis_s), float(is_h), int(cluster), int(omega0), int(acc_prob))
     Kn = len(model_ids)
     B = int(tokens.shape[0])
     if stream is None:
-        stream = torch.cuda.current_stream().cuda_stream
+        stream = torch.cuda.current_stream(int(device)).cuda_stream
     elif isinstance(stream, torch.cuda.Stream):
         stream = stream.cuda_stream
     rc = _lib.mds_verify_noalloc(ctypes.byref(cfg), int(device), _ptr(target), _draft_ptrs(drafts, Kn),
@@ -214,6 +222,24 @@ def mds_status(ctx):
 
 def mds_cluster_size(ctx):
     return _lib.mds_cluster_size(ctx)
+
+
+PHASES = ("kernel", "wait_full", "task_list", "task_stats", "task_resid", "task_full", "dec_stats",
+          "dec_combine", "dec_stages", "dec_resid", "dec_full", "dec_bonus", "push", "sched_poll",
+          "sched_empty", "tasks", "decisions")
+
+
+def mds_phase_timers(device=0):
+    """Phase counters of an instrumented build (None for the default build):
+    a dict of SM cycles summed over CTAs per phase, and the task and decision
+    counts; reading clears them."""
+    buf = (ctypes.c_uint64 * 64)()
+    rc = _lib.mds_phase_timers(int(device), buf, 64)
+    if rc == MDS_EUNSUP:
+        return None
+    if rc < 0:
+        raise MdsError(rc, "mds_phase_timers")
+    return {name: int(buf[i]) for i, name in enumerate(PHASES[:rc])}
 
 
 def mds_destroy(ctx):
@@ -243,7 +269,9 @@ class Verifier:
         else:
             out_tokens, out_accept, out_diag = out
         check_buffers(self.K, self.L, self.V, self.dtype, target, drafts, model_ids, tokens, temps, out_tokens,
-                      out_accept, out_diag, "cuda")
+                      out_accept, out_diag, "cuda", device=self.device.index)
+        if stream is None:
+            stream = torch.cuda.current_stream(self.device)
         mds_verify(self.ctx, target, drafts, model_ids, tokens, temps, scheme, seed, out_tokens, out_accept,
                    out_diag, stream)
         return out_tokens, out_accept, out_diag

@@ -82,3 +82,43 @@ def test_bad_buffers_are_rejected(mds):
     bad[4] = w.temps.double()                                               # float64 temperatures
     expect(mds.MDS_EINVAL, bad)
     expect(mds.MDS_EINVAL, good, placement="cuda")                          # host tensors to the device entry
+
+
+class _OnDevice:
+    """A host tensor that reports a CUDA placement (shape, type and layout are
+    the tensor's): stands in for a tensor on another GPU without needing one."""
+
+    def __init__(self, t, index):
+        self._t = t
+        self.device = torch.device("cuda", index)
+
+    shape = property(lambda self: self._t.shape)
+    dtype = property(lambda self: self._t.dtype)
+
+    def dim(self):
+        return self._t.dim()
+
+    def is_contiguous(self):
+        return self._t.is_contiguous()
+
+
+def test_tensors_on_another_device_are_rejected(mds):
+    from synth import WORKLOADS, make_workload
+    spec = WORKLOADS["tiny"].with_(B=2, V=64)
+    w = make_workload(spec, device="cpu")
+    on = lambda t, i: _OnDevice(t, i)  # noqa: E731
+    outs = _outs(spec.B, spec.L)
+    args = [on(w.target, 0), [on(d, 0) for d in w.draft_list()], w.model_ids, on(w.tokens, 0), on(w.temps, 0)]
+    good_outs = [on(outs[0], 0), on(outs[1], 0), on(outs[2], 0)]
+    mds.check_buffers(spec.K, spec.L, spec.V, spec.dtype, *args, *good_outs, placement="cuda", device=0)
+    for i in range(len(good_outs)):
+        bad = list(good_outs)
+        bad[i] = on(outs[i], 1)
+        with pytest.raises(mds.MdsError) as e:
+            mds.check_buffers(spec.K, spec.L, spec.V, spec.dtype, *args, *bad, placement="cuda", device=0)
+        assert e.value.code == mds.MDS_EINVAL
+    bad_args = list(args)
+    bad_args[0] = on(w.target, 1)
+    with pytest.raises(mds.MdsError) as e:
+        mds.check_buffers(spec.K, spec.L, spec.V, spec.dtype, *bad_args, *good_outs, placement="cuda", device=0)
+    assert e.value.code == mds.MDS_EINVAL

@@ -120,6 +120,32 @@ def test_mixed_models_and_temperatures():
         check(run_both(spec, scheme, seed=13), scheme)
 
 
+def test_more_draft_models_than_a_candidate_list_holds():
+    # five distinct draft models: six rows per depth, more than the candidate
+    # list carries, so every WIS stage is a full-vocabulary pass; also the
+    # stage LP with s = 8 (pair state outside the five-token fast path)
+    spec = WorkloadSpec("five", B=12, K=5, L=3, V=3000, dtype="bf16", model_ids=[0, 1, 2, 3, 4], target_scale=3.0,
+                        draft_sigma=[0.4, 0.8, 1.2, 1.6, 2.0], t_target=1.0, t_draft=[1.0, 1.3, 0.8, 1.1, 0.9],
+                        data_seed=29)
+    for wis_s in (5, 8):
+        check(run_both(spec, "WIS", seed=21, wis_s=wis_s), "WIS")
+    check(run_both(spec, "single", seed=21), "single")
+
+
+def test_small_slices_and_flat_rows():
+    # small batches cut each row into many small slices (threads without a
+    # unit), and nearly flat target rows put many tokens at the top: the
+    # candidate threshold and its overflow path
+    spec = WorkloadSpec("flat", B=4, K=4, L=3, V=1283, dtype="bf16", model_ids=[0] * 4, target_scale=0.02,
+                        draft_sigma=[0.01], t_target=1.0, t_draft=[1.0], data_seed=31)
+    for scheme in ("WIS", "single"):
+        check(run_both(spec, scheme, seed=2), scheme)
+    spec = WorkloadSpec("ramp", B=3, K=3, L=2, V=4096, dtype="f32", model_ids=[0] * 3, target_scale=0.0,
+                        draft_sigma=[0.5], t_target=1.0, t_draft=[1.0], data_seed=33)
+    for scheme in ("WIS", "single"):
+        check(run_both(spec, scheme, seed=4), scheme)
+
+
 FULL = [
     ("tiny", ["IS", "WIS", "single", "SpecTr"], None),
     ("llama2-32k", ["IS", "WIS"], [0, 1, 31, 63]),
