@@ -52,6 +52,10 @@ def parse():
     ap.add_argument("--K", type=int, default=0, help="override the branch count, keeping the first K branches' "
                                                     "draft models (profiling on a small case)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-cpu-all", action="store_true", help="skip the all-core oracle baseline")
+    ap.add_argument("--table", action="store_true", help="every workload x scheme (not the driver's bench line)")
+    ap.add_argument("--table-out", default=None)
+    ap.add_argument("--only", default=None, help="--table: comma-separated workloads or workload/scheme")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-parity", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
@@ -66,6 +70,7 @@ def walk_accounting(tokens, model_ids, out_tokens, acc, V, esize, scheme="WIS", 
     """Rows the walk consumed per sequence, replayed from the outputs:
     returns (vocab_rows, algorithmic_bytes) summed over the batch.  A depth
     verifies its target row and one row per distinct draft model (vocab-rows);
+    the single-draft scheme needs only the lowest valid branch's draft row;
     the truncated alphabet reads only the target row in full and each draft
     row at the at most omega0 tokens of Omega_0, which is what its bytes count."""
     B, K, L = tokens.shape
@@ -78,7 +83,7 @@ def walk_accounting(tokens, model_ids, out_tokens, acc, V, esize, scheme="WIS", 
             if j == L:
                 rows += 1
                 break
-            d = len(np.unique(mids[valid]))
+            d = 1 if scheme == "single" else len(np.unique(mids[valid]))
             rows += 1 + d
             point += d
             z = out_tokens[b, j]
@@ -144,6 +149,13 @@ class ClockSampler:
 
 
 # ----------------------------------------------------------------- peaks / traffic
+
+
+def kernel_name(scheme, cluster):
+    """The kernel a call ran: the slice-dataflow engine's for single, WIS and
+    WIS0 (the library reports cluster size 0 for it), the per-sequence
+    engine's otherwise."""
+    return "flow_kernel" if cluster == 0 and scheme in ("single", "WIS", "WIS0") else "verify_kernel"
 
 
 def hbm_peak():
@@ -212,6 +224,51 @@ def oracle_rate(w, scheme, seconds, seqs=None, omega0=20):
     return rows / t_total, f"{len(done)} of {spec.B} sequences (first {len(done)}), {t_total:.1f} s", outs
 
 
+def _oracle_seq(job):
+    """One sequence through the oracle (a worker of the all-core baseline)."""
+    host, scheme, seed, b, omega0, V, es = job
+    from oracle.verify import oracle_verify
+    o, a, _ = oracle_verify(*host, scheme, seed, seq_ids=[b], omega0=omega0)
+    out = np.asarray(o[b])[None]
+    r, _ = walk_accounting(host[3], host[2], out, np.array([a[b]]), V, es, scheme, omega0)
+    return r
+
+
+def oracle_rate_all_cores(w, scheme, seconds, omega0=20, cores=None):
+    """The oracle, as it stands, on every host core: one process per core
+    (spawned, so no CUDA state is inherited), sequences handed out in order
+    until the time budget is spent; the rate is the rows finished over the
+    wall time of the timed region (pool start-up excluded)."""
+    import multiprocessing as mp
+    from synth import host_copy
+    spec = w.spec
+    es = 4 if spec.dtype == "f32" else 2
+    cores = cores or os.cpu_count() or 1
+    ctx = mp.get_context("spawn")
+    with ctx.Pool(cores) as pool:
+        pool.map(_warm, range(cores))
+        pending, rows, done = [], 0, 0
+        t0 = time.perf_counter()
+        b = 0
+        while True:
+            while b < spec.B and len(pending) < 2 * cores and time.perf_counter() - t0 < seconds:
+                job = (host_copy(w, [b]), scheme, spec.verify_seed, b, omega0, spec.V, es)
+                job = ((job[0][0], job[0][1], job[0][2], job[0][3], job[0][4]), *job[1:])
+                pending.append(pool.apply_async(_oracle_seq, (job,)))
+                b += 1
+            if not pending:
+                break
+            rows += pending.pop(0).get()
+            done += 1
+        wall = time.perf_counter() - t0
+    return rows / wall, f"{done} of {spec.B} sequences on {cores} processes, {wall:.1f} s", cores
+
+
+def _warm(_):
+    import oracle.verify  # noqa: F401
+    return 0
+
+
 def agreement(g_tok, g_acc, outs):
     """GPU vs oracle on the sequences the oracle finished: identical, within
     the band (first differing decision flagged by the oracle), or mismatched."""
@@ -252,11 +309,102 @@ def combine_ranks(rows, abytes, ms, world, device):
     return int(round(t[0].item())), int(round(t[1].item())), float(m[0].item())
 
 
+# ----------------------------------------------------------------- table of every workload and scheme
+
+TABLE = [("tiny", "IS"), ("llama2-32k", "IS"), ("llama2-32k", "WIS"), ("two-models-50k", "WIS"),
+         ("two-models-50k", "SpecTr"), ("llama3-128k", "WIS"), ("llama3-128k", "WIS0"),
+         ("serving-152k", "single"), ("serving-152k", "IS"), ("serving-152k", "WIS"), ("serving-152k", "SpecTr"),
+         ("serving-152k-k2", "single"), ("serving-152k-k2", "IS"), ("serving-152k-k2", "WIS"),
+         ("serving-152k-k2", "SpecTr")]
+
+
+def table(args):
+    """Every workload x scheme of the benchmark set on one GPU: median step
+    time (CUDA events, L2 flushed between steps), rows/s, algorithmic GB/s and
+    its fraction of the measured HBM peak, oracle agreement and the oracle's
+    one-core rate on a bounded sample.  One JSON line per entry, then a
+    markdown table (to --table-out if given)."""
+    import torch
+    from paper_2410_18234_gb300 import mds
+    from synth import WORKLOADS, make_workload
+    dev = torch.device("cuda", 0)
+    peak, peak_kind = hbm_peak()
+    flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+    rows_md = []
+    want = None if not args.only else set(args.only.split(","))
+    for name, scheme in TABLE:
+        if want and f"{name}/{scheme}" not in want and name not in want:
+            continue
+        spec = WORKLOADS[name]
+        es = 4 if spec.dtype == "f32" else 2
+        w = make_workload(spec, device=dev)
+        v = mds.Verifier(spec.B, spec.K, spec.L, spec.V, dtype=spec.dtype, device=0, omega0=args.omega0)
+        out_tokens = torch.empty(spec.B, spec.L + 1, dtype=torch.int32, device=dev)
+        out_acc = torch.empty(spec.B, dtype=torch.int32, device=dev)
+        stream = torch.cuda.current_stream(dev)
+
+        def step():
+            mds.mds_verify(v.ctx, w.target, w.draft_list(), w.model_ids, w.tokens, w.temps, scheme,
+                           spec.verify_seed, out_tokens, out_acc, None, stream)
+
+        for _ in range(args.warmup):
+            flush.fill_(1.0)
+            step()
+        torch.cuda.synchronize()
+        times = []
+        for _ in range(args.steps):
+            flush.fill_(1.0)
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            step()
+            b.record(stream)
+            torch.cuda.synchronize()
+            times.append(a.elapsed_time(b))
+        ms = float(np.median(times))
+        tok = w.tokens.cpu().numpy()
+        o_tok, o_acc = out_tokens.cpu().numpy(), out_acc.cpu().numpy()
+        rows, abytes = walk_accounting(tok, w.model_ids, o_tok, o_acc, spec.V, es, scheme, args.omega0)
+        gbs = abytes / (ms * 1e-3) / 1e9
+        rate, desc, outs = oracle_rate(w, scheme, args.cpu_seconds, omega0=args.omega0)
+        par = agreement(o_tok, o_acc, outs)
+        bits, _ = v.status()
+        cn = v.cluster_size
+        v.close()
+        line = {"workload": name, "scheme": scheme, "B": spec.B, "K": spec.K, "L": spec.L, "V": spec.V,
+                "logits": spec.dtype, "ms_per_step": ms, "ms_mean": float(np.mean(times)),
+                "rows_per_s": rows / (ms * 1e-3), "vocab_rows_per_step": rows, "gb_per_s": gbs,
+                "hbm_frac": gbs / peak, "peak": peak, "peak_kind": peak_kind, "kernel": kernel_name(scheme, cn),
+                "block_efficiency": float(np.mean(o_acc + 1)), "oracle_agreement": par,
+                "cpu_1core_rows_per_s": rate, "cpu_sample": desc, "status_bits": bits}
+        print(json.dumps(line), flush=True)
+        rows_md.append(line)
+        del w
+        torch.cuda.empty_cache()
+    md = ["| workload | scheme | kernel | ms/step (median) | vocab-rows/s | GB/s | frac of measured HBM | "
+          "block eff. | oracle agreement (identical/band/mismatch of n) | oracle 1 core rows/s |",
+          "|---|---|---|---|---|---|---|---|---|---|"]
+    for r in rows_md:
+        a = r["oracle_agreement"]
+        md.append(f"| {r['workload']} | {r['scheme']} | {r['kernel']} | {r['ms_per_step']:.3f} | "
+                  f"{r['rows_per_s'] / 1e6:.2f}M | {r['gb_per_s']:.0f} | {r['hbm_frac']:.3f} | "
+                  f"{r['block_efficiency']:.2f} | {a['identical']}/{a['band']}/{a['mismatch']} of {a['sequences']} | "
+                  f"{r['cpu_1core_rows_per_s']:.1f} |")
+    text = "\n".join(md)
+    if args.table_out:
+        with open(args.table_out, "w") as fh:
+            fh.write(text + "\n")
+    else:
+        print(text)
+    return 0
+
+
 # ----------------------------------------------------------------- main
 
 
 def main():
     args = parse()
+    if args.table:
+        return table(args)
     import torch
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -348,7 +496,8 @@ def main():
         dist.barrier()
     clk = clocks.stop() if clocks else None
     times = [s.elapsed_time(e) for s, e in zip(starts, ends)]
-    ms_own = float(np.mean(times))
+    ms_own = float(np.median(times))
+    ms_mean = float(np.mean(times))
 
     tok = w.tokens.cpu().numpy()
     o_tok = out_tokens.cpu().numpy()
@@ -389,12 +538,16 @@ def main():
 
     # ------------------------------------------------------------- oracle agreement + cpu baseline
     cpu = None
+    cpu_all = None
     parity = None
     if rank == 0 and world == 1 and not (args.no_cpu_baseline and args.no_parity):
         rate, desc, outs = oracle_rate(w, scheme, args.cpu_seconds, omega0=args.omega0)
         parity = agreement(o_tok, o_acc, outs)
         if not args.no_cpu_baseline:
             cpu = {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc}
+            if not args.no_cpu_all:
+                r_all, d_all, cores = oracle_rate_all_cores(w, scheme, args.cpu_seconds, omega0=args.omega0)
+                cpu_all = {"value": r_all, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": d_all}
 
     bits, msg = v.status()
     cn = v.cluster_size
@@ -402,7 +555,8 @@ def main():
     if rank == 0:
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "warmup": args.warmup, "ms_per_step": ms, "ms_mean": ms_mean, "higher_is_better": True,
+            "scaling": "weak",
             "vs_baseline": None, "dtype": "f32", "data": "synthetic",
             "config": {"workload": spec.name, "B": spec.B, "K": spec.K, "L": spec.L, "V": spec.V,
                        "logits": spec.dtype, "scheme": scheme, "cluster": cn, "l2_flush": True,
@@ -411,8 +565,9 @@ def main():
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "peak_kind": peak_kind,
                          "traffic": None if (args.B or args.K) else recorded_traffic(spec.name, scheme),
-                         "algorithmic_bytes_per_launch": int(abytes), "kernel": "verify_kernel"},
+                         "algorithmic_bytes_per_launch": int(abytes), "kernel": kernel_name(scheme, cn)},
             "cpu_baseline": cpu,
+            "cpu_baseline_all_cores": cpu_all,
             "e2e": e2e,
             "gpu_launches": args.steps,
             "clocks": clk,

@@ -47,11 +47,10 @@ constexpr int kCW = 8;                 // compute warps
 constexpr int kCT = kCW * 32;          // compute threads
 constexpr int kBlock = kCT + 32;       // + the scheduler warp
 constexpr int kNBuf = 2;               // slice buffers per CTA
-constexpr int kCandCap = 1024;         // candidate tokens one slice may set aside
+constexpr int kCandCap = 512;          // candidate tokens one slice may set aside
 constexpr int kListMax = 64;           // candidate list length at most
 constexpr int kHdr = 2 * kMaxRows + 2; // record: (max, sum) per row, tau, list length
 constexpr int kTopF = 8;               // per-thread candidates of a full stage (>= MDS_MAX_S)
-constexpr int kTopW = 8;               // thread maxima each warp offers to the slice's threshold
 constexpr unsigned long long kWaitNs = 2000000000ull;   // 2 s bound on every wait
 constexpr unsigned FULLM = 0xffffffffu;
 static_assert(kHdr % 4 == 0, "record header keeps 16-byte alignment");
@@ -76,6 +75,12 @@ enum : int {
   kPhPush,              // publishing the next pass
   kPhSchedPoll,         // scheduler waiting for a published task
   kPhSchedEmpty,        // scheduler waiting for a free buffer
+  kPhListA,             // list tasks: maxima and the candidate threshold
+  kPhListB,             // list tasks: the sums and the candidates
+  kPhListC,             // list tasks: ranking and the record
+  kPhPublish,           // a task's record publication (fence, pass counter)
+  kPhLp,                // the stage LPs (one thread)
+  kPhLpCalls,           // count: stage LPs
   kPhTasks,             // count: slice tasks
   kPhDecisions,         // count: decisions
   kPhaseN
@@ -119,10 +124,11 @@ struct __align__(16) FSeq {
   FWalk W;
 };
 
-struct FDesc {
+struct __align__(16) FDesc {
   FPass P;
   int b, slice, exit, pad;
 };
+static_assert(sizeof(FDesc) % 16 == 0, "descriptor moves in 16-byte chunks");
 
 struct Cand {  // full-stage candidate: larger key first, then smaller token id
   float key;
@@ -139,6 +145,8 @@ struct DState {                // the decision's working state (shared memory)
   FWalk W;
   int nv;
   int vbr[MDS_MAX_K], X[MDS_MAX_K], vrow[MDS_MAX_K];
+  float xl[MDS_MAX_K][kMaxRows];   // every row's logit at each valid draft token (X[k])
+  int xl_ok;
   // candidate list (token-id order)
   int n, cand_all;
   float cand_q, cand_tau;
@@ -156,6 +164,8 @@ struct DState {                // the decision's working state (shared memory)
   float A2, B2;
   int Y, fast_ok;
   Cand fin[kTopF];
+  float lp_rs[kMaxPairs], lp_fl[kMaxPairs], lp_fh[kMaxPairs];   // LP pair state in shared memory
+  float lp_rd[MDS_MAX_S];
   // search
   int seg, cross, lastp, tok;
   float run;
@@ -170,12 +180,12 @@ struct DState {                // the decision's working state (shared memory)
 struct FShared {
   uint64_t full[kNBuf], empty[kNBuf];
   FDesc desc[kNBuf];
+  FDesc pend;                  // the scheduler's next task, resolved ahead
   float red[kCW * 2 * kMaxRows];
   float mrow[kMaxRows];
   float wth[kCW];
   int ncand, last, issued, consumed;
-  float theta, addtau;
-  unsigned tkey[kCW * 8];       // the warps' largest thread maxima (order-preserving keys)
+  float addtau;
   float add[kMaxRows];
   uint32_t bitmap[64];         // one bit per 16-byte unit of a slice holding a special token
   Cand wcand[kCW * kTopF];
@@ -203,6 +213,11 @@ __device__ __forceinline__ unsigned ld_relaxed(const unsigned* a) {
   unsigned v;
   asm volatile("ld.relaxed.gpu.u32 %0, [%1];" : "=r"(v) : "l"(a) : "memory");
   return v;
+}
+__device__ __forceinline__ unsigned atom_add_acq_rel(unsigned* a, unsigned v) {
+  unsigned old;
+  asm volatile("atom.add.acq_rel.gpu.u32 %0, [%1], %2;" : "=r"(old) : "l"(a), "r"(v) : "memory");
+  return old;
 }
 __device__ __forceinline__ unsigned long long now_ns() {
   unsigned long long t;
@@ -273,8 +288,17 @@ struct Eng {
   __device__ __forceinline__ uint4 raw(const char* b, int r, int u) const {
     return *reinterpret_cast<const uint4*>(srow(b, r) + 16 * u);
   }
+  // Logit of row r at token x: from the decision's cache when x is one of
+  // the depth's draft tokens (the intermediate token always is), else a load.
+  __device__ __forceinline__ float logit_at(const FPass& P, int r, int x) const {
+    const DState& D = S.D;
+    if (D.xl_ok)
+      for (int k = 0; k < D.nv; ++k)
+        if (D.X[k] == x) return D.xl[k][r];
+    return E::global(P.row[r].ptr, x);
+  }
   __device__ __forceinline__ float prob_row(const FPass& P, int r, int x) const {
-    return prob_of(E::global(P.row[r].ptr, x), P.row[r].M, P.row[r].c, P.row[r].invZ);
+    return prob_of(logit_at(P, r, x), P.row[r].M, P.row[r].c, P.row[r].invZ);
   }
   __device__ __forceinline__ float spec_lookup(const FPass& P, int tok, float fallback) const {
     for (int i = 0; i < P.nspec; ++i)
@@ -382,9 +406,212 @@ struct Eng {
     }
   }
 
-  __device__ void scheduler() {
+  // Warp-parallel plan_rows (one lane per branch): the same rows in the same
+  // order, the valid branches, their tokens and rows; then every row's logit
+  // at each draft token into the decision's cache.  Warp 0 of a decision.
+  __device__ void plan_warp(int b, int j, unsigned valid, bool bonus, bool set_pass) {
+    DState& D = S.D;
+    FPass& P = D.P;
+    const int lane = threadIdx.x & 31;
+    const int K = p.K;
+    const bool v = !bonus && lane < K && ((valid >> lane) & 1u);
+    const int m = v ? (int)p.model_of[lane] : 64 + lane;
+    const unsigned same = __match_any_sync(FULLM, m);
+    const bool first = v && (__ffs(same) - 1) == lane;
+    const unsigned fm = __ballot_sync(FULLM, first);
+    const unsigned vm = __ballot_sync(FULLM, v);
+    const int nr = 1 + __popc(fm);
+    const int myrow = first ? 1 + __popc(fm & ((1u << lane) - 1u)) : 0;
+    const int row = __shfl_sync(FULLM, myrow, __ffs(same) - 1);
+    if (v) {
+      const int i = __popc(vm & ((1u << lane) - 1u));
+      int x = p.tokens[((size_t)b * K + lane) * p.L + j];
+      if (x < 0 || x >= p.V) {
+        atomicOr(p.status, MDS_ST_BADTOKEN);
+        x = 0;
+      }
+      D.vbr[i] = lane;
+      D.X[i] = x;
+      D.vrow[i] = row;
+    }
+    if (set_pass && first) {
+      P.row[myrow].ptr = p.drafts[lane] + (((size_t)b * p.L + j) * (size_t)p.V) * p.esize;
+      float td = p.temps[(size_t)b * (1 + K) + 1 + lane];
+      if (!(td > 0.f) || !(td < kPosInf)) {
+        atomicOr(p.status, MDS_ST_BADTEMP);
+        td = 1.f;
+      }
+      P.row[myrow].c = __fdiv_rn(kLog2e, td);
+      P.row[myrow].M = 0.f;
+      P.row[myrow].invZ = 0.f;
+      P.row[myrow].gamma = 0.f;
+    }
+    if (lane == 0) {
+      D.nv = __popc(vm);
+      if (set_pass) {
+        const int kstar = __ffs(valid) - 1;
+        P.row[0].ptr = p.target + ((((size_t)b * K + kstar) * (p.L + 1) + j) * (size_t)p.V) * p.esize;
+        float tq = p.temps[(size_t)b * (1 + K)];
+        if (!(tq > 0.f) || !(tq < kPosInf)) {
+          atomicOr(p.status, MDS_ST_BADTEMP);
+          tq = 1.f;
+        }
+        P.row[0].c = __fdiv_rn(kLog2e, tq);
+        P.row[0].M = 0.f;
+        P.row[0].invZ = 0.f;
+        P.row[0].gamma = 0.f;
+        P.nrows = nr;
+        P.j = j;
+        P.nspec = 0;
+        P.rb = 0;
+        P.cut = 0.f;
+        P.all0 = 0;
+        if (bonus) {
+          P.kind = kBonus;
+          P.nstream = 1;
+          P.list = 0;
+        } else {
+          P.kind = kStats;
+          if (p.scheme == MDS_WIS0) {
+            P.nstream = 1;
+            P.list = 1;
+          } else if (p.scheme == MDS_WIS) {
+            P.nstream = nr;
+            P.list = (__popc(vm) > 1 && nr <= kListRowsMax && p.ln > 0) ? 1 : 0;
+          } else {
+            P.nstream = min(2, nr);
+            P.list = 0;
+          }
+        }
+      }
+    }
+    __syncwarp();
+    // the cache: row r's logit at X[k] for every valid branch k
+    const int nv = D.nv, nrow = P.nrows;
+    for (int i = lane; i < nv * nrow; i += 32) {
+      const int k = i / nrow, r = i - k * nrow;
+      D.xl[k][r] = E::global(P.row[r].ptr, D.X[k]);
+    }
+    if (lane == 0) D.xl_ok = bonus ? 0 : 1;
+    __syncwarp();
+  }
+
+  // Warp-parallel plan of a sequence's depth-0 pass (every branch valid):
+  // lane k < K takes branch k, and a draft model's row is that of its first
+  // branch (the same rows, in the same order, as plan_rows).
+  __device__ void plan_depth0_warp(int b, FPass& P) const {
+    const int lane = threadIdx.x & 31;
+    const int K = p.K;
+    const int m = (lane < K) ? (int)p.model_of[lane] : 64 + lane;
+    const unsigned same = __match_any_sync(FULLM, m);
+    const bool first = lane < K && (__ffs(same) - 1) == lane;
+    const unsigned fm = __ballot_sync(FULLM, first);
+    const int nr = 1 + __popc(fm);
+    if (first) {
+      const int r = 1 + __popc(fm & ((1u << lane) - 1u));
+      P.row[r].ptr = p.drafts[lane] + ((size_t)b * p.L * (size_t)p.V) * p.esize;
+      float td = p.temps[(size_t)b * (1 + K) + 1 + lane];
+      if (!(td > 0.f) || !(td < kPosInf)) {
+        atomicOr(p.status, MDS_ST_BADTEMP);
+        td = 1.f;
+      }
+      P.row[r].c = __fdiv_rn(kLog2e, td);
+      P.row[r].M = 0.f;
+      P.row[r].invZ = 0.f;
+      P.row[r].gamma = 0.f;
+    }
+    if (lane == 0) {
+      P.row[0].ptr = p.target + ((size_t)b * K * (p.L + 1) * (size_t)p.V) * p.esize;
+      float tq = p.temps[(size_t)b * (1 + K)];
+      if (!(tq > 0.f) || !(tq < kPosInf)) {
+        atomicOr(p.status, MDS_ST_BADTEMP);
+        tq = 1.f;
+      }
+      P.row[0].c = __fdiv_rn(kLog2e, tq);
+      P.row[0].M = 0.f;
+      P.row[0].invZ = 0.f;
+      P.row[0].gamma = 0.f;
+      P.nrows = nr;
+      P.j = 0;
+      P.nspec = 0;
+      P.rb = 0;
+      P.cut = 0.f;
+      P.all0 = 0;
+      P.kind = kStats;
+      if (p.scheme == MDS_WIS0) {
+        P.nstream = 1;
+        P.list = 1;
+      } else if (p.scheme == MDS_WIS) {
+        P.nstream = nr;
+        P.list = (K > 1 && nr <= kListRowsMax && p.ln > 0) ? 1 : 0;
+      } else {
+        P.nstream = min(2, nr);
+        P.list = 0;
+      }
+    }
+  }
+
+  // Claim the next task number and resolve it into Pd: the sequence, the
+  // slice and the sequence's pass descriptor (depth-0 tasks are implicit:
+  // task t < B * ns is slice t % ns of sequence t / ns).  Returns 0 when no
+  // work is left (every sequence finished, or an abort).  Warp-wide.
+  __device__ int resolve(FDesc& Pd) {
     const int lane = threadIdx.x & 31;
     const unsigned N0 = (unsigned)p.B * (unsigned)p.ns;
+    int have = 0, b = 0, s = 0;
+    if (lane == 0 && !aborted()) {
+      const unsigned t = atomicAdd(&p.ctl[kCtlHead], 1u);
+      if (t < N0) {
+        b = (int)(t / (unsigned)p.ns);
+        s = (int)(t % (unsigned)p.ns);
+        st_release(&p.ring_rtag[t % (unsigned)p.ring_cap], tag_of(t));
+        have = 1;
+      } else {
+        const unsigned slot = t % (unsigned)p.ring_cap;
+        const unsigned long long want = tag_of(t);
+        const unsigned long long t0 = now_ns();
+        PT_T0(t_poll);
+        for (int it = 0;; ++it) {
+          if (ld_acquire(&p.ring_tag[slot]) == want) {
+            const unsigned pay = __ldcg(&p.ring_pay[slot]);
+            b = (int)(pay >> 16);
+            s = (int)(pay & 0xffffu);
+            st_release(&p.ring_rtag[slot], want);
+            have = 2;
+            break;
+          }
+          if (ld_relaxed(&p.ctl[kCtlDone]) >= (unsigned)p.B || aborted()) break;
+          if ((it & 15) == 15 && now_ns() - t0 > kWaitNs) {
+            set_abort(MDS_ST_TIMEOUT);
+            break;
+          }
+          __nanosleep(it < 16 ? 32 : 256);
+        }
+        PT_ADD(kPhSchedPoll, t_poll);
+      }
+    }
+    have = __shfl_sync(FULLM, have, 0);
+    b = __shfl_sync(FULLM, b, 0);
+    s = __shfl_sync(FULLM, s, 0);
+    if (have == 1)
+      plan_depth0_warp(b, Pd.P);
+    else if (have == 2)
+      copy_in(&Pd.P, &reinterpret_cast<const FSeq*>(p.seq)[b].P, (int)sizeof(FPass), lane, 32);
+    if (lane == 0) {
+      Pd.b = b;
+      Pd.slice = s;
+      Pd.exit = have ? 0 : 1;
+    }
+    __syncwarp();
+    return have != 0;
+  }
+
+  // The scheduler warp: the next task is resolved ahead (while the compute
+  // warps work on the other buffer), so that a freed buffer only waits for
+  // the descriptor move and the bulk copies.
+  __device__ void scheduler() {
+    const int lane = threadIdx.x & 31;
+    int have = resolve(S.pend);
     for (int k = 0;; ++k) {
       const int bi = k % kNBuf;
       FDesc& D = S.desc[bi];
@@ -399,52 +626,15 @@ struct Eng {
         if (lane == 0) set_abort(MDS_ST_TIMEOUT);
         return;
       }
-      unsigned t = 0;
-      int have = 0, b = 0, s = 0;
-      if (lane == 0 && !aborted()) {
-        t = atomicAdd(&p.ctl[kCtlHead], 1u);
-        if (t < N0) {
-          b = (int)(t / (unsigned)p.ns);
-          s = (int)(t % (unsigned)p.ns);
-          st_release(&p.ring_rtag[t % (unsigned)p.ring_cap], tag_of(t));
-          plan_rows(b, 0, (p.K >= 32) ? FULLM : ((1u << p.K) - 1u), false, &D.P, nullptr, nullptr, nullptr, nullptr);
-          have = 1;
-        } else {
-          const unsigned slot = t % (unsigned)p.ring_cap;
-          const unsigned long long want = tag_of(t);
-          const unsigned long long t0 = now_ns();
-          PT_T0(t_poll);
-          for (int it = 0;; ++it) {
-            if (ld_acquire(&p.ring_tag[slot]) == want) {
-              const unsigned pay = __ldcg(&p.ring_pay[slot]);
-              b = (int)(pay >> 16);
-              s = (int)(pay & 0xffffu);
-              st_release(&p.ring_rtag[slot], want);
-              have = 2;
-              break;
-            }
-            if (ld_relaxed(&p.ctl[kCtlDone]) >= (unsigned)p.B || aborted()) break;
-            if ((it & 15) == 15 && now_ns() - t0 > kWaitNs) {
-              set_abort(MDS_ST_TIMEOUT);
-              break;
-            }
-            __nanosleep(it < 16 ? 32 : 256);
-          }
-          PT_ADD(kPhSchedPoll, t_poll);
-        }
-      }
-      have = __shfl_sync(FULLM, have, 0);
-      b = __shfl_sync(FULLM, b, 0);
-      s = __shfl_sync(FULLM, s, 0);
-      if (have == 2) copy_in(&D.P, &reinterpret_cast<const FSeq*>(p.seq)[b].P, (int)sizeof(FPass), lane, 32);
-      if (lane == 0) {
-        D.b = b;
-        D.slice = s;
-        D.exit = have ? 0 : 1;
+      {
+        const int4* src = reinterpret_cast<const int4*>(&S.pend);
+        int4* dst = reinterpret_cast<int4*>(&D);
+        for (int i = lane; i < (int)(sizeof(FDesc) / 16); i += 32) dst[i] = src[i];
       }
       __syncwarp();
       if (lane == 0) {
         if (have && p.bulk) {
+          const int s = D.slice;
           const int tok0 = s * p.T;
           const int n = min(p.T, p.V - tok0);
           const uint32_t bytes = (uint32_t)n * (uint32_t)p.esize;
@@ -459,6 +649,7 @@ struct Eng {
       }
       __syncwarp();
       if (!have) return;
+      have = resolve(S.pend);
     }
   }
 
@@ -542,18 +733,30 @@ struct Eng {
 
   // -------------------------------------------------------------- stats task
   // R rows (compile time, at most kListRowsMax) with or without the candidate
-  // list.  Record: (max, sum) per row, tau (largest target logit of the slice
-  // outside its list), list length, then the list (larger target logit
-  // first, ties to the smaller id): ids, then each row's logits.
+  // list, in two passes over the slice in shared memory.  Pass A: every
+  // row's maximum (the slice's exponent reference) and the candidate
+  // threshold theta: the smallest of the warps' largest target logits, so
+  // that at least one token per warp is >= theta (theta = -inf for a slice
+  // of at most kCandCap tokens: every token is a candidate).  Pass B: every
+  // row's sum of 2^(l c - m c) over the tokens that are not candidates (the
+  // candidates, target logit > theta, are set aside with every row's logit).
+  // Then the candidates are ranked (larger target logit first, ties to the
+  // smaller id): the first LN form the slice's list, the others rejoin the
+  // sums in rank order.  tau = the largest target logit outside the list.
+  // Should more than kCandCap tokens pass theta, theta is raised to the
+  // kCandCap-th largest target logit (bisection) and pass B repeated.
+  // Record: (max, sum) per row, tau, list length, then the list: ids, then
+  // each row's logits.
   template <int R, bool LIST>
   __device__ void stats_small(const FPass& P, const char* b, int tok0, int n, float* rec) {
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int U = (n + VE - 1) / VE;
-    const int LN = p.ln;
+    const int LN = p.lns;   // this slice's list length
     float c[R];
 #pragma unroll
     for (int r = 0; r < R; ++r) c[r] = P.row[r].c;
-    // phase A: maxima
+    // pass A: maxima
+    PT_T0(t_a);
     float tmax = kNegInf;
 #pragma unroll
     for (int r = 0; r < R; ++r) {
@@ -564,40 +767,20 @@ struct Eng {
       if (lane == 0) S.red[warp * kMaxRows + r] = mx;
     }
     if constexpr (LIST) {
-      // each warp's kTopW largest thread maxima (distinct tokens) ...
+      // this warp's k-th largest thread maximum (distinct tokens), k = LN / kCW
+      // rounded up: every warp then holds k tokens >= its value
+      const int k = (LN + kCW - 1) / kCW;
       unsigned key = (tmax > kNegInf) ? ord_key(__fadd_rn(tmax, 0.f)) : 0u;
-      for (int t = 0; t < kTopW; ++t) {
-        const unsigned km = __reduce_max_sync(FULLM, key);
-        const unsigned who = __ballot_sync(FULLM, km != 0u && key == km);
-        if (lane == 0) S.tkey[warp * kTopW + t] = km;
-        if (who && lane == __ffs(who) - 1) key = 0u;
+      unsigned km = 0u;
+      for (int t = 0; t < k; ++t) {
+        km = __reduce_max_sync(FULLM, key);
+        if (!km) break;
+        const unsigned who = __ballot_sync(FULLM, key == km);
+        if (lane == __ffs(who) - 1) key = 0u;
       }
+      if (lane == 0) S.wth[warp] = km ? ord_val(km) : kNegInf;
     }
-    if (tid == 0) S.ncand = 0;
     cbar();
-    if constexpr (LIST) {
-      // ... and theta = the LN-th largest of them: at least LN tokens of the
-      // slice are >= theta (-inf if fewer than LN thread maxima are finite)
-      if (warp == 0) {
-        unsigned k2[kTopW * kCW / 32];
-        int rk2[kTopW * kCW / 32];
-#pragma unroll
-        for (int i = 0; i < kTopW * kCW / 32; ++i) {
-          k2[i] = S.tkey[lane + 32 * i];
-          rk2[i] = 0;
-        }
-        for (int q = 0; q < kTopW * kCW; ++q) {
-          const unsigned kq = S.tkey[q];
-#pragma unroll
-          for (int i = 0; i < kTopW * kCW / 32; ++i)
-            rk2[i] += (kq > k2[i] || (kq == k2[i] && q < lane + 32 * i)) ? 1 : 0;
-        }
-#pragma unroll
-        for (int i = 0; i < kTopW * kCW / 32; ++i)
-          if (rk2[i] == LN - 1) S.theta = (k2[i] != 0u) ? ord_val(k2[i]) : kNegInf;
-      }
-      cbar();
-    }
     float m[R];
 #pragma unroll
     for (int r = 0; r < R; ++r) {
@@ -606,12 +789,27 @@ struct Eng {
       for (int w = 0; w < kCW; ++w) t = fmaxf(t, S.red[w * kMaxRows + r]);
       m[r] = t;
     }
+    // theta: the smallest of the warps' k-th largest thread maxima (warps
+    // with fewer than k tokens left out), so at least LN tokens are >= theta
+    // when every warp takes part; -inf (every token a candidate) for a slice
+    // of at most kCandCap tokens
     float theta = kNegInf;
-    if constexpr (LIST) theta = S.theta;
+    if constexpr (LIST) {
+      if (n > kCandCap) {
+        theta = kPosInf;
+#pragma unroll
+        for (int w = 0; w < kCW; ++w) {
+          const float wm = S.wth[w];
+          if (wm > kNegInf) theta = fminf(theta, wm);
+        }
+        if (theta == kPosInf) theta = kNegInf;
+      }
+    }
+    if (LIST) PT_ADD(kPhListA, t_a);
+    PT_T0(t_b);
     float sm[R], tau;
     int nc = 0;
     for (int attempt = 0; attempt < 2; ++attempt) {
-      // phase B: sums of the tokens outside the candidates; candidates set aside
 #pragma unroll
       for (int r = 0; r < R; ++r) sm[r] = 0.f;
       tau = kNegInf;
@@ -630,14 +828,17 @@ struct Eng {
               else
                 tau = fmaxf(tau, v0[e]);
             }
+            const int cnt = __popc(cm);
+            const int pos = atomicAdd(&S.ncand, cnt);
+            int q = pos;
 #pragma unroll
             for (int e = 0; e < VE; ++e)
               if (cm >> e & 1u) {
-                const int pos = atomicAdd(&S.ncand, 1);
-                if (pos < kCandCap) {
-                  cid[pos] = tok0 + u * VE + e;
-                  cl[pos] = v0[e];
+                if (q < kCandCap) {
+                  cid[q] = tok0 + u * VE + e;
+                  cl[q] = v0[e];
                 }
+                ++q;
               }
           } else {
             tau = fmaxf(tau, um);
@@ -670,11 +871,11 @@ struct Eng {
       cbar();
       nc = S.ncand;
       if (!LIST || nc <= kCandCap) break;
-      // too many tokens above the threshold (ties or adversarial orderings):
-      // raise it to the kCandCap-th largest target logit by bisection on
-      // order-preserving keys, then redo the pass
+      // more than kCandCap tokens above theta: raise it to the kCandCap-th
+      // largest target logit (bisection on order-preserving keys over every
+      // bit: keys of negative logits use the low bits too) and repeat
       unsigned t = 0u;
-      for (int bit = 31; bit >= 0; --bit) {   // keys of negative logits use every bit
+      for (int bit = 31; bit >= 0; --bit) {
         const unsigned cand = t | (1u << bit);
         int cnt = 0;
         for (int u = tid; u < U; u += kCT) {
@@ -698,6 +899,8 @@ struct Eng {
       cbar();
     }
     nc = min(nc, kCandCap);   // the bisection leaves fewer than kCandCap; never read past the arrays
+    if (LIST) PT_ADD(kPhListB, t_b);
+    PT_T0(t_c);
     // block sums of the rows (fixed order)
     float tot[R];
 #pragma unroll
@@ -721,13 +924,14 @@ struct Eng {
       tau = kNegInf;
 #pragma unroll
       for (int w = 0; w < kCW; ++w) tau = fmaxf(tau, S.wth[w]);
-      // phase C: ranks; the first LN go to the record, the rest back to the sums
+      // ranks; the first LN go to the record, the rest back to the sums
       for (int i = tid; i < nc; i += kCT) {
         const float li = cl[i];
         const int ii = cid[i];
         int rk = 0;
         for (int q = 0; q < nc; ++q) rk += better(cl[q], cid[q], li, ii) ? 1 : 0;
         crank[i] = rk;
+        if (rk >= LN) cord[rk - LN] = i;
       }
       cbar();
       int* rid = reinterpret_cast<int*>(rec + kHdr);
@@ -748,44 +952,40 @@ struct Eng {
               if (e == loc % VE) l = v[e];
             __stcg(rec + kHdr + LN * (1 + r) + rk, l);
           }
-        } else {
-          cord[rk - LN] = i;
         }
       }
-      cbar();
       const int nd = nc - LN;
-      if (nd > 0 && warp == 0) {
-        float add[R];
+      if (nd > 0) {
+        if (warp == 0) {
+          float add[R];
 #pragma unroll
-        for (int r = 0; r < R; ++r) add[r] = 0.f;
-        float at = kNegInf;
-        for (int t = lane; t < nd; t += 32) {
-          const int i = cord[t];
-          const int id = cid[i];
-          const int loc = id - tok0;
-          at = fmaxf(at, cl[i]);
+          for (int r = 0; r < R; ++r) add[r] = 0.f;
+          float at = kNegInf;
+          for (int t = lane; t < nd; t += 32) {
+            const int i = cord[t];
+            const int loc = cid[i] - tok0;
+            at = fmaxf(at, cl[i]);
 #pragma unroll
-          for (int r = 0; r < R; ++r) {
-            float v[VE];
-            E::unpack(raw(b, r, loc / VE), v);
-            float l = v[0];
+            for (int r = 0; r < R; ++r) {
+              float v[VE];
+              E::unpack(raw(b, r, loc / VE), v);
+              float l = v[0];
 #pragma unroll
-            for (int e = 1; e < VE; ++e)
-              if (e == loc % VE) l = v[e];
-            if (m[r] > kNegInf) add[r] = __fadd_rn(add[r], ex2(__fmaf_rn(l, c[r], -__fmul_rn(m[r], c[r]))));
+              for (int e = 1; e < VE; ++e)
+                if (e == loc % VE) l = v[e];
+              if (m[r] > kNegInf) add[r] = __fadd_rn(add[r], exp_term(l, m[r], c[r]));
+            }
+          }
+#pragma unroll
+          for (int r = 0; r < R; ++r) add[r] = warp_sum(add[r]);
+          at = warp_max(at);
+          if (lane == 0) {
+#pragma unroll
+            for (int r = 0; r < R; ++r) S.add[r] = add[r];
+            S.addtau = at;
           }
         }
-#pragma unroll
-        for (int r = 0; r < R; ++r) add[r] = warp_sum(add[r]);
-        at = warp_max(at);
-        if (lane == 0) {
-#pragma unroll
-          for (int r = 0; r < R; ++r) S.add[r] = add[r];
-          S.addtau = at;
-        }
-      }
-      cbar();
-      if (nd > 0) {
+        cbar();
 #pragma unroll
         for (int r = 0; r < R; ++r) tot[r] = __fadd_rn(tot[r], S.add[r]);
         tau = fmaxf(tau, S.addtau);
@@ -799,7 +999,9 @@ struct Eng {
       }
       __stcg(rec + 2 * kMaxRows, tau);
       __stcg(reinterpret_cast<int*>(rec) + 2 * kMaxRows + 1, LIST ? min(nc, LN) : 0);
+      S.ncand = 0;   // for the next slice (every reader is past the barriers above)
     }
+    if (LIST) PT_ADD(kPhListC, t_c);
   }
 
   // Stats of any number of rows, one row at a time, no candidate list.
@@ -1066,14 +1268,15 @@ struct Eng {
       for (int j = threadIdx.x; j <= p.L; j += kCT) __stcg(p.out_tokens + (size_t)seqb * (p.L + 1) + j, -1);
       if (threadIdx.x == 0) __stcg(p.out_accept + seqb, -1);
     }
-    __threadfence();
+    // publish the record: the barrier orders every thread's record writes
+    // before thread 0's release (acq_rel: the last arriver also acquires the
+    // other slices' records)
+    PT_T0(t_pub);
     cbar();
-    if (threadIdx.x == 0) S.last = (atomicAdd(&p.cnt[seqb], 1u) == (unsigned)(p.ns - 1)) ? 1 : 0;
+    if (threadIdx.x == 0) S.last = (atom_add_acq_rel(&p.cnt[seqb], 1u) == (unsigned)(p.ns - 1)) ? 1 : 0;
     cbar();
-    if (S.last) {
-      __threadfence();
-      decide(Dd, b);
-    }
+    PT_ADD(kPhPublish, t_pub);
+    if (S.last) decide(Dd, b);
   }
 
   __device__ void compute() {
@@ -1178,6 +1381,7 @@ struct Eng {
         D.W.zres = 0;
         plan_rows(b, j + 1, nv, j + 1 == p.L, &D.P, &D.nv, D.vbr, D.X, D.vrow);
       }
+      D.xl_ok = 0;
     }
     cbar();
     const int next = D.tok;
@@ -1190,29 +1394,29 @@ struct Eng {
   // Combine the records of a stats pass: every row's M and 1/Z, and with
   // candidate lists the sequence's list (the first LN of the slices' lists
   // by (logit, id)), its complement masses and tau.
-  __device__ void combine_stats(const FDesc& Dd, int b, char* scratch) {
-    DState& D = S.D;
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int ns = p.ns, R = Dd.P.nstream, LN = p.ln;
-    const bool list = Dd.P.list != 0;
+  // The records of a stats pass into the scratch buffer (threads t of nt):
+  // per row the slice maxima and sums, and with lists each slice's tau,
+  // list length and entries.
+  __device__ void stage_records(const FDesc& Dd, int b, char* scratch, int t, int nt) const {
+    const int ns = p.ns, R = Dd.P.nstream, LN = p.lns;
     const float* recb = p.rec + (size_t)b * ns * p.rec_floats;
-    float* hm = reinterpret_cast<float*>(scratch);        // [R][ns] slice maxima
-    float* hs = hm + R * ns;                              // [R][ns] slice sums
-    float* htau = hs + R * ns;                            // [ns]
-    int* hnl = reinterpret_cast<int*>(htau + ns);         // [ns]
-    int* eid = hnl + ns;                                  // [ns][LN]
-    float* el = reinterpret_cast<float*>(eid + ns * LN);  // [R][ns][LN]
-    for (int i = tid; i < R * ns; i += kCT) {
+    float* hm = reinterpret_cast<float*>(scratch);
+    float* hs = hm + R * ns;
+    float* htau = hs + R * ns;
+    int* hnl = reinterpret_cast<int*>(htau + ns);
+    int* eid = hnl + ns;
+    float* el = reinterpret_cast<float*>(eid + ns * LN);
+    for (int i = t; i < R * ns; i += nt) {
       const int r = i / ns, s = i - r * ns;
       hm[i] = __ldcg(recb + (size_t)s * p.rec_floats + 2 * r);
       hs[i] = __ldcg(recb + (size_t)s * p.rec_floats + 2 * r + 1);
     }
-    if (list) {
-      for (int s = tid; s < ns; s += kCT) {
+    if (Dd.P.list) {
+      for (int s = t; s < ns; s += nt) {
         htau[s] = __ldcg(recb + (size_t)s * p.rec_floats + 2 * kMaxRows);
         hnl[s] = __ldcg(reinterpret_cast<const int*>(recb + (size_t)s * p.rec_floats) + 2 * kMaxRows + 1);
       }
-      for (int i = tid; i < ns * LN * (1 + R); i += kCT) {
+      for (int i = t; i < ns * LN * (1 + R); i += nt) {
         const int f = i / (ns * LN), rest = i - f * ns * LN;
         const int s = rest / LN, q = rest - s * LN;
         const float v = __ldcg(recb + (size_t)s * p.rec_floats + kHdr + f * LN + q);
@@ -1222,7 +1426,20 @@ struct Eng {
           el[(f - 1) * ns * LN + rest] = v;
       }
     }
-    cbar();
+  }
+
+  // Combine the staged records (stage_records) of a stats pass.
+  __device__ void combine_stats(const FDesc& Dd, int b, char* scratch) {
+    DState& D = S.D;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int ns = p.ns, R = Dd.P.nstream, LN = p.lns, LF = p.ln;   // a slice's list, the sequence's
+    const bool list = Dd.P.list != 0;
+    float* hm = reinterpret_cast<float*>(scratch);        // [R][ns] slice maxima
+    float* hs = hm + R * ns;                              // [R][ns] slice sums
+    float* htau = hs + R * ns;                            // [ns]
+    int* hnl = reinterpret_cast<int*>(htau + ns);         // [ns]
+    int* eid = hnl + ns;                                  // [ns][LN]
+    float* el = reinterpret_cast<float*>(eid + ns * LN);  // [R][ns][LN]
     // row maxima
     if (tid < R) {
       float M = kNegInf;
@@ -1254,7 +1471,7 @@ struct Eng {
       int h = 0;
       unsigned key = (h < nl) ? ord_key(__fadd_rn(el[lane * LN], 0.f)) : 0u;
       int nf = 0;
-      for (int t = 0; t < LN; ++t) {
+      for (int t = 0; t < LF; ++t) {
         const unsigned km = __reduce_max_sync(FULLM, key);
         if (!km) break;
         const unsigned who = __ballot_sync(FULLM, key == km);
@@ -1298,13 +1515,19 @@ struct Eng {
         D.pc[r] = __fadd_rn(C, add);
       }
     }
-    // the list by token id (positions by counting)
+    // the list: in merge order (larger logit first) for the weighted scheme,
+    // whose stages break key ties on the id; by token id for the truncated
+    // alphabet, whose draws scan Omega_0 in token order
     if (warp == 0) {
+      const bool by_id = p.scheme == MDS_WIS0;
       for (int t = lane; t < nf; t += 32) {
         const int idx = D.fin_s[t] * LN + D.fin_i[t];
         const int id = eid[idx];
-        int pos = 0;
-        for (int q = 0; q < nf; ++q) pos += (eid[D.fin_s[q] * LN + D.fin_i[q]] < id) ? 1 : 0;
+        int pos = t;
+        if (by_id) {
+          pos = 0;
+          for (int q = 0; q < nf; ++q) pos += (eid[D.fin_s[q] * LN + D.fin_i[q]] < id) ? 1 : 0;
+        }
         D.cm_id[pos] = id;
         D.cm_l0[pos] = el[idx];
         for (int r = 0; r < R; ++r) D.cm_e[r][pos] = exp_term(el[r * ns * LN + idx], D.P.row[r].M, D.P.row[r].c);
@@ -1342,10 +1565,10 @@ struct Eng {
   // not above every key outside the list (each such key is <= its q <= q(tau)).
   __device__ bool wis_stage_list(int A, int Btok, int rb, float u) {
     DState& D = S.D;
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
     const int s = min(p.wis_s, p.V);
     const int n = D.n;
-    if (warp == 0) {
+    {
       const float iz0 = D.P.row[0].invZ, izb = D.P.row[rb].invZ;
       const bool have = lane < n;
       float q = 0.f, a = 0.f, bq = 0.f, key = kNegInf;
@@ -1360,13 +1583,17 @@ struct Eng {
         bq = __fmul_rn(D.cm_e[rb][lane], izb);
         key = __fadd_rn(__fmaf_rn(-a, bq, q), 0.f);   // -0 -> +0: keys compare as floats
       }
+      // Omega_1: s rounds of a warp max over order-preserving keys, ties to
+      // the smaller token id (the list is in logit order, not id order)
+      const int myid = have ? D.cm_id[lane] : 0x7fffffff;
       unsigned kk = have ? ord_key(key) : 0u;
       uint32_t selm = 0u;
       float kth = kNegInf;
       for (int t = 0; t < s; ++t) {
         const unsigned km = __reduce_max_sync(FULLM, kk);
-        const uint32_t who = __ballot_sync(FULLM, km != 0u && kk == km);
-        if (!who) break;
+        if (!km) break;
+        const int idm = __reduce_min_sync(FULLM, (kk == km) ? myid : 0x7fffffff);
+        const uint32_t who = __ballot_sync(FULLM, kk == km && myid == idm);
         const int wl = __ffs(who) - 1;
         selm |= 1u << wl;
         if (lane == wl) kk = 0u;
@@ -1380,7 +1607,9 @@ struct Eng {
       if (!ok) {
         if (lane == 0) D.fast_ok = 0;
       } else {
-        const int rk = __popc(selm & ((1u << lane) - 1u));
+        // position in Omega_1 by token id
+        int rk = 0;
+        for (uint32_t mm = selm; mm; mm &= mm - 1u) rk += (__shfl_sync(FULLM, myid, __ffs(mm) - 1) < myid) ? 1 : 0;
         if (lane >= s && lane < MDS_MAX_S) {
           D.om[lane] = -1;
           D.om_q[lane] = 0.f;
@@ -1418,17 +1647,34 @@ struct Eng {
         if (lane == 0) gamma_update(rb, A2, B2);
       }
     }
-    cbar();
+    __syncwarp();
     return D.fast_ok != 0;
   }
 
-  __device__ int solve(int s, float A2, float B2, int A, int Btok, float u) {
+  // The stage LP on one thread.  Out of line, so that it has the kernel's
+  // whole register budget: s <= 5 keeps its pair state in registers, larger
+  // s in shared memory.
+  __device__ __noinline__ int solve5(int s, float A2, float B2, int A, int Btok, float u) {
     DState& D = S.D;
     bool capped = false;
-    const int y = (s <= 5) ? stage_solve<5>(s, A2, B2, A, Btok, u, D.om, D.om_q, D.om_a, D.om_b, D.om_x, &capped)
-                           : stage_solve<MDS_MAX_S>(s, A2, B2, A, Btok, u, D.om, D.om_q, D.om_a, D.om_b, D.om_x,
-                                                    &capped);
+    const int y = stage_solve_split<5>(s, A2, B2, A, Btok, u, D.om, D.om_q, D.om_a, D.om_b, D.om_x, &capped, D.lp_rs,
+                                       D.lp_fl, D.lp_fh, D.lp_rd);
     if (capped) atomicOr(p.status, MDS_ST_LP_CAP);
+    return y;
+  }
+  __device__ __noinline__ int solve8(int s, float A2, float B2, int A, int Btok, float u) {
+    DState& D = S.D;
+    bool capped = false;
+    const int y = stage_solve<MDS_MAX_S>(s, A2, B2, A, Btok, u, D.om, D.om_q, D.om_a, D.om_b, D.om_x, &capped,
+                                         D.lp_rs, D.lp_fl, D.lp_fh);
+    if (capped) atomicOr(p.status, MDS_ST_LP_CAP);
+    return y;
+  }
+  __device__ int solve(int s, float A2, float B2, int A, int Btok, float u) {
+    PT_T0(t_lp);
+    const int y = (s <= 5) ? solve5(s, A2, B2, A, Btok, u) : solve8(s, A2, B2, A, Btok, u);
+    PT_ADD(kPhLp, t_lp);
+    PT_CNT(kPhLpCalls);
     return y;
   }
 
@@ -1487,15 +1733,20 @@ struct Eng {
 
   __device__ void decide_stats(const FDesc& Dd, int b, char* scratch) {
     DState& D = S.D;
-    const int tid = threadIdx.x;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int j = Dd.P.j;
-    if (tid == 0) {
-      if (j == 0) {
+    // warp 0 plans the depth (and caches the logits at the draft tokens)
+    // while the other warps stage the records
+    if (warp == 0) {
+      if (j == 0 && lane == 0) {
         D.W = FWalk{};
         D.W.valid = (p.K >= 32) ? FULLM : ((1u << p.K) - 1u);
         D.W.Yp = -1;
       }
-      plan_rows(b, j, D.W.valid, false, &D.P, &D.nv, D.vbr, D.X, D.vrow);
+      __syncwarp();
+      plan_warp(b, j, D.W.valid, false, true);
+    } else {
+      stage_records(Dd, b, scratch, tid - 32, kCT - 32);
     }
     cbar();
     PT_T0(t_comb);
@@ -1517,44 +1768,47 @@ struct Eng {
       return;
     }
     // WIS: the pairwise stages (Remark 4) on the candidate list while it
-    // certifies Omega_1; from the first stage it cannot, full-vocabulary passes
-    if (tid == 0) {
-      for (int r = 0; r < D.P.nrows; ++r) D.P.row[r].gamma = 0.f;
-      D.P.row[D.vrow[0]].gamma = 1.f;
-      D.P.nspec = 0;
-    }
-    cbar();
-    int A = D.X[0];
-    bool fast = Dd.P.list != 0;
-    int m = 1;
+    // certifies Omega_1 (warp 0 alone); from the first stage it cannot,
+    // full-vocabulary passes
     PT_T0(t_stg);
-    if (fast) {
-      for (; m < D.nv; ++m) {
-        const float u = draw_uniform(p.seed, b, j, kDrawSelect + m - 1);
-        if (!wis_stage_list(A, D.X[m], D.vrow[m], u)) break;
-        A = D.Y;
+    if (warp == 0) {
+      if (lane == 0) {
+        for (int r = 0; r < D.P.nrows; ++r) D.P.row[r].gamma = 0.f;
+        D.P.row[D.vrow[0]].gamma = 1.f;
+        D.P.nspec = 0;
       }
-      if (tid == 0) list_to_table();
-      cbar();
-    }
-    PT_ADD(kPhDecStages, t_stg);
-    if (m < D.nv) {
-      if (tid == 0) {
+      __syncwarp();
+      int A = D.X[0];
+      int m = 1;
+      if (Dd.P.list) {
+        // every stage's selection uniform at once (lane m - 1 draws stage m's)
+        const float ul = (lane + 1 < D.nv) ? draw_uniform(p.seed, b, j, kDrawSelect + lane) : 0.f;
+        for (; m < D.nv; ++m) {
+          const float u = __shfl_sync(FULLM, ul, m - 1);
+          if (!wis_stage_list(A, D.X[m], D.vrow[m], u)) break;
+          A = D.Y;
+        }
+        if (lane == 0) list_to_table();
+      }
+      if (lane == 0) {
         D.W.stage = m;
         D.W.A = A;
-        D.P.rb = D.vrow[m];
-        D.P.nstream = D.P.nrows;
+        if (m < D.nv) {
+          D.P.rb = D.vrow[m];
+          D.P.nstream = D.P.nrows;
+        } else {
+          D.W.Y = A;
+          D.W.qY = prob_row(D.P, 0, A);
+          D.W.pIY = law_at(D.P, A);
+        }
       }
-      cbar();
+    }
+    cbar();
+    PT_ADD(kPhDecStages, t_stg);
+    if (D.W.stage < D.nv) {
       push(b, kFull);
       return;
     }
-    if (tid == 0) {
-      D.W.Y = A;
-      D.W.qY = prob_row(D.P, 0, A);
-      D.W.pIY = law_at(D.P, A);
-    }
-    cbar();
     accept_step(b);
   }
 
@@ -1562,7 +1816,7 @@ struct Eng {
     DState& D = S.D;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int j = D.P.j, ns = p.ns;
-    if (tid == 0) plan_rows(b, j, D.W.valid, false, nullptr, &D.nv, D.vbr, D.X, D.vrow);
+    if (warp == 0) plan_warp(b, j, D.W.valid, false, false);
     cbar();
     const int m = D.W.stage;
     const int A = D.W.A, Btok = D.X[m], rb = D.vrow[m];
@@ -1846,7 +2100,7 @@ struct Eng {
   __device__ void decide_resid(int b, char* scratch) {
     DState& D = S.D;
     const int tid = threadIdx.x;
-    if (tid == 0) plan_rows(b, D.P.j, D.W.valid, false, nullptr, &D.nv, D.vbr, D.X, D.vrow);
+    if ((tid >> 5) == 0) plan_warp(b, D.P.j, D.W.valid, false, false);
     float* Rs = S.Rs;
     const float R = slice_masses(b, Rs);
     int Z = D.W.Y;
@@ -1874,7 +2128,7 @@ struct Eng {
   __device__ void decide_replace(int b, char* scratch) {
     DState& D = S.D;
     const int tid = threadIdx.x;
-    if (tid == 0) plan_rows(b, D.P.j, D.W.valid, false, nullptr, &D.nv, D.vbr, D.X, D.vrow);
+    if ((tid >> 5) == 0) plan_warp(b, D.P.j, D.W.valid, false, false);
     float* Rs = S.Rs;
     const float R = slice_masses(b, Rs);
     int Z;
@@ -2157,6 +2411,8 @@ struct Eng {
       copy_in(&D.W, &g->W, (int)sizeof(FWalk), threadIdx.x, kCT);
       cbar();
     }
+    if (threadIdx.x == 0) D.xl_ok = 0;
+    cbar();
     PT_T0(t_dec);
     PT_CNT(kPhDecisions);
     switch (kind) {
@@ -2192,6 +2448,7 @@ __global__ void __launch_bounds__(kBlock, 2) flow_kernel(const __grid_constant__
     }
     S.issued = 0;
     S.consumed = 0;
+    S.ncand = 0;
 #ifdef MDS_PHASE_TIMERS
     for (int i = 0; i < kPhaseN; ++i) S.tm[i] = 0ull;
 #endif
@@ -2321,13 +2578,24 @@ bool plan_geometry(Params& p, int grid) {
   p.ns = ns;
   p.ln = list ? ((p.scheme == MDS_WIS0 && p.omega0 >= 32) ? 64 : 32) : 0;
   if (p.ln > kListMax) return false;
+  // a slice's list: enough that the slices' lists together hold the
+  // sequence's list whenever its tokens are spread over the slices (a slice
+  // holding more of them only shortens the certified list)
+  if (list) {
+    const int base = (p.scheme == MDS_WIS0) ? 16 : 8;
+    int lns = (2 * p.ln + ns - 1) / ns;
+    lns = (lns + 7) / 8 * 8;
+    p.lns = lns < base ? base : (lns > p.ln ? p.ln : lns);
+  } else {
+    p.lns = 0;
+  }
   const int lrows = list ? nstream : 0;
-  int rf = kHdr + p.ln * (1 + lrows);
+  int rf = kHdr + p.lns * (1 + lrows);
   if (rf < 4 + 4 * kTopF) rf = 4 + 4 * kTopF;
   p.rec_floats = (rf + 3) & ~3;
   p.hdr_floats = kHdr;
   // the decision stages one stats pass's records in one slice buffer
-  const size_t stage = (size_t)(2 * nstream * ns + 2 * ns + ns * p.ln * (1 + lrows)) * 4;
+  const size_t stage = (size_t)(2 * nstream * ns + 2 * ns + ns * p.lns * (1 + lrows)) * 4;
   if (stage > (size_t)kBufBytes) return false;
   return true;
 }

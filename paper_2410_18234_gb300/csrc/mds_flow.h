@@ -48,7 +48,8 @@ struct Params {
   int wis_s, omega0, acc_prob;
   int T;                               // tokens per slice (multiple of kSliceQuantum)
   int ns;                              // slices per row
-  int ln;                              // candidate list length (0: no candidate lists)
+  int ln;                              // candidate list length of a sequence (0: no candidate lists)
+  int lns;                             // candidate list length of one slice (<= ln)
   int rec_floats;                      // record stride per slice
   int hdr_floats;                      // start of a record's list entries
   int ring_cap;

@@ -73,6 +73,11 @@ WORKLOADS = {
                                  target_scale=4.0, draft_sigma=[0.3, 1.0, 2.0], t_target=1.0, t_draft=[1.0],
                                  sigma_per_seq=True, temp_per_seq=(0.5, 1.5),
                                  schemes=["single", "IS", "WIS", "SpecTr"], data_seed=1004),
+    # the same serving sweep with K = 2 draft branches (its other arm)
+    "serving-152k-k2": WorkloadSpec("serving-152k-k2", B=1024, K=2, L=8, V=151936, dtype="bf16", model_ids=[0] * 2,
+                                    target_scale=4.0, draft_sigma=[0.3, 1.0, 2.0], t_target=1.0, t_draft=[1.0],
+                                    sigma_per_seq=True, temp_per_seq=(0.5, 1.5),
+                                    schemes=["single", "IS", "WIS", "SpecTr"], data_seed=1005),
 }
 
 
