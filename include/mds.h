@@ -179,7 +179,8 @@ int mds_verify_host(mds_ctx* ctx, const void* target_logits, const void* const* 
  * number of slices per row, about V / 8192) lives in a file-scope device
  * array of MDS_NOALLOC_SCRATCH_BYTES (8 MiB) that every GPU loading the
  * library holds until the process exits; a call whose scratch exceeds it
- * (for llama3-like rows, beyond roughly 900 sequences per call) is rejected
+ * (for llama3-like rows of 128k bf16 logits, beyond roughly 1,500 sequences
+ * per call) is rejected
  * with MDS_ESHAPE before any launch.  The first call on a device looks up
  * that array's device address and sets kernel attributes, so make it before
  * any stream capture.  Every call clears the parts of the scratch that must

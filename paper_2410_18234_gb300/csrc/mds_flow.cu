@@ -32,6 +32,7 @@
 // bit-reproducible.  Every wait is bounded in time; a wait that gives up sets
 // MDS_ST_TIMEOUT and an abort flag on which every CTA leaves, after waiting
 // for its own copies in flight.
+#include <cstdlib>
 #include <cuda_bf16.h>
 
 #include "mds_device.cuh"
@@ -47,6 +48,7 @@ constexpr int kCW = 8;                 // compute warps
 constexpr int kCT = kCW * 32;          // compute threads
 constexpr int kBlock = kCT + 32;       // + the scheduler warp
 constexpr int kNBuf = 2;               // slice buffers per CTA
+constexpr int kCtasPerSm = 2;          // resident CTAs per SM (the launch bound)
 constexpr int kCandCap = 512;          // candidate tokens one slice may set aside
 constexpr int kListMax = 64;           // candidate list length at most
 constexpr int kHdr = 2 * kMaxRows + 2; // record: (max, sum) per row, tau, list length
@@ -57,6 +59,12 @@ static_assert(kHdr % 4 == 0, "record header keeps 16-byte alignment");
 static_assert(kTopF >= MDS_MAX_S, "full-stage candidates");
 
 enum : int { kNone = 0, kStats = 1, kResid = 2, kBonus = 3, kFull = 4, kReplace = 5 };
+
+// A decision request: sequence (16 bits), kind (3), depth (7), rows (5), list (1).
+__host__ __device__ constexpr unsigned dec_payload(int b, int kind, int j, int R, int list) {
+  return ((unsigned)b << 16) | ((unsigned)kind << 13) | ((unsigned)j << 6) | ((unsigned)R << 1) | (unsigned)(list != 0);
+}
+static_assert(MDS_MAX_L < 127 && kMaxRows < 32, "decision request fields");
 
 // Phase-timer slots (SM cycles summed over CTAs, or counts).
 enum : int {
@@ -75,6 +83,12 @@ enum : int {
   kPhPush,              // publishing the next pass
   kPhSchedPoll,         // scheduler waiting for a published task
   kPhSchedEmpty,        // scheduler waiting for a free buffer
+  kPhDecPoll,           // decision warps waiting for a request
+  kPhDecPlan,           // decisions: planning a pass (rows, tokens, cached logits)
+  kPhDecLoad,           // decisions: staging a stats pass's records
+  kPhDecSelect,         // decisions: WIS stage selection and masses (list)
+  kPhDecAccept,         // decisions: the accept step (with its push or walk)
+  kPhDecWalk,           // decisions: the walk to the next depth
   kPhListA,             // list tasks: maxima and the candidate threshold
   kPhListB,             // list tasks: the sums and the candidates
   kPhListC,             // list tasks: ranking and the record
@@ -196,7 +210,6 @@ struct FShared {
 #ifdef MDS_PHASE_TIMERS
   unsigned long long tm[kPhaseN];
 #endif
-  DState D;
 };
 
 // ------------------------------------------------------------------ memory helpers
@@ -254,10 +267,20 @@ __device__ unsigned long long g_phase[kPhaseN];
   do {                                            \
     if ((threadIdx.x & 0xff) == 0) S.tm[i] += 1ull; \
   } while (0)
+#define PT_ADDW(i, v)                                                               \
+  do {                                                                              \
+    if ((threadIdx.x & 31) == 0) atomicAdd(&S.tm[i], (unsigned long long)(clock64() - (v))); \
+  } while (0)
+#define PT_CNTW(i)                                         \
+  do {                                                     \
+    if ((threadIdx.x & 31) == 0) atomicAdd(&S.tm[i], 1ull); \
+  } while (0)
 #else
 #define PT_T0(v)
 #define PT_ADD(i, v)
 #define PT_CNT(i)
+#define PT_ADDW(i, v)
+#define PT_CNTW(i)
 #endif
 
 // ------------------------------------------------------------------ the engine
@@ -288,113 +311,11 @@ struct Eng {
   __device__ __forceinline__ uint4 raw(const char* b, int r, int u) const {
     return *reinterpret_cast<const uint4*>(srow(b, r) + 16 * u);
   }
-  // Logit of row r at token x: from the decision's cache when x is one of
-  // the depth's draft tokens (the intermediate token always is), else a load.
-  __device__ __forceinline__ float logit_at(const FPass& P, int r, int x) const {
-    const DState& D = S.D;
-    if (D.xl_ok)
-      for (int k = 0; k < D.nv; ++k)
-        if (D.X[k] == x) return D.xl[k][r];
-    return E::global(P.row[r].ptr, x);
-  }
-  __device__ __forceinline__ float prob_row(const FPass& P, int r, int x) const {
-    return prob_of(logit_at(P, r, x), P.row[r].M, P.row[r].c, P.row[r].invZ);
-  }
+  // Explicit value of a special token of the current law, else fallback.
   __device__ __forceinline__ float spec_lookup(const FPass& P, int tok, float fallback) const {
     for (int i = 0; i < P.nspec; ++i)
       if (P.spec_id[i] == tok) return P.spec_val[i];
     return fallback;
-  }
-  // Point value of the current law p_I (WIS): explicit value of a special
-  // token, else sum_r gamma_r p_r(x) in row order.
-  __device__ float law_at(const FPass& P, int x) const {
-    float a = 0.f;
-    for (int r = 1; r < P.nrows; ++r)
-      if (P.row[r].gamma != 0.f) a = __fmaf_rn(P.row[r].gamma, prob_row(P, r, x), a);
-    return spec_lookup(P, x, a);
-  }
-
-  // -------------------------------------------------------------- planning
-  // Rows of depth j for the valid branches (the lowest valid branch's target
-  // row, then one row per distinct draft model in branch order) into *P (if
-  // given) and, if X is given, the valid branches, their tokens and rows.
-  // One thread.
-  __device__ void plan_rows(int b, int j, unsigned valid, bool bonus, FPass* P, int* nv, int* vbr, int* X,
-                            int* vrow) const {
-    const int K = p.K, L = p.L, V = p.V;
-    const int kstar = __ffs(valid) - 1;
-    if (P) {
-      P->row[0].ptr = p.target + ((((size_t)b * K + kstar) * (L + 1) + j) * (size_t)V) * p.esize;
-      float tq = p.temps[(size_t)b * (1 + K)];
-      if (!(tq > 0.f) || !(tq < kPosInf)) {
-        atomicOr(p.status, MDS_ST_BADTEMP);
-        tq = 1.f;
-      }
-      P->row[0].c = __fdiv_rn(kLog2e, tq);
-    }
-    int mrow[MDS_MAX_K];
-    for (int m = 0; m < MDS_MAX_K; ++m) mrow[m] = -1;
-    int nr = 1, n = 0;
-    if (!bonus) {
-      for (int k = 0; k < K; ++k) {
-        if (!(valid >> k & 1u)) continue;
-        const int m = p.model_of[k];
-        if (mrow[m] < 0) {
-          mrow[m] = nr;
-          if (P) {
-            P->row[nr].ptr = p.drafts[k] + (((size_t)b * L + j) * (size_t)V) * p.esize;
-            float td = p.temps[(size_t)b * (1 + K) + 1 + k];
-            if (!(td > 0.f) || !(td < kPosInf)) {
-              atomicOr(p.status, MDS_ST_BADTEMP);
-              td = 1.f;
-            }
-            P->row[nr].c = __fdiv_rn(kLog2e, td);
-          }
-          ++nr;
-        }
-        if (X) {
-          int x = p.tokens[((size_t)b * K + k) * L + j];
-          if (x < 0 || x >= V) {
-            atomicOr(p.status, MDS_ST_BADTOKEN);
-            x = 0;
-          }
-          vbr[n] = k;
-          X[n] = x;
-          vrow[n] = mrow[m];
-        }
-        ++n;
-      }
-    }
-    if (nv) *nv = n;
-    if (!P) return;
-    for (int r = 0; r < nr; ++r) {
-      P->row[r].M = 0.f;
-      P->row[r].invZ = 0.f;
-      P->row[r].gamma = 0.f;
-    }
-    P->nrows = nr;
-    P->j = j;
-    P->nspec = 0;
-    P->rb = 0;
-    P->cut = 0.f;
-    P->all0 = 0;
-    if (bonus) {
-      P->kind = kBonus;
-      P->nstream = 1;
-      P->list = 0;
-    } else {
-      P->kind = kStats;
-      if (p.scheme == MDS_WIS0) {
-        P->nstream = 1;
-        P->list = 1;
-      } else if (p.scheme == MDS_WIS) {
-        P->nstream = nr;
-        P->list = (n > 1 && nr <= kListRowsMax && p.ln > 0) ? 1 : 0;
-      } else {
-        P->nstream = min(2, nr);
-        P->list = 0;
-      }
-    }
   }
 
   // -------------------------------------------------------------- scheduler warp
@@ -404,96 +325,6 @@ struct Eng {
       if (mbar_try_wait(bar, parity)) return true;
       if ((it & 63) == 63 && now_ns() - t0 > kWaitNs) return false;
     }
-  }
-
-  // Warp-parallel plan_rows (one lane per branch): the same rows in the same
-  // order, the valid branches, their tokens and rows; then every row's logit
-  // at each draft token into the decision's cache.  Warp 0 of a decision.
-  __device__ void plan_warp(int b, int j, unsigned valid, bool bonus, bool set_pass) {
-    DState& D = S.D;
-    FPass& P = D.P;
-    const int lane = threadIdx.x & 31;
-    const int K = p.K;
-    const bool v = !bonus && lane < K && ((valid >> lane) & 1u);
-    const int m = v ? (int)p.model_of[lane] : 64 + lane;
-    const unsigned same = __match_any_sync(FULLM, m);
-    const bool first = v && (__ffs(same) - 1) == lane;
-    const unsigned fm = __ballot_sync(FULLM, first);
-    const unsigned vm = __ballot_sync(FULLM, v);
-    const int nr = 1 + __popc(fm);
-    const int myrow = first ? 1 + __popc(fm & ((1u << lane) - 1u)) : 0;
-    const int row = __shfl_sync(FULLM, myrow, __ffs(same) - 1);
-    if (v) {
-      const int i = __popc(vm & ((1u << lane) - 1u));
-      int x = p.tokens[((size_t)b * K + lane) * p.L + j];
-      if (x < 0 || x >= p.V) {
-        atomicOr(p.status, MDS_ST_BADTOKEN);
-        x = 0;
-      }
-      D.vbr[i] = lane;
-      D.X[i] = x;
-      D.vrow[i] = row;
-    }
-    if (set_pass && first) {
-      P.row[myrow].ptr = p.drafts[lane] + (((size_t)b * p.L + j) * (size_t)p.V) * p.esize;
-      float td = p.temps[(size_t)b * (1 + K) + 1 + lane];
-      if (!(td > 0.f) || !(td < kPosInf)) {
-        atomicOr(p.status, MDS_ST_BADTEMP);
-        td = 1.f;
-      }
-      P.row[myrow].c = __fdiv_rn(kLog2e, td);
-      P.row[myrow].M = 0.f;
-      P.row[myrow].invZ = 0.f;
-      P.row[myrow].gamma = 0.f;
-    }
-    if (lane == 0) {
-      D.nv = __popc(vm);
-      if (set_pass) {
-        const int kstar = __ffs(valid) - 1;
-        P.row[0].ptr = p.target + ((((size_t)b * K + kstar) * (p.L + 1) + j) * (size_t)p.V) * p.esize;
-        float tq = p.temps[(size_t)b * (1 + K)];
-        if (!(tq > 0.f) || !(tq < kPosInf)) {
-          atomicOr(p.status, MDS_ST_BADTEMP);
-          tq = 1.f;
-        }
-        P.row[0].c = __fdiv_rn(kLog2e, tq);
-        P.row[0].M = 0.f;
-        P.row[0].invZ = 0.f;
-        P.row[0].gamma = 0.f;
-        P.nrows = nr;
-        P.j = j;
-        P.nspec = 0;
-        P.rb = 0;
-        P.cut = 0.f;
-        P.all0 = 0;
-        if (bonus) {
-          P.kind = kBonus;
-          P.nstream = 1;
-          P.list = 0;
-        } else {
-          P.kind = kStats;
-          if (p.scheme == MDS_WIS0) {
-            P.nstream = 1;
-            P.list = 1;
-          } else if (p.scheme == MDS_WIS) {
-            P.nstream = nr;
-            P.list = (__popc(vm) > 1 && nr <= kListRowsMax && p.ln > 0) ? 1 : 0;
-          } else {
-            P.nstream = min(2, nr);
-            P.list = 0;
-          }
-        }
-      }
-    }
-    __syncwarp();
-    // the cache: row r's logit at X[k] for every valid branch k
-    const int nv = D.nv, nrow = P.nrows;
-    for (int i = lane; i < nv * nrow; i += 32) {
-      const int k = i / nrow, r = i - k * nrow;
-      D.xl[k][r] = E::global(P.row[r].ptr, D.X[k]);
-    }
-    if (lane == 0) D.xl_ok = bonus ? 0 : 1;
-    __syncwarp();
   }
 
   // Warp-parallel plan of a sequence's depth-0 pass (every branch valid):
@@ -1227,6 +1058,28 @@ struct Eng {
   }
 
   // -------------------------------------------------------------- compute warps
+  // The pass of a sequence is complete: publish a decision request (thread
+  // 0, after acquiring every slice's record through the pass counter; the
+  // release of the request's tag passes them on to the decision warp).
+  __device__ void post_decision(unsigned pay) const {
+    const unsigned t = atomicAdd(&p.ctl[kCtlDecTail], 1u);
+    const unsigned slot = t % (unsigned)p.dec_cap;
+    if (t >= (unsigned)p.dec_cap) {
+      const unsigned long long prev = tag_of(t - (unsigned)p.dec_cap);
+      const unsigned long long t0 = now_ns();
+      for (int it = 0; ld_acquire(&p.dec_rtag[slot]) != prev; ++it) {
+        if (aborted()) break;
+        if ((it & 15) == 15 && now_ns() - t0 > kWaitNs) {
+          set_abort(MDS_ST_TIMEOUT);
+          break;
+        }
+        __nanosleep(64);
+      }
+    }
+    __stcg(p.dec_pay + slot, pay);
+    st_release(&p.dec_tag[slot], tag_of(t));
+  }
+
   __device__ void process(int bi) {
     FDesc& Dd = S.desc[bi];
     char* b = buf(bi);
@@ -1273,10 +1126,9 @@ struct Eng {
     // other slices' records)
     PT_T0(t_pub);
     cbar();
-    if (threadIdx.x == 0) S.last = (atom_add_acq_rel(&p.cnt[seqb], 1u) == (unsigned)(p.ns - 1)) ? 1 : 0;
-    cbar();
+    if (threadIdx.x == 0 && atom_add_acq_rel(&p.cnt[seqb], 1u) == (unsigned)(p.ns - 1))
+      post_decision(dec_payload(seqb, P.kind, P.j, P.nstream, P.list));
     PT_ADD(kPhPublish, t_pub);
-    if (S.last) decide(Dd, b);
   }
 
   __device__ void compute() {
@@ -1308,25 +1160,251 @@ struct Eng {
     }
   }
 
-  // ============================================================== decisions
-  // Run by the compute warps of the CTA that completed a pass of sequence b.
+};
 
+// ================================================================== decisions
+// One decision warp (on a decision SM) runs one sequence's decision at a
+// time: the records of the pass just completed, the importance step, the
+// accept test and the inverse-CDF search, then the sequence's next pass.
+// Single-warp code throughout (lane 0 for the serial steps); its state and
+// scratch are this warp's own shared memory.
+
+constexpr int kDecStage = 6656;        // bytes of a decision's staged records
+constexpr int kDecScratch = kDecStage + 2 * kMaxSlices * 4 + 64 * 4;   // + slice masses, maxima, bitmap
+
+template <int DT>
+struct Dec {
+  using E = Elt<DT>;
+  static constexpr int VE = E::VE;
+
+  const Params& p;
+  FShared& S;      // the CTA's shared state (phase timers)
+  DState& D;       // this warp's decision state
+  char* scr;       // this warp's scratch: staged records
+  float* Rs;       // slice masses of a search [kMaxSlices]
+  float* Hm;       // slice maxima of the bonus draw [kMaxSlices]
+  uint32_t* bm;    // special-token bits of a re-read slice [64]
+  int lane;
+
+  __device__ __forceinline__ unsigned long long tag_of(unsigned t) const {
+    return ((unsigned long long)p.epoch << 32) | (unsigned long long)(t + 1u);
+  }
+  __device__ __forceinline__ bool aborted() const { return ld_relaxed(&p.ctl[kCtlAbort]) != 0u; }
+  __device__ __forceinline__ void set_abort(unsigned bits) const {
+    atomicOr(p.status, bits);
+    atomicExch(&p.ctl[kCtlAbort], 1u);
+  }
+
+  // -------------------------------------------------------------- point values
+  __device__ __forceinline__ float logit_at(const FPass& P, int r, int x) const {
+    if (D.xl_ok)
+      for (int k = 0; k < D.nv; ++k)
+        if (D.X[k] == x) return D.xl[k][r];
+    return E::global(P.row[r].ptr, x);
+  }
+  __device__ __forceinline__ float prob_row(const FPass& P, int r, int x) const {
+    return prob_of(logit_at(P, r, x), P.row[r].M, P.row[r].c, P.row[r].invZ);
+  }
+  __device__ __forceinline__ float spec_lookup(const FPass& P, int tok, float fallback) const {
+    for (int i = 0; i < P.nspec; ++i)
+      if (P.spec_id[i] == tok) return P.spec_val[i];
+    return fallback;
+  }
+  // Point value of the current law p_I (WIS): explicit value of a special
+  // token, else sum_r gamma_r p_r(x) in row order.
+  __device__ float law_at(const FPass& P, int x) const {
+    float a = 0.f;
+    for (int r = 1; r < P.nrows; ++r)
+      if (P.row[r].gamma != 0.f) a = __fmaf_rn(P.row[r].gamma, prob_row(P, r, x), a);
+    return spec_lookup(P, x, a);
+  }
+
+  // -------------------------------------------------------------- planning
+  // Rows of depth j for the valid branches (the lowest valid branch's target
+  // row, then one row per distinct draft model in branch order) into *P (if
+  // given) and, if X is given, the valid branches, their tokens and rows.
+  // One lane.
+  __device__ void plan_rows(int b, int j, unsigned valid, bool bonus, FPass* P, int* nv, int* vbr, int* X,
+                            int* vrow) const {
+    const int K = p.K, L = p.L, V = p.V;
+    const int kstar = __ffs(valid) - 1;
+    if (P) {
+      P->row[0].ptr = p.target + ((((size_t)b * K + kstar) * (L + 1) + j) * (size_t)V) * p.esize;
+      float tq = p.temps[(size_t)b * (1 + K)];
+      if (!(tq > 0.f) || !(tq < kPosInf)) {
+        atomicOr(p.status, MDS_ST_BADTEMP);
+        tq = 1.f;
+      }
+      P->row[0].c = __fdiv_rn(kLog2e, tq);
+    }
+    int mrow[MDS_MAX_K];
+    for (int m = 0; m < MDS_MAX_K; ++m) mrow[m] = -1;
+    int nr = 1, n = 0;
+    if (!bonus) {
+      for (int k = 0; k < K; ++k) {
+        if (!(valid >> k & 1u)) continue;
+        const int m = p.model_of[k];
+        if (mrow[m] < 0) {
+          mrow[m] = nr;
+          if (P) {
+            P->row[nr].ptr = p.drafts[k] + (((size_t)b * L + j) * (size_t)V) * p.esize;
+            float td = p.temps[(size_t)b * (1 + K) + 1 + k];
+            if (!(td > 0.f) || !(td < kPosInf)) {
+              atomicOr(p.status, MDS_ST_BADTEMP);
+              td = 1.f;
+            }
+            P->row[nr].c = __fdiv_rn(kLog2e, td);
+          }
+          ++nr;
+        }
+        if (X) {
+          int x = p.tokens[((size_t)b * K + k) * L + j];
+          if (x < 0 || x >= V) {
+            atomicOr(p.status, MDS_ST_BADTOKEN);
+            x = 0;
+          }
+          vbr[n] = k;
+          X[n] = x;
+          vrow[n] = mrow[m];
+        }
+        ++n;
+      }
+    }
+    if (nv) *nv = n;
+    if (!P) return;
+    for (int r = 0; r < nr; ++r) {
+      P->row[r].M = 0.f;
+      P->row[r].invZ = 0.f;
+      P->row[r].gamma = 0.f;
+    }
+    P->nrows = nr;
+    P->j = j;
+    P->nspec = 0;
+    P->rb = 0;
+    P->cut = 0.f;
+    P->all0 = 0;
+    if (bonus) {
+      P->kind = kBonus;
+      P->nstream = 1;
+      P->list = 0;
+    } else {
+      P->kind = kStats;
+      if (p.scheme == MDS_WIS0) {
+        P->nstream = 1;
+        P->list = 1;
+      } else if (p.scheme == MDS_WIS) {
+        P->nstream = nr;
+        P->list = (n > 1 && nr <= kListRowsMax && p.ln > 0) ? 1 : 0;
+      } else {
+        P->nstream = min(2, nr);
+        P->list = 0;
+      }
+    }
+  }
+
+  // Warp-parallel plan_rows (one lane per branch): the same rows in the same
+  // order, the valid branches, their tokens and rows; then every row's logit
+  // at each draft token into the cache.
+  __device__ void plan_warp(int b, int j, unsigned valid, bool bonus, bool set_pass) {
+    FPass& P = D.P;
+    const int K = p.K;
+    const bool v = !bonus && lane < K && ((valid >> lane) & 1u);
+    const int m = v ? (int)p.model_of[lane] : 64 + lane;
+    const unsigned same = __match_any_sync(FULLM, m);
+    const bool first = v && (__ffs(same) - 1) == lane;
+    const unsigned fm = __ballot_sync(FULLM, first);
+    const unsigned vm = __ballot_sync(FULLM, v);
+    const int nr = 1 + __popc(fm);
+    const int myrow = first ? 1 + __popc(fm & ((1u << lane) - 1u)) : 0;
+    const int row = __shfl_sync(FULLM, myrow, __ffs(same) - 1);
+    if (v) {
+      const int i = __popc(vm & ((1u << lane) - 1u));
+      int x = p.tokens[((size_t)b * K + lane) * p.L + j];
+      if (x < 0 || x >= p.V) {
+        atomicOr(p.status, MDS_ST_BADTOKEN);
+        x = 0;
+      }
+      D.vbr[i] = lane;
+      D.X[i] = x;
+      D.vrow[i] = row;
+    }
+    if (set_pass && first) {
+      P.row[myrow].ptr = p.drafts[lane] + (((size_t)b * p.L + j) * (size_t)p.V) * p.esize;
+      float td = p.temps[(size_t)b * (1 + K) + 1 + lane];
+      if (!(td > 0.f) || !(td < kPosInf)) {
+        atomicOr(p.status, MDS_ST_BADTEMP);
+        td = 1.f;
+      }
+      P.row[myrow].c = __fdiv_rn(kLog2e, td);
+      P.row[myrow].M = 0.f;
+      P.row[myrow].invZ = 0.f;
+      P.row[myrow].gamma = 0.f;
+    }
+    if (lane == 0) {
+      D.nv = __popc(vm);
+      if (set_pass) {
+        const int kstar = __ffs(valid) - 1;
+        P.row[0].ptr = p.target + ((((size_t)b * K + kstar) * (p.L + 1) + j) * (size_t)p.V) * p.esize;
+        float tq = p.temps[(size_t)b * (1 + K)];
+        if (!(tq > 0.f) || !(tq < kPosInf)) {
+          atomicOr(p.status, MDS_ST_BADTEMP);
+          tq = 1.f;
+        }
+        P.row[0].c = __fdiv_rn(kLog2e, tq);
+        P.row[0].M = 0.f;
+        P.row[0].invZ = 0.f;
+        P.row[0].gamma = 0.f;
+        P.nrows = nr;
+        P.j = j;
+        P.nspec = 0;
+        P.rb = 0;
+        P.cut = 0.f;
+        P.all0 = 0;
+        if (bonus) {
+          P.kind = kBonus;
+          P.nstream = 1;
+          P.list = 0;
+        } else {
+          P.kind = kStats;
+          if (p.scheme == MDS_WIS0) {
+            P.nstream = 1;
+            P.list = 1;
+          } else if (p.scheme == MDS_WIS) {
+            P.nstream = nr;
+            P.list = (__popc(vm) > 1 && nr <= kListRowsMax && p.ln > 0) ? 1 : 0;
+          } else {
+            P.nstream = min(2, nr);
+            P.list = 0;
+          }
+        }
+      }
+    }
+    __syncwarp();
+    const int nv = D.nv, nrow = P.nrows;
+    for (int i = lane; i < nv * nrow; i += 32) {
+      const int k = i / nrow, r = i - k * nrow;
+      D.xl[k][r] = E::global(P.row[r].ptr, D.X[k]);
+    }
+    if (lane == 0) D.xl_ok = bonus ? 0 : 1;
+    __syncwarp();
+  }
+
+  // -------------------------------------------------------------- publishing
   __device__ void push(int b, int kind) {
-    DState& D = S.D;
-    const int tid = threadIdx.x;
     PT_T0(t_push);
-    if (tid == 0) D.P.kind = kind;
-    cbar();
+    if (lane == 0) D.P.kind = kind;
+    __syncwarp();
     FSeq* g = &reinterpret_cast<FSeq*>(p.seq)[b];
-    copy_out(&g->P, &D.P, (int)sizeof(FPass), tid, kCT);
-    copy_out(&g->W, &D.W, (int)sizeof(FWalk), tid, kCT);
-    if (tid == 0) __stcg(p.cnt + b, 0u);
-    __threadfence();
-    cbar();
-    if (tid == 0) D.tbase = (unsigned)p.B * (unsigned)p.ns + atomicAdd(&p.ctl[kCtlTail], (unsigned)p.ns);
-    cbar();
-    for (int i = tid; i < p.ns; i += kCT) {
-      const unsigned t = D.tbase + (unsigned)i;
+    copy_out(&g->P, &D.P, (int)sizeof(FPass), lane, 32);
+    copy_out(&g->W, &D.W, (int)sizeof(FWalk), lane, 32);
+    if (lane == 0) __stcg(p.cnt + b, 0u);
+    __threadfence();   // every lane's state writes before any publication
+    __syncwarp();
+    unsigned base = 0u;
+    if (lane == 0) base = (unsigned)p.B * (unsigned)p.ns + atomicAdd(&p.ctl[kCtlTail], (unsigned)p.ns);
+    base = __shfl_sync(FULLM, base, 0);
+    for (int i = lane; i < p.ns; i += 32) {
+      const unsigned t = base + (unsigned)i;
       const unsigned slot = t % (unsigned)p.ring_cap;
       if (t >= (unsigned)p.ring_cap) {
         // the slot's previous task must have been taken
@@ -1344,25 +1422,28 @@ struct Eng {
       __stcg(p.ring_pay + slot, ((unsigned)b << 16) | (unsigned)i);
       st_release(&p.ring_tag[slot], tag_of(t));
     }
-    PT_ADD(kPhPush, t_push);
+    __syncwarp();
+    PT_ADDW(kPhPush, t_push);
   }
 
   __device__ void finish(int b, int acc_len) {
-    if (threadIdx.x == 0) {
+    if (lane == 0) {
       __stcg(p.out_accept + b, acc_len);
       __stcg(p.cnt + b, 0u);
       __threadfence();
       atomicAdd(&p.ctl[kCtlDone], 1u);
     }
+    __syncwarp();
   }
 
   // Z decided at the current depth: outputs, then the next depth's pass,
   // the bonus pass, or the end of the sequence.
   __device__ void walk(int b, int Z, float R, float qY, float pIY, int Ydiag) {
-    DState& D = S.D;
     const int j = D.P.j;
-    cbar();   // every thread has read the depth before thread 0 re-plans
-    if (threadIdx.x == 0) {
+    PT_T0(t_walk);
+    __syncwarp();
+    int next = kNone;
+    if (lane == 0) {
       __stcg(p.out_tokens + (size_t)b * (p.L + 1) + j, Z);
       if (p.out_diag) {
         float* dg = p.out_diag + ((size_t)b * (p.L + 1) + j) * 4;
@@ -1375,7 +1456,7 @@ struct Eng {
       for (int i = 0; i < D.nv; ++i)
         if (D.X[i] == Z) nv |= 1u << D.vbr[i];
       D.W.valid = nv;
-      D.tok = nv ? ((j + 1 == p.L) ? kBonus : kStats) : kNone;
+      next = nv ? ((j + 1 == p.L) ? kBonus : kStats) : kNone;
       if (nv) {
         D.W.stage = 0;
         D.W.zres = 0;
@@ -1383,40 +1464,38 @@ struct Eng {
       }
       D.xl_ok = 0;
     }
-    cbar();
-    const int next = D.tok;
+    next = __shfl_sync(FULLM, next, 0);
+    __syncwarp();
     if (next == kNone)
       finish(b, j);
     else
       push(b, next);
+    PT_ADDW(kPhDecWalk, t_walk);
   }
 
-  // Combine the records of a stats pass: every row's M and 1/Z, and with
-  // candidate lists the sequence's list (the first LN of the slices' lists
-  // by (logit, id)), its complement masses and tau.
-  // The records of a stats pass into the scratch buffer (threads t of nt):
-  // per row the slice maxima and sums, and with lists each slice's tau,
-  // list length and entries.
-  __device__ void stage_records(const FDesc& Dd, int b, char* scratch, int t, int nt) const {
-    const int ns = p.ns, R = Dd.P.nstream, LN = p.lns;
+  // -------------------------------------------------------------- stats decision
+  // The records of a stats pass into the scratch: per row the slice maxima
+  // and sums, and with lists each slice's tau, list length and entries.
+  __device__ void stage_records(int R, bool list, int b) const {
+    const int ns = p.ns, LN = p.lns;
     const float* recb = p.rec + (size_t)b * ns * p.rec_floats;
-    float* hm = reinterpret_cast<float*>(scratch);
+    float* hm = reinterpret_cast<float*>(scr);
     float* hs = hm + R * ns;
     float* htau = hs + R * ns;
     int* hnl = reinterpret_cast<int*>(htau + ns);
     int* eid = hnl + ns;
     float* el = reinterpret_cast<float*>(eid + ns * LN);
-    for (int i = t; i < R * ns; i += nt) {
+    for (int i = lane; i < R * ns; i += 32) {
       const int r = i / ns, s = i - r * ns;
       hm[i] = __ldcg(recb + (size_t)s * p.rec_floats + 2 * r);
       hs[i] = __ldcg(recb + (size_t)s * p.rec_floats + 2 * r + 1);
     }
-    if (Dd.P.list) {
-      for (int s = t; s < ns; s += nt) {
+    if (list) {
+      for (int s = lane; s < ns; s += 32) {
         htau[s] = __ldcg(recb + (size_t)s * p.rec_floats + 2 * kMaxRows);
         hnl[s] = __ldcg(reinterpret_cast<const int*>(recb + (size_t)s * p.rec_floats) + 2 * kMaxRows + 1);
       }
-      for (int i = t; i < ns * LN * (1 + R); i += nt) {
+      for (int i = lane; i < ns * LN * (1 + R); i += 32) {
         const int f = i / (ns * LN), rest = i - f * ns * LN;
         const int s = rest / LN, q = rest - s * LN;
         const float v = __ldcg(recb + (size_t)s * p.rec_floats + kHdr + f * LN + q);
@@ -1426,79 +1505,78 @@ struct Eng {
           el[(f - 1) * ns * LN + rest] = v;
       }
     }
+    __syncwarp();
   }
 
-  // Combine the staged records (stage_records) of a stats pass.
-  __device__ void combine_stats(const FDesc& Dd, int b, char* scratch) {
-    DState& D = S.D;
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int ns = p.ns, R = Dd.P.nstream, LN = p.lns, LF = p.ln;   // a slice's list, the sequence's
-    const bool list = Dd.P.list != 0;
-    float* hm = reinterpret_cast<float*>(scratch);        // [R][ns] slice maxima
-    float* hs = hm + R * ns;                              // [R][ns] slice sums
-    float* htau = hs + R * ns;                            // [ns]
-    int* hnl = reinterpret_cast<int*>(htau + ns);         // [ns]
-    int* eid = hnl + ns;                                  // [ns][LN]
+  __device__ void finish_row(int r, float Z) {
+    if (!(Z > 0.f) || !(Z < kPosInf) || Z != Z) {
+      atomicOr(p.status, MDS_ST_NONFINITE);
+      Z = 1.f;
+    }
+    D.P.row[r].invZ = __frcp_rn(Z);
+  }
+
+  // Combine the staged records of a stats pass: every row's M and 1/Z, and
+  // with candidate lists the sequence's list (the first LF of the slices'
+  // lists by (logit, id)), its complement masses and tau.
+  __device__ void combine_stats(int R, bool list) {
+    const int ns = p.ns, LN = p.lns, LF = p.ln;   // a slice's list, the sequence's
+    float* hm = reinterpret_cast<float*>(scr);        // [R][ns] slice maxima
+    float* hs = hm + R * ns;                          // [R][ns] slice sums
+    float* htau = hs + R * ns;                        // [ns]
+    int* hnl = reinterpret_cast<int*>(htau + ns);     // [ns]
+    int* eid = hnl + ns;                              // [ns][LN]
     float* el = reinterpret_cast<float*>(eid + ns * LN);  // [R][ns][LN]
     // row maxima
-    if (tid < R) {
+    for (int r = lane; r < R; r += 32) {
       float M = kNegInf;
-      for (int s = 0; s < ns; ++s) M = fmaxf(M, hm[tid * ns + s]);
+      for (int s = 0; s < ns; ++s) M = fmaxf(M, hm[r * ns + s]);
       if (!(M > kNegInf) || M != M) {
         atomicOr(p.status, MDS_ST_NONFINITE);
         M = 0.f;
       }
-      D.P.row[tid].M = M;
+      D.P.row[r].M = M;
     }
-    cbar();
+    __syncwarp();
     if (!list) {
-      if (tid < R) {
-        const float M = D.P.row[tid].M, c = D.P.row[tid].c;
+      for (int r = lane; r < R; r += 32) {
+        const float M = D.P.row[r].M, c = D.P.row[r].c;
         float Z = 0.f;
         for (int s = 0; s < ns; ++s) {
-          const float ms = hm[tid * ns + s];
-          if (ms > kNegInf) Z = __fadd_rn(Z, __fmul_rn(hs[tid * ns + s], ref_shift(ms, M, c)));
+          const float ms = hm[r * ns + s];
+          if (ms > kNegInf) Z = __fadd_rn(Z, __fmul_rn(hs[r * ns + s], ref_shift(ms, M, c)));
         }
-        finish_row(tid, Z);
+        finish_row(r, Z);
       }
-      cbar();
+      __syncwarp();
       return;
     }
-    // merge of the slices' lists (warp 0): lane s holds slice s's head; ties
-    // of the logit go to the lower slice, which holds the lower token ids
-    if (warp == 0) {
-      const int nl = (lane < ns) ? hnl[lane] : 0;
-      int h = 0;
-      unsigned key = (h < nl) ? ord_key(__fadd_rn(el[lane * LN], 0.f)) : 0u;
-      int nf = 0;
-      for (int t = 0; t < LF; ++t) {
-        const unsigned km = __reduce_max_sync(FULLM, key);
-        if (!km) break;
-        const unsigned who = __ballot_sync(FULLM, key == km);
-        if (lane == __ffs(who) - 1) {
-          D.fin_s[t] = lane;
-          D.fin_i[t] = h;
-          ++h;
-          key = (h < nl) ? ord_key(__fadd_rn(el[lane * LN + h], 0.f)) : 0u;
-        }
-        nf = t + 1;
+    // merge of the slices' lists: lane s holds slice s's head; ties of the
+    // logit go to the lower slice, which holds the lower token ids
+    const int nl = (lane < ns) ? hnl[lane] : 0;
+    int h = 0;
+    unsigned key = (h < nl) ? ord_key(__fadd_rn(el[lane * LN], 0.f)) : 0u;
+    int nf = 0;
+    for (int t = 0; t < LF; ++t) {
+      const unsigned km = __reduce_max_sync(FULLM, key);
+      if (!km) break;
+      const unsigned who = __ballot_sync(FULLM, key == km);
+      if (lane == __ffs(who) - 1) {
+        D.fin_s[t] = lane;
+        D.fin_i[t] = h;
+        ++h;
+        key = (h < nl) ? ord_key(__fadd_rn(el[lane * LN + h], 0.f)) : 0u;
       }
-      if (lane < ns) D.ksl[lane] = h;
-      // tau: the largest target logit left out (slices' own and dropped entries)
-      float tau = (lane < ns) ? htau[lane] : kNegInf;
-      for (int q = h; q < nl; ++q) tau = fmaxf(tau, el[lane * LN + q]);
-      tau = warp_max(tau);
-      if (lane == 0) {
-        D.n = nf;
-        D.cand_tau = tau;
-        D.cand_all = (nf == p.V) ? 1 : 0;
-      }
+      nf = t + 1;
     }
-    cbar();
-    const int nf = D.n;
-    // dropped entries' masses per row (warp r, fixed order) and the slices' sums
-    if (warp < R) {
-      const int r = warp;
+    if (lane < ns) D.ksl[lane] = h;
+    // tau: the largest target logit left out (slices' own and dropped entries)
+    float tau = (lane < ns) ? htau[lane] : kNegInf;
+    for (int q = h; q < nl; ++q) tau = fmaxf(tau, el[lane * LN + q]);
+    tau = warp_max(tau);
+    __syncwarp();
+    // dropped entries' masses per row (fixed order) and the slices' sums
+    for (int r = 0; r < R; ++r) {
       const float M = D.P.row[r].M, c = D.P.row[r].c;
       float add = 0.f;
       for (int i = lane; i < ns * LN; i += 32) {
@@ -1518,56 +1596,45 @@ struct Eng {
     // the list: in merge order (larger logit first) for the weighted scheme,
     // whose stages break key ties on the id; by token id for the truncated
     // alphabet, whose draws scan Omega_0 in token order
-    if (warp == 0) {
-      const bool by_id = p.scheme == MDS_WIS0;
-      for (int t = lane; t < nf; t += 32) {
-        const int idx = D.fin_s[t] * LN + D.fin_i[t];
-        const int id = eid[idx];
-        int pos = t;
-        if (by_id) {
-          pos = 0;
-          for (int q = 0; q < nf; ++q) pos += (eid[D.fin_s[q] * LN + D.fin_i[q]] < id) ? 1 : 0;
-        }
-        D.cm_id[pos] = id;
-        D.cm_l0[pos] = el[idx];
-        for (int r = 0; r < R; ++r) D.cm_e[r][pos] = exp_term(el[r * ns * LN + idx], D.P.row[r].M, D.P.row[r].c);
-        D.cm_sp[pos] = 0;
-        D.cm_a[pos] = 0.f;
+    const bool by_id = p.scheme == MDS_WIS0;
+    for (int t = lane; t < nf; t += 32) {
+      const int idx = D.fin_s[t] * LN + D.fin_i[t];
+      const int id = eid[idx];
+      int pos = t;
+      if (by_id) {
+        pos = 0;
+        for (int q = 0; q < nf; ++q) pos += (eid[D.fin_s[q] * LN + D.fin_i[q]] < id) ? 1 : 0;
       }
+      D.cm_id[pos] = id;
+      D.cm_l0[pos] = el[idx];
+      for (int r = 0; r < R; ++r) D.cm_e[r][pos] = exp_term(el[r * ns * LN + idx], D.P.row[r].M, D.P.row[r].c);
+      D.cm_sp[pos] = 0;
+      D.cm_a[pos] = 0.f;
     }
-    cbar();
-    if (warp < R) {
-      const int r = warp;
+    __syncwarp();
+    for (int r = 0; r < R; ++r) {
       float z = 0.f;
       for (int t = lane; t < nf; t += 32) z = __fadd_rn(z, D.cm_e[r][t]);
       z = warp_sum(z);
       if (lane == 0) finish_row(r, __fadd_rn(D.pc[r], z));
     }
-    cbar();
-    if (tid == 0) {
-      const float tau = D.cand_tau;
+    __syncwarp();
+    if (lane == 0) {
+      D.n = nf;
+      D.cand_tau = tau;
+      D.cand_all = (nf == p.V) ? 1 : 0;
       D.cand_q = (tau > kNegInf) ? exp_term(tau, D.P.row[0].M, D.P.row[0].c) : 0.f;
     }
-    cbar();
+    __syncwarp();
   }
-
-  __device__ void finish_row(int r, float Z) {
-    if (!(Z > 0.f) || !(Z < kPosInf) || Z != Z) {
-      atomicOr(p.status, MDS_ST_NONFINITE);
-      Z = 1.f;
-    }
-    S.D.P.row[r].invZ = __frcp_rn(Z);
-  }
-
   // -------------------------------------------------------------- WIS stage on the candidate list
-  // Warp 0, one list entry per lane.  Returns false (changing nothing) if
+  // One list entry per lane.  Returns false (changing nothing) if
   // the list cannot certify Omega_1: fewer than s entries, or the s-th key
   // not above every key outside the list (each such key is <= its q <= q(tau)).
   __device__ bool wis_stage_list(int A, int Btok, int rb, float u) {
-    DState& D = S.D;
-    const int lane = threadIdx.x & 31;
     const int s = min(p.wis_s, p.V);
     const int n = D.n;
+    PT_T0(t_sel);
     {
       const float iz0 = D.P.row[0].invZ, izb = D.P.row[rb].invZ;
       const bool have = lane < n;
@@ -1623,6 +1690,7 @@ struct Eng {
           D.om_b[rk] = bq;
         }
         __syncwarp();
+        PT_ADDW(kPhDecSelect, t_sel);
         if (lane == 0) {
           // Omega_2 masses: complement (generic law) + list entries outside Omega_1
           float sa = 0.f;
@@ -1655,7 +1723,6 @@ struct Eng {
   // whole register budget: s <= 5 keeps its pair state in registers, larger
   // s in shared memory.
   __device__ __noinline__ int solve5(int s, float A2, float B2, int A, int Btok, float u) {
-    DState& D = S.D;
     bool capped = false;
     const int y = stage_solve_split<5>(s, A2, B2, A, Btok, u, D.om, D.om_q, D.om_a, D.om_b, D.om_x, &capped, D.lp_rs,
                                        D.lp_fl, D.lp_fh, D.lp_rd);
@@ -1663,7 +1730,6 @@ struct Eng {
     return y;
   }
   __device__ __noinline__ int solve8(int s, float A2, float B2, int A, int Btok, float u) {
-    DState& D = S.D;
     bool capped = false;
     const int y = stage_solve<MDS_MAX_S>(s, A2, B2, A, Btok, u, D.om, D.om_q, D.om_a, D.om_b, D.om_x, &capped,
                                          D.lp_rs, D.lp_fl, D.lp_fh);
@@ -1673,14 +1739,13 @@ struct Eng {
   __device__ int solve(int s, float A2, float B2, int A, int Btok, float u) {
     PT_T0(t_lp);
     const int y = (s <= 5) ? solve5(s, A2, B2, A, Btok, u) : solve8(s, A2, B2, A, Btok, u);
-    PT_ADD(kPhLp, t_lp);
-    PT_CNT(kPhLpCalls);
+    PT_ADDW(kPhLp, t_lp);
+    PT_CNTW(kPhLpCalls);
     return y;
   }
 
   // Generic law after a stage: gamma <- (B2/2) gamma + (A2/2) e_rb.  One thread.
   __device__ void gamma_update(int rb, float A2, float B2) {
-    DState& D = S.D;
     const float hB = __fmul_rn(0.5f, B2), hA = __fmul_rn(0.5f, A2);
     for (int r = 1; r < D.P.nrows; ++r) D.P.row[r].gamma = __fmul_rn(hB, D.P.row[r].gamma);
     D.P.row[rb].gamma = __fadd_rn(D.P.row[rb].gamma, hA);
@@ -1689,7 +1754,6 @@ struct Eng {
   // The list's special tokens into the table form used by the residual and
   // the point lookups.  One thread.
   __device__ void list_to_table() {
-    DState& D = S.D;
     int k = 0;
     for (int i = 0; i < D.n && k < kMaxSpecial; ++i)
       if (D.cm_sp[i]) {
@@ -1702,16 +1766,17 @@ struct Eng {
 
   // -------------------------------------------------------------- decisions per pass kind
   __device__ void accept_step(int b) {
-    DState& D = S.D;
-    if (threadIdx.x == 0) {
+    PT_T0(t_acc);
+    int walk_now = 0;
+    if (lane == 0) {
       const int j = D.P.j;
       const float u = draw_uniform(p.seed, b, j, kDrawAccept);
       const float ratio = D.W.pIY > 0.f ? __fdiv_rn(D.W.qY, D.W.pIY) : kPosInf;
       const bool acc = u < fminf(1.f, ratio);
       D.W.acc = acc ? 1 : 0;
       D.W.Ydiag = D.W.Y;
-      D.tok = (acc && !p.acc_prob) ? 1 : 0;
-      if (!D.tok) {
+      walk_now = (acc && !p.acc_prob) ? 1 : 0;
+      if (!walk_now) {
         D.W.ures = acc ? 0.f : draw_uniform(p.seed, b, j, kDrawResidual);
         if (p.scheme == MDS_SINGLE || D.nv == 1 || p.scheme != MDS_WIS) {
           // residual against one draft law: rows 0 and the first valid branch's
@@ -1724,111 +1789,103 @@ struct Eng {
         }
       }
     }
-    cbar();
-    if (D.tok)
+    walk_now = __shfl_sync(FULLM, walk_now, 0);
+    __syncwarp();
+    if (walk_now)
       walk(b, D.W.Y, 0.f, D.W.qY, D.W.pIY, D.W.Y);
     else
       push(b, kResid);
+    PT_ADDW(kPhDecAccept, t_acc);
   }
 
-  __device__ void decide_stats(const FDesc& Dd, int b, char* scratch) {
-    DState& D = S.D;
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int j = Dd.P.j;
-    // warp 0 plans the depth (and caches the logits at the draft tokens)
-    // while the other warps stage the records
-    if (warp == 0) {
-      if (j == 0 && lane == 0) {
-        D.W = FWalk{};
-        D.W.valid = (p.K >= 32) ? FULLM : ((1u << p.K) - 1u);
-        D.W.Yp = -1;
-      }
-      __syncwarp();
-      plan_warp(b, j, D.W.valid, false, true);
-    } else {
-      stage_records(Dd, b, scratch, tid - 32, kCT - 32);
+  __device__ void decide_stats(int b, int j, int R, bool list) {
+    if (j == 0 && lane == 0) {
+      D.W = FWalk{};
+      D.W.valid = (p.K >= 32) ? FULLM : ((1u << p.K) - 1u);
+      D.W.Yp = -1;
     }
-    cbar();
+    __syncwarp();
+    PT_T0(t_plan);
+    plan_warp(b, j, D.W.valid, false, true);
+    PT_ADDW(kPhDecPlan, t_plan);
+    PT_T0(t_load);
+    stage_records(R, list, b);
+    PT_ADDW(kPhDecLoad, t_load);
     PT_T0(t_comb);
-    combine_stats(Dd, b, scratch);
-    PT_ADD(kPhDecCombine, t_comb);
+    combine_stats(R, list);
+    PT_ADDW(kPhDecCombine, t_comb);
     if (p.scheme == MDS_WIS0) {
       wis0_decide(b);
       return;
     }
     if (p.scheme == MDS_SINGLE || D.nv == 1) {
-      if (tid == 0) {
+      if (lane == 0) {
         const int Y = D.X[0];
         D.W.Y = Y;
         D.W.qY = prob_row(D.P, 0, Y);
         D.W.pIY = prob_row(D.P, D.vrow[0], Y);
       }
-      cbar();
+      __syncwarp();
       accept_step(b);
       return;
     }
     // WIS: the pairwise stages (Remark 4) on the candidate list while it
-    // certifies Omega_1 (warp 0 alone); from the first stage it cannot,
-    // full-vocabulary passes
+    // certifies Omega_1; from the first stage it cannot, full-vocabulary passes
     PT_T0(t_stg);
-    if (warp == 0) {
-      if (lane == 0) {
-        for (int r = 0; r < D.P.nrows; ++r) D.P.row[r].gamma = 0.f;
-        D.P.row[D.vrow[0]].gamma = 1.f;
-        D.P.nspec = 0;
+    if (lane == 0) {
+      for (int r = 0; r < D.P.nrows; ++r) D.P.row[r].gamma = 0.f;
+      D.P.row[D.vrow[0]].gamma = 1.f;
+      D.P.nspec = 0;
+    }
+    __syncwarp();
+    int A = D.X[0];
+    int m = 1;
+    if (list) {
+      // every stage's selection uniform at once (lane m - 1 draws stage m's)
+      const float ul = (lane + 1 < D.nv) ? draw_uniform(p.seed, b, j, kDrawSelect + lane) : 0.f;
+      for (; m < D.nv; ++m) {
+        const float u = __shfl_sync(FULLM, ul, m - 1);
+        if (!wis_stage_list(A, D.X[m], D.vrow[m], u)) break;
+        A = D.Y;
       }
-      __syncwarp();
-      int A = D.X[0];
-      int m = 1;
-      if (Dd.P.list) {
-        // every stage's selection uniform at once (lane m - 1 draws stage m's)
-        const float ul = (lane + 1 < D.nv) ? draw_uniform(p.seed, b, j, kDrawSelect + lane) : 0.f;
-        for (; m < D.nv; ++m) {
-          const float u = __shfl_sync(FULLM, ul, m - 1);
-          if (!wis_stage_list(A, D.X[m], D.vrow[m], u)) break;
-          A = D.Y;
-        }
-        if (lane == 0) list_to_table();
-      }
-      if (lane == 0) {
-        D.W.stage = m;
-        D.W.A = A;
-        if (m < D.nv) {
-          D.P.rb = D.vrow[m];
-          D.P.nstream = D.P.nrows;
-        } else {
-          D.W.Y = A;
-          D.W.qY = prob_row(D.P, 0, A);
-          D.W.pIY = law_at(D.P, A);
-        }
+      if (lane == 0) list_to_table();
+    }
+    if (lane == 0) {
+      D.W.stage = m;
+      D.W.A = A;
+      if (m < D.nv) {
+        D.P.rb = D.vrow[m];
+        D.P.nstream = D.P.nrows;
+      } else {
+        D.W.Y = A;
+        D.W.qY = prob_row(D.P, 0, A);
+        D.W.pIY = law_at(D.P, A);
       }
     }
-    cbar();
-    PT_ADD(kPhDecStages, t_stg);
-    if (D.W.stage < D.nv) {
+    __syncwarp();
+    PT_ADDW(kPhDecStages, t_stg);
+    if (m < D.nv) {
       push(b, kFull);
       return;
     }
     accept_step(b);
   }
 
-  __device__ void decide_full(const FDesc& Dd, int b) {
-    DState& D = S.D;
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  // One full-vocabulary stage's decision: Omega_1 = the top s of the slices'
+  // top s (s rounds of a warp argmax), the Omega_2 masses (the slices' rests
+  // plus their entries not taken), the LP, the selection and the law update.
+  __device__ void decide_full(int b) {
     const int j = D.P.j, ns = p.ns;
-    if (warp == 0) plan_warp(b, j, D.W.valid, false, false);
-    cbar();
+    plan_warp(b, j, D.W.valid, false, false);
     const int m = D.W.stage;
     const int A = D.W.A, Btok = D.X[m], rb = D.vrow[m];
     const float u = draw_uniform(p.seed, b, j, kDrawSelect + m - 1);
     const int s = min(p.wis_s, p.V);
     const float* recb = p.rec + (size_t)b * ns * p.rec_floats;
-    // Omega_1: the top s of every slice's top s (s rounds of a block argmax)
-    float ra = 0.f, rbs = 0.f;
     for (int r = 0; r < s; ++r) {
       float bk = kNegInf;
       int bid = 0x7fffffff, bi = -1;
-      for (int i = tid; i < ns * kTopF; i += kCT) {
+      for (int i = lane; i < ns * kTopF; i += 32) {
         const int sl = i / kTopF, t = i - sl * kTopF;
         if (t >= s) continue;
         const float* rc = recb + (size_t)sl * p.rec_floats;
@@ -1854,162 +1911,186 @@ struct Eng {
           bi = oi;
         }
       }
-      cbar();
       if (lane == 0) {
-        S.red[warp * 3] = bk;
-        S.red[warp * 3 + 1] = __int_as_float(bid);
-        S.red[warp * 3 + 2] = __int_as_float(bi);
-      }
-      cbar();
-      if (tid == 0) {
-        float k2 = kNegInf;
-        int id2 = 0x7fffffff, i2 = -1;
-        for (int w = 0; w < kCW; ++w) {
-          const float kw = S.red[w * 3];
-          const int iw = __float_as_int(S.red[w * 3 + 1]);
-          if (better(kw, iw, k2, id2)) {
-            k2 = kw;
-            id2 = iw;
-            i2 = __float_as_int(S.red[w * 3 + 2]);
-          }
-        }
         Cand c = CAND_NONE;
-        if (i2 >= 0) {
-          const float* rc = recb + (size_t)(i2 / kTopF) * p.rec_floats;
-          const int t = i2 % kTopF;
-          c = Cand{k2, id2, __ldcg(rc + 4 + 2 * kTopF + t), __ldcg(rc + 4 + 3 * kTopF + t)};
+        if (bi >= 0) {
+          const float* rc = recb + (size_t)(bi / kTopF) * p.rec_floats;
+          const int t = bi % kTopF;
+          c = Cand{bk, bid, __ldcg(rc + 4 + 2 * kTopF + t), __ldcg(rc + 4 + 3 * kTopF + t)};
         }
         D.fin[r] = c;
       }
-      cbar();
+      __syncwarp();
     }
     // Omega_2 masses: the slices' rests plus their top-s entries not taken
-    {
-      float sa = 0.f, sb = 0.f;
-      for (int i = tid; i < ns * kTopF; i += kCT) {
-        const int sl = i / kTopF, t = i - sl * kTopF;
-        const float* rc = recb + (size_t)sl * p.rec_floats;
-        if (t == 0) {
-          sa = __fadd_rn(sa, __ldcg(rc + 0));
-          sb = __fadd_rn(sb, __ldcg(rc + 1));
-        }
-        if (t >= s) continue;
-        const int id = __ldcg(reinterpret_cast<const int*>(rc) + 4 + kTopF + t);
-        if (id == 0x7fffffff) continue;
-        bool taken = false;
-        for (int q = 0; q < s; ++q) taken |= (D.fin[q].id == id);
-        if (taken) continue;
-        sa = __fadd_rn(sa, __ldcg(rc + 4 + 2 * kTopF + t));
-        sb = __fadd_rn(sb, __ldcg(rc + 4 + 3 * kTopF + t));
+    float sa = 0.f, sb = 0.f;
+    for (int i = lane; i < ns * kTopF; i += 32) {
+      const int sl = i / kTopF, t = i - sl * kTopF;
+      const float* rc = recb + (size_t)sl * p.rec_floats;
+      if (t == 0) {
+        sa = __fadd_rn(sa, __ldcg(rc + 0));
+        sb = __fadd_rn(sb, __ldcg(rc + 1));
       }
-      ra = block_sum(sa, S.red);
-      rbs = block_sum(sb, S.red + kCW);
+      if (t >= s) continue;
+      const int id = __ldcg(reinterpret_cast<const int*>(rc) + 4 + kTopF + t);
+      if (id == 0x7fffffff) continue;
+      bool taken = false;
+      for (int q = 0; q < s; ++q) taken |= (D.fin[q].id == id);
+      if (taken) continue;
+      sa = __fadd_rn(sa, __ldcg(rc + 4 + 2 * kTopF + t));
+      sb = __fadd_rn(sb, __ldcg(rc + 4 + 3 * kTopF + t));
     }
-    if (warp == 0) {
-      if (lane < s) {
-        int id = D.fin[lane].id;
-        if (id < 0 || id >= p.V) id = 0;   // only with non-finite keys (status already set)
-        D.fin[lane].id = id;
-        D.om_q[lane] = prob_row(D.P, 0, id);
-      }
-      __syncwarp();
-      if (lane == 0) {
-        // Omega_1 by token id; q follows its token
-        int om[MDS_MAX_S];
-        float ak[MDS_MAX_S], bk[MDS_MAX_S], qk[MDS_MAX_S];
-        for (int t = 0; t < MDS_MAX_S; ++t) {
-          om[t] = (t < s) ? D.fin[t].id : 0x7fffffff;
-          ak[t] = (t < s) ? D.fin[t].a : 0.f;
-          bk[t] = (t < s) ? D.fin[t].b : 0.f;
-          qk[t] = (t < s) ? D.om_q[t] : 0.f;
-        }
-        for (int x = 1; x < MDS_MAX_S; ++x)   // insertion sort by id (at most 8 entries)
-          for (int y = x; y > 0 && om[y] < om[y - 1]; --y) {
-            const int ti = om[y];
-            om[y] = om[y - 1];
-            om[y - 1] = ti;
-            float tf = ak[y];
-            ak[y] = ak[y - 1];
-            ak[y - 1] = tf;
-            tf = bk[y];
-            bk[y] = bk[y - 1];
-            bk[y - 1] = tf;
-            tf = qk[y];
-            qk[y] = qk[y - 1];
-            qk[y - 1] = tf;
-          }
-        for (int t = 0; t < MDS_MAX_S; ++t) {
-          D.om[t] = om[t];
-          D.om_a[t] = ak[t];
-          D.om_b[t] = bk[t];
-          D.om_q[t] = qk[t];
-        }
-        D.Y = solve(s, ra, rbs, A, Btok, u);
-        D.A2 = ra;
-        D.B2 = rbs;
-      }
-      __syncwarp();
-      // law update: special tokens outside Omega_1, gamma, Omega_1 values
-      const float A2 = D.A2, B2 = D.B2;
-      for (int i = lane; i < D.P.nspec; i += 32) {
-        const int tokn = D.P.spec_id[i];
-        bool in1 = false;
-        for (int t = 0; t < s; ++t) in1 |= (D.om[t] == tokn);
-        if (!in1)
-          D.P.spec_val[i] =
-              __fmul_rn(0.5f, __fadd_rn(__fmul_rn(D.P.spec_val[i], B2), __fmul_rn(prob_row(D.P, rb, tokn), A2)));
-      }
-      __syncwarp();
-      if (lane == 0) {
-        gamma_update(rb, A2, B2);
-        for (int t = 0; t < s; ++t) {
-          int i = 0;
-          while (i < D.P.nspec && D.P.spec_id[i] != D.om[t]) ++i;
-          if (i == D.P.nspec && D.P.nspec < kMaxSpecial) {
-            D.P.spec_id[i] = D.om[t];
-            ++D.P.nspec;
-          }
-          if (i < kMaxSpecial) D.P.spec_val[i] = D.om_x[t];
-        }
-        D.W.A = D.Y;
-        D.W.stage = m + 1;
-        if (m + 1 < D.nv) D.P.rb = D.vrow[m + 1];
-      }
+    const float ra = warp_sum(sa), rbs = warp_sum(sb);
+    if (lane < s) {
+      int id = D.fin[lane].id;
+      if (id < 0 || id >= p.V) id = 0;   // only with non-finite keys (status already set)
+      D.fin[lane].id = id;
+      D.om_q[lane] = prob_row(D.P, 0, id);
     }
-    cbar();
+    __syncwarp();
+    if (lane == 0) {
+      // Omega_1 by token id; q follows its token
+      int om[MDS_MAX_S];
+      float ak[MDS_MAX_S], bk[MDS_MAX_S], qk[MDS_MAX_S];
+      for (int t = 0; t < MDS_MAX_S; ++t) {
+        om[t] = (t < s) ? D.fin[t].id : 0x7fffffff;
+        ak[t] = (t < s) ? D.fin[t].a : 0.f;
+        bk[t] = (t < s) ? D.fin[t].b : 0.f;
+        qk[t] = (t < s) ? D.om_q[t] : 0.f;
+      }
+      for (int x = 1; x < MDS_MAX_S; ++x)   // insertion sort by id (at most 8 entries)
+        for (int y = x; y > 0 && om[y] < om[y - 1]; --y) {
+          const int ti = om[y];
+          om[y] = om[y - 1];
+          om[y - 1] = ti;
+          float tf = ak[y];
+          ak[y] = ak[y - 1];
+          ak[y - 1] = tf;
+          tf = bk[y];
+          bk[y] = bk[y - 1];
+          bk[y - 1] = tf;
+          tf = qk[y];
+          qk[y] = qk[y - 1];
+          qk[y - 1] = tf;
+        }
+      for (int t = 0; t < MDS_MAX_S; ++t) {
+        D.om[t] = om[t];
+        D.om_a[t] = ak[t];
+        D.om_b[t] = bk[t];
+        D.om_q[t] = qk[t];
+      }
+      D.Y = solve(s, ra, rbs, A, Btok, u);
+      D.A2 = ra;
+      D.B2 = rbs;
+    }
+    __syncwarp();
+    // law update: special tokens outside Omega_1, gamma, Omega_1 values
+    const float A2 = D.A2, B2 = D.B2;
+    for (int i = lane; i < D.P.nspec; i += 32) {
+      const int tokn = D.P.spec_id[i];
+      bool in1 = false;
+      for (int t = 0; t < s; ++t) in1 |= (D.om[t] == tokn);
+      if (!in1)
+        D.P.spec_val[i] =
+            __fmul_rn(0.5f, __fadd_rn(__fmul_rn(D.P.spec_val[i], B2), __fmul_rn(prob_row(D.P, rb, tokn), A2)));
+    }
+    __syncwarp();
+    if (lane == 0) {
+      gamma_update(rb, A2, B2);
+      for (int t = 0; t < s; ++t) {
+        int i = 0;
+        while (i < D.P.nspec && D.P.spec_id[i] != D.om[t]) ++i;
+        if (i == D.P.nspec && D.P.nspec < kMaxSpecial) {
+          D.P.spec_id[i] = D.om[t];
+          ++D.P.nspec;
+        }
+        if (i < kMaxSpecial) D.P.spec_val[i] = D.om_x[t];
+      }
+      D.W.A = D.Y;
+      D.W.stage = m + 1;
+      if (m + 1 < D.nv) D.P.rb = D.vrow[m + 1];
+    }
+    __syncwarp();
     if (m + 1 < D.nv) {
       push(b, kFull);
       return;
     }
-    if (tid == 0) {
+    if (lane == 0) {
       const int Y = D.W.A;
       D.W.Y = Y;
       D.W.qY = prob_row(D.P, 0, Y);
       D.W.pIY = law_at(D.P, Y);
     }
-    cbar();
+    __syncwarp();
     accept_step(b);
   }
 
-  // Inverse-CDF search over the weights of pass kind P.kind: the slice by
-  // the per-slice masses Rs[0..ns) (slice order), the token by one re-read of
-  // that slice in token order (contiguous runs per thread, a fixed-order
-  // exclusive scan, then the owning run).  Returns the smallest token whose
-  // running mass exceeds T, else the last token with positive weight.
-  __device__ int search(FPass& P, const float* Rs, float T, char* scratch) {
-    DState& D = S.D;
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    if (tid == 0) {
+  // -------------------------------------------------------------- inverse-CDF search
+  // Weights of unit u (tokens tok0 + u*VE + e) of a re-read slice, read from
+  // global memory: the residual max(0, q - p_I) (kResid), the target mass
+  // outside Omega_0 (kReplace) or the target mass (kBonus); tokens past the
+  // slice weigh 0.
+  __device__ void weights_g(const FPass& P, int u, int tok0, int n, float* w) const {
+    auto load = [&](int r, float* v) {
+      const char* row = P.row[r].ptr;
+      const int t0 = tok0 + u * VE;
+      if (p.aligned && u * VE + VE <= n) {
+        E::unit_global(row + (size_t)t0 * p.esize, v);
+      } else {
+#pragma unroll
+        for (int e = 0; e < VE; ++e) v[e] = (u * VE + e < n) ? E::global(row, t0 + e) : kNegInf;
+      }
+    };
+    float v0[VE];
+    load(0, v0);
+    const float M0 = P.row[0].M, c0 = P.row[0].c, iz0 = P.row[0].invZ;
+    if (P.kind == kResid) {
+      float a[VE];
+#pragma unroll
+      for (int e = 0; e < VE; ++e) a[e] = 0.f;
+      for (int r = 1; r < P.nstream; ++r) {
+        const float g = P.row[r].gamma;
+        if (g == 0.f) continue;
+        float v[VE];
+        load(r, v);
+        const float M = P.row[r].M, c = P.row[r].c, iz = P.row[r].invZ;
+#pragma unroll
+        for (int e = 0; e < VE; ++e) a[e] = __fmaf_rn(g, prob_of(v[e], M, c, iz), a[e]);
+      }
+      if (P.nspec > 0 && ((bm[u >> 5] >> (u & 31)) & 1u)) {
+#pragma unroll
+        for (int e = 0; e < VE; ++e) a[e] = spec_lookup(P, tok0 + u * VE + e, a[e]);
+      }
+#pragma unroll
+      for (int e = 0; e < VE; ++e) w[e] = fmaxf(0.f, __fsub_rn(prob_of(v0[e], M0, c0, iz0), a[e]));
+    } else if (P.kind == kReplace) {
+#pragma unroll
+      for (int e = 0; e < VE; ++e) w[e] = (P.all0 || v0[e] > P.cut) ? 0.f : prob_of(v0[e], M0, c0, iz0);
+    } else {
+#pragma unroll
+      for (int e = 0; e < VE; ++e) w[e] = prob_of(v0[e], M0, c0, iz0);
+    }
+  }
+
+  // The smallest token whose running mass exceeds T, else the last token
+  // with positive weight: the slice by the masses Rs[0..ns) (in slice order),
+  // then inside it three levels in token order: contiguous runs of units per
+  // lane, the units of the owning run (one per lane), the owning unit's
+  // tokens.  Every level sums in a fixed order.
+  __device__ int search(FPass& P, float T) {
+    int s = 0;
+    float base = 0.f;
+    if (lane == 0) {
       float run = 0.f, run_last = 0.f, run_hit = 0.f;
       int hit = -1, last = -1;
-      for (int s = 0; s < p.ns; ++s) {
-        const float v = Rs[s];
+      for (int q = 0; q < p.ns; ++q) {
+        const float v = Rs[q];
         if (v > 0.f) {
-          last = s;
+          last = q;
           run_last = run;
         }
         if (hit < 0 && __fadd_rn(run, v) > T) {
-          hit = s;
+          hit = q;
           run_hit = run;
         }
         run = __fadd_rn(run, v);
@@ -2018,98 +2099,120 @@ struct Eng {
         hit = max(last, 0);
         run_hit = run_last;
       }
-      D.seg = hit;
-      D.run = run_hit;
-      D.cross = kCT;
-      D.lastp = -1;
+      s = hit;
+      base = run_hit;
     }
-    cbar();
-    const int s = D.seg;
-    const float base = D.run;
+    s = __shfl_sync(FULLM, s, 0);
+    base = __shfl_sync(FULLM, base, 0);
     const int tok0 = s * p.T, n = min(p.T, p.V - tok0);
-    const int nst = (P.kind == kResid) ? P.nstream : 1;
-    load_plain(P, nst, scratch, tok0, n);
-    if (P.kind == kResid && P.nspec > 0) build_bitmap(P, tok0, n);
     const int U = (n + VE - 1) / VE;
-    const int upt = (U + kCT - 1) / kCT;
-    const int u0 = min(U, tid * upt), u1 = min(U, u0 + upt);
+    if (P.kind == kResid && P.nspec > 0) {
+      for (int i = lane; i < 64; i += 32) bm[i] = 0u;
+      __syncwarp();
+      for (int i = lane; i < P.nspec; i += 32) {
+        const int loc = P.spec_id[i] - tok0;
+        if (loc >= 0 && loc < n) atomicOr(&bm[(loc / VE) >> 5], 1u << ((loc / VE) & 31));
+      }
+      __syncwarp();
+    }
+    // level 1: lane runs of upl units
+    const int upl = (U + 31) / 32;
+    const int u0 = min(U, lane * upl), u1 = min(U, u0 + upl);
     float part = 0.f;
     for (int u = u0; u < u1; ++u) {
       float w[VE];
-      weights(P, scratch, u, tok0, w);
+      weights_g(P, u, tok0, n, w);
 #pragma unroll
       for (int e = 0; e < VE; ++e) part = __fadd_rn(part, w[e]);
     }
-    // exclusive scan over the threads (warp scans, then warps in order)
     float incl = part;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
       const float t = __shfl_up_sync(FULLM, incl, o);
       if (lane >= o) incl = __fadd_rn(incl, t);
     }
-    if (lane == 31) S.red[warp] = incl;
-    cbar();
-    float wbase = base;
-    for (int w = 0; w < warp; ++w) wbase = __fadd_rn(wbase, S.red[w]);
-    const float excl = __fadd_rn(wbase, __fsub_rn(incl, part));
-    const float end = __fadd_rn(wbase, incl);
-    if (end > T && part > 0.f) atomicMin(&D.cross, tid);
-    if (part > 0.f) atomicMax(&D.lastp, tid);
-    cbar();
-    // the first run whose end passes T; if rounding left the slice short, the
-    // last run with mass (its last positive token); -1: no mass at all
-    const int owner = (D.cross < kCT) ? D.cross : D.lastp;
-    if (tid == (owner < 0 ? 0 : owner)) {
-      int tok = -1, last = -1;
-      float acc = excl;
-      if (owner >= 0) {
-        for (int u = u0; u < u1 && tok < 0; ++u) {
-          float w[VE];
-          weights(P, scratch, u, tok0, w);
+    const float excl = __fadd_rn(base, __fsub_rn(incl, part));
+    const unsigned hit1 = __ballot_sync(FULLM, __fadd_rn(base, incl) > T && part > 0.f);
+    const unsigned pos1 = __ballot_sync(FULLM, part > 0.f);
+    if (!pos1) return tok0;   // no mass in the slice (only by rounding)
+    const int own = hit1 ? __ffs(hit1) - 1 : 31 - __clz(pos1);
+    // level 2: the owning run's units, one per lane (chunks of 32)
+    float run = __shfl_sync(FULLM, excl, own);
+    const int v0 = __shfl_sync(FULLM, u0, own), v1 = __shfl_sync(FULLM, u1, own);
+    int unit = -1, ulast = -1;
+    float ubase = 0.f, ubase_last = 0.f;
+    for (int c0 = v0; c0 < v1 && unit < 0; c0 += 32) {
+      const int u = c0 + lane;
+      float w[VE], us = 0.f;
+      if (u < v1) {
+        weights_g(P, u, tok0, n, w);
 #pragma unroll
-          for (int e = 0; e < VE; ++e) {
-            if (w[e] > 0.f) last = tok0 + u * VE + e;
-            acc = __fadd_rn(acc, w[e]);
-            if (tok < 0 && acc > T && w[e] > 0.f) tok = tok0 + u * VE + e;
-          }
-        }
+        for (int e = 0; e < VE; ++e) us = __fadd_rn(us, w[e]);
       }
-      if (tok < 0) tok = last;
-      if (tok < 0) tok = tok0;
-      D.tok = min(tok, p.V - 1);
+      float ui = us;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const float t = __shfl_up_sync(FULLM, ui, o);
+        if (lane >= o) ui = __fadd_rn(ui, t);
+      }
+      const float uex = __fadd_rn(run, __fsub_rn(ui, us));
+      const unsigned h2 = __ballot_sync(FULLM, __fadd_rn(run, ui) > T && us > 0.f);
+      const unsigned p2 = __ballot_sync(FULLM, us > 0.f);
+      if (h2) {
+        const int l2 = __ffs(h2) - 1;
+        unit = c0 + l2;
+        ubase = __shfl_sync(FULLM, uex, l2);
+      } else if (p2) {
+        const int l2 = 31 - __clz(p2);
+        ulast = c0 + l2;
+        ubase_last = __shfl_sync(FULLM, uex, l2);
+      }
+      run = __shfl_sync(FULLM, __fadd_rn(run, ui), 31);
     }
-    cbar();
-    return D.tok;
+    if (unit < 0) {
+      unit = ulast;
+      ubase = ubase_last;
+    }
+    // level 3: the owning unit's tokens (one lane)
+    int tok = tok0;
+    if (lane == 0 && unit >= 0) {
+      float w[VE];
+      weights_g(P, unit, tok0, n, w);
+      float acc = ubase;
+      int hit = -1, last = -1;
+#pragma unroll
+      for (int e = 0; e < VE; ++e) {
+        if (w[e] > 0.f) last = e;
+        acc = __fadd_rn(acc, w[e]);
+        if (hit < 0 && acc > T && w[e] > 0.f) hit = e;
+      }
+      if (hit < 0) hit = last < 0 ? 0 : last;
+      tok = min(tok0 + unit * VE + hit, p.V - 1);
+    }
+    return __shfl_sync(FULLM, tok, 0);
   }
 
-  // Slice masses of pass `kind` from the records (Rs in shared memory) and
-  // their total in slice order.
-  __device__ float slice_masses(int b, float* Rs) {
+  // Slice masses of the pass just completed (Rs) and their total in slice order.
+  __device__ float slice_masses(int b) {
     const float* recb = p.rec + (size_t)b * p.ns * p.rec_floats;
-    for (int s = threadIdx.x; s < p.ns; s += kCT) Rs[s] = __ldcg(recb + (size_t)s * p.rec_floats);
-    cbar();
-    if (threadIdx.x == 0) {
-      float R = 0.f;
-      for (int s = 0; s < p.ns; ++s) R = __fadd_rn(R, Rs[s]);
-      S.D.rtot = R;
-    }
-    cbar();
-    return S.D.rtot;
+    for (int q = lane; q < p.ns; q += 32) Rs[q] = __ldcg(recb + (size_t)q * p.rec_floats);
+    __syncwarp();
+    float R = 0.f;
+    if (lane == 0)
+      for (int q = 0; q < p.ns; ++q) R = __fadd_rn(R, Rs[q]);
+    return __shfl_sync(FULLM, R, 0);
   }
 
-  __device__ void decide_resid(int b, char* scratch) {
-    DState& D = S.D;
-    const int tid = threadIdx.x;
-    if ((tid >> 5) == 0) plan_warp(b, D.P.j, D.W.valid, false, false);
-    float* Rs = S.Rs;
-    const float R = slice_masses(b, Rs);
+  __device__ void decide_resid(int b) {
+    plan_warp(b, D.P.j, D.W.valid, false, false);
+    const float R = slice_masses(b);
     int Z = D.W.Y;
     if (!D.W.acc) {
       if (R > 0.f) {
-        Z = search(D.P, Rs, __fmul_rn(D.W.ures, R), scratch);
+        Z = search(D.P, __fmul_rn(D.W.ures, R));
       } else {
         // zero residual mass (only by rounding): sample the target row
-        if (tid == 0) {
+        if (lane == 0) {
           atomicOr(p.status, MDS_ST_ZERO_RESID);
           D.W.zres = 1;
           D.W.R = R;
@@ -2117,7 +2220,7 @@ struct Eng {
           D.P.all0 = 0;
           D.P.nstream = 1;
         }
-        cbar();
+        __syncwarp();
         push(b, kReplace);
         return;
       }
@@ -2125,74 +2228,64 @@ struct Eng {
     walk(b, Z, R, D.W.qY, D.W.pIY, D.W.Ydiag);
   }
 
-  __device__ void decide_replace(int b, char* scratch) {
-    DState& D = S.D;
-    const int tid = threadIdx.x;
-    if ((tid >> 5) == 0) plan_warp(b, D.P.j, D.W.valid, false, false);
-    float* Rs = S.Rs;
-    const float R = slice_masses(b, Rs);
+  __device__ void decide_replace(int b) {
+    plan_warp(b, D.P.j, D.W.valid, false, false);
+    const float R = slice_masses(b);
     int Z;
     if (R > 0.f) {
-      Z = search(D.P, Rs, __fmul_rn(D.W.ures, R), scratch);
+      Z = search(D.P, __fmul_rn(D.W.ures, R));
     } else if (!D.W.zres && D.W.Yp >= 0) {
       Z = D.W.Yp;   // no target mass outside Omega_0
     } else if (!D.W.zres) {
-      if (tid == 0) {
+      if (lane == 0) {
         atomicOr(p.status, MDS_ST_ZERO_RESID);
         D.W.zres = 1;
         D.P.cut = kPosInf;
         D.P.all0 = 0;
       }
-      cbar();
+      __syncwarp();
       push(b, kReplace);
       return;
     } else {
-      if (tid == 0) atomicOr(p.status, MDS_ST_NONFINITE);
+      if (lane == 0) atomicOr(p.status, MDS_ST_NONFINITE);
       Z = 0;
     }
     const float Rd = (p.scheme == MDS_WIS0) ? D.W.R : (D.W.zres ? D.W.R : R);
     walk(b, Z, Rd, D.W.qY, D.W.pIY, D.W.Ydiag);
   }
 
-  __device__ void decide_bonus(const FDesc& Dd, int b, char* scratch) {
-    DState& D = S.D;
-    const int tid = threadIdx.x;
+  __device__ void decide_bonus(int b) {
     const float* recb = p.rec + (size_t)b * p.ns * p.rec_floats;
-    float* hm = S.hm;
-    float* Rs = S.Rs;
-    for (int s = tid; s < p.ns; s += kCT) {
-      hm[s] = __ldcg(recb + (size_t)s * p.rec_floats);
-      Rs[s] = __ldcg(recb + (size_t)s * p.rec_floats + 1);
+    for (int q = lane; q < p.ns; q += 32) {
+      Hm[q] = __ldcg(recb + (size_t)q * p.rec_floats);
+      Rs[q] = __ldcg(recb + (size_t)q * p.rec_floats + 1);
     }
-    cbar();
-    if (tid == 0) {
+    __syncwarp();
+    if (lane == 0) {
       float M = kNegInf;
-      for (int s = 0; s < p.ns; ++s) M = fmaxf(M, hm[s]);
+      for (int q = 0; q < p.ns; ++q) M = fmaxf(M, Hm[q]);
       if (!(M > kNegInf) || M != M) {
         atomicOr(p.status, MDS_ST_NONFINITE);
         M = 0.f;
       }
       const float c = D.P.row[0].c;
       float Z = 0.f;
-      for (int s = 0; s < p.ns; ++s)
-        if (hm[s] > kNegInf) Z = __fadd_rn(Z, __fmul_rn(Rs[s], ref_shift(hm[s], M, c)));
+      for (int q = 0; q < p.ns; ++q)
+        if (Hm[q] > kNegInf) Z = __fadd_rn(Z, __fmul_rn(Rs[q], ref_shift(Hm[q], M, c)));
       D.P.row[0].M = M;
       finish_row(0, Z);
     }
-    cbar();
+    __syncwarp();
     const float M = D.P.row[0].M, c = D.P.row[0].c, iz = D.P.row[0].invZ;
-    for (int s = tid; s < p.ns; s += kCT)
-      Rs[s] = (hm[s] > kNegInf) ? __fmul_rn(__fmul_rn(Rs[s], ref_shift(hm[s], M, c)), iz) : 0.f;
-    cbar();
-    if (tid == 0) {
-      float Q = 0.f;
-      for (int s = 0; s < p.ns; ++s) Q = __fadd_rn(Q, Rs[s]);
-      D.rtot = Q;
-    }
-    cbar();
-    const float Q = D.rtot;
-    const int Z = search(D.P, Rs, __fmul_rn(draw_uniform(p.seed, b, p.L, kDrawBonus), Q), scratch);
-    if (tid == 0) {
+    for (int q = lane; q < p.ns; q += 32)
+      Rs[q] = (Hm[q] > kNegInf) ? __fmul_rn(__fmul_rn(Rs[q], ref_shift(Hm[q], M, c)), iz) : 0.f;
+    __syncwarp();
+    float Q = 0.f;
+    if (lane == 0)
+      for (int q = 0; q < p.ns; ++q) Q = __fadd_rn(Q, Rs[q]);
+    Q = __shfl_sync(FULLM, Q, 0);
+    const int Z = search(D.P, __fmul_rn(draw_uniform(p.seed, b, p.L, kDrawBonus), Q));
+    if (lane == 0) {
       __stcg(p.out_tokens + (size_t)b * (p.L + 1) + p.L, Z);
       if (p.out_diag) {
         float* dg = p.out_diag + ((size_t)b * (p.L + 1) + p.L) * 4;
@@ -2204,14 +2297,12 @@ struct Eng {
     }
     finish(b, p.L);
   }
-
   // -------------------------------------------------------------- truncated alphabet
   // Warp-wide inverse CDF over one weight per lane (lane order = token-id
   // order of the list): the smallest lane whose running sum exceeds
   // u * total, the last lane with positive weight if rounding leaves none,
   // -1 if the total is not positive.
-  __device__ __forceinline__ static int lane_cdf(float w, float u01, float* total) {
-    const int lane = threadIdx.x & 31;
+  __device__ __forceinline__ int lane_cdf(float w, float u01, float* total) const {
     float c = w;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
@@ -2237,10 +2328,8 @@ struct Eng {
   // logits there), then Algorithm 1 against q~.  Y' is kept with probability
   // p_a, else a replace pass draws from the tokens outside Omega_0 by q.
   __device__ void wis0_decide(int b) {
-    DState& D = S.D;
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int j = D.P.j;
-    if (warp == 0) {
+    {
       const int n = D.n;
       const bool have = lane < n;
       const int id = have ? D.cm_id[lane] : 0;
@@ -2394,44 +2483,91 @@ struct Eng {
         }
       }
     }
-    cbar();
+    __syncwarp();
     if (D.tok)
       walk(b, D.W.Yp, D.W.R, D.W.qY, D.W.pIY, D.W.Ydiag);
     else
       push(b, kReplace);
   }
 
-  __device__ void decide(const FDesc& Dd, char* scratch) {
-    DState& D = S.D;
-    const int b = Dd.b;
-    const int kind = Dd.P.kind;
-    if (!(kind == kStats && Dd.P.j == 0)) {
+  // -------------------------------------------------------------- one decision
+  // Request fields: the sequence, the kind, depth, row count and list flag of
+  // the pass that just completed.
+  __device__ void decide(int b, int kind, int j, int R, bool list) {
+    if (!(kind == kStats && j == 0)) {
       const FSeq* g = &reinterpret_cast<const FSeq*>(p.seq)[b];
-      copy_in(&D.P, &g->P, (int)sizeof(FPass), threadIdx.x, kCT);
-      copy_in(&D.W, &g->W, (int)sizeof(FWalk), threadIdx.x, kCT);
-      cbar();
+      copy_in(&D.P, &g->P, (int)sizeof(FPass), lane, 32);
+      copy_in(&D.W, &g->W, (int)sizeof(FWalk), lane, 32);
     }
-    if (threadIdx.x == 0) D.xl_ok = 0;
-    cbar();
+    if (lane == 0) D.xl_ok = 0;
+    __syncwarp();
     PT_T0(t_dec);
-    PT_CNT(kPhDecisions);
+    PT_CNTW(kPhDecisions);
     switch (kind) {
-      case kStats: decide_stats(Dd, b, scratch); break;
-      case kResid: decide_resid(b, scratch); break;
-      case kReplace: decide_replace(b, scratch); break;
-      case kFull: decide_full(Dd, b); break;
-      case kBonus: decide_bonus(Dd, b, scratch); break;
+      case kStats: decide_stats(b, j, R, list); break;
+      case kResid: decide_resid(b); break;
+      case kReplace: decide_replace(b); break;
+      case kFull: decide_full(b); break;
+      case kBonus: decide_bonus(b); break;
       default: break;
     }
-    cbar();
-    PT_ADD(kind == kStats ? kPhDecStats
-                          : (kind == kFull ? kPhDecFull : (kind == kBonus ? kPhDecBonus : kPhDecResid)),
-           t_dec);
+    __syncwarp();
+    PT_ADDW(kind == kStats ? kPhDecStats
+                           : (kind == kFull ? kPhDecFull : (kind == kBonus ? kPhDecBonus : kPhDecResid)),
+            t_dec);
+  }
+
+  // The decision warp's loop: take request numbers from the decision ring,
+  // wait for each request's publication, decide.  Leaves when every sequence
+  // is finished (or on an abort).
+  __device__ __noinline__ void loop() {
+    for (;;) {
+      int have = 0;
+      unsigned pay = 0u;
+      if (lane == 0 && !aborted()) {
+        const unsigned t = atomicAdd(&p.ctl[kCtlDecHead], 1u);
+        const unsigned slot = t % (unsigned)p.dec_cap;
+        const unsigned long long want = tag_of(t);
+        const unsigned long long t0 = now_ns();
+        PT_T0(t_poll);
+        for (int it = 0;; ++it) {
+          if (ld_acquire(&p.dec_tag[slot]) == want) {
+            pay = __ldcg(&p.dec_pay[slot]);
+            st_release(&p.dec_rtag[slot], want);
+            have = 1;
+            break;
+          }
+          if (ld_relaxed(&p.ctl[kCtlDone]) >= (unsigned)p.B || aborted()) break;
+          if ((it & 15) == 15 && now_ns() - t0 > kWaitNs) {
+            set_abort(MDS_ST_TIMEOUT);
+            break;
+          }
+          __nanosleep(it < 16 ? 32 : 256);
+        }
+        PT_ADDW(kPhDecPoll, t_poll);
+      }
+      have = __shfl_sync(FULLM, have, 0);
+      pay = __shfl_sync(FULLM, pay, 0);
+      if (!have) return;
+      const int b = (int)(pay >> 16);
+      const int kind = (int)((pay >> 13) & 7u);
+      const int j = (int)((pay >> 6) & 127u);
+      const int R = (int)((pay >> 1) & 31u);
+      const bool list = (pay & 1u) != 0u;
+      decide(b, kind, j, R, list);
+    }
   }
 };
 
+
+constexpr int kDStateBytes = (int)((sizeof(DState) + 127) / 128 * 128);
+constexpr int kDecPerWarp = kDStateBytes + (kDecScratch + 127) / 128 * 128;
+constexpr int kDynBytes = kNBuf * kBufBytes + 4 * kCandCap * 4;
+constexpr int kDecWarps = (kDynBytes / kDecPerWarp < kBlock / 32) ? kDynBytes / kDecPerWarp : kBlock / 32;
+static_assert(kDecWarps >= 2, "decision warps per decision CTA");
+
 template <int DT>
-__global__ void __launch_bounds__(kBlock, 2) flow_kernel(const __grid_constant__ Params p) {
+__global__ void __launch_bounds__(kBlock, kCtasPerSm) flow_kernel(const __grid_constant__ Params p) {
   extern __shared__ __align__(128) char dsm[];
   __shared__ FShared S;
   Eng<DT> e{p, S};
@@ -2454,12 +2590,34 @@ __global__ void __launch_bounds__(kBlock, 2) flow_kernel(const __grid_constant__
 #endif
     mbar_init_fence();
   }
+  // Roles: the CTAs on the first dec_sms SMs run decisions (kDecWarps
+  // decision warps each, the rest of their warps idle), every other CTA
+  // streams slices (one scheduler warp, eight compute warps).  Decisions are
+  // serial code: on their own SMs they do not wait behind the streaming warps.
+  __shared__ int role;
+  if (threadIdx.x == 0) {
+    unsigned smid;
+    asm volatile("mov.u32 %0, %%smid;" : "=r"(smid));
+    role = (smid < (unsigned)p.dec_sms) ? 1 : 0;
+  }
   __syncthreads();
   PT_T0(t_kernel);
-  if (threadIdx.x >= kCT)
+  if (role) {
+    const int w = threadIdx.x >> 5;
+    if (w < kDecWarps) {
+      char* base = dsm + (size_t)w * kDecPerWarp;
+      char* scr = base + kDStateBytes;
+      Dec<DT> d{p, S, *reinterpret_cast<DState*>(base), scr, reinterpret_cast<float*>(scr + kDecStage),
+                reinterpret_cast<float*>(scr + kDecStage) + kMaxSlices,
+                reinterpret_cast<uint32_t*>(reinterpret_cast<float*>(scr + kDecStage) + 2 * kMaxSlices),
+                (int)(threadIdx.x & 31)};
+      d.loop();
+    }
+  } else if (threadIdx.x >= kCT) {
     e.scheduler();
-  else
+  } else {
     e.compute();
+  }
   __syncthreads();
   // copies issued but never consumed (only after an abort): wait for them
   if (threadIdx.x == kCT) {
@@ -2480,6 +2638,8 @@ __global__ void __launch_bounds__(kBlock, 2) flow_kernel(const __grid_constant__
         for (int b = 0; b < p.B; ++b) p.cnt[b] = 0u;
       p.ctl[kCtlHead] = 0u;
       p.ctl[kCtlTail] = 0u;
+      p.ctl[kCtlDecHead] = 0u;
+      p.ctl[kCtlDecTail] = 0u;
       p.ctl[kCtlDone] = 0u;
       p.ctl[kCtlAbort] = 0u;
       __threadfence();
@@ -2488,7 +2648,7 @@ __global__ void __launch_bounds__(kBlock, 2) flow_kernel(const __grid_constant__
   }
 }
 
-size_t dyn_smem() { return (size_t)kNBuf * kBufBytes + 4 * (size_t)kCandCap * 4; }
+size_t dyn_smem() { return (size_t)kDynBytes; }
 
 }  // namespace
 
@@ -2497,15 +2657,18 @@ size_t seq_bytes() { return sizeof(FSeq); }
 namespace {
 size_t up256(size_t x) { return (x + 255) / 256 * 256; }
 struct Layout {
-  size_t ctl, tag, pay, cnt, seq, rec;
-  size_t cap;
+  size_t ctl, tag, pay, dtag, dpay, cnt, seq, rec;
+  size_t cap, dcap;
 };
 Layout layout(const Params& p, int nseq, int grid) {
   Layout L;
   L.cap = (size_t)nseq * p.ns + (size_t)grid + 64;
+  L.dcap = (size_t)nseq + (size_t)grid * kDecWarps + 64;   // one request per sequence, plus the claims
   L.ctl = 256;
   L.tag = up256(L.cap * 8);
   L.pay = up256(L.cap * 4);
+  L.dtag = up256(L.dcap * 8);
+  L.dpay = up256(L.dcap * 4);
   L.cnt = up256((size_t)nseq * 4);
   L.seq = up256((size_t)nseq * sizeof(FSeq));
   L.rec = up256((size_t)nseq * p.ns * p.rec_floats * 4);
@@ -2515,12 +2678,12 @@ Layout layout(const Params& p, int nseq, int grid) {
 
 size_t workspace_bytes(const Params& p, int nseq, int grid) {
   const Layout L = layout(p, nseq, grid);
-  return L.ctl + 2 * L.tag + L.pay + L.cnt + L.seq + L.rec;
+  return L.ctl + 2 * L.tag + L.pay + 2 * L.dtag + L.dpay + L.cnt + L.seq + L.rec;
 }
 
 size_t clear_bytes(const Params& p, int nseq, int grid) {
   const Layout L = layout(p, nseq, grid);
-  return L.ctl + 2 * L.tag + L.pay + L.cnt;
+  return L.ctl + 2 * L.tag + L.pay + 2 * L.dtag + L.dpay + L.cnt;
 }
 
 void carve_workspace(Params& p, char* w, int nseq, int grid) {
@@ -2533,12 +2696,34 @@ void carve_workspace(Params& p, char* w, int nseq, int grid) {
   w += L.tag;
   p.ring_pay = reinterpret_cast<unsigned*>(w);
   w += L.pay;
+  p.dec_tag = reinterpret_cast<unsigned long long*>(w);
+  w += L.dtag;
+  p.dec_rtag = reinterpret_cast<unsigned long long*>(w);
+  w += L.dtag;
+  p.dec_pay = reinterpret_cast<unsigned*>(w);
+  w += L.dpay;
   p.cnt = reinterpret_cast<unsigned*>(w);
   w += L.cnt;
   p.seq = w;
   w += L.seq;
   p.rec = reinterpret_cast<float*>(w);
   p.ring_cap = (int)L.cap;
+  p.dec_cap = (int)L.dcap;
+}
+
+// SMs whose CTAs run the decisions: about a tenth of the grid's SMs, at
+// least one and never all of them.  The environment variable MDS_DEC_SMS
+// overrides the count (read once per process), for tuning.
+int decision_sms(int grid) {
+  static const int env = [] {
+    const char* e = getenv("MDS_DEC_SMS");
+    return e ? atoi(e) : 0;
+  }();
+  const int sms = grid / kCtasPerSm;
+  int d = env > 0 ? env : (sms + 5) / 10;
+  if (d < 1) d = 1;
+  if (d > sms - 1) d = sms - 1;
+  return d;
 }
 
 bool plan_geometry(Params& p, int grid) {
@@ -2594,10 +2779,11 @@ bool plan_geometry(Params& p, int grid) {
   if (rf < 4 + 4 * kTopF) rf = 4 + 4 * kTopF;
   p.rec_floats = (rf + 3) & ~3;
   p.hdr_floats = kHdr;
-  // the decision stages one stats pass's records in one slice buffer
+  // a decision stages one stats pass's records in its warp's staging area
   const size_t stage = (size_t)(2 * nstream * ns + 2 * ns + ns * p.lns * (1 + lrows)) * 4;
-  if (stage > (size_t)kBufBytes) return false;
-  return true;
+  if (stage > (size_t)kDecStage) return false;
+  p.dec_sms = decision_sms(grid);
+  return p.dec_sms > 0;
 }
 
 int grid_size(int device) {

@@ -23,7 +23,8 @@ constexpr int kSliceQuantum = 256;     // T is a multiple of this many tokens
 
 // Control words (ctl[]): task head and tail, finished sequences, abort flag,
 // CTAs that left the kernel.  All zero between launches.
-enum { kCtlHead = 0, kCtlTail = 1, kCtlDone = 2, kCtlAbort = 3, kCtlExit = 4, kCtlWords = 16 };
+enum { kCtlHead = 0, kCtlTail = 1, kCtlDone = 2, kCtlAbort = 3, kCtlExit = 4, kCtlDecHead = 5, kCtlDecTail = 6,
+       kCtlWords = 16 };
 
 struct Params {
   const char* target;                  // [B][K][L+1][V]
@@ -38,6 +39,9 @@ struct Params {
   unsigned long long* ring_tag;        // [ring_cap] published task tags
   unsigned long long* ring_rtag;       // [ring_cap] tags of tasks taken
   unsigned* ring_pay;                  // [ring_cap] (sequence << 16) | slice
+  unsigned long long* dec_tag;         // [dec_cap] published decision requests
+  unsigned long long* dec_rtag;        // [dec_cap] tags of requests taken
+  unsigned* dec_pay;                   // [dec_cap] the requests
   unsigned* cnt;                       // [B] slices of the current pass completed
   char* seq;                           // [B] per-sequence pass and walk state
   float* rec;                          // [B][ns][rec_floats] slice records
@@ -53,6 +57,8 @@ struct Params {
   int rec_floats;                      // record stride per slice
   int hdr_floats;                      // start of a record's list entries
   int ring_cap;
+  int dec_cap;
+  int dec_sms;                         // SMs (ids 0..dec_sms-1) whose CTAs run the decisions
   int bulk;                            // rows are fetched with bulk copies (device memory, 16-byte aligned rows)
   int aligned;                         // rows start 16-byte aligned and V * esize is a multiple of 16
   int n_models;

@@ -471,6 +471,7 @@ struct Kernel {
   int xbuf;
   int clbuf;           // which copy of the CTA list the next candidate pass publishes
   uint32_t wphase;     // parity of each stage of this warp's ring
+  int bail;            // this warp's ring gave up on a copy: it streams nothing more
 
   __device__ float prob_row(int r, int x) const {
     return prob_of(E::global(S.gptr[r], x), S.M[r], S.c[r], S.invZ[r]);
@@ -525,7 +526,7 @@ struct Kernel {
     }
     const int nchunk = (Uv + su - 1) / su;
     const int nk = (nchunk - warp + kWarps - 1) / kWarps;   // this warp's chunks: warp, warp + kWarps, ...
-    if (nk <= 0) return;
+    if (nk <= 0 || bail) return;
     if (lane == 0) {
       fence_proxy_async();
       for (int k = 0; k < nk && k < kWStages; ++k) issue_stage(k, mask, su);
@@ -535,11 +536,29 @@ struct Kernel {
       const int stage = k % kWStages;
       const char* base = ring + (size_t)(warp * kWStages + stage) * (p.ring_bytes / kWarps / kWStages);
       long long spins = 0;
+      bool ok = true;
       while (!mbar_try_wait(&S.wbar[warp][stage], (wphase >> stage) & 1u)) {
         if (++spins > kWaitLimit) {
-          if (lane == 0) atomicOr(p.status, MDS_ST_TIMEOUT);
+          ok = false;
           break;
         }
+      }
+      if (!__all_sync(0xffffffffu, ok)) {
+        // A copy never landed: flag the launch (every sequence still to be
+        // written is then marked -1), issue nothing more from this warp and
+        // give the copies already issued one more bounded wait before the
+        // warp's ring is left for good.
+        if (lane == 0) {
+          atomicOr(p.status, MDS_ST_TIMEOUT);
+          for (int kk = k; kk < nk && kk < k + kWStages; ++kk) {
+            const int st = kk % kWStages;
+            for (long long w = 0; w <= kWaitLimit && !mbar_try_wait(&S.wbar[warp][st], (wphase >> st) & 1u); ++w) {
+            }
+          }
+        }
+        __syncwarp();
+        bail = 1;
+        return;
       }
       wphase ^= 1u << stage;
       const int cu0 = (warp + k * kWarps) * su, cu1 = min(cu0 + su, Uv);
@@ -2648,9 +2667,20 @@ struct Kernel {
       valid = nvld;
     }
     if (rank == 0 && tid == 0) {
-      p.out_accept[b] = acc_len;
-      for (int j = acc_len + 1; j <= L; ++j) p.out_tokens[(size_t)b * (L + 1) + j] = -1;
+      if (*reinterpret_cast<volatile unsigned*>(p.status) & MDS_ST_TIMEOUT) {
+        abandon(b);   // a ring wait gave up during the launch: this walk is not trusted
+      } else {
+        p.out_accept[b] = acc_len;
+        for (int j = acc_len + 1; j <= L; ++j) p.out_tokens[(size_t)b * (L + 1) + j] = -1;
+      }
     }
+  }
+
+  // Outputs of a sequence the launch gives up on: accept length -1, every
+  // token -1 (the diagnostics are left as they are).
+  __device__ void abandon(int b) const {
+    p.out_accept[b] = -1;
+    for (int j = 0; j <= p.L; ++j) p.out_tokens[(size_t)b * (p.L + 1) + j] = -1;
   }
 
   // residual weight max(0, q - p_I) for WIS (generic gamma law + special table)
@@ -2857,6 +2887,7 @@ __global__ void __launch_bounds__(kThreads, SCHEME == MDS_IS ? 1 : 2) verify_ker
   k.xbuf = 0;
   k.clbuf = 0;
   k.wphase = 0u;
+  k.bail = 0;
   if (threadIdx.x == 0) {
     for (int w = 0; w < kWarps; ++w)
       for (int i = 0; i < kWStages; ++i) mbar_init(&S.wbar[w][i]);
@@ -2868,7 +2899,11 @@ __global__ void __launch_bounds__(kThreads, SCHEME == MDS_IS ? 1 : 2) verify_ker
   if (p.cn > 1) cluster_sync_all();
   for (;;) {
     if (k.rank == 0 && threadIdx.x == 0) {
-      const int b = (int)(atomicAdd(p.queue, 1u) - p.ticket0);
+      int b = (int)(atomicAdd(p.queue, 1u) - p.ticket0);
+      if (b < p.B && (*reinterpret_cast<volatile unsigned*>(p.status) & MDS_ST_TIMEOUT)) {
+        k.abandon(b);   // after a ring wait gave up, the remaining sequences are only marked
+        b = -1;
+      }
       if (p.cn > 1) {
         for (int q = 0; q < p.cn; ++q) st_dsmem(&S.next_b, (uint32_t)q, b);
       } else {
@@ -2882,6 +2917,11 @@ __global__ void __launch_bounds__(kThreads, SCHEME == MDS_IS ? 1 : 2) verify_ker
     const int b = *(volatile int*)&S.next_b;
     __syncthreads();
     if (b >= p.B) break;
+    if (b < 0) {
+      // every CTA of the cluster has read S.next_b before rank 0 writes it again
+      if (p.cn > 1) cluster_sync_all();
+      continue;
+    }
     k.run_sequence(b);
   }
 }

@@ -2,7 +2,7 @@
 
 Some callers cannot call cudaMalloc: code running where device memory is
 fixed once at start-up (a serving loop under an allocator that forbids growth
-after warm-up), or code that must not create a context at all.  For them the
+after warm-up), and so cannot create an mds_ctx (no cudaMalloc).  For them the
 library offers a context-free variant whose scratch lives in a static device
 array.  This test calls it through the C ABI twice in a row and checks that
 both calls reproduce the context-based entry point's outputs (the same kernel
