@@ -1172,6 +1172,15 @@ struct Eng {
 constexpr int kDecStage = 6656;        // bytes of a decision's staged records
 constexpr int kDecScratch = kDecStage + 2 * kMaxSlices * 4 + 64 * 4;   // + slice masses, maxima, bitmap
 
+// Each kind of decision out of line (its own register allocation); each
+// rebuilds the warp's view of its shared state.
+template <int DT> __device__ __noinline__ void dec_stats_nl(int b, int j, int R, bool list);
+template <int DT> __device__ __noinline__ void dec_resid_nl(int b);
+template <int DT> __device__ __noinline__ void dec_replace_nl(int b);
+template <int DT> __device__ __noinline__ void dec_full_nl(int b);
+template <int DT> __device__ __noinline__ void dec_bonus_nl(int b);
+template <int DT> __device__ __noinline__ void dec_wis0_nl(int b);
+
 template <int DT>
 struct Dec {
   using E = Elt<DT>;
@@ -1815,7 +1824,7 @@ struct Dec {
     combine_stats(R, list);
     PT_ADDW(kPhDecCombine, t_comb);
     if (p.scheme == MDS_WIS0) {
-      wis0_decide(b);
+      dec_wis0_nl<DT>(b);
       return;
     }
     if (p.scheme == MDS_SINGLE || D.nv == 1) {
@@ -2504,11 +2513,11 @@ struct Dec {
     PT_T0(t_dec);
     PT_CNTW(kPhDecisions);
     switch (kind) {
-      case kStats: decide_stats(b, j, R, list); break;
-      case kResid: decide_resid(b); break;
-      case kReplace: decide_replace(b); break;
-      case kFull: decide_full(b); break;
-      case kBonus: decide_bonus(b); break;
+      case kStats: dec_stats_nl<DT>(b, j, R, list); break;
+      case kResid: dec_resid_nl<DT>(b); break;
+      case kReplace: dec_replace_nl<DT>(b); break;
+      case kFull: dec_full_nl<DT>(b); break;
+      case kBonus: dec_bonus_nl<DT>(b); break;
       default: break;
     }
     __syncwarp();
@@ -2520,7 +2529,7 @@ struct Dec {
   // The decision warp's loop: take request numbers from the decision ring,
   // wait for each request's publication, decide.  Leaves when every sequence
   // is finished (or on an abort).
-  __device__ __noinline__ void loop() {
+  __device__ __forceinline__ void loop() {
     for (;;) {
       int have = 0;
       unsigned pay = 0u;
@@ -2560,16 +2569,46 @@ struct Dec {
 };
 
 
+// Shared memory of a CTA, at file scope so that the decision code (out of
+// line) addresses it as shared memory: the dynamic buffers, the CTA state and,
+// in decision CTAs, a copy of the launch parameters.
+extern __shared__ __align__(128) char g_dsm[];
+__shared__ FShared g_S;
+__shared__ Params g_dp;
+
 constexpr int kDStateBytes = (int)((sizeof(DState) + 127) / 128 * 128);
 constexpr int kDecPerWarp = kDStateBytes + (kDecScratch + 127) / 128 * 128;
 constexpr int kDynBytes = kNBuf * kBufBytes + 4 * kCandCap * 4;
 constexpr int kDecWarps = (kDynBytes / kDecPerWarp < kBlock / 32) ? kDynBytes / kDecPerWarp : kBlock / 32;
 static_assert(kDecWarps >= 2, "decision warps per decision CTA");
 
+// The calling warp's decision view: its state and scratch in the CTA's
+// dynamic shared memory, the parameters from the CTA's shared copy.
+template <int DT>
+__device__ __forceinline__ Dec<DT> dec_view() {
+  char* base = g_dsm + (size_t)(threadIdx.x >> 5) * kDecPerWarp;
+  char* scr = base + kDStateBytes;
+  float* rs = reinterpret_cast<float*>(scr + kDecStage);
+  return Dec<DT>{g_dp, g_S, *reinterpret_cast<DState*>(base), scr, rs, rs + kMaxSlices,
+                 reinterpret_cast<uint32_t*>(rs + 2 * kMaxSlices), (int)(threadIdx.x & 31)};
+}
+template <int DT> __device__ __noinline__ void dec_stats_nl(int b, int j, int R, bool list) {
+  dec_view<DT>().decide_stats(b, j, R, list);
+}
+template <int DT> __device__ __noinline__ void dec_resid_nl(int b) { dec_view<DT>().decide_resid(b); }
+template <int DT> __device__ __noinline__ void dec_replace_nl(int b) { dec_view<DT>().decide_replace(b); }
+template <int DT> __device__ __noinline__ void dec_full_nl(int b) { dec_view<DT>().decide_full(b); }
+template <int DT> __device__ __noinline__ void dec_bonus_nl(int b) { dec_view<DT>().decide_bonus(b); }
+template <int DT> __device__ __noinline__ void dec_wis0_nl(int b) { dec_view<DT>().wis0_decide(b); }
+
+// A decision warp's loop, out of line with the whole register budget.
+template <int DT>
+__device__ __noinline__ void decision_warp() { dec_view<DT>().loop(); }
+
 template <int DT>
 __global__ void __launch_bounds__(kBlock, kCtasPerSm) flow_kernel(const __grid_constant__ Params p) {
-  extern __shared__ __align__(128) char dsm[];
-  __shared__ FShared S;
+  char* dsm = g_dsm;
+  FShared& S = g_S;
   Eng<DT> e{p, S};
   e.bufs = dsm;
   char* c = dsm + (size_t)kNBuf * kBufBytes;
@@ -2603,16 +2642,13 @@ __global__ void __launch_bounds__(kBlock, kCtasPerSm) flow_kernel(const __grid_c
   __syncthreads();
   PT_T0(t_kernel);
   if (role) {
+    // the parameters into shared memory, where the decision code reads them
+    static_assert(sizeof(Params) % 4 == 0, "parameter copy in words");
+    for (int i = threadIdx.x; i < (int)(sizeof(Params) / 4); i += kBlock)
+      reinterpret_cast<int*>(&g_dp)[i] = reinterpret_cast<const int*>(&p)[i];
+    __syncthreads();
     const int w = threadIdx.x >> 5;
-    if (w < kDecWarps) {
-      char* base = dsm + (size_t)w * kDecPerWarp;
-      char* scr = base + kDStateBytes;
-      Dec<DT> d{p, S, *reinterpret_cast<DState*>(base), scr, reinterpret_cast<float*>(scr + kDecStage),
-                reinterpret_cast<float*>(scr + kDecStage) + kMaxSlices,
-                reinterpret_cast<uint32_t*>(reinterpret_cast<float*>(scr + kDecStage) + 2 * kMaxSlices),
-                (int)(threadIdx.x & 31)};
-      d.loop();
-    }
+    if (w < kDecWarps) decision_warp<DT>();
   } else if (threadIdx.x >= kCT) {
     e.scheduler();
   } else {
