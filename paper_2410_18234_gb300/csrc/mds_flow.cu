@@ -53,6 +53,7 @@ constexpr int kCandCap = 512;          // candidate tokens one slice may set asi
 constexpr int kListMax = 64;           // candidate list length at most
 constexpr int kHdr = 2 * kMaxRows + 2; // record: (max, sum) per row, tau, list length
 constexpr int kTopF = 8;               // per-thread candidates of a full stage (>= MDS_MAX_S)
+constexpr int kMaxEntries = 512;       // slices x slice list length, at most
 constexpr unsigned long long kWaitNs = 2000000000ull;   // 2 s bound on every wait
 constexpr unsigned FULLM = 0xffffffffu;
 static_assert(kHdr % 4 == 0, "record header keeps 16-byte alignment");
@@ -85,7 +86,7 @@ enum : int {
   kPhSchedEmpty,        // scheduler waiting for a free buffer
   kPhDecPoll,           // decision warps waiting for a request
   kPhDecPlan,           // decisions: planning a pass (rows, tokens, cached logits)
-  kPhDecLoad,           // decisions: staging a stats pass's records
+  kPhDecLoad,           // decisions: staging the state, inputs and records
   kPhDecSelect,         // decisions: WIS stage selection and masses (list)
   kPhDecAccept,         // decisions: the accept step (with its push or walk)
   kPhDecWalk,           // decisions: the walk to the next depth
@@ -186,10 +187,17 @@ struct DState {                // the decision's working state (shared memory)
   // truncated alphabet
   int k_lane[MDS_MAX_K], k_row[MDS_MAX_K];
   int o0_n, o0_all, o0_Yp;
+  // inputs of the sequence staged by the decision: draft tokens at the
+  // depth (tk0) and the next depth (tk1), temperatures (target, drafts)
+  int tk0[MDS_MAX_K], tk1[MDS_MAX_K];
+  float tmp[MDS_MAX_K + 1];
+  int xl_wait;                 // the row logits at the draft tokens are still in flight
   float o0_cut, o0_pa, o0_R;
   float rtot;
   unsigned tbase;
 };
+static_assert(offsetof(DState, W) == offsetof(DState, P) + sizeof(FPass) && offsetof(FSeq, W) == sizeof(FPass),
+              "a sequence's state copies into the decision state in one piece");
 
 struct FShared {
   uint64_t full[kNBuf], empty[kNBuf];
@@ -250,6 +258,17 @@ __device__ __forceinline__ void copy_out(void* dst, const void* src, int bytes, 
   int4* d = reinterpret_cast<int4*>(dst);
   for (int i = t; i < bytes / 16; i += nt) __stcg(d + i, s[i]);
 }
+
+// Asynchronous copies global -> shared (the issuing thread's own copies
+// complete at cpa_wait): 16 bytes through L2 only (data other SMs write
+// during the launch), 4 bytes cached (inputs only).
+__device__ __forceinline__ void cpa16(void* dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cpa4(void* dst, const void* src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cpa_wait() { asm volatile("cp.async.wait_all;" ::: "memory"); }
 
 // ------------------------------------------------------------------ phase timers
 // Built with -DMDS_PHASE_TIMERS, every CTA accumulates SM cycles per phase
@@ -899,18 +918,41 @@ struct Eng {
     }
   }
 
+  // The slice's mass (record[0]) and its 32 run masses (record[4 + q]): run q
+  // is units [q * upl, (q + 1) * upl), upl = ceil(units / 32), the runs the
+  // decision's search walks.  A unit's mass adds its tokens in order, a run's
+  // its chunks of 32 units (each a butterfly over the units), the slice's
+  // its runs in order.
   __device__ void resid_task(const FPass& P, const char* b, int tok0, int n, float* rec) {
     if (P.kind == kResid && P.nspec > 0) build_bitmap(P, tok0, n);
     const int U = (n + VE - 1) / VE;
-    float part = 0.f;
-    for (int u = threadIdx.x; u < U; u += kCT) {
-      float w[VE];
-      weights(P, b, u, tok0, w);
+    const int upl = (U + 31) / 32;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    for (int q = warp; q < 32; q += kCW) {
+      const int u0 = min(U, q * upl), u1 = min(U, u0 + upl);
+      float run = 0.f;
+      for (int c = u0; c < u1; c += 32) {
+        const int u = c + lane;
+        float us = 0.f;
+        if (u < u1) {
+          float w[VE];
+          weights(P, b, u, tok0, w);
 #pragma unroll
-      for (int e = 0; e < VE; ++e) part = __fadd_rn(part, w[e]);
+          for (int e = 0; e < VE; ++e) us = __fadd_rn(us, w[e]);
+        }
+        run = __fadd_rn(run, warp_sum(us));
+      }
+      if (lane == 0) {
+        S.red[q] = run;
+        __stcg(rec + 4 + q, run);
+      }
     }
-    part = block_sum(part, S.red);
-    if (threadIdx.x == 0) __stcg(rec, part);
+    cbar();
+    if (threadIdx.x == 0) {
+      float tot = 0.f;
+      for (int q = 0; q < 32; ++q) tot = __fadd_rn(tot, S.red[q]);
+      __stcg(rec, tot);
+    }
   }
 
   // -------------------------------------------------------------- full-vocabulary stage task
@@ -1169,7 +1211,7 @@ struct Eng {
 // Single-warp code throughout (lane 0 for the serial steps); its state and
 // scratch are this warp's own shared memory.
 
-constexpr int kDecStage = 6656;        // bytes of a decision's staged records
+constexpr int kDecStage = 8192;        // bytes of a decision's staged records
 constexpr int kDecScratch = kDecStage + 2 * kMaxSlices * 4 + 64 * 4;   // + slice masses, maxima, bitmap
 
 // Each kind of decision out of line (its own register allocation); each
@@ -1180,6 +1222,8 @@ template <int DT> __device__ __noinline__ void dec_replace_nl(int b);
 template <int DT> __device__ __noinline__ void dec_full_nl(int b);
 template <int DT> __device__ __noinline__ void dec_bonus_nl(int b);
 template <int DT> __device__ __noinline__ void dec_wis0_nl(int b);
+__device__ __noinline__ int lp_solve5(int s, float A2, float B2, int A, int Btok, float u);
+__device__ __noinline__ int lp_solve8(int s, float A2, float B2, int A, int Btok, float u);
 
 template <int DT>
 struct Dec {
@@ -1311,10 +1355,12 @@ struct Dec {
     }
   }
 
-  // Warp-parallel plan_rows (one lane per branch): the same rows in the same
-  // order, the valid branches, their tokens and rows; then every row's logit
-  // at each draft token into the cache.
-  __device__ void plan_warp(int b, int j, unsigned valid, bool bonus, bool set_pass) {
+  // Rows of depth j for the valid branches (the lowest valid branch's target
+  // row, then one row per distinct draft model in branch order), one lane per
+  // branch; the valid branches, their tokens (tk: the staged tokens of depth
+  // j) and rows; with want_xl, every row's logit at each draft token, by
+  // asynchronous copies that xl_sync completes.
+  __device__ void plan_warp(int b, int j, unsigned valid, bool bonus, bool set_pass, bool want_xl, const int* tk) {
     FPass& P = D.P;
     const int K = p.K;
     const bool v = !bonus && lane < K && ((valid >> lane) & 1u);
@@ -1328,7 +1374,7 @@ struct Dec {
     const int row = __shfl_sync(FULLM, myrow, __ffs(same) - 1);
     if (v) {
       const int i = __popc(vm & ((1u << lane) - 1u));
-      int x = p.tokens[((size_t)b * K + lane) * p.L + j];
+      int x = tk[lane];
       if (x < 0 || x >= p.V) {
         atomicOr(p.status, MDS_ST_BADTOKEN);
         x = 0;
@@ -1339,7 +1385,7 @@ struct Dec {
     }
     if (set_pass && first) {
       P.row[myrow].ptr = p.drafts[lane] + (((size_t)b * p.L + j) * (size_t)p.V) * p.esize;
-      float td = p.temps[(size_t)b * (1 + K) + 1 + lane];
+      float td = D.tmp[1 + lane];
       if (!(td > 0.f) || !(td < kPosInf)) {
         atomicOr(p.status, MDS_ST_BADTEMP);
         td = 1.f;
@@ -1354,7 +1400,7 @@ struct Dec {
       if (set_pass) {
         const int kstar = __ffs(valid) - 1;
         P.row[0].ptr = p.target + ((((size_t)b * K + kstar) * (p.L + 1) + j) * (size_t)p.V) * p.esize;
-        float tq = p.temps[(size_t)b * (1 + K)];
+        float tq = D.tmp[0];
         if (!(tq > 0.f) || !(tq < kPosInf)) {
           atomicOr(p.status, MDS_ST_BADTEMP);
           tq = 1.f;
@@ -1388,13 +1434,49 @@ struct Dec {
         }
       }
     }
-    __syncwarp();
-    const int nv = D.nv, nrow = P.nrows;
-    for (int i = lane; i < nv * nrow; i += 32) {
-      const int k = i / nrow, r = i - k * nrow;
-      D.xl[k][r] = E::global(P.row[r].ptr, D.X[k]);
+    if (lane == 0) {
+      D.xl_ok = 0;
+      D.xl_wait = 0;
     }
-    if (lane == 0) D.xl_ok = bonus ? 0 : 1;
+    __syncwarp();
+    if (want_xl && !bonus) {
+      const int nv = D.nv, nrow = P.nrows;
+      for (int i = lane; i < nv * nrow; i += 32) {
+        const int k = i / nrow, r = i - k * nrow;
+        const char* at = P.row[r].ptr + (size_t)D.X[k] * p.esize;
+        if (p.bulk)
+          cpa4(&D.xl[k][r], reinterpret_cast<const char*>(reinterpret_cast<uintptr_t>(at) & ~uintptr_t(3)));
+        else
+          D.xl[k][r] = E::global(P.row[r].ptr, D.X[k]);
+      }
+      if (lane == 0) D.xl_wait = 1;
+      __syncwarp();
+    }
+  }
+
+  // Complete plan_warp's copies of the row logits at the draft tokens (the
+  // 4-byte word holding a 16-bit logit is copied, its half taken here).
+  // Warp-wide; afterwards logit_at answers those points from the cache.
+  __device__ void xl_sync() {
+    if (!D.xl_wait) return;
+    cpa_wait();
+    __syncwarp();
+    if (p.bulk) {
+      const int nv = D.nv, nrow = D.P.nrows;
+      for (int i = lane; i < nv * nrow; i += 32) {
+        const int k = i / nrow, r = i - k * nrow;
+        if constexpr (DT == MDS_BF16) {
+          const uint32_t w = __float_as_uint(D.xl[k][r]);
+          const uintptr_t at = reinterpret_cast<uintptr_t>(D.P.row[r].ptr) + (uintptr_t)D.X[k] * 2u;
+          D.xl[k][r] = __uint_as_float((at & 2u) ? (w & 0xffff0000u) : (w << 16));
+        }
+      }
+    }
+    __syncwarp();
+    if (lane == 0) {
+      D.xl_wait = 0;
+      D.xl_ok = 1;
+    }
     __syncwarp();
   }
 
@@ -1469,12 +1551,12 @@ struct Dec {
       if (nv) {
         D.W.stage = 0;
         D.W.zres = 0;
-        plan_rows(b, j + 1, nv, j + 1 == p.L, &D.P, &D.nv, D.vbr, D.X, D.vrow);
       }
-      D.xl_ok = 0;
     }
     next = __shfl_sync(FULLM, next, 0);
     __syncwarp();
+    // the next depth's pass, planned from the staged tokens of depth j + 1
+    if (next != kNone) plan_warp(b, j + 1, D.W.valid, next == kBonus, true, false, D.tk1);
     if (next == kNone)
       finish(b, j);
     else
@@ -1485,38 +1567,6 @@ struct Dec {
   // -------------------------------------------------------------- stats decision
   // The records of a stats pass into the scratch: per row the slice maxima
   // and sums, and with lists each slice's tau, list length and entries.
-  __device__ void stage_records(int R, bool list, int b) const {
-    const int ns = p.ns, LN = p.lns;
-    const float* recb = p.rec + (size_t)b * ns * p.rec_floats;
-    float* hm = reinterpret_cast<float*>(scr);
-    float* hs = hm + R * ns;
-    float* htau = hs + R * ns;
-    int* hnl = reinterpret_cast<int*>(htau + ns);
-    int* eid = hnl + ns;
-    float* el = reinterpret_cast<float*>(eid + ns * LN);
-    for (int i = lane; i < R * ns; i += 32) {
-      const int r = i / ns, s = i - r * ns;
-      hm[i] = __ldcg(recb + (size_t)s * p.rec_floats + 2 * r);
-      hs[i] = __ldcg(recb + (size_t)s * p.rec_floats + 2 * r + 1);
-    }
-    if (list) {
-      for (int s = lane; s < ns; s += 32) {
-        htau[s] = __ldcg(recb + (size_t)s * p.rec_floats + 2 * kMaxRows);
-        hnl[s] = __ldcg(reinterpret_cast<const int*>(recb + (size_t)s * p.rec_floats) + 2 * kMaxRows + 1);
-      }
-      for (int i = lane; i < ns * LN * (1 + R); i += 32) {
-        const int f = i / (ns * LN), rest = i - f * ns * LN;
-        const int s = rest / LN, q = rest - s * LN;
-        const float v = __ldcg(recb + (size_t)s * p.rec_floats + kHdr + f * LN + q);
-        if (f == 0)
-          eid[rest] = __float_as_int(v);
-        else
-          el[(f - 1) * ns * LN + rest] = v;
-      }
-    }
-    __syncwarp();
-  }
-
   __device__ void finish_row(int r, float Z) {
     if (!(Z > 0.f) || !(Z < kPosInf) || Z != Z) {
       atomicOr(p.status, MDS_ST_NONFINITE);
@@ -1525,100 +1575,170 @@ struct Dec {
     D.P.row[r].invZ = __frcp_rn(Z);
   }
 
-  // Combine the staged records of a stats pass: every row's M and 1/Z, and
-  // with candidate lists the sequence's list (the first LF of the slices'
-  // lists by (logit, id)), its complement masses and tau.
+  // Combine the staged records of a stats pass (scr: [ns][rec_floats]):
+  // every row's M and 1/Z, and with candidate lists the sequence's list (the
+  // first LF of the slices' lists by (logit, id)), its complement masses and
+  // tau.  Sums over slices and entries run in fixed orders (lane-strided
+  // partial sums, then a butterfly).
   __device__ void combine_stats(int R, bool list) {
-    const int ns = p.ns, LN = p.lns, LF = p.ln;   // a slice's list, the sequence's
-    float* hm = reinterpret_cast<float*>(scr);        // [R][ns] slice maxima
-    float* hs = hm + R * ns;                          // [R][ns] slice sums
-    float* htau = hs + R * ns;                        // [ns]
-    int* hnl = reinterpret_cast<int*>(htau + ns);     // [ns]
-    int* eid = hnl + ns;                              // [ns][LN]
-    float* el = reinterpret_cast<float*>(eid + ns * LN);  // [R][ns][LN]
+    const int ns = p.ns, LN = p.lns, LF = p.ln, rf = p.rec_floats;
+    const float* rec = reinterpret_cast<const float*>(scr);
+    auto HM = [&](int r, int sl) { return rec[sl * rf + 2 * r]; };
+    auto HS = [&](int r, int sl) { return rec[sl * rf + 2 * r + 1]; };
     // row maxima
-    for (int r = lane; r < R; r += 32) {
+    for (int r = 0; r < R; ++r) {
       float M = kNegInf;
-      for (int s = 0; s < ns; ++s) M = fmaxf(M, hm[r * ns + s]);
-      if (!(M > kNegInf) || M != M) {
-        atomicOr(p.status, MDS_ST_NONFINITE);
-        M = 0.f;
+      for (int sl = lane; sl < ns; sl += 32) M = fmaxf(M, HM(r, sl));
+      M = warp_max(M);
+      if (lane == 0) {
+        if (!(M > kNegInf) || M != M) {
+          atomicOr(p.status, MDS_ST_NONFINITE);
+          M = 0.f;
+        }
+        D.P.row[r].M = M;
       }
-      D.P.row[r].M = M;
     }
     __syncwarp();
-    if (!list) {
-      for (int r = lane; r < R; r += 32) {
-        const float M = D.P.row[r].M, c = D.P.row[r].c;
-        float Z = 0.f;
-        for (int s = 0; s < ns; ++s) {
-          const float ms = hm[r * ns + s];
-          if (ms > kNegInf) Z = __fadd_rn(Z, __fmul_rn(hs[r * ns + s], ref_shift(ms, M, c)));
-        }
-        finish_row(r, Z);
+    // every row's slice sums at its maximum
+    float C[kListRowsMax];
+    const int RC = list ? R : 0;
+    for (int r = 0; r < R; ++r) {
+      const float M = D.P.row[r].M, c = D.P.row[r].c;
+      float z = 0.f;
+      for (int sl = lane; sl < ns; sl += 32) {
+        const float ms = HM(r, sl);
+        if (ms > kNegInf) z = __fadd_rn(z, __fmul_rn(HS(r, sl), ref_shift(ms, M, c)));
       }
+      z = warp_sum(z);
+      if (!list) {
+        if (lane == 0) finish_row(r, z);
+      } else if (r < kListRowsMax) {
+        C[r] = z;
+      }
+    }
+    if (!list) {
       __syncwarp();
       return;
     }
-    // merge of the slices' lists: lane s holds slice s's head; ties of the
-    // logit go to the lower slice, which holds the lower token ids
-    const int nl = (lane < ns) ? hnl[lane] : 0;
-    int h = 0;
-    unsigned key = (h < nl) ? ord_key(__fadd_rn(el[lane * LN], 0.f)) : 0u;
-    int nf = 0;
-    for (int t = 0; t < LF; ++t) {
-      const unsigned km = __reduce_max_sync(FULLM, key);
-      if (!km) break;
-      const unsigned who = __ballot_sync(FULLM, key == km);
-      if (lane == __ffs(who) - 1) {
-        D.fin_s[t] = lane;
-        D.fin_i[t] = h;
-        ++h;
-        key = (h < nl) ? ord_key(__fadd_rn(el[lane * LN + h], 0.f)) : 0u;
+    // the list: entry i = sl * LN + q is slice sl's q-th entry (valid for
+    // q < its list length), keyed by its target logit; the first LF entries in
+    // the order (larger logit, lower slice, lower position) -- the slices hold
+    // increasing token ids and sort their own lists the same way
+    const int NE = ns * LN;
+    constexpr int kPer = kMaxEntries / 32;
+    unsigned key[kPer];
+    int nvalid = 0;
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) {
+      const int i = lane + 32 * k;
+      key[k] = 0u;
+      if (i < NE) {
+        const int sl = i / LN, q = i - sl * LN;
+        const int nl = __float_as_int(rec[sl * rf + 2 * kMaxRows + 1]);
+        if (q < nl) key[k] = ord_key(__fadd_rn(rec[sl * rf + kHdr + LN + q], 0.f));
       }
-      nf = t + 1;
+      nvalid += key[k] ? 1 : 0;
     }
-    if (lane < ns) D.ksl[lane] = h;
-    // tau: the largest target logit left out (slices' own and dropped entries)
-    float tau = (lane < ns) ? htau[lane] : kNegInf;
-    for (int q = h; q < nl; ++q) tau = fmaxf(tau, el[lane * LN + q]);
-    tau = warp_max(tau);
+    nvalid = __reduce_add_sync(FULLM, nvalid);
+    // theta: the LF-th largest key (0: take every valid entry)
+    unsigned theta = 0u;
+    if (nvalid > LF) {
+      for (int bit = 31; bit >= 0; --bit) {
+        const unsigned c = theta | (1u << bit);
+        int cnt = 0;
+#pragma unroll
+        for (int k = 0; k < kPer; ++k) cnt += (key[k] >= c) ? 1 : 0;
+        if (__reduce_add_sync(FULLM, cnt) >= LF) theta = c;
+      }
+    }
+    // taken: keys above theta, then ties at theta in entry order
+    int above = 0;
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) above += (key[k] > theta) ? 1 : 0;
+    above = __reduce_add_sync(FULLM, above);
+    const int nf = min(LF, nvalid);
+    int tie_base = 0, pos_base = 0;
+    const unsigned lt = (1u << lane) - 1u;
+    if (lane < ns) D.ksl[lane] = 0;
     __syncwarp();
-    // dropped entries' masses per row (fixed order) and the slices' sums
+    int* sk = reinterpret_cast<int*>(D.cm_sp);   // taken entries' keys, then their indices (scratch)
+    int* si = D.fin_i;
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) {
+      const bool tie = theta != 0u && key[k] == theta;
+      const unsigned tb = __ballot_sync(FULLM, tie);
+      const bool take = key[k] != 0u && (key[k] > theta || (tie && above + tie_base + __popc(tb & lt) < nf));
+      tie_base += __popc(tb);
+      const unsigned kb = __ballot_sync(FULLM, take);
+      if (take) {
+        const int pos = pos_base + __popc(kb & lt);
+        sk[pos] = (int)key[k];
+        si[pos] = lane + 32 * k;
+        atomicAdd(&D.ksl[(lane + 32 * k) / LN], 1);
+      }
+      pos_base += __popc(kb);
+    }
+    __syncwarp();
+    // merge order of the taken entries
+    for (int t = lane; t < nf; t += 32) {
+      const unsigned kt = (unsigned)sk[t];
+      const int it = si[t];
+      int rank = 0;
+      for (int u = 0; u < nf; ++u) {
+        const unsigned ku = (unsigned)sk[u];
+        rank += (ku > kt || (ku == kt && si[u] < it)) ? 1 : 0;
+      }
+      D.fin_s[rank] = it;   // entry index, by merge position
+    }
+    __syncwarp();
+    // tau: the largest target logit left out (the slices' own and the entries not taken)
+    float tau = kNegInf;
+    for (int sl = lane; sl < ns; sl += 32) tau = fmaxf(tau, rec[sl * rf + 2 * kMaxRows]);
+    for (int i = lane; i < NE; i += 32) {
+      const int sl = i / LN, q = i - sl * LN;
+      const int nl = __float_as_int(rec[sl * rf + 2 * kMaxRows + 1]);
+      if (q >= D.ksl[sl] && q < nl) tau = fmaxf(tau, rec[sl * rf + kHdr + LN + q]);
+    }
+    tau = warp_max(tau);
+    // complement masses per row: the slice sums plus the entries not taken
     for (int r = 0; r < R; ++r) {
       const float M = D.P.row[r].M, c = D.P.row[r].c;
       float add = 0.f;
-      for (int i = lane; i < ns * LN; i += 32) {
-        const int s = i / LN, q = i - s * LN;
-        if (q >= D.ksl[s] && q < hnl[s]) add = __fadd_rn(add, exp_term(el[r * ns * LN + i], M, c));
+      for (int i = lane; i < NE; i += 32) {
+        const int sl = i / LN, q = i - sl * LN;
+        const int nl = __float_as_int(rec[sl * rf + 2 * kMaxRows + 1]);
+        if (q >= D.ksl[sl] && q < nl) add = __fadd_rn(add, exp_term(rec[sl * rf + kHdr + (1 + r) * LN + q], M, c));
       }
       add = warp_sum(add);
-      if (lane == 0) {
-        float C = 0.f;
-        for (int s = 0; s < ns; ++s) {
-          const float ms = hm[r * ns + s];
-          if (ms > kNegInf) C = __fadd_rn(C, __fmul_rn(hs[r * ns + s], ref_shift(ms, M, c)));
-        }
-        D.pc[r] = __fadd_rn(C, add);
-      }
+      if (lane == 0) D.pc[r] = __fadd_rn(C[r], add);
     }
     // the list: in merge order (larger logit first) for the weighted scheme,
     // whose stages break key ties on the id; by token id for the truncated
     // alphabet, whose draws scan Omega_0 in token order
     const bool by_id = p.scheme == MDS_WIS0;
+    __syncwarp();
     for (int t = lane; t < nf; t += 32) {
-      const int idx = D.fin_s[t] * LN + D.fin_i[t];
-      const int id = eid[idx];
+      const int i = D.fin_s[t];
+      const int sl = i / LN, q = i - sl * LN;
+      const float* e = rec + sl * rf + kHdr;
+      const int id = __float_as_int(e[q]);
       int pos = t;
       if (by_id) {
         pos = 0;
-        for (int q = 0; q < nf; ++q) pos += (eid[D.fin_s[q] * LN + D.fin_i[q]] < id) ? 1 : 0;
+        for (int u = 0; u < nf; ++u) {
+          const int iu = D.fin_s[u];
+          const int su = iu / LN, qu = iu - su * LN;
+          pos += (__float_as_int(rec[su * rf + kHdr + qu]) < id) ? 1 : 0;
+        }
       }
       D.cm_id[pos] = id;
-      D.cm_l0[pos] = el[idx];
-      for (int r = 0; r < R; ++r) D.cm_e[r][pos] = exp_term(el[r * ns * LN + idx], D.P.row[r].M, D.P.row[r].c);
-      D.cm_sp[pos] = 0;
-      D.cm_a[pos] = 0.f;
+      D.cm_l0[pos] = e[LN + q];
+      for (int r = 0; r < R; ++r) D.cm_e[r][pos] = exp_term(e[(1 + r) * LN + q], D.P.row[r].M, D.P.row[r].c);
+    }
+    __syncwarp();
+    for (int t = lane; t < nf; t += 32) {
+      D.cm_sp[t] = 0;
+      D.cm_a[t] = 0.f;
     }
     __syncwarp();
     for (int r = 0; r < R; ++r) {
@@ -1731,23 +1851,9 @@ struct Dec {
   // The stage LP on one thread.  Out of line, so that it has the kernel's
   // whole register budget: s <= 5 keeps its pair state in registers, larger
   // s in shared memory.
-  __device__ __noinline__ int solve5(int s, float A2, float B2, int A, int Btok, float u) {
-    bool capped = false;
-    const int y = stage_solve_split<5>(s, A2, B2, A, Btok, u, D.om, D.om_q, D.om_a, D.om_b, D.om_x, &capped, D.lp_rs,
-                                       D.lp_fl, D.lp_fh, D.lp_rd);
-    if (capped) atomicOr(p.status, MDS_ST_LP_CAP);
-    return y;
-  }
-  __device__ __noinline__ int solve8(int s, float A2, float B2, int A, int Btok, float u) {
-    bool capped = false;
-    const int y = stage_solve<MDS_MAX_S>(s, A2, B2, A, Btok, u, D.om, D.om_q, D.om_a, D.om_b, D.om_x, &capped,
-                                         D.lp_rs, D.lp_fl, D.lp_fh);
-    if (capped) atomicOr(p.status, MDS_ST_LP_CAP);
-    return y;
-  }
   __device__ int solve(int s, float A2, float B2, int A, int Btok, float u) {
     PT_T0(t_lp);
-    const int y = (s <= 5) ? solve5(s, A2, B2, A, Btok, u) : solve8(s, A2, B2, A, Btok, u);
+    const int y = (s <= 5) ? lp_solve5(s, A2, B2, A, Btok, u) : lp_solve8(s, A2, B2, A, Btok, u);
     PT_ADDW(kPhLp, t_lp);
     PT_CNTW(kPhLpCalls);
     return y;
@@ -1815,13 +1921,11 @@ struct Dec {
     }
     __syncwarp();
     PT_T0(t_plan);
-    plan_warp(b, j, D.W.valid, false, true);
+    plan_warp(b, j, D.W.valid, false, true, true, D.tk0);
     PT_ADDW(kPhDecPlan, t_plan);
-    PT_T0(t_load);
-    stage_records(R, list, b);
-    PT_ADDW(kPhDecLoad, t_load);
     PT_T0(t_comb);
     combine_stats(R, list);
+    xl_sync();
     PT_ADDW(kPhDecCombine, t_comb);
     if (p.scheme == MDS_WIS0) {
       dec_wis0_nl<DT>(b);
@@ -1885,7 +1989,7 @@ struct Dec {
   // plus their entries not taken), the LP, the selection and the law update.
   __device__ void decide_full(int b) {
     const int j = D.P.j, ns = p.ns;
-    plan_warp(b, j, D.W.valid, false, false);
+    plan_warp(b, j, D.W.valid, false, false, false, D.tk0);
     const int m = D.W.stage;
     const int A = D.W.A, Btok = D.X[m], rb = D.vrow[m];
     const float u = draw_uniform(p.seed, b, j, kDrawSelect + m - 1);
@@ -2081,38 +2185,51 @@ struct Dec {
     }
   }
 
-  // The smallest token whose running mass exceeds T, else the last token
-  // with positive weight: the slice by the masses Rs[0..ns) (in slice order),
-  // then inside it three levels in token order: contiguous runs of units per
-  // lane, the units of the owning run (one per lane), the owning unit's
-  // tokens.  Every level sums in a fixed order.
-  __device__ int search(FPass& P, float T) {
-    int s = 0;
-    float base = 0.f;
-    if (lane == 0) {
-      float run = 0.f, run_last = 0.f, run_hit = 0.f;
-      int hit = -1, last = -1;
-      for (int q = 0; q < p.ns; ++q) {
-        const float v = Rs[q];
-        if (v > 0.f) {
-          last = q;
-          run_last = run;
-        }
-        if (hit < 0 && __fadd_rn(run, v) > T) {
-          hit = q;
-          run_hit = run;
-        }
-        run = __fadd_rn(run, v);
-      }
-      if (hit < 0) {
-        hit = max(last, 0);
-        run_hit = run_last;
-      }
-      s = hit;
-      base = run_hit;
+  // Inclusive warp scan (fixed order) of v over the lanes.
+  __device__ __forceinline__ static float scan_incl(float v, int lane) {
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const float t = __shfl_up_sync(FULLM, v, o);
+      if (lane >= o) v = __fadd_rn(v, t);
     }
-    s = __shfl_sync(FULLM, s, 0);
-    base = __shfl_sync(FULLM, base, 0);
+    return v;
+  }
+
+  // The smallest token whose running mass exceeds T, else the last token
+  // with positive weight.  Four levels in token order, each a warp scan:
+  // the slices (masses Rs[0..ns)), the slice's 32 runs of upl units (masses
+  // from its staged record when `runs`, else summed from a re-read), the
+  // owning run's units (re-read, one per lane), the owning unit's tokens (in
+  // that lane's registers).
+  __device__ int search(FPass& P, float T, bool runs) {
+    // level 0: slices
+    int s = -1, slast = -1;
+    float base = 0.f, blast = 0.f;
+    {
+      float run = 0.f;
+      for (int c = 0; c < p.ns && s < 0; c += 32) {
+        const int q = c + lane;
+        const float v = q < p.ns ? Rs[q] : 0.f;
+        const float incl = scan_incl(v, lane);
+        const float ex = __fadd_rn(run, __fsub_rn(incl, v));
+        const unsigned h = __ballot_sync(FULLM, __fadd_rn(run, incl) > T && v > 0.f);
+        const unsigned pz = __ballot_sync(FULLM, v > 0.f);
+        if (h) {
+          const int l = __ffs(h) - 1;
+          s = c + l;
+          base = __shfl_sync(FULLM, ex, l);
+        } else if (pz) {
+          const int l = 31 - __clz(pz);
+          slast = c + l;
+          blast = __shfl_sync(FULLM, ex, l);
+        }
+        run = __shfl_sync(FULLM, __fadd_rn(run, incl), 31);
+      }
+      if (s < 0) {
+        s = max(slast, 0);
+        base = blast;
+      }
+    }
     const int tok0 = s * p.T, n = min(p.T, p.V - tok0);
     const int U = (n + VE - 1) / VE;
     if (P.kind == kResid && P.nspec > 0) {
@@ -2124,70 +2241,76 @@ struct Dec {
       }
       __syncwarp();
     }
-    // level 1: lane runs of upl units
+    // level 1: runs of upl units, one per lane
     const int upl = (U + 31) / 32;
     const int u0 = min(U, lane * upl), u1 = min(U, u0 + upl);
     float part = 0.f;
-    for (int u = u0; u < u1; ++u) {
-      float w[VE];
-      weights_g(P, u, tok0, n, w);
+    if (runs) {
+      part = reinterpret_cast<const float*>(scr)[s * p.rec_floats + 4 + lane];
+    } else {
+      for (int u = u0; u < u1; ++u) {
+        float w[VE];
+        weights_g(P, u, tok0, n, w);
 #pragma unroll
-      for (int e = 0; e < VE; ++e) part = __fadd_rn(part, w[e]);
+        for (int e = 0; e < VE; ++e) part = __fadd_rn(part, w[e]);
+      }
     }
-    float incl = part;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const float t = __shfl_up_sync(FULLM, incl, o);
-      if (lane >= o) incl = __fadd_rn(incl, t);
-    }
+    const float incl = scan_incl(part, lane);
     const float excl = __fadd_rn(base, __fsub_rn(incl, part));
     const unsigned hit1 = __ballot_sync(FULLM, __fadd_rn(base, incl) > T && part > 0.f);
     const unsigned pos1 = __ballot_sync(FULLM, part > 0.f);
     if (!pos1) return tok0;   // no mass in the slice (only by rounding)
     const int own = hit1 ? __ffs(hit1) - 1 : 31 - __clz(pos1);
-    // level 2: the owning run's units, one per lane (chunks of 32)
+    // level 2: the owning run's units, one per lane (chunks of 32); level 3
+    // in the owning lane
     float run = __shfl_sync(FULLM, excl, own);
     const int v0 = __shfl_sync(FULLM, u0, own), v1 = __shfl_sync(FULLM, u1, own);
-    int unit = -1, ulast = -1;
-    float ubase = 0.f, ubase_last = 0.f;
-    for (int c0 = v0; c0 < v1 && unit < 0; c0 += 32) {
+    int ulast = -1;
+    float ubase_last = 0.f;
+    for (int c0 = v0; c0 < v1; c0 += 32) {
       const int u = c0 + lane;
       float w[VE], us = 0.f;
+#pragma unroll
+      for (int e = 0; e < VE; ++e) w[e] = 0.f;
       if (u < v1) {
         weights_g(P, u, tok0, n, w);
 #pragma unroll
         for (int e = 0; e < VE; ++e) us = __fadd_rn(us, w[e]);
       }
-      float ui = us;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const float t = __shfl_up_sync(FULLM, ui, o);
-        if (lane >= o) ui = __fadd_rn(ui, t);
-      }
+      const float ui = scan_incl(us, lane);
       const float uex = __fadd_rn(run, __fsub_rn(ui, us));
       const unsigned h2 = __ballot_sync(FULLM, __fadd_rn(run, ui) > T && us > 0.f);
       const unsigned p2 = __ballot_sync(FULLM, us > 0.f);
       if (h2) {
         const int l2 = __ffs(h2) - 1;
-        unit = c0 + l2;
-        ubase = __shfl_sync(FULLM, uex, l2);
-      } else if (p2) {
+        int tok = 0;
+        if (lane == l2) {
+          float acc = uex;
+          int hit = -1, last = -1;
+#pragma unroll
+          for (int e = 0; e < VE; ++e) {
+            if (w[e] > 0.f) last = e;
+            acc = __fadd_rn(acc, w[e]);
+            if (hit < 0 && acc > T && w[e] > 0.f) hit = e;
+          }
+          if (hit < 0) hit = last < 0 ? 0 : last;
+          tok = min(tok0 + u * VE + hit, p.V - 1);
+        }
+        return __shfl_sync(FULLM, tok, l2);
+      }
+      if (p2) {
         const int l2 = 31 - __clz(p2);
         ulast = c0 + l2;
         ubase_last = __shfl_sync(FULLM, uex, l2);
       }
       run = __shfl_sync(FULLM, __fadd_rn(run, ui), 31);
     }
-    if (unit < 0) {
-      unit = ulast;
-      ubase = ubase_last;
-    }
-    // level 3: the owning unit's tokens (one lane)
+    // T beyond the run's mass (only by rounding): the last unit with mass
     int tok = tok0;
-    if (lane == 0 && unit >= 0) {
+    if (lane == 0 && ulast >= 0) {
       float w[VE];
-      weights_g(P, unit, tok0, n, w);
-      float acc = ubase;
+      weights_g(P, ulast, tok0, n, w);
+      float acc = ubase_last;
       int hit = -1, last = -1;
 #pragma unroll
       for (int e = 0; e < VE; ++e) {
@@ -2196,15 +2319,15 @@ struct Dec {
         if (hit < 0 && acc > T && w[e] > 0.f) hit = e;
       }
       if (hit < 0) hit = last < 0 ? 0 : last;
-      tok = min(tok0 + unit * VE + hit, p.V - 1);
+      tok = min(tok0 + ulast * VE + hit, p.V - 1);
     }
     return __shfl_sync(FULLM, tok, 0);
   }
 
   // Slice masses of the pass just completed (Rs) and their total in slice order.
   __device__ float slice_masses(int b) {
-    const float* recb = p.rec + (size_t)b * p.ns * p.rec_floats;
-    for (int q = lane; q < p.ns; q += 32) Rs[q] = __ldcg(recb + (size_t)q * p.rec_floats);
+    const float* rec = reinterpret_cast<const float*>(scr);
+    for (int q = lane; q < p.ns; q += 32) Rs[q] = rec[q * p.rec_floats];
     __syncwarp();
     float R = 0.f;
     if (lane == 0)
@@ -2213,12 +2336,12 @@ struct Dec {
   }
 
   __device__ void decide_resid(int b) {
-    plan_warp(b, D.P.j, D.W.valid, false, false);
+    plan_warp(b, D.P.j, D.W.valid, false, false, false, D.tk0);
     const float R = slice_masses(b);
     int Z = D.W.Y;
     if (!D.W.acc) {
       if (R > 0.f) {
-        Z = search(D.P, __fmul_rn(D.W.ures, R));
+        Z = search(D.P, __fmul_rn(D.W.ures, R), true);
       } else {
         // zero residual mass (only by rounding): sample the target row
         if (lane == 0) {
@@ -2238,11 +2361,11 @@ struct Dec {
   }
 
   __device__ void decide_replace(int b) {
-    plan_warp(b, D.P.j, D.W.valid, false, false);
+    plan_warp(b, D.P.j, D.W.valid, false, false, false, D.tk0);
     const float R = slice_masses(b);
     int Z;
     if (R > 0.f) {
-      Z = search(D.P, __fmul_rn(D.W.ures, R));
+      Z = search(D.P, __fmul_rn(D.W.ures, R), true);
     } else if (!D.W.zres && D.W.Yp >= 0) {
       Z = D.W.Yp;   // no target mass outside Omega_0
     } else if (!D.W.zres) {
@@ -2264,10 +2387,10 @@ struct Dec {
   }
 
   __device__ void decide_bonus(int b) {
-    const float* recb = p.rec + (size_t)b * p.ns * p.rec_floats;
+    const float* rec = reinterpret_cast<const float*>(scr);
     for (int q = lane; q < p.ns; q += 32) {
-      Hm[q] = __ldcg(recb + (size_t)q * p.rec_floats);
-      Rs[q] = __ldcg(recb + (size_t)q * p.rec_floats + 1);
+      Hm[q] = rec[q * p.rec_floats];
+      Rs[q] = rec[q * p.rec_floats + 1];
     }
     __syncwarp();
     if (lane == 0) {
@@ -2293,7 +2416,7 @@ struct Dec {
     if (lane == 0)
       for (int q = 0; q < p.ns; ++q) Q = __fadd_rn(Q, Rs[q]);
     Q = __shfl_sync(FULLM, Q, 0);
-    const int Z = search(D.P, __fmul_rn(draw_uniform(p.seed, b, p.L, kDrawBonus), Q));
+    const int Z = search(D.P, __fmul_rn(draw_uniform(p.seed, b, p.L, kDrawBonus), Q), false);
     if (lane == 0) {
       __stcg(p.out_tokens + (size_t)b * (p.L + 1) + p.L, Z);
       if (p.out_diag) {
@@ -2503,13 +2626,35 @@ struct Dec {
   // Request fields: the sequence, the kind, depth, row count and list flag of
   // the pass that just completed.
   __device__ void decide(int b, int kind, int j, int R, bool list) {
+    // One round of asynchronous copies: the sequence's state (a depth-0
+    // stats pass has none yet), its draft tokens at depths j and j + 1, its
+    // temperatures and the slice records of the pass.
+    const int K = p.K, L = p.L;
+    PT_T0(t_load);
     if (!(kind == kStats && j == 0)) {
-      const FSeq* g = &reinterpret_cast<const FSeq*>(p.seq)[b];
-      copy_in(&D.P, &g->P, (int)sizeof(FPass), lane, 32);
-      copy_in(&D.W, &g->W, (int)sizeof(FWalk), lane, 32);
+      const int4* src = reinterpret_cast<const int4*>(reinterpret_cast<const FSeq*>(p.seq) + b);
+      int4* dst = reinterpret_cast<int4*>(&D.P);
+      for (int i = lane; i < (int)(sizeof(FSeq) / 16); i += 32) cpa16(dst + i, src + i);
     }
-    if (lane == 0) D.xl_ok = 0;
+    if (lane < K) {
+      const int32_t* tk = p.tokens + ((size_t)b * K + lane) * L;
+      cpa4(&D.tk0[lane], tk + j);
+      if (j + 1 < L) cpa4(&D.tk1[lane], tk + j + 1);
+    }
+    if (lane <= K) cpa4(&D.tmp[lane], p.temps + (size_t)b * (1 + K) + lane);
+    {
+      const float* recb = p.rec + (size_t)b * p.ns * p.rec_floats;
+      const int n16 = p.ns * p.rec_floats / 4;
+      for (int i = lane; i < n16; i += 32) cpa16(scr + 16 * i, recb + 4 * i);
+    }
+    cpa_wait();
     __syncwarp();
+    if (lane == 0) {
+      D.xl_ok = 0;
+      D.xl_wait = 0;
+    }
+    __syncwarp();
+    PT_ADDW(kPhDecLoad, t_load);
     PT_T0(t_dec);
     PT_CNTW(kPhDecisions);
     switch (kind) {
@@ -2600,6 +2745,25 @@ template <int DT> __device__ __noinline__ void dec_replace_nl(int b) { dec_view<
 template <int DT> __device__ __noinline__ void dec_full_nl(int b) { dec_view<DT>().decide_full(b); }
 template <int DT> __device__ __noinline__ void dec_bonus_nl(int b) { dec_view<DT>().decide_bonus(b); }
 template <int DT> __device__ __noinline__ void dec_wis0_nl(int b) { dec_view<DT>().wis0_decide(b); }
+
+// The stage LP of the calling warp's decision (one lane), on its Omega_1
+// tables: pair state in registers for s <= 5, in shared memory above.
+__device__ __noinline__ int lp_solve5(int s, float A2, float B2, int A, int Btok, float u) {
+  DState& D = *reinterpret_cast<DState*>(g_dsm + (size_t)(threadIdx.x >> 5) * kDecPerWarp);
+  bool capped = false;
+  float RS[10], FL[10], FH[10];
+  const int y = stage_solve<5>(s, A2, B2, A, Btok, u, D.om, D.om_q, D.om_a, D.om_b, D.om_x, &capped, RS, FL, FH);
+  if (capped) atomicOr(g_dp.status, MDS_ST_LP_CAP);
+  return y;
+}
+__device__ __noinline__ int lp_solve8(int s, float A2, float B2, int A, int Btok, float u) {
+  DState& D = *reinterpret_cast<DState*>(g_dsm + (size_t)(threadIdx.x >> 5) * kDecPerWarp);
+  bool capped = false;
+  const int y = stage_solve<MDS_MAX_S>(s, A2, B2, A, Btok, u, D.om, D.om_q, D.om_a, D.om_b, D.om_x, &capped,
+                                       D.lp_rs, D.lp_fl, D.lp_fh);
+  if (capped) atomicOr(g_dp.status, MDS_ST_LP_CAP);
+  return y;
+}
 
 // A decision warp's loop, out of line with the whole register budget.
 template <int DT>
@@ -2778,7 +2942,7 @@ bool plan_geometry(Params& p, int grid) {
     return false;
   }
   if (nstream > kMaxRows) return false;
-  int Tmax = kBufBytes / (nstream * es);
+  int Tmax = kBufBytes / (nstream * es);   // the slice buffer's bound
   Tmax = (Tmax / kSliceQuantum) * kSliceQuantum;
   if (Tmax < kSliceQuantum) return false;
   const int cap = list ? kMaxSlicesList : kMaxSlices;
@@ -2792,32 +2956,40 @@ bool plan_geometry(Params& p, int grid) {
     int T = (p.V + nsw - 1) / nsw;
     T = ((T + kSliceQuantum - 1) / kSliceQuantum) * kSliceQuantum;
     if (T < kSliceQuantum) T = kSliceQuantum;
-    if (T < Tmax) Tmax = T;
-    ns = (p.V + Tmax - 1) / Tmax;
+    if (T > Tmax) T = Tmax;
+    ns = (p.V + T - 1) / T;
   }
-  p.T = Tmax;
-  p.ns = ns;
   p.ln = list ? ((p.scheme == MDS_WIS0 && p.omega0 >= 32) ? 64 : 32) : 0;
   if (p.ln > kListMax) return false;
-  // a slice's list: enough that the slices' lists together hold the
-  // sequence's list whenever its tokens are spread over the slices (a slice
-  // holding more of them only shortens the certified list)
-  if (list) {
-    const int base = (p.scheme == MDS_WIS0) ? 16 : 8;
-    int lns = (2 * p.ln + ns - 1) / ns;
-    lns = (lns + 7) / 8 * 8;
-    p.lns = lns < base ? base : (lns > p.ln ? p.ln : lns);
-  } else {
-    p.lns = 0;
-  }
   const int lrows = list ? nstream : 0;
-  int rf = kHdr + p.lns * (1 + lrows);
-  if (rf < 4 + 4 * kTopF) rf = 4 + 4 * kTopF;
-  p.rec_floats = (rf + 3) & ~3;
-  p.hdr_floats = kHdr;
-  // a decision stages one stats pass's records in its warp's staging area
-  const size_t stage = (size_t)(2 * nstream * ns + 2 * ns + ns * p.lns * (1 + lrows)) * 4;
-  if (stage > (size_t)kDecStage) return false;
+  // a decision stages a pass's records ([ns][rec_floats]) in its warp's
+  // staging area: fewer, longer slices where they would not fit
+  const int ns_min = (p.V + Tmax - 1) / Tmax;
+  for (;; --ns) {
+    if (ns < ns_min) return false;
+    int T = (p.V + ns - 1) / ns;
+    T = ((T + kSliceQuantum - 1) / kSliceQuantum) * kSliceQuantum;
+    if (T > Tmax) return false;
+    ns = (p.V + T - 1) / T;
+    p.T = T;
+    p.ns = ns;
+    // a slice's list: enough that the slices' lists together hold the
+    // sequence's list whenever its tokens are spread over the slices (a
+    // slice holding more of them only shortens the certified list)
+    if (list) {
+      const int base = (p.scheme == MDS_WIS0) ? 16 : 8;
+      int lns = (2 * p.ln + ns - 1) / ns;
+      lns = (lns + 7) / 8 * 8;
+      p.lns = lns < base ? base : (lns > p.ln ? p.ln : lns);
+    } else {
+      p.lns = 0;
+    }
+    int rf = kHdr + p.lns * (1 + lrows);
+    if (rf < 4 + 4 * kTopF) rf = 4 + 4 * kTopF;
+    p.rec_floats = (rf + 3) & ~3;
+    p.hdr_floats = kHdr;
+    if ((size_t)ns * p.rec_floats * 4 <= (size_t)kDecStage && ns * p.lns <= kMaxEntries) break;
+  }
   p.dec_sms = decision_sms(grid);
   return p.dec_sms > 0;
 }
