@@ -54,6 +54,13 @@ constexpr int kListMax = 64;           // candidate list length at most
 constexpr int kHdr = 2 * kMaxRows + 2; // record: (max, sum) per row, tau, list length
 constexpr int kTopF = 8;               // per-thread candidates of a full stage (>= MDS_MAX_S)
 constexpr int kMaxEntries = 512;       // slices x slice list length, at most
+constexpr int kDecStage = 8192;        // bytes of a pass's slice records ([ns][rec_floats]) at most
+// A stats pass's combined record (written over the sequence's slice records
+// by the CTA that completes the pass): per row M, 1/Z and the complement
+// mass, the list's length, tau, completeness and q(tau), then the list:
+// ids, target logits and per row exp terms (token order of the merge).
+constexpr int kCmbM = 0, kCmbIz = kMaxRows, kCmbPc = 2 * kMaxRows, kCmbN = 2 * kMaxRows + kListRowsMax;
+constexpr int kCmbHdr = kCmbN + 4;
 constexpr unsigned long long kWaitNs = 2000000000ull;   // 2 s bound on every wait
 constexpr unsigned FULLM = 0xffffffffu;
 static_assert(kHdr % 4 == 0, "record header keeps 16-byte alignment");
@@ -94,6 +101,7 @@ enum : int {
   kPhListB,             // list tasks: the sums and the candidates
   kPhListC,             // list tasks: ranking and the record
   kPhPublish,           // a task's record publication (fence, pass counter)
+  kPhCombine,           // combining a completed stats pass (the last task's CTA)
   kPhLp,                // the stage LPs (one thread)
   kPhLpCalls,           // count: stage LPs
   kPhTasks,             // count: slice tasks
@@ -207,6 +215,8 @@ struct FShared {
   float mrow[kMaxRows];
   float wth[kCW];
   int ncand, last, issued, consumed;
+  int cmb_n, cmb_nv;           // combine of a pass: entries taken, valid entries
+  unsigned cmb_tau;            // ... order key of tau
   float addtau;
   float add[kMaxRows];
   uint32_t bitmap[64];         // one bit per 16-byte unit of a slice holding a special token
@@ -955,6 +965,186 @@ struct Eng {
     }
   }
 
+  // -------------------------------------------------------------- a stats pass's combine
+  // Run by the CTA that completes a stats pass, with the pass's slice records
+  // (rec, [ns][rec_floats]) in global memory: every row's M and 1/Z and, with
+  // candidate lists, the sequence's list (the first LF of the slices' lists
+  // by (logit, then slice, then position: the slices hold increasing token
+  // ids and sort their own lists that way)), its complement masses and tau;
+  // written over the records as the combined record.  Scratch: the task's
+  // slice buffer b.  Sums over slices and entries run in fixed orders.
+  __device__ __noinline__ void combine_pass(const FPass& P, char* b, float* rec) {
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int ns = p.ns, rf = p.rec_floats, LN = p.lns, LF = p.ln;
+    const int R = P.nstream;
+    const bool list = P.list != 0;
+    float* sr = reinterpret_cast<float*>(b);                       // records [ns][rf]
+    unsigned* sk = reinterpret_cast<unsigned*>(b + kDecStage);     // entry keys [ns * LN]
+    int* fin = reinterpret_cast<int*>(sk + kMaxEntries);           // taken entries by merge rank [LF]
+    int* ksl = fin + kListMax;                                     // entries taken per slice [ns]
+    float* part = reinterpret_cast<float*>(ksl + kMaxSlices);      // per-warp partials [kCW][3 * kListRowsMax]
+    for (int i = tid; i < ns * rf / 4; i += kCT)
+      reinterpret_cast<float4*>(sr)[i] = __ldcg(reinterpret_cast<const float4*>(rec) + i);
+    if (tid < ns) ksl[tid] = 0;
+    if (tid == 0) {
+      S.cmb_nv = 0;
+      S.cmb_tau = 0u;
+    }
+    cbar();
+    // rows: warp w takes rows w, w + kCW, ...
+    float* hdr = part + kCW * 3 * kListRowsMax;   // combined header being built [kCmbHdr]
+    for (int r = warp; r < R; r += kCW) {
+      float M = kNegInf;
+      for (int sl = lane; sl < ns; sl += 32) M = fmaxf(M, sr[sl * rf + 2 * r]);
+      M = warp_max(M);
+      if (!(M > kNegInf) || M != M) {
+        if (lane == 0) atomicOr(p.status, MDS_ST_NONFINITE);
+        M = 0.f;
+      }
+      const float c = P.row[r].c;
+      float z = 0.f;
+      for (int sl = lane; sl < ns; sl += 32) {
+        const float ms = sr[sl * rf + 2 * r];
+        if (ms > kNegInf) z = __fadd_rn(z, __fmul_rn(sr[sl * rf + 2 * r + 1], ref_shift(ms, M, c)));
+      }
+      z = warp_sum(z);
+      if (lane == 0) {
+        hdr[kCmbM + r] = M;
+        hdr[kCmbPc + (r < kListRowsMax ? r : 0)] = z;   // the slices' sums (list passes add the entries left out)
+        if (!list) {
+          if (!(z > 0.f) || !(z < kPosInf) || z != z) {
+            atomicOr(p.status, MDS_ST_NONFINITE);
+            z = 1.f;
+          }
+          hdr[kCmbIz + r] = __frcp_rn(z);
+        }
+      }
+    }
+    if (!list) {
+      cbar();
+      for (int i = tid; i < 2 * kMaxRows; i += kCT) __stcg(rec + i, hdr[i]);
+      return;
+    }
+    // entries: keys (0: no entry), the valid count
+    const int NE = ns * LN;
+    for (int i0 = warp * 32; i0 < NE; i0 += kCT) {   // warp-uniform trips (the ballot below)
+      const int i = i0 + lane;
+      unsigned k = 0u;
+      if (i < NE) {
+        const int sl = i / LN, q = i - sl * LN;
+        if (q < __float_as_int(sr[sl * rf + 2 * kMaxRows + 1]))
+          k = ord_key(__fadd_rn(sr[sl * rf + kHdr + LN + q], 0.f));
+        sk[i] = k;
+      }
+      const unsigned vb = __ballot_sync(FULLM, k != 0u);
+      if (lane == 0 && vb) atomicAdd(&S.cmb_nv, __popc(vb));
+    }
+    cbar();
+    const int nf = min(LF, S.cmb_nv);
+    // rank of each valid entry in the merge order; the first nf are taken
+    for (int i = tid; i < NE; i += kCT) {
+      const unsigned k = sk[i];
+      if (k == 0u) continue;
+      int rank = 0;
+      for (int u = 0; u < NE; ++u) {
+        const unsigned ku = sk[u];
+        rank += (ku > k || (ku == k && u < i)) ? 1 : 0;
+      }
+      if (rank < nf) {
+        fin[rank] = i;
+        atomicAdd(&ksl[i / LN], 1);
+      }
+    }
+    cbar();
+    // tau and the complement masses: entries not taken (and the slices' own tau)
+    float add[kListRowsMax];
+#pragma unroll
+    for (int r = 0; r < kListRowsMax; ++r) add[r] = 0.f;
+    float tau = kNegInf;
+    for (int sl = tid; sl < ns; sl += kCT) tau = fmaxf(tau, sr[sl * rf + 2 * kMaxRows]);
+    for (int i = tid; i < NE; i += kCT) {
+      const int sl = i / LN, q = i - sl * LN;
+      if (q >= ksl[sl] && q < __float_as_int(sr[sl * rf + 2 * kMaxRows + 1])) {
+        const float* e = sr + sl * rf + kHdr + q;
+        tau = fmaxf(tau, e[LN]);
+#pragma unroll
+        for (int r = 0; r < kListRowsMax; ++r)
+          if (r < R) add[r] = __fadd_rn(add[r], exp_term(e[(1 + r) * LN], hdr[kCmbM + r], P.row[r].c));
+      }
+    }
+    tau = warp_max(tau);
+#pragma unroll
+    for (int r = 0; r < kListRowsMax; ++r) add[r] = warp_sum(add[r]);
+    if (lane == 0) {
+      if (tau > kNegInf) atomicMax(&S.cmb_tau, ord_key(tau));
+#pragma unroll
+      for (int r = 0; r < kListRowsMax; ++r) part[warp * 3 * kListRowsMax + r] = add[r];
+    }
+    // the list into the combined record: merge order for the weighted
+    // scheme, token-id order for the truncated alphabet
+    const bool by_id = p.scheme == MDS_WIS0;
+    float* out_id = rec + kCmbHdr;
+    float* out_l0 = out_id + LF;
+    float* out_e = out_l0 + LF;
+    float z[kListRowsMax];
+#pragma unroll
+    for (int r = 0; r < kListRowsMax; ++r) z[r] = 0.f;
+    for (int t = tid; t < nf; t += kCT) {
+      const int i = fin[t];
+      const int sl = i / LN, q = i - sl * LN;
+      const float* e = sr + sl * rf + kHdr + q;
+      const int id = __float_as_int(e[0]);
+      int pos = t;
+      if (by_id) {
+        pos = 0;
+        for (int u = 0; u < nf; ++u) {
+          const int iu = fin[u];
+          const int su = iu / LN, qu = iu - su * LN;
+          pos += (__float_as_int(sr[su * rf + kHdr + qu]) < id) ? 1 : 0;
+        }
+      }
+      __stcg(out_id + pos, __int_as_float(id));
+      __stcg(out_l0 + pos, e[LN]);
+#pragma unroll
+      for (int r = 0; r < kListRowsMax; ++r)
+        if (r < R) {
+          const float ev = exp_term(e[(1 + r) * LN], hdr[kCmbM + r], P.row[r].c);
+          __stcg(out_e + r * LF + pos, ev);
+          z[r] = __fadd_rn(z[r], ev);
+        }
+    }
+#pragma unroll
+    for (int r = 0; r < kListRowsMax; ++r) {
+      z[r] = warp_sum(z[r]);
+      if (lane == 0) part[warp * 3 * kListRowsMax + kListRowsMax + r] = z[r];
+    }
+    cbar();
+    if (tid == 0) {
+      for (int r = 0; r < R; ++r) {
+        float a = 0.f, zz = 0.f;
+        for (int w = 0; w < kCW; ++w) {
+          a = __fadd_rn(a, part[w * 3 * kListRowsMax + r]);
+          zz = __fadd_rn(zz, part[w * 3 * kListRowsMax + kListRowsMax + r]);
+        }
+        const float pc = __fadd_rn(hdr[kCmbPc + r], a);
+        float Z = __fadd_rn(pc, zz);
+        if (!(Z > 0.f) || !(Z < kPosInf) || Z != Z) {
+          atomicOr(p.status, MDS_ST_NONFINITE);
+          Z = 1.f;
+        }
+        hdr[kCmbPc + r] = pc;
+        hdr[kCmbIz + r] = __frcp_rn(Z);
+      }
+      const float t = S.cmb_tau ? ord_val(S.cmb_tau) : kNegInf;
+      hdr[kCmbN] = __int_as_float(nf);
+      hdr[kCmbN + 1] = t;
+      hdr[kCmbN + 2] = __int_as_float(nf == p.V ? 1 : 0);
+      hdr[kCmbN + 3] = (t > kNegInf) ? exp_term(t, hdr[kCmbM], P.row[0].c) : 0.f;
+    }
+    cbar();
+    for (int i = tid; i < kCmbHdr; i += kCT) __stcg(rec + i, hdr[i]);
+  }
+
   // -------------------------------------------------------------- full-vocabulary stage task
   __device__ __forceinline__ static void cand_insert(Cand (&top)[kTopF], const Cand& c, float& ra, float& rb) {
     if (better(c.key, c.id, top[kTopF - 1].key, top[kTopF - 1].id)) {
@@ -1168,9 +1358,20 @@ struct Eng {
     // other slices' records)
     PT_T0(t_pub);
     cbar();
-    if (threadIdx.x == 0 && atom_add_acq_rel(&p.cnt[seqb], 1u) == (unsigned)(p.ns - 1))
-      post_decision(dec_payload(seqb, P.kind, P.j, P.nstream, P.list));
+    if (threadIdx.x == 0) S.last = (atom_add_acq_rel(&p.cnt[seqb], 1u) == (unsigned)(p.ns - 1)) ? 1 : 0;
+    cbar();
     PT_ADD(kPhPublish, t_pub);
+    if (S.last) {
+      // thread 0 acquired the other slices' records; the barrier passes that on
+      PT_T0(t_cmb);
+      if (P.kind == kStats) combine_pass(P, b, rec - (size_t)s * p.rec_floats);
+      cbar();
+      if (threadIdx.x == 0) {
+        __threadfence();   // the combined record before the request
+        post_decision(dec_payload(seqb, P.kind, P.j, P.nstream, P.list));
+      }
+      PT_ADD(kPhCombine, t_cmb);
+    }
   }
 
   __device__ void compute() {
@@ -1211,7 +1412,6 @@ struct Eng {
 // Single-warp code throughout (lane 0 for the serial steps); its state and
 // scratch are this warp's own shared memory.
 
-constexpr int kDecStage = 8192;        // bytes of a decision's staged records
 constexpr int kDecScratch = kDecStage + 2 * kMaxSlices * 4 + 64 * 4;   // + slice masses, maxima, bitmap
 
 // Each kind of decision out of line (its own register allocation); each
@@ -1222,6 +1422,8 @@ template <int DT> __device__ __noinline__ void dec_replace_nl(int b);
 template <int DT> __device__ __noinline__ void dec_full_nl(int b);
 template <int DT> __device__ __noinline__ void dec_bonus_nl(int b);
 template <int DT> __device__ __noinline__ void dec_wis0_nl(int b);
+template <int DT> __device__ __noinline__ void dec_accept_nl(int b);
+template <int DT> __device__ __noinline__ bool dec_stage_nl(int A, int Btok, int rb, float u);
 __device__ __noinline__ int lp_solve5(int s, float A2, float B2, int A, int Btok, float u);
 __device__ __noinline__ int lp_solve8(int s, float A2, float B2, int A, int Btok, float u);
 
@@ -1575,187 +1777,36 @@ struct Dec {
     D.P.row[r].invZ = __frcp_rn(Z);
   }
 
-  // Combine the staged records of a stats pass (scr: [ns][rec_floats]):
-  // every row's M and 1/Z, and with candidate lists the sequence's list (the
-  // first LF of the slices' lists by (logit, id)), its complement masses and
-  // tau.  Sums over slices and entries run in fixed orders (lane-strided
-  // partial sums, then a butterfly).
-  __device__ void combine_stats(int R, bool list) {
-    const int ns = p.ns, LN = p.lns, LF = p.ln, rf = p.rec_floats;
-    const float* rec = reinterpret_cast<const float*>(scr);
-    auto HM = [&](int r, int sl) { return rec[sl * rf + 2 * r]; };
-    auto HS = [&](int r, int sl) { return rec[sl * rf + 2 * r + 1]; };
-    // row maxima
-    for (int r = 0; r < R; ++r) {
-      float M = kNegInf;
-      for (int sl = lane; sl < ns; sl += 32) M = fmaxf(M, HM(r, sl));
-      M = warp_max(M);
+  // The combined record of a stats pass (staged in scr; written by the CTA
+  // that completed the pass): every row's M and 1/Z and, with candidate
+  // lists, the sequence's list, its complement masses and tau.
+  __device__ void adopt_combined(int R, bool list) {
+    const float* c = reinterpret_cast<const float*>(scr);
+    for (int r = lane; r < R; r += 32) {
+      D.P.row[r].M = c[kCmbM + r];
+      D.P.row[r].invZ = c[kCmbIz + r];
+      if (list) D.pc[r] = c[kCmbPc + r];
+    }
+    if (list) {
+      const int LF = p.ln;
+      const int n = __float_as_int(c[kCmbN]);
+      for (int t = lane; t < n; t += 32) {
+        D.cm_id[t] = __float_as_int(c[kCmbHdr + t]);
+        D.cm_l0[t] = c[kCmbHdr + LF + t];
+        for (int r = 0; r < R; ++r) D.cm_e[r][t] = c[kCmbHdr + (2 + r) * LF + t];
+        D.cm_sp[t] = 0;
+        D.cm_a[t] = 0.f;
+      }
       if (lane == 0) {
-        if (!(M > kNegInf) || M != M) {
-          atomicOr(p.status, MDS_ST_NONFINITE);
-          M = 0.f;
-        }
-        D.P.row[r].M = M;
+        D.n = n;
+        D.cand_tau = c[kCmbN + 1];
+        D.cand_all = __float_as_int(c[kCmbN + 2]);
+        D.cand_q = c[kCmbN + 3];
       }
-    }
-    __syncwarp();
-    // every row's slice sums at its maximum
-    float C[kListRowsMax];
-    const int RC = list ? R : 0;
-    for (int r = 0; r < R; ++r) {
-      const float M = D.P.row[r].M, c = D.P.row[r].c;
-      float z = 0.f;
-      for (int sl = lane; sl < ns; sl += 32) {
-        const float ms = HM(r, sl);
-        if (ms > kNegInf) z = __fadd_rn(z, __fmul_rn(HS(r, sl), ref_shift(ms, M, c)));
-      }
-      z = warp_sum(z);
-      if (!list) {
-        if (lane == 0) finish_row(r, z);
-      } else if (r < kListRowsMax) {
-        C[r] = z;
-      }
-    }
-    if (!list) {
-      __syncwarp();
-      return;
-    }
-    // the list: entry i = sl * LN + q is slice sl's q-th entry (valid for
-    // q < its list length), keyed by its target logit; the first LF entries in
-    // the order (larger logit, lower slice, lower position) -- the slices hold
-    // increasing token ids and sort their own lists the same way
-    const int NE = ns * LN;
-    constexpr int kPer = kMaxEntries / 32;
-    unsigned key[kPer];
-    int nvalid = 0;
-#pragma unroll
-    for (int k = 0; k < kPer; ++k) {
-      const int i = lane + 32 * k;
-      key[k] = 0u;
-      if (i < NE) {
-        const int sl = i / LN, q = i - sl * LN;
-        const int nl = __float_as_int(rec[sl * rf + 2 * kMaxRows + 1]);
-        if (q < nl) key[k] = ord_key(__fadd_rn(rec[sl * rf + kHdr + LN + q], 0.f));
-      }
-      nvalid += key[k] ? 1 : 0;
-    }
-    nvalid = __reduce_add_sync(FULLM, nvalid);
-    // theta: the LF-th largest key (0: take every valid entry)
-    unsigned theta = 0u;
-    if (nvalid > LF) {
-      for (int bit = 31; bit >= 0; --bit) {
-        const unsigned c = theta | (1u << bit);
-        int cnt = 0;
-#pragma unroll
-        for (int k = 0; k < kPer; ++k) cnt += (key[k] >= c) ? 1 : 0;
-        if (__reduce_add_sync(FULLM, cnt) >= LF) theta = c;
-      }
-    }
-    // taken: keys above theta, then ties at theta in entry order
-    int above = 0;
-#pragma unroll
-    for (int k = 0; k < kPer; ++k) above += (key[k] > theta) ? 1 : 0;
-    above = __reduce_add_sync(FULLM, above);
-    const int nf = min(LF, nvalid);
-    int tie_base = 0, pos_base = 0;
-    const unsigned lt = (1u << lane) - 1u;
-    if (lane < ns) D.ksl[lane] = 0;
-    __syncwarp();
-    int* sk = reinterpret_cast<int*>(D.cm_sp);   // taken entries' keys, then their indices (scratch)
-    int* si = D.fin_i;
-#pragma unroll
-    for (int k = 0; k < kPer; ++k) {
-      const bool tie = theta != 0u && key[k] == theta;
-      const unsigned tb = __ballot_sync(FULLM, tie);
-      const bool take = key[k] != 0u && (key[k] > theta || (tie && above + tie_base + __popc(tb & lt) < nf));
-      tie_base += __popc(tb);
-      const unsigned kb = __ballot_sync(FULLM, take);
-      if (take) {
-        const int pos = pos_base + __popc(kb & lt);
-        sk[pos] = (int)key[k];
-        si[pos] = lane + 32 * k;
-        atomicAdd(&D.ksl[(lane + 32 * k) / LN], 1);
-      }
-      pos_base += __popc(kb);
-    }
-    __syncwarp();
-    // merge order of the taken entries
-    for (int t = lane; t < nf; t += 32) {
-      const unsigned kt = (unsigned)sk[t];
-      const int it = si[t];
-      int rank = 0;
-      for (int u = 0; u < nf; ++u) {
-        const unsigned ku = (unsigned)sk[u];
-        rank += (ku > kt || (ku == kt && si[u] < it)) ? 1 : 0;
-      }
-      D.fin_s[rank] = it;   // entry index, by merge position
-    }
-    __syncwarp();
-    // tau: the largest target logit left out (the slices' own and the entries not taken)
-    float tau = kNegInf;
-    for (int sl = lane; sl < ns; sl += 32) tau = fmaxf(tau, rec[sl * rf + 2 * kMaxRows]);
-    for (int i = lane; i < NE; i += 32) {
-      const int sl = i / LN, q = i - sl * LN;
-      const int nl = __float_as_int(rec[sl * rf + 2 * kMaxRows + 1]);
-      if (q >= D.ksl[sl] && q < nl) tau = fmaxf(tau, rec[sl * rf + kHdr + LN + q]);
-    }
-    tau = warp_max(tau);
-    // complement masses per row: the slice sums plus the entries not taken
-    for (int r = 0; r < R; ++r) {
-      const float M = D.P.row[r].M, c = D.P.row[r].c;
-      float add = 0.f;
-      for (int i = lane; i < NE; i += 32) {
-        const int sl = i / LN, q = i - sl * LN;
-        const int nl = __float_as_int(rec[sl * rf + 2 * kMaxRows + 1]);
-        if (q >= D.ksl[sl] && q < nl) add = __fadd_rn(add, exp_term(rec[sl * rf + kHdr + (1 + r) * LN + q], M, c));
-      }
-      add = warp_sum(add);
-      if (lane == 0) D.pc[r] = __fadd_rn(C[r], add);
-    }
-    // the list: in merge order (larger logit first) for the weighted scheme,
-    // whose stages break key ties on the id; by token id for the truncated
-    // alphabet, whose draws scan Omega_0 in token order
-    const bool by_id = p.scheme == MDS_WIS0;
-    __syncwarp();
-    for (int t = lane; t < nf; t += 32) {
-      const int i = D.fin_s[t];
-      const int sl = i / LN, q = i - sl * LN;
-      const float* e = rec + sl * rf + kHdr;
-      const int id = __float_as_int(e[q]);
-      int pos = t;
-      if (by_id) {
-        pos = 0;
-        for (int u = 0; u < nf; ++u) {
-          const int iu = D.fin_s[u];
-          const int su = iu / LN, qu = iu - su * LN;
-          pos += (__float_as_int(rec[su * rf + kHdr + qu]) < id) ? 1 : 0;
-        }
-      }
-      D.cm_id[pos] = id;
-      D.cm_l0[pos] = e[LN + q];
-      for (int r = 0; r < R; ++r) D.cm_e[r][pos] = exp_term(e[(1 + r) * LN + q], D.P.row[r].M, D.P.row[r].c);
-    }
-    __syncwarp();
-    for (int t = lane; t < nf; t += 32) {
-      D.cm_sp[t] = 0;
-      D.cm_a[t] = 0.f;
-    }
-    __syncwarp();
-    for (int r = 0; r < R; ++r) {
-      float z = 0.f;
-      for (int t = lane; t < nf; t += 32) z = __fadd_rn(z, D.cm_e[r][t]);
-      z = warp_sum(z);
-      if (lane == 0) finish_row(r, __fadd_rn(D.pc[r], z));
-    }
-    __syncwarp();
-    if (lane == 0) {
-      D.n = nf;
-      D.cand_tau = tau;
-      D.cand_all = (nf == p.V) ? 1 : 0;
-      D.cand_q = (tau > kNegInf) ? exp_term(tau, D.P.row[0].M, D.P.row[0].c) : 0.f;
     }
     __syncwarp();
   }
+
   // -------------------------------------------------------------- WIS stage on the candidate list
   // One list entry per lane.  Returns false (changing nothing) if
   // the list cannot certify Omega_1: fewer than s entries, or the s-th key
@@ -1924,7 +1975,7 @@ struct Dec {
     plan_warp(b, j, D.W.valid, false, true, true, D.tk0);
     PT_ADDW(kPhDecPlan, t_plan);
     PT_T0(t_comb);
-    combine_stats(R, list);
+    adopt_combined(R, list);
     xl_sync();
     PT_ADDW(kPhDecCombine, t_comb);
     if (p.scheme == MDS_WIS0) {
@@ -1939,7 +1990,7 @@ struct Dec {
         D.W.pIY = prob_row(D.P, D.vrow[0], Y);
       }
       __syncwarp();
-      accept_step(b);
+      dec_accept_nl<DT>(b);
       return;
     }
     // WIS: the pairwise stages (Remark 4) on the candidate list while it
@@ -1958,7 +2009,7 @@ struct Dec {
       const float ul = (lane + 1 < D.nv) ? draw_uniform(p.seed, b, j, kDrawSelect + lane) : 0.f;
       for (; m < D.nv; ++m) {
         const float u = __shfl_sync(FULLM, ul, m - 1);
-        if (!wis_stage_list(A, D.X[m], D.vrow[m], u)) break;
+        if (!dec_stage_nl<DT>(A, D.X[m], D.vrow[m], u)) break;
         A = D.Y;
       }
       if (lane == 0) list_to_table();
@@ -1981,7 +2032,7 @@ struct Dec {
       push(b, kFull);
       return;
     }
-    accept_step(b);
+    dec_accept_nl<DT>(b);
   }
 
   // One full-vocabulary stage's decision: Omega_1 = the top s of the slices'
@@ -2135,7 +2186,7 @@ struct Dec {
       D.W.pIY = law_at(D.P, Y);
     }
     __syncwarp();
-    accept_step(b);
+    dec_accept_nl<DT>(b);
   }
 
   // -------------------------------------------------------------- inverse-CDF search
@@ -2745,6 +2796,10 @@ template <int DT> __device__ __noinline__ void dec_replace_nl(int b) { dec_view<
 template <int DT> __device__ __noinline__ void dec_full_nl(int b) { dec_view<DT>().decide_full(b); }
 template <int DT> __device__ __noinline__ void dec_bonus_nl(int b) { dec_view<DT>().decide_bonus(b); }
 template <int DT> __device__ __noinline__ void dec_wis0_nl(int b) { dec_view<DT>().wis0_decide(b); }
+template <int DT> __device__ __noinline__ void dec_accept_nl(int b) { dec_view<DT>().accept_step(b); }
+template <int DT> __device__ __noinline__ bool dec_stage_nl(int A, int Btok, int rb, float u) {
+  return dec_view<DT>().wis_stage_list(A, Btok, rb, u);
+}
 
 // The stage LP of the calling warp's decision (one lane), on its Omega_1
 // tables: pair state in registers for s <= 5, in shared memory above.
@@ -2988,7 +3043,9 @@ bool plan_geometry(Params& p, int grid) {
     if (rf < 4 + 4 * kTopF) rf = 4 + 4 * kTopF;
     p.rec_floats = (rf + 3) & ~3;
     p.hdr_floats = kHdr;
-    if ((size_t)ns * p.rec_floats * 4 <= (size_t)kDecStage && ns * p.lns <= kMaxEntries) break;
+    if ((size_t)ns * p.rec_floats * 4 <= (size_t)kDecStage && ns * p.lns <= kMaxEntries &&
+        kCmbHdr + p.ln * (2 + lrows) <= ns * p.rec_floats)
+      break;
   }
   p.dec_sms = decision_sms(grid);
   return p.dec_sms > 0;

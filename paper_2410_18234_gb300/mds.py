@@ -227,7 +227,7 @@ def mds_cluster_size(ctx):
 PHASES = ("kernel", "wait_full", "task_list", "task_stats", "task_resid", "task_full", "dec_stats",
           "dec_combine", "dec_stages", "dec_resid", "dec_full", "dec_bonus", "push", "sched_poll",
           "sched_empty", "dec_poll", "dec_plan", "dec_load", "dec_select", "dec_accept",
-          "dec_walk", "list_a", "list_b", "list_c", "publish", "lp", "lp_calls", "tasks",
+          "dec_walk", "list_a", "list_b", "list_c", "publish", "combine", "lp", "lp_calls", "tasks",
           "decisions")
 
 
