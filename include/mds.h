@@ -205,6 +205,26 @@ int mds_status(mds_ctx* ctx, const char** msg);
  * slice-dataflow engine, where every CTA works on every sequence's slices. */
 int mds_cluster_size(const mds_ctx* ctx);
 
+/* Softmax export for tests (Sec. 3: q = softmax of the target row, p = of a
+ * draft row, both at their temperatures, Sec. 5).  mds_debug_row_stats
+ * makes the context's later calls served by the slice-dataflow engine
+ * (single, WIS, WIS0; see mds_cluster_size) write, for every depth a
+ * sequence's walk visits with a statistics pass, the statistics the kernel
+ * derived for each row of that pass: `row_stats` is caller-owned device
+ * memory of max_B * (L + 1) * MDS_DEBUG_ROWS * 4 floats, laid out
+ * [b][j][r][4] = {M, 1/Z, c = log2(e) / T, source}, source = k for the target
+ * row of branch k (r = 0) and 100 + k for the draft row of branch k (r > 0);
+ * entries of depths and rows not visited are left untouched.  NULL turns it
+ * off.  The per-sequence engine (IS, SpecTr, cluster sizes > 0) writes
+ * nothing.  mds_debug_probs then writes, for one row of V logits of
+ * `dtype` in device memory, the probability the kernel assigns to every
+ * token under such statistics: out[x] = 2^(l_x c - M c) / Z, evaluated by the
+ * same device function as every probability on the verification path.
+ * Asynchronous on `stream`; MDS_EINVAL for bad arguments. */
+#define MDS_DEBUG_ROWS 4
+int mds_debug_row_stats(mds_ctx* ctx, float* row_stats);
+int mds_debug_probs(const void* row, int dtype, int V, float M, float invZ, float c, float* out, void* stream);
+
 /* Diagnostics of an instrumented build (compiled with MDS_PHASE_TIMERS; the
  * default build returns MDS_EUNSUP): synchronises device `device`, copies
  * up to n phase counters of the slice-dataflow engine (SM cycles summed over

@@ -32,6 +32,7 @@ struct mds_ctx {
   size_t f_bytes;
   unsigned epoch;
   int f_grid;
+  float* dbg_rows;         // test export of row statistics (caller-owned), or null
 };
 
 namespace {
@@ -252,6 +253,7 @@ int flow_verify(mds_ctx* ctx, const void* target_logits, const void* const* draf
   mds::flow_buffers(p, target_logits, draft_logits, draft_tokens, temperatures, out_tokens, out_accept_len, out_diag,
                     B, philox_seed);
   p.status = ctx->work;
+  p.dbg_rows = ctx->dbg_rows;
   ctx->epoch = (ctx->epoch + 1u == 0u) ? 1u : ctx->epoch + 1u;
   p.epoch = ctx->epoch;
   const cudaError_t le = mds::flow::launch(p, ctx->f_grid, static_cast<cudaStream_t>(stream));
@@ -461,6 +463,19 @@ int mds_status(mds_ctx* ctx, const char** msg) {
 }
 
 int mds_cluster_size(const mds_ctx* ctx) { return ctx ? ctx->last_cn : 0; }
+
+int mds_debug_row_stats(mds_ctx* ctx, float* row_stats) {
+  if (!ctx) return MDS_EINVAL;
+  ctx->dbg_rows = row_stats;
+  return MDS_OK;
+}
+
+int mds_debug_probs(const void* row, int dtype, int V, float M, float invZ, float c, float* out, void* stream) {
+  if (!row || !out || V <= 0 || (dtype != MDS_F32 && dtype != MDS_BF16)) return MDS_EINVAL;
+  const cudaError_t e = mds::flow::launch_probs(row, dtype, V, M, invZ, c, out, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "mds_debug_probs");
+  return MDS_OK;
+}
 
 int mds_phase_timers(int device, unsigned long long* cycles, int n) {
   if (!cycles || n < 0) return MDS_EINVAL;

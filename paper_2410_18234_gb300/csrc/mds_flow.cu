@@ -1777,6 +1777,28 @@ struct Dec {
     D.P.row[r].invZ = __frcp_rn(Z);
   }
 
+  // Test export: the statistics of the depth's rows (M, 1/Z, c, source:
+  // the target row's branch, or 100 + the branch whose draft row it is).
+  __device__ void debug_rows(int b, int j, int R) const {
+    for (int r = lane; r < R && r < MDS_DEBUG_ROWS; r += 32) {
+      int src = __ffs(D.W.valid) - 1;
+      if (r > 0) {
+        src = -1;
+        for (int i = 0; i < D.nv; ++i)
+          if (D.vrow[i] == r) {
+            src = 100 + D.vbr[i];
+            break;
+          }
+      }
+      float* o = p.dbg_rows + (((size_t)b * (p.L + 1) + j) * MDS_DEBUG_ROWS + r) * 4;
+      o[0] = D.P.row[r].M;
+      o[1] = D.P.row[r].invZ;
+      o[2] = D.P.row[r].c;
+      o[3] = (float)src;
+    }
+    __syncwarp();
+  }
+
   // The combined record of a stats pass (staged in scr; written by the CTA
   // that completed the pass): every row's M and 1/Z and, with candidate
   // lists, the sequence's list, its complement masses and tau.
@@ -1976,6 +1998,7 @@ struct Dec {
     PT_ADDW(kPhDecPlan, t_plan);
     PT_T0(t_comb);
     adopt_combined(R, list);
+    if (p.dbg_rows) debug_rows(b, j, R);
     xl_sync();
     PT_ADDW(kPhDecCombine, t_comb);
     if (p.scheme == MDS_WIS0) {
@@ -2459,6 +2482,13 @@ struct Dec {
       finish_row(0, Z);
     }
     __syncwarp();
+    if (p.dbg_rows && lane == 0) {
+      float* o = p.dbg_rows + (((size_t)b * (p.L + 1) + p.L) * MDS_DEBUG_ROWS) * 4;
+      o[0] = D.P.row[0].M;
+      o[1] = D.P.row[0].invZ;
+      o[2] = D.P.row[0].c;
+      o[3] = (float)(__ffs(D.W.valid) - 1);
+    }
     const float M = D.P.row[0].M, c = D.P.row[0].c, iz = D.P.row[0].invZ;
     for (int q = lane; q < p.ns; q += 32)
       Rs[q] = (Hm[q] > kNegInf) ? __fmul_rn(__fmul_rn(Rs[q], ref_shift(Hm[q], M, c)), iz) : 0.f;
@@ -3049,6 +3079,23 @@ bool plan_geometry(Params& p, int grid) {
   }
   p.dec_sms = decision_sms(grid);
   return p.dec_sms > 0;
+}
+
+// Every token's probability under given row statistics, by prob_of.
+template <int DT>
+__global__ void probs_kernel(const char* row, int V, float M, float invZ, float c, float* out) {
+  for (int x = blockIdx.x * blockDim.x + threadIdx.x; x < V; x += gridDim.x * blockDim.x)
+    out[x] = prob_of(Elt<DT>::global(row, x), M, c, invZ);
+}
+
+cudaError_t launch_probs(const void* row, int dtype, int V, float M, float invZ, float c, float* out,
+                         cudaStream_t stream) {
+  const int blocks = (V + 255) / 256 < 1024 ? (V + 255) / 256 : 1024;
+  if (dtype == MDS_BF16)
+    probs_kernel<MDS_BF16><<<blocks, 256, 0, stream>>>(static_cast<const char*>(row), V, M, invZ, c, out);
+  else
+    probs_kernel<MDS_F32><<<blocks, 256, 0, stream>>>(static_cast<const char*>(row), V, M, invZ, c, out);
+  return cudaGetLastError();
 }
 
 int grid_size(int device) {

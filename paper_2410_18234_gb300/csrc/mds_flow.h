@@ -45,6 +45,7 @@ struct Params {
   unsigned* cnt;                       // [B] slices of the current pass completed
   char* seq;                           // [B] per-sequence pass and walk state
   float* rec;                          // [B][ns][rec_floats] slice records
+  float* dbg_rows;                     // [B][L+1][MDS_DEBUG_ROWS][4] row statistics, or null
   unsigned long long seed;
   unsigned epoch;                      // launch number (tags of the ring)
   int B, K, L, V;
@@ -96,6 +97,10 @@ int read_phase_timers(unsigned long long* out, int n);
 
 // Launch on `stream` with `grid` CTAs.
 cudaError_t launch(const Params& p, int grid, cudaStream_t stream);
+
+// Every token's probability of one row under given statistics (test export).
+cudaError_t launch_probs(const void* row, int dtype, int V, float M, float invZ, float c, float* out,
+                         cudaStream_t stream);
 
 }  // namespace flow
 }  // namespace mds

@@ -34,7 +34,8 @@ MDS_MAX_OMEGA0 = 30
 
 # every symbol include/mds.h declares
 EXPORTS = ("mds_create", "mds_verify", "mds_verify_host", "mds_verify_noalloc", "mds_status",
-           "mds_cluster_size", "mds_phase_timers", "mds_error_string", "mds_destroy")
+           "mds_cluster_size", "mds_phase_timers", "mds_debug_row_stats", "mds_debug_probs", "mds_error_string",
+           "mds_destroy")
 
 
 class MdsConfig(ctypes.Structure):
@@ -72,6 +73,11 @@ def load_library(path=LIB_PATH):
     lib.mds_cluster_size.restype = ctypes.c_int
     lib.mds_phase_timers.argtypes = [ctypes.c_int, ctypes.POINTER(ctypes.c_uint64), ctypes.c_int]
     lib.mds_phase_timers.restype = ctypes.c_int
+    lib.mds_debug_row_stats.argtypes = [vp, vp]
+    lib.mds_debug_row_stats.restype = ctypes.c_int
+    lib.mds_debug_probs.argtypes = [vp, ctypes.c_int, ctypes.c_int, ctypes.c_float, ctypes.c_float, ctypes.c_float,
+                                    vp, vp]
+    lib.mds_debug_probs.restype = ctypes.c_int
     lib.mds_error_string.argtypes = [ctypes.c_int]
     lib.mds_error_string.restype = ctypes.c_char_p
     lib.mds_destroy.argtypes = [vp]
@@ -242,6 +248,37 @@ def mds_phase_timers(device=0):
     if rc < 0:
         raise MdsError(rc, "mds_phase_timers")
     return {name: int(buf[i]) for i, name in enumerate(PHASES[:rc])}
+
+
+DEBUG_ROWS = 4   # MDS_DEBUG_ROWS
+
+
+def mds_debug_row_stats(ctx, row_stats):
+    """Have the context's later dataflow-engine calls write every visited
+    row's statistics into row_stats (float32 CUDA tensor [max_B][L+1][4][4]:
+    M, 1/Z, c, source), or stop with None.  Test export."""
+    ptr = None if row_stats is None else ctypes.c_void_p(row_stats.data_ptr())
+    rc = _lib.mds_debug_row_stats(ctx, ptr)
+    if rc != MDS_OK:
+        raise MdsError(rc, "mds_debug_row_stats")
+
+
+def mds_debug_probs(row, M, invZ, c, out, stream=None):
+    """The kernel's probability of every token of one logit row (CUDA tensor
+    of V logits) under row statistics (M, 1/Z, c), into out (float32, V)."""
+    if not (row.is_cuda and out.is_cuda and row.is_contiguous() and out.is_contiguous()):
+        raise MdsError(MDS_EINVAL, "mds_debug_probs: contiguous CUDA tensors")
+    if out.dtype != torch.float32 or out.numel() != row.numel():
+        raise MdsError(MDS_EINVAL, "mds_debug_probs: out must be float32 of the row's length")
+    dt = {torch.float32: MDS_F32, torch.bfloat16: MDS_BF16}.get(row.dtype)
+    if dt is None:
+        raise MdsError(MDS_EINVAL, "mds_debug_probs: logits must be float32 or bfloat16")
+    if stream is None:
+        stream = torch.cuda.current_stream(row.device)
+    rc = _lib.mds_debug_probs(ctypes.c_void_p(row.data_ptr()), dt, int(row.numel()), float(M), float(invZ),
+                              float(c), ctypes.c_void_p(out.data_ptr()), ctypes.c_void_p(stream.cuda_stream))
+    if rc != MDS_OK:
+        raise MdsError(rc, "mds_debug_probs")
 
 
 def mds_destroy(ctx):
