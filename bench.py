@@ -35,6 +35,9 @@ sys.path.insert(0, ROOT)
 METRIC = "verified vocab-rows/sec and achieved HBM GB/s vs GB300 peak; oracle agreement"
 UNIT = "vocab-rows/s"
 DEFAULT_WORKLOAD = "llama3-128k"
+# ex2 (MUFU) throughput of the GPU: 152 SMs x 32 results per clock (GB300
+# doubles Blackwell's 16) x 2.07 GHz
+EX2_PEAK = 152 * 32 * 2.07e9
 FALLBACK_HBM = 6800.0
 
 
@@ -347,10 +350,16 @@ def table(args):
             mds.mds_verify(v.ctx, w.target, w.draft_list(), w.model_ids, w.tokens, w.temps, scheme,
                            spec.verify_seed, out_tokens, out_acc, None, stream)
 
+        # classical IS is bound by its quadrature's exponentials: the kernel
+        # counts them (nodes chosen on the device x V x draft rows)
+        exps = torch.zeros(1, dtype=torch.int64, device=dev) if scheme == "IS" else None
+
         for _ in range(args.warmup):
             flush.fill_(1.0)
             step()
         torch.cuda.synchronize()
+        if exps is not None:
+            mds.mds_debug_exp_count(v.ctx, exps)
         times = []
         for _ in range(args.steps):
             flush.fill_(1.0)
@@ -361,6 +370,13 @@ def table(args):
             torch.cuda.synchronize()
             times.append(a.elapsed_time(b))
         ms = float(np.median(times))
+        ex2 = None
+        if exps is not None:
+            mds.mds_debug_exp_count(v.ctx, None)
+            per_step = float(exps.item()) / args.steps
+            rate = per_step / (ms * 1e-3)
+            ex2 = {"exps_per_step": per_step, "ex2_per_s": rate, "peak": EX2_PEAK, "frac": rate / EX2_PEAK,
+                   "peak_kind": "derived: 152 SMs x 32 ex2/clk x 2.07 GHz"}
         tok = w.tokens.cpu().numpy()
         o_tok, o_acc = out_tokens.cpu().numpy(), out_acc.cpu().numpy()
         rows, abytes = walk_accounting(tok, w.model_ids, o_tok, o_acc, spec.V, es, scheme, args.omega0)
@@ -375,18 +391,21 @@ def table(args):
                 "rows_per_s": rows / (ms * 1e-3), "vocab_rows_per_step": rows, "gb_per_s": gbs,
                 "hbm_frac": gbs / peak, "peak": peak, "peak_kind": peak_kind, "kernel": kernel_name(scheme, cn),
                 "block_efficiency": float(np.mean(o_acc + 1)), "oracle_agreement": par,
-                "cpu_1core_rows_per_s": rate, "cpu_sample": desc, "status_bits": bits}
+                "cpu_1core_rows_per_s": rate, "cpu_sample": desc, "status_bits": bits, "ex2_roofline": ex2}
         print(json.dumps(line), flush=True)
         rows_md.append(line)
         del w
         torch.cuda.empty_cache()
     md = ["| workload | scheme | kernel | ms/step (median) | vocab-rows/s | GB/s | frac of measured HBM | "
-          "block eff. | oracle agreement (identical/band/mismatch of n) | oracle 1 core rows/s |",
-          "|---|---|---|---|---|---|---|---|---|---|"]
+          "ex2/s (frac of derived) | block eff. | oracle agreement (identical/band/mismatch of n) | "
+          "oracle 1 core rows/s |",
+          "|---|---|---|---|---|---|---|---|---|---|---|"]
     for r in rows_md:
         a = r["oracle_agreement"]
+        e = r["ex2_roofline"]
+        ex = f"{e['ex2_per_s'] / 1e12:.2f} T ({e['frac']:.3f})" if e else "-"
         md.append(f"| {r['workload']} | {r['scheme']} | {r['kernel']} | {r['ms_per_step']:.3f} | "
-                  f"{r['rows_per_s'] / 1e6:.2f}M | {r['gb_per_s']:.0f} | {r['hbm_frac']:.3f} | "
+                  f"{r['rows_per_s'] / 1e6:.2f}M | {r['gb_per_s']:.0f} | {r['hbm_frac']:.3f} | {ex} | "
                   f"{r['block_efficiency']:.2f} | {a['identical']}/{a['band']}/{a['mismatch']} of {a['sequences']} | "
                   f"{r['cpu_1core_rows_per_s']:.1f} |")
     text = "\n".join(md)

@@ -223,6 +223,14 @@ int mds_cluster_size(const mds_ctx* ctx);
  * Asynchronous on `stream`; MDS_EINVAL for bad arguments. */
 #define MDS_DEBUG_ROWS 4
 int mds_debug_row_stats(mds_ctx* ctx, float* row_stats);
+
+/* Measurement export for classical IS (Sec. 3, the law p_I of the selected
+ * token by the quadrature of its Laplace identity): mds_debug_exp_count
+ * makes the context's later IS calls add to *counter (caller-owned device
+ * memory, one unsigned 64-bit word) the exponentials of their quadrature
+ * node sums, nodes x V x draft rows per visited depth and per residual draw,
+ * with the node count each depth chose on the device.  NULL turns it off. */
+int mds_debug_exp_count(mds_ctx* ctx, unsigned long long* counter);
 int mds_debug_probs(const void* row, int dtype, int V, float M, float invZ, float c, float* out, void* stream);
 
 /* Diagnostics of an instrumented build (compiled with MDS_PHASE_TIMERS; the

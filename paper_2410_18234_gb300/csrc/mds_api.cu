@@ -33,6 +33,7 @@ struct mds_ctx {
   unsigned epoch;
   int f_grid;
   float* dbg_rows;         // test export of row statistics (caller-owned), or null
+  unsigned long long* dbg_exps;   // count of IS quadrature exponentials (caller-owned), or null
 };
 
 namespace {
@@ -311,6 +312,7 @@ static int verify_impl(mds_ctx* ctx, const void* target_logits, const void* cons
   p.out_diag = out_diag;
   p.status = ctx->work;
   p.queue = ctx->work + 1;
+  p.dbg_exps = ctx->dbg_exps;
   p.seed = philox_seed;
   p.B = B;
   p.K = c.K;
@@ -467,6 +469,12 @@ int mds_cluster_size(const mds_ctx* ctx) { return ctx ? ctx->last_cn : 0; }
 int mds_debug_row_stats(mds_ctx* ctx, float* row_stats) {
   if (!ctx) return MDS_EINVAL;
   ctx->dbg_rows = row_stats;
+  return MDS_OK;
+}
+
+int mds_debug_exp_count(mds_ctx* ctx, unsigned long long* counter) {
+  if (!ctx) return MDS_EINVAL;
+  ctx->dbg_exps = counter;
   return MDS_OK;
 }
 

@@ -46,6 +46,7 @@ struct Params {
   int bulk_ok;                         // rows may be read with bulk copies (device memory, not mapped host memory)
   int cand_cap;                        // WIS candidate list capacity (kListN; 0: no candidate path)
   int cand_stage;                      // WIS staging capacity (every CTA's list: cn * kListN)
+  unsigned long long* dbg_exps;        // IS: quadrature exponentials evaluated (test export), or null
   int8_t model_of[MDS_MAX_K];          // remapped model id per branch
 };
 

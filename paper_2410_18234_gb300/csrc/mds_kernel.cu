@@ -2104,6 +2104,12 @@ struct Kernel {
       if (mhi - mlo + 1 > kIsNodesMax) mhi = mlo + kIsNodesMax - 1;
       S.is_mlo = mlo;
       S.is_n = mhi - mlo + 1;
+      if (p.dbg_exps && rank == 0) {
+        // the node sums below: one exponential per node, token and draft row
+        int rows = 0;
+        for (int r = 1; r < S.nrows; ++r) rows += S.is_cnt[r] ? 1 : 0;
+        atomicAdd(p.dbg_exps, (unsigned long long)S.is_n * (unsigned long long)p.V * (unsigned long long)rows);
+      }
     }
     __syncthreads();
     const int nn = S.is_n;
@@ -2603,8 +2609,14 @@ struct Kernel {
           if constexpr (SCHEME == MDS_IS) {
             if (S.nv > 1) {
               uint32_t mask = 1u;
+              int rows = 0;
               for (int r = 1; r < S.nrows; ++r)
-                if (S.is_cnt[r]) mask |= 1u << r;
+                if (S.is_cnt[r]) {
+                  mask |= 1u << r;
+                  ++rows;
+                }
+              if (p.dbg_exps && rank == 0 && tid == 0)   // p_I at every token: one exponential per node and row
+                atomicAdd(p.dbg_exps, (unsigned long long)S.is_n * (unsigned long long)p.V * (unsigned long long)rows);
               Z = sample_cdf(mask, [&](int, const auto& L, float* r) { residual_is(L, r); }, ures, &tot);
               done = true;
             }

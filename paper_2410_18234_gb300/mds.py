@@ -34,8 +34,8 @@ MDS_MAX_OMEGA0 = 30
 
 # every symbol include/mds.h declares
 EXPORTS = ("mds_create", "mds_verify", "mds_verify_host", "mds_verify_noalloc", "mds_status",
-           "mds_cluster_size", "mds_phase_timers", "mds_debug_row_stats", "mds_debug_probs", "mds_error_string",
-           "mds_destroy")
+           "mds_cluster_size", "mds_phase_timers", "mds_debug_row_stats", "mds_debug_exp_count", "mds_debug_probs",
+           "mds_error_string", "mds_destroy")
 
 
 class MdsConfig(ctypes.Structure):
@@ -75,6 +75,8 @@ def load_library(path=LIB_PATH):
     lib.mds_phase_timers.restype = ctypes.c_int
     lib.mds_debug_row_stats.argtypes = [vp, vp]
     lib.mds_debug_row_stats.restype = ctypes.c_int
+    lib.mds_debug_exp_count.argtypes = [vp, vp]
+    lib.mds_debug_exp_count.restype = ctypes.c_int
     lib.mds_debug_probs.argtypes = [vp, ctypes.c_int, ctypes.c_int, ctypes.c_float, ctypes.c_float, ctypes.c_float,
                                     vp, vp]
     lib.mds_debug_probs.restype = ctypes.c_int
@@ -261,6 +263,15 @@ def mds_debug_row_stats(ctx, row_stats):
     rc = _lib.mds_debug_row_stats(ctx, ptr)
     if rc != MDS_OK:
         raise MdsError(rc, "mds_debug_row_stats")
+
+
+def mds_debug_exp_count(ctx, counter):
+    """Have the context's later IS calls add their quadrature exponentials to
+    counter (int64 CUDA tensor of one element), or stop with None."""
+    ptr = None if counter is None else ctypes.c_void_p(counter.data_ptr())
+    rc = _lib.mds_debug_exp_count(ctx, ptr)
+    if rc != MDS_OK:
+        raise MdsError(rc, "mds_debug_exp_count")
 
 
 def mds_debug_probs(row, M, invZ, c, out, stream=None):
