@@ -112,7 +112,10 @@ typedef struct {
                       acceptance probability (Theorem 1's objective for the
                       depth's draft laws); costs one more pass over the rows
                       at accepted depths.  0: R only after a rejection (0 when
-                      accepted).  Used by MDS_SINGLE, MDS_IS and MDS_WIS.     */
+                      accepted).  Used by MDS_SINGLE, MDS_IS and MDS_WIS; for
+                      MDS_SPECTR out_diag[b][j][2] is prod_i R_i, the
+                      probability that every round rejects (with 1 the rounds
+                      after an acceptance are computed too).                  */
 } mds_config;
 
 /* Create a context on CUDA device `device`.  Allocates the context's device

@@ -2758,11 +2758,19 @@ struct Kernel {
   }
 
   // Sequential rejection over the valid drafts (baseline).  Returns Z.
+  // *Rd: the product of the rounds' residual masses, the probability that
+  // every round rejects (1 - the depth's acceptance probability); with
+  // acc_prob the rounds after an acceptance are computed for it too, without
+  // changing the token.
   __device__ int spectr(int b, int j, float* qY, float* pIY, int* Yd, float* Rd) {
     const int nv = S.nv;
+    int zacc = -1;
+    float prodR = 1.f;
     for (int i = 0; i < nv; ++i) {
-      // point value of the running target at X_i
-      if (threadIdx.x == 0) {
+      // point value of the running target at X_i (the accept test, until a
+      // round accepts)
+      if (threadIdx.x == 0) S.sp_rows[i] = S.vrow[i];
+      if (threadIdx.x == 0 && zacc < 0) {
         const int x = S.X[i];
         float qi = prob_row(0, x);
         for (int k = 0; k < i; ++k) {
@@ -2777,16 +2785,18 @@ struct Kernel {
           S.pIY = pv;
         }
         S.accepted = (u < fminf(1.f, ratio)) ? 1 : 0;
-        S.sp_rows[i] = S.vrow[i];
       }
       __syncthreads();
       *qY = S.qY;
       *pIY = S.pIY;
       *Yd = S.X[0];
-      if (S.accepted) {
-        const int z = S.X[i];
-        __syncthreads();
-        return z;
+      if (zacc < 0 && S.accepted) {
+        zacc = S.X[i];
+        if (!p.acc_prob) {
+          __syncthreads();
+          *Rd = 0.f;
+          return zacc;
+        }
       }
       // residual mass of this round
       float part = 0.f;
@@ -2816,15 +2826,19 @@ struct Kernel {
         float R = 0.f;
         for (int q = 0; q < cn; ++q) R = __fadd_rn(R, S.gat[q]);
         S.sp_invR[i] = R > 0.f ? __frcp_rn(R) : 0.f;
+        S.red[kWarps] = R;
       }
       __syncthreads();
+      prodR = __fmul_rn(prodR, S.red[kWarps]);
+      __syncthreads();
     }
+    *Rd = prodR;
+    if (zacc >= 0) return zacc;
     float tot;
     uint32_t mask = 1u;
     for (int k = 0; k < nv; ++k) mask |= 1u << S.sp_rows[k];
     const int z = sample_cdf(mask, [&](int, const auto& L, float* r) { spectr_target(L, nv, r); },
                              draw_uniform(p.seed, b, j, kDrawResidual), &tot);
-    *Rd = tot;
     return z;
   }
 

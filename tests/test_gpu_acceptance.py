@@ -81,3 +81,37 @@ def test_full_size_sampled():
                 break
             assert abs(diag[b, r.j, 2] - r.R) <= R_ATOL["WIS"]
 
+
+
+@pytest.mark.parametrize("name,kw,cluster", [
+    ("two-models-50k", dict(B=8, V=7001), 0),
+    ("llama2-32k", dict(B=8, V=5003), 0),
+    ("serving-152k", dict(B=6, V=6007, L=4), 2),
+], ids=lambda x: x if isinstance(x, str) else "")
+def test_spectr_rejection_probability(name, kw, cluster):
+    # The sequential-rejection reading: out_diag[b][j][2] = prod_i R_i, the
+    # probability that every round rejects, at every visited depth below L
+    # (the rounds after an acceptance computed too), against the oracle's
+    # analytic 1 - acceptance on the same rows; tokens unchanged.
+    from oracle.acceptance import scheme_acceptance
+    from oracle.verify import softmax_t
+    spec = WORKLOADS[name].with_(**kw)
+    w, out, acc, diag = run(spec, "SpecTr", 5, acc_prob=1, cluster=cluster)
+    _, out0, acc0, _ = run(spec, "SpecTr", 5, acc_prob=0, cluster=cluster)
+    np.testing.assert_array_equal(out, out0)
+    np.testing.assert_array_equal(acc, acc0)
+    target, drafts, mids, tokens, temps = host_copy(w)
+    checked = 0
+    for b in range(spec.B):
+        valid = list(range(spec.K))
+        for j in range(min(int(acc[b]) + 1, spec.L)):
+            k0 = valid[0]
+            q = softmax_t(target[b, k0, j], temps[b, 0])
+            dists = [softmax_t(drafts[k][b, j], temps[b, 1 + k]) for k in valid]
+            R = 1.0 - scheme_acceptance(q, dists, [mids[k] for k in valid], "SpecTr")
+            assert abs(diag[b, j, 2] - R) <= 2e-5 * len(valid), (b, j, float(diag[b, j, 2]), R)
+            checked += 1
+            valid = [k for k in valid if tokens[b, k, j] == out[b, j]]
+            if not valid:
+                break
+    assert checked >= spec.B
