@@ -66,7 +66,8 @@ extern "C" {
 #define MDS_MAX_L 64      /* draft positions per branch                     */
 #define MDS_MAX_S 8       /* LP truncation threshold s (|Omega_1|)          */
 #define MDS_MAX_IS_MODELS 4  /* distinct draft models for plain IS          */
-#define MDS_MAX_OMEGA0 30 /* |Omega_0| of the truncated alphabet, MDS_WIS0  */
+#define MDS_MAX_OMEGA0 62 /* |Omega_0| of the truncated alphabet, MDS_WIS0  */
+#define MDS_MAX_OMEGA0_CLUSTER 30 /* ... with a cluster size set (per-sequence engine) */
 
 typedef struct mds_ctx mds_ctx;
 
@@ -105,7 +106,11 @@ typedef struct {
   int cluster;     /* CTAs per sequence: 1, 2, 4, 8 or 16 (0: chosen from max_B and the device) */
   int omega0;      /* |Omega_0| for MDS_WIS0, 1..MDS_MAX_OMEGA0 (0: 20; the paper's
                       runs use 10 to 50, Section 5, Table "Effect of LP
-                      Truncation and Alphabet Truncation")                    */
+                      Truncation and Alphabet Truncation").  Sizes above
+                      MDS_MAX_OMEGA0_CLUSTER run on the slice-dataflow engine
+                      only: an MDS_WIS0 call that engine does not serve (a
+                      cluster size set, see mds_cluster_size) returns
+                      MDS_EUNSUP.                                             */
   int acc_prob;    /* 1: out_diag[b][j][2] holds the residual mass R = sum_k
                       max(0, q_k - p_I(k)) at every visited depth below L, so
                       that 1 - R = sum_k min(q_k, p_I(k)) is the depth's

@@ -301,6 +301,8 @@ static int verify_impl(mds_ctx* ctx, const void* target_logits, const void* cons
                                 scheme, philox_seed, out_tokens, out_accept_len, out_diag, B, stream, bulk_ok, tma_ok);
     if (frc != mds::kNotServed) return frc;
   }
+  // the per-sequence engine's list holds 32 entries: |Omega_0| <= 30 there
+  if (scheme == MDS_WIS0 && c.omega0 > MDS_MAX_OMEGA0_CLUSTER) return MDS_EUNSUP;
   p.dtype = c.dtype;
   int rc = geometry(ctx, scheme, n_models, p);
   if (rc != MDS_OK) return rc;

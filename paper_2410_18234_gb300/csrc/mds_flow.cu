@@ -2515,19 +2515,34 @@ struct Dec {
   // order of the list): the smallest lane whose running sum exceeds
   // u * total, the last lane with positive weight if rounding leaves none,
   // -1 if the total is not positive.
-  __device__ __forceinline__ int lane_cdf(float w, float u01, float* total) const {
-    float c = w;
+  // Inverse CDF over the list entries in token order, two per lane (entry
+  // lane and 32 + lane; weights w0, w1): the first entry whose running sum
+  // exceeds u01 * total, else the last with positive weight; -1 when the
+  // total is 0.  Sums: a warp scan of each half, the halves in order.
+  __device__ __forceinline__ int lane_cdf2(float w0, float w1, float u01, float* total) const {
+    float c0 = w0, c1 = w1;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
-      const float t = __shfl_up_sync(FULLM, c, o);
-      if (lane >= o) c = __fadd_rn(c, t);
+      const float t0 = __shfl_up_sync(FULLM, c0, o);
+      const float t1 = __shfl_up_sync(FULLM, c1, o);
+      if (lane >= o) {
+        c0 = __fadd_rn(c0, t0);
+        c1 = __fadd_rn(c1, t1);
+      }
     }
-    const float tot = __shfl_sync(FULLM, c, 31);
+    const float h0 = __shfl_sync(FULLM, c0, 31);
+    c1 = __fadd_rn(h0, c1);
+    const float tot = __shfl_sync(FULLM, c1, 31);
     *total = tot;
     if (!(tot > 0.f)) return -1;
-    const unsigned who = __ballot_sync(FULLM, c > __fmul_rn(u01, tot));
-    if (who) return __ffs(who) - 1;
-    return 31 - __clz(__ballot_sync(FULLM, w > 0.f));
+    const float T = __fmul_rn(u01, tot);
+    const unsigned who0 = __ballot_sync(FULLM, c0 > T);
+    if (who0) return __ffs(who0) - 1;
+    const unsigned who1 = __ballot_sync(FULLM, c1 > T);
+    if (who1) return 32 + __ffs(who1) - 1;
+    const unsigned p1 = __ballot_sync(FULLM, w1 > 0.f);
+    if (p1) return 32 + 31 - __clz(p1);
+    return 31 - __clz(__ballot_sync(FULLM, w0 > 0.f));
   }
 
   // One depth of the truncated-alphabet scheme (Section 4, read with the
@@ -2535,23 +2550,33 @@ struct Dec {
   // Omega_0 = the target tokens above the (M+1)-th largest target logit, read
   // off the candidate list (exact when the list's (M+1)-th entry is >= tau,
   // the list holds the whole vocabulary, or every token outside it is -inf;
-  // otherwise the tokens above tau, with MDS_ST_OMEGA0).  Warp 0 runs the
+  // otherwise the tokens above tau, with MDS_ST_OMEGA0).  The warp runs the
   // WIS stages on Omega_0 against q~ = q / p_a with the kept inputs' draft
   // laws restricted to Omega_0 and renormalised (point loads of the draft
   // logits there), then Algorithm 1 against q~.  Y' is kept with probability
   // p_a, else a replace pass draws from the tokens outside Omega_0 by q.
+  // The list (token-id order, up to 64 entries) sits two entries per lane:
+  // entry lane (half 0) and 32 + lane (half 1).
   __device__ void wis0_decide(int b) {
     const int j = D.P.j;
     {
       const int n = D.n;
-      const bool have = lane < n;
-      const int id = have ? D.cm_id[lane] : 0;
-      const float l = have ? D.cm_l0[lane] : kNegInf;
-      int rk = 0;   // rank in the list by (larger logit, then lower id)
-      for (int t = 0; t < 32; ++t) {
-        const float lt = __shfl_sync(FULLM, l, t);
-        const int it = __shfl_sync(FULLM, id, t);
-        rk += (t < n && better(lt, it, l, id)) ? 1 : 0;
+      bool have[2], in0[2];
+      int id[2], rk[2] = {0, 0};
+      float l[2], q[2], qt[2];
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int e = lane + 32 * h;
+        have[h] = e < n;
+        id[h] = have[h] ? D.cm_id[e] : 0;
+        l[h] = have[h] ? D.cm_l0[e] : kNegInf;
+      }
+      // rank in the list by (larger logit, then lower id)
+      for (int t = 0; t < n; ++t) {
+        const float lt = D.cm_l0[t];
+        const int it = D.cm_id[t];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) rk[h] += better(lt, it, l[h], id[h]) ? 1 : 0;
       }
       const int M = p.omega0;
       const bool all0 = M >= p.V;
@@ -2560,51 +2585,54 @@ struct Dec {
       if (all0) {
         cert = D.cand_all != 0;
       } else {
-        const unsigned who = __ballot_sync(FULLM, have && rk == M);
-        if (who) cut = __shfl_sync(FULLM, l, __ffs(who) - 1);
+        const unsigned w0 = __ballot_sync(FULLM, have[0] && rk[0] == M);
+        const unsigned w1 = __ballot_sync(FULLM, have[1] && rk[1] == M);
+        const bool found = (w0 | w1) != 0u;
+        if (w0)
+          cut = __shfl_sync(FULLM, l[0], __ffs(w0) - 1);
+        else if (w1)
+          cut = __shfl_sync(FULLM, l[1], __ffs(w1) - 1);
         const float tau = D.cand_tau;
-        cert = D.cand_all || (who ? cut >= tau : !(tau > kNegInf));
+        cert = D.cand_all || (found ? cut >= tau : !(tau > kNegInf));
         if (!cert) cut = fmaxf(cut, tau);
       }
-      const bool in0 = have && (all0 || l > cut);
-      const int n0 = __popc(__ballot_sync(FULLM, in0));
-      const float q = in0 ? prob_of(l, D.P.row[0].M, D.P.row[0].c, D.P.row[0].invZ) : 0.f;
-      const float pa = warp_sum(q);
-      const float qt = (in0 && pa > 0.f) ? __fdiv_rn(q, pa) : 0.f;
-      // draft laws restricted to Omega_0 (exponents against their own maximum
-      // there; the rows' full normalisers cancel)
-      float ew[MDS_MAX_K];
 #pragma unroll
-      for (int k = 0; k < MDS_MAX_K; ++k) ew[k] = 0.f;
-      for (int r = 1; r < D.P.nrows; ++r) {
-        const float lr = in0 ? E::global(D.P.row[r].ptr, id) : kNegInf;
-        const float ref = warp_max(lr);
-        const float cr = D.P.row[r].c;
-        const float e = (in0 && ref > kNegInf) ? exp_term(lr, ref, cr) : 0.f;
-        const float Pm = warp_sum(e);
-        if (lane == 0 && Pm != Pm) atomicOr(p.status, MDS_ST_NONFINITE);
-        const float lw = (Pm > 0.f) ? __fdiv_rn(e, Pm) : 0.f;
-#pragma unroll
-        for (int k = 0; k < MDS_MAX_K; ++k)
-          if (k == r - 1) ew[k] = lw;
+      for (int h = 0; h < 2; ++h) {
+        in0[h] = have[h] && (all0 || l[h] > cut);
+        q[h] = in0[h] ? prob_of(l[h], D.P.row[0].M, D.P.row[0].c, D.P.row[0].invZ) : 0.f;
       }
-      auto law = [&](int r) -> float {
-        float v = 0.f;
+      const int n0 = __popc(__ballot_sync(FULLM, in0[0])) + __popc(__ballot_sync(FULLM, in0[1]));
+      const float pa = warp_sum(__fadd_rn(q[0], q[1]));
 #pragma unroll
-        for (int k = 0; k < MDS_MAX_K; ++k)
-          if (k == r - 1) v = ew[k];
-        return v;
-      };
+      for (int h = 0; h < 2; ++h) qt[h] = (in0[h] && pa > 0.f) ? __fdiv_rn(q[h], pa) : 0.f;
+      // draft laws restricted to Omega_0 (exponents against their own maximum
+      // there; the rows' full normalisers cancel), per row and entry, in the
+      // warp's scratch (the staged records are spent)
+      float* ew = reinterpret_cast<float*>(scr);   // [nrows][64]
+      for (int r = 1; r < D.P.nrows; ++r) {
+        float lr[2], e[2];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) lr[h] = in0[h] ? E::global(D.P.row[r].ptr, id[h]) : kNegInf;
+        const float ref = warp_max(fmaxf(lr[0], lr[1]));
+        const float cr = D.P.row[r].c;
+#pragma unroll
+        for (int h = 0; h < 2; ++h) e[h] = (in0[h] && ref > kNegInf) ? exp_term(lr[h], ref, cr) : 0.f;
+        const float Pm = warp_sum(__fadd_rn(e[0], e[1]));
+        if (lane == 0 && Pm != Pm) atomicOr(p.status, MDS_ST_NONFINITE);
+#pragma unroll
+        for (int h = 0; h < 2; ++h) ew[r * 64 + lane + 32 * h] = (Pm > 0.f) ? __fdiv_rn(e[h], Pm) : 0.f;
+      }
+      __syncwarp();
       // kept inputs: valid branches (branch order) whose token lies in Omega_0
       int nk = 0;
       for (int i = 0; i < D.nv; ++i) {
-        const unsigned w = __ballot_sync(FULLM, in0 && id == D.X[i]);
-        if (!w) continue;
-        const int li = __ffs(w) - 1;
-        const float lv = __shfl_sync(FULLM, law(D.vrow[i]), li);
-        if (!(lv > 0.f)) continue;   // impossible draw: dropped
+        const unsigned w0 = __ballot_sync(FULLM, in0[0] && id[0] == D.X[i]);
+        const unsigned w1 = __ballot_sync(FULLM, in0[1] && id[1] == D.X[i]);
+        if (!(w0 | w1)) continue;
+        const int ei = w0 ? __ffs(w0) - 1 : 32 + __ffs(w1) - 1;
+        if (!(ew[D.vrow[i] * 64 + ei] > 0.f)) continue;   // impossible draw: dropped
         if (lane == 0) {
-          D.k_lane[nk] = li;
+          D.k_lane[nk] = ei;
           D.k_row[nk] = D.vrow[i];
         }
         ++nk;
@@ -2614,63 +2642,89 @@ struct Dec {
       float qY = 0.f, pIY = 0.f, R = 0.f;
       if (n0 > 0 && nk == 0) {
         float t;
-        yl = lane_cdf(qt, draw_uniform(p.seed, b, j, kDrawResidual), &t);
+        yl = lane_cdf2(qt[0], qt[1], draw_uniform(p.seed, b, j, kDrawResidual), &t);
       } else if (n0 > 0) {
-        float a = law(D.k_row[0]);
+        float a[2];
+        {
+          const float* w = ew + D.k_row[0] * 64;
+          a[0] = w[lane];
+          a[1] = w[lane + 32];
+        }
         int A = D.k_lane[0];
         const int s = min(p.wis_s, n0);
+        const unsigned lt = (1u << lane) - 1u;
         for (int m = 1; m < nk; ++m) {
           const int Bl = D.k_lane[m];
-          const float bb = law(D.k_row[m]);
+          const float* wb = ew + D.k_row[m] * 64;
+          const float bb[2] = {wb[lane], wb[lane + 32]};
           const float u = draw_uniform(p.seed, b, j, kDrawSelect + m - 1);
-          unsigned kk = in0 ? ord_key(__fadd_rn(__fmaf_rn(-a, bb, qt), 0.f)) : 0u;
-          uint32_t selm = 0u;
+          unsigned kk[2];
+#pragma unroll
+          for (int h = 0; h < 2; ++h) kk[h] = in0[h] ? ord_key(__fadd_rn(__fmaf_rn(-a[h], bb[h], qt[h]), 0.f)) : 0u;
+          // Omega_1: s rounds of the largest key, ties to the smaller id
+          // (the lower entry)
+          uint32_t sel0 = 0u, sel1 = 0u;
           for (int t = 0; t < s; ++t) {
-            const unsigned km = __reduce_max_sync(FULLM, kk);
-            const uint32_t who = __ballot_sync(FULLM, km != 0u && kk == km);
-            if (!who) break;
-            const int wl = __ffs(who) - 1;
-            selm |= 1u << wl;
-            if (lane == wl) kk = 0u;
+            const unsigned km = __reduce_max_sync(FULLM, max(kk[0], kk[1]));
+            if (!km) break;
+            const uint32_t w0 = __ballot_sync(FULLM, kk[0] == km);
+            if (w0) {
+              const int wl = __ffs(w0) - 1;
+              sel0 |= 1u << wl;
+              if (lane == wl) kk[0] = 0u;
+            } else {
+              const int wl = __ffs(__ballot_sync(FULLM, kk[1] == km)) - 1;
+              sel1 |= 1u << wl;
+              if (lane == wl) kk[1] = 0u;
+            }
           }
-          const bool sel = (selm >> lane) & 1u;
-          const int sn = __popc(selm);
-          const float A2 = warp_sum((in0 && !sel) ? a : 0.f);
-          const float B2 = warp_sum((in0 && !sel) ? bb : 0.f);
-          const int rk1 = __popc(selm & ((1u << lane) - 1u));
+          const bool sl[2] = {((sel0 >> lane) & 1u) != 0u, ((sel1 >> lane) & 1u) != 0u};
+          const int sn = __popc(sel0) + __popc(sel1);
+          const float A2 = warp_sum(__fadd_rn((in0[0] && !sl[0]) ? a[0] : 0.f, (in0[1] && !sl[1]) ? a[1] : 0.f));
+          const float B2 = warp_sum(__fadd_rn((in0[0] && !sl[0]) ? bb[0] : 0.f, (in0[1] && !sl[1]) ? bb[1] : 0.f));
+          const int rk1[2] = {__popc(sel0 & lt), __popc(sel0) + __popc(sel1 & lt)};
           if (lane >= sn && lane < MDS_MAX_S) {
             D.om[lane] = -1;
             D.om_q[lane] = 0.f;
             D.om_a[lane] = 0.f;
             D.om_b[lane] = 0.f;
           }
-          if (sel) {
-            D.om[rk1] = id;
-            D.om_q[rk1] = qt;
-            D.om_a[rk1] = a;
-            D.om_b[rk1] = bb;
-          }
+#pragma unroll
+          for (int h = 0; h < 2; ++h)
+            if (sl[h]) {
+              D.om[rk1[h]] = id[h];
+              D.om_q[rk1[h]] = qt[h];
+              D.om_a[rk1[h]] = a[h];
+              D.om_b[rk1[h]] = bb[h];
+            }
           __syncwarp();
           if (lane == 0) D.Y = solve(sn, A2, B2, D.cm_id[A], D.cm_id[Bl], u);
           __syncwarp();
           const int Yt = D.Y;
-          A = max(0, __ffs(__ballot_sync(FULLM, in0 && id == Yt)) - 1);
-          a = sel ? D.om_x[rk1] : (in0 ? __fmul_rn(0.5f, __fadd_rn(__fmul_rn(a, B2), __fmul_rn(bb, A2))) : 0.f);
+          const unsigned y0 = __ballot_sync(FULLM, in0[0] && id[0] == Yt);
+          const unsigned y1 = __ballot_sync(FULLM, in0[1] && id[1] == Yt);
+          A = y0 ? __ffs(y0) - 1 : (y1 ? 32 + __ffs(y1) - 1 : 0);
+#pragma unroll
+          for (int h = 0; h < 2; ++h)
+            a[h] = sl[h] ? D.om_x[rk1[h]]
+                         : (in0[h] ? __fmul_rn(0.5f, __fadd_rn(__fmul_rn(a[h], B2), __fmul_rn(bb[h], A2))) : 0.f);
           __syncwarp();
         }
         Yl = A;
-        qY = __shfl_sync(FULLM, qt, A);
-        pIY = __shfl_sync(FULLM, a, A);
+        const int Ah = A >> 5, Alane = A & 31;
+        qY = __shfl_sync(FULLM, Ah ? qt[1] : qt[0], Alane);
+        pIY = __shfl_sync(FULLM, Ah ? a[1] : a[0], Alane);
         const float ratio = pIY > 0.f ? __fdiv_rn(qY, pIY) : kPosInf;
         if (draw_uniform(p.seed, b, j, kDrawAccept) < fminf(1.f, ratio)) {
           yl = A;
         } else {
           const float ures = draw_uniform(p.seed, b, j, kDrawResidual);
-          yl = lane_cdf(in0 ? fmaxf(0.f, __fsub_rn(qt, a)) : 0.f, ures, &R);
+          yl = lane_cdf2(in0[0] ? fmaxf(0.f, __fsub_rn(qt[0], a[0])) : 0.f,
+                         in0[1] ? fmaxf(0.f, __fsub_rn(qt[1], a[1])) : 0.f, ures, &R);
           if (yl < 0) {   // only by rounding: sample q~
             if (lane == 0) atomicOr(p.status, MDS_ST_ZERO_RESID);
             float t;
-            yl = lane_cdf(qt, ures, &t);
+            yl = lane_cdf2(qt[0], qt[1], ures, &t);
           }
         }
       }
@@ -3071,11 +3125,12 @@ bool plan_geometry(Params& p, int grid) {
     }
     int rf = kHdr + p.lns * (1 + lrows);
     if (rf < 4 + 4 * kTopF) rf = 4 + 4 * kTopF;
+    // the combined record of a pass is written over the pass's records
+    const int cmb = (kCmbHdr + p.ln * (2 + lrows) + ns - 1) / ns;
+    if (rf < cmb) rf = cmb;
     p.rec_floats = (rf + 3) & ~3;
     p.hdr_floats = kHdr;
-    if ((size_t)ns * p.rec_floats * 4 <= (size_t)kDecStage && ns * p.lns <= kMaxEntries &&
-        kCmbHdr + p.ln * (2 + lrows) <= ns * p.rec_floats)
-      break;
+    if ((size_t)ns * p.rec_floats * 4 <= (size_t)kDecStage && ns * p.lns <= kMaxEntries) break;
   }
   p.dec_sms = decision_sms(grid);
   return p.dec_sms > 0;

@@ -135,6 +135,7 @@ extern "C" int mds_verify_noalloc(const mds_config* cfg_in, int device, const vo
     }
   }
   p.dtype = c.dtype;
+  if (rc == MDS_OK && scheme == MDS_WIS0 && c.omega0 > MDS_MAX_OMEGA0_CLUSTER) rc = MDS_EUNSUP;
   if (rc == MDS_OK) rc = mds::launch_geometry(c, device, scheme, n_models, p);
   if (rc == MDS_OK) {
     p.target = static_cast<const char*>(target_logits);

@@ -30,7 +30,8 @@ MDS_ST_NONFINITE, MDS_ST_BADTEMP, MDS_ST_ZERO_RESID, MDS_ST_TIMEOUT, MDS_ST_LP_C
     1, 2, 4, 8, 16, 32
 MDS_ST_OMEGA0 = 64
 MDS_MAX_K = 16
-MDS_MAX_OMEGA0 = 30
+MDS_MAX_OMEGA0 = 62
+MDS_MAX_OMEGA0_CLUSTER = 30   # with a cluster size set (the per-sequence engine)
 
 # every symbol include/mds.h declares
 EXPORTS = ("mds_create", "mds_verify", "mds_verify_host", "mds_verify_noalloc", "mds_status",

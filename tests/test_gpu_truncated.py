@@ -42,6 +42,36 @@ def test_largest_omega0_on_f32_rows():
     # f32 logits have no ties, so the cut of the largest Omega_0 is certified
     spec = small("tiny", B=8, V=5000)
     ok(run_both(spec, "WIS0", seed=3, omega0=mds.MDS_MAX_OMEGA0))
+    ok(run_both(spec, "WIS0", seed=4, omega0=mds.MDS_MAX_OMEGA0_CLUSTER, cluster=2))
+
+
+@pytest.mark.parametrize("name,kw", [
+    ("llama3-128k", dict(B=12, V=9000)),
+    ("two-models-50k", dict(B=12, V=7001, dtype="f32")),
+    ("serving-152k", dict(B=10, V=6007, L=4)),
+], ids=lambda x: x if isinstance(x, str) else "")
+def test_paper_omega0_sizes(name, kw):
+    # |Omega_0| = 40 and 50 (Section 5's runs) and the largest size: a
+    # 64-entry list, two entries per lane of the decision warp (bf16 ties at
+    # the cut may leave it uncertified)
+    spec = small(name, **kw)
+    for M in (31, 40, 50, mds.MDS_MAX_OMEGA0):
+        ok(run_both(spec, "WIS0", seed=M, omega0=M), allow_uncertified=(spec.dtype == "bf16"))
+
+
+def test_large_omega0_needs_the_dataflow_engine():
+    # the per-sequence engine's list holds 32 entries: a cluster size with
+    # |Omega_0| above 30 is refused before any launch
+    spec = small("tiny", B=4, V=3000)
+    from synth import make_workload
+    w = make_workload(spec, device="cuda:0")
+    v = mds.Verifier(spec.B, spec.K, spec.L, spec.V, dtype=spec.dtype, cluster=2, omega0=40)
+    with pytest.raises(mds.MdsError) as e:
+        v.verify(w.target, w.draft_list(), w.model_ids, w.tokens, w.temps, "WIS0", 1)
+    assert e.value.code == mds.MDS_EUNSUP
+    v.verify(w.target, w.draft_list(), w.model_ids, w.tokens, w.temps, "WIS", 1)   # other schemes run
+    torch.cuda.synchronize()
+    v.close()
 
 
 @pytest.mark.parametrize("cluster", [1, 2, 4, 8, 16])
@@ -57,10 +87,10 @@ def test_tiny_vocabularies(V):
     for dtype in ("f32", "bf16"):
         spec = WorkloadSpec(f"v{V}", B=24, K=3, L=3, V=V, dtype=dtype, model_ids=[0, 0, 1], target_scale=2.0,
                             draft_sigma=[0.5, 1.0], t_target=1.0, t_draft=[1.0, 1.3], data_seed=V)
-        for M in (1, 5, 30):
-            # bf16 ties at the cut can leave the largest Omega_0 uncertified
+        for M in (1, 5, 30, 45):
+            # bf16 ties at the cut can leave the larger Omega_0 uncertified
             ok(run_both(spec, "WIS0", seed=V + M, omega0=M, wis_s=min(5, max(1, V))),
-               allow_uncertified=(dtype == "bf16" and M == 30))
+               allow_uncertified=(dtype == "bf16" and M >= 30))
 
 
 def test_more_draft_models_than_one_pass_holds():
