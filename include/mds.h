@@ -194,7 +194,7 @@ int mds_verify_host(mds_ctx* ctx, const void* target_logits, const void* const* 
  * any stream capture.  Every call clears the parts of the scratch that must
  * start at zero on `stream`, then launches; all calls share the one array,
  * so calls that overlap on the GPU race.  The status word is not reported
- * (use a context for mds_status).  The paper has no counterpart to this entry
+ * (use mds_noalloc_status).  The paper has no counterpart to this entry
  * point: it exists only for callers that cannot allocate. */
 #define MDS_NOALLOC_SCRATCH_BYTES (8u << 20)
 int mds_verify_noalloc(const mds_config* cfg, int device, const void* target_logits,
@@ -202,6 +202,13 @@ int mds_verify_noalloc(const mds_config* cfg, int device, const void* target_log
                        const int32_t* draft_tokens, const float* temperatures, int scheme,
                        uint64_t philox_seed, int32_t* out_tokens, int32_t* out_accept_len, float* out_diag,
                        int B, void* stream);
+
+/* The status word of the last mds_verify_noalloc call on `device`: copies it
+ * to the host on `stream` (after that call's kernel) and synchronises the
+ * stream, allocating nothing.  Returns the MDS_ST_* bits (>= 0) or a negative
+ * code; *msg (if not NULL) as for mds_status.  The word is cleared by the
+ * next mds_verify_noalloc call on the device, not by this one. */
+int mds_noalloc_status(int device, void* stream, const char** msg);
 
 /* Synchronise the device, read and clear the status word.  Returns the
  * MDS_ST_* bits (>= 0) or a negative code; *msg (if not NULL) receives a

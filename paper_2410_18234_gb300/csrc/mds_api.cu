@@ -453,16 +453,7 @@ int mds_status(mds_ctx* ctx, const char** msg) {
     if (msg) *msg = "CUDA runtime error while reading the status word";
     return MDS_ECUDA;
   }
-  if (msg) {
-    if (st & MDS_ST_OMEGA0) *msg = "Omega_0 cut not certified by the candidate list; certified subset used";
-    else if (st & MDS_ST_BADTOKEN) *msg = "draft token outside [0, V); token 0 used";
-    else if (st & MDS_ST_LP_CAP) *msg = "stage LP reached its augmentation cap";
-    else if (st & MDS_ST_TIMEOUT) *msg = "a bounded wait on a bulk copy gave up";
-    else if (st & MDS_ST_ZERO_RESID) *msg = "zero residual mass after a rejection; target row sampled";
-    else if (st & MDS_ST_BADTEMP) *msg = "temperature <= 0 or not finite (1.0 used)";
-    else if (st & MDS_ST_NONFINITE) *msg = "non-finite logits or normaliser";
-    else *msg = "ok";
-  }
+  if (msg) *msg = mds::status_message(st);
   return (int)st;
 }
 
@@ -517,6 +508,17 @@ int launch_geometry(const mds_config& cfg, int device, int scheme, int n_models,
 }
 int prepare_kernels(int dtype) { return ensure_configured(dtype); }
 int record_cuda_error(cudaError_t e, const char* where) { return cuda_fail(e, where); }
+
+const char* status_message(unsigned st) {
+  if (st & MDS_ST_OMEGA0) return "Omega_0 cut not certified by the candidate list; certified subset used";
+  if (st & MDS_ST_BADTOKEN) return "draft token outside [0, V); token 0 used";
+  if (st & MDS_ST_LP_CAP) return "stage LP reached its augmentation cap";
+  if (st & MDS_ST_TIMEOUT) return "a bounded wait gave up";
+  if (st & MDS_ST_ZERO_RESID) return "zero residual mass after a rejection; target row sampled";
+  if (st & MDS_ST_BADTEMP) return "temperature <= 0 or not finite (1.0 used)";
+  if (st & MDS_ST_NONFINITE) return "non-finite logits or normaliser";
+  return "ok";
+}
 
 bool flow_params(const mds_config& c, int grid, int scheme, const int8_t* model_of, int n_models, bool bulk_ok,
                  bool aligned16, flow::Params& p) {

@@ -75,6 +75,9 @@ int prepare_kernels(int dtype);
 // reports for this host thread); returns MDS_ECUDA.
 int record_cuda_error(cudaError_t e, const char* where);
 
+// Description of the highest status bit set (static string).
+const char* status_message(unsigned status);
+
 namespace flow {
 struct Params;
 }

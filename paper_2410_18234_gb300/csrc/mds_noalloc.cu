@@ -169,3 +169,31 @@ extern "C" int mds_verify_noalloc(const mds_config* cfg_in, int device, const vo
   if (prev >= 0 && prev != device) cudaSetDevice(prev);
   return rc;
 }
+
+extern "C" int mds_noalloc_status(int device, void* stream, const char** msg) {
+  int count = 0;
+  if (cudaGetDeviceCount(&count) != cudaSuccess || device < 0 || device >= count || device >= kMaxDevices) {
+    cudaGetLastError();
+    return MDS_EINVAL;
+  }
+  int prev = -1;
+  cudaGetDevice(&prev);
+  if (prev != device) {
+    const cudaError_t se = cudaSetDevice(device);
+    if (se != cudaSuccess) return mds::record_cuda_error(se, "cudaSetDevice");
+  }
+  unsigned char* scratch = nullptr;
+  int grid = 0;
+  int rc = scratch_for(device, &scratch, &grid);
+  unsigned st = 0;
+  if (rc == MDS_OK) {
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaMemcpyAsync(&st, scratch, sizeof(st), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) rc = mds::record_cuda_error(e, "mds_noalloc_status");
+  }
+  if (prev >= 0 && prev != device) cudaSetDevice(prev);
+  if (rc != MDS_OK) return rc;
+  if (msg) *msg = mds::status_message(st);
+  return (int)st;
+}

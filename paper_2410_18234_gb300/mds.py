@@ -34,7 +34,7 @@ MDS_MAX_OMEGA0 = 62
 MDS_MAX_OMEGA0_CLUSTER = 30   # with a cluster size set (the per-sequence engine)
 
 # every symbol include/mds.h declares
-EXPORTS = ("mds_create", "mds_verify", "mds_verify_host", "mds_verify_noalloc", "mds_status",
+EXPORTS = ("mds_create", "mds_verify", "mds_verify_host", "mds_verify_noalloc", "mds_noalloc_status", "mds_status",
            "mds_cluster_size", "mds_phase_timers", "mds_debug_row_stats", "mds_debug_exp_count", "mds_debug_probs",
            "mds_error_string", "mds_destroy")
 
@@ -68,6 +68,8 @@ def load_library(path=LIB_PATH):
     lib.mds_verify_noalloc.argtypes = [ctypes.POINTER(MdsConfig), ctypes.c_int, vp, ctypes.POINTER(vp), i32p, vp, vp,
                                        ctypes.c_int, ctypes.c_uint64, vp, vp, f32p, ctypes.c_int, vp]
     lib.mds_verify_noalloc.restype = ctypes.c_int
+    lib.mds_noalloc_status.argtypes = [ctypes.c_int, vp, ctypes.POINTER(ctypes.c_char_p)]
+    lib.mds_noalloc_status.restype = ctypes.c_int
     lib.mds_status.argtypes = [vp, ctypes.POINTER(ctypes.c_char_p)]
     lib.mds_status.restype = ctypes.c_int
     lib.mds_cluster_size.argtypes = [vp]
@@ -219,6 +221,20 @@ def mds_verify_noalloc(max_B, K, L, V, target, drafts, model_ids, tokens, temps,
                                  ctypes.c_void_p(int(stream)))
     if rc != MDS_OK:
         raise MdsError(rc, "mds_verify_noalloc")
+
+
+def mds_noalloc_status(device=0, stream=None):
+    """(bits, message) of the last mds_verify_noalloc call on `device`, read
+    without allocating (see include/mds.h)."""
+    if stream is None:
+        stream = torch.cuda.current_stream(int(device)).cuda_stream
+    elif isinstance(stream, torch.cuda.Stream):
+        stream = stream.cuda_stream
+    msg = ctypes.c_char_p()
+    rc = _lib.mds_noalloc_status(int(device), ctypes.c_void_p(int(stream)), ctypes.byref(msg))
+    if rc < 0:
+        raise MdsError(rc, "mds_noalloc_status")
+    return rc, (msg.value or b"").decode()
 
 
 def mds_status(ctx):

@@ -62,3 +62,24 @@ def test_noalloc_rejects_bad_arguments_without_launching():
         mds.mds_verify_noalloc(spec.B, spec.K, spec.L, spec.V, w.target, w.draft_list(), w.model_ids, w.tokens,
                                w.temps, 9, 0, out, acc, dtype=spec.dtype)
     assert e.value.code == mds.MDS_EINVAL
+
+
+def test_noalloc_status_word():
+    # The status bits of a no-allocation call, read without allocating: a
+    # draft token outside [0, V) (a host-side input; the kernel replaces it by
+    # token 0 and flags it), then a clean call, whose clearing resets them.
+    spec = WORKLOADS["llama2-32k"].with_(B=4, V=4099)
+    w = make_workload(spec, device="cuda:0")
+    out = torch.empty(spec.B, spec.L + 1, dtype=torch.int32, device="cuda:0")
+    acc = torch.empty(spec.B, dtype=torch.int32, device="cuda:0")
+    bad = w.tokens.clone()
+    bad[1, :, 0] = spec.V + 5
+    for scheme in ("WIS", "SpecTr"):
+        mds.mds_verify_noalloc(spec.B, spec.K, spec.L, spec.V, w.target, w.draft_list(), w.model_ids, bad,
+                               w.temps, scheme, 3, out, acc, dtype=spec.dtype)
+        bits, msg = mds.mds_noalloc_status(0)
+        assert bits & mds.MDS_ST_BADTOKEN, (scheme, bits, msg)
+        assert int(out.max()) < spec.V and int(acc.min()) >= 0   # every output still a valid token
+        mds.mds_verify_noalloc(spec.B, spec.K, spec.L, spec.V, w.target, w.draft_list(), w.model_ids, w.tokens,
+                               w.temps, scheme, 3, out, acc, dtype=spec.dtype)
+        assert mds.mds_noalloc_status(0) == (0, "ok")
