@@ -383,245 +383,6 @@ __device__ __forceinline__ bool lp_maxflow(int s, float (&rd)[SM], float (&RS)[S
   return false;
 }
 
-// The augmenting phase (b) of lp_maxflow on pair state in shared memory
-// (dynamic indices) with bitmask breadth-first search: the same paths, in the
-// same order, with the same arithmetic on every pair.  RS, FL, FH are indexed
-// by pidx(., ., SM); rd by token.  One thread.  Returns false at the cap.
-template <int SM>
-__device__ __forceinline__ bool lp_augment_smem(int s, float* RS, float* FL, float* FH, float* rd, float eps) {
-  static_assert(SM <= 8, "8 bits of adjacency per token");
-  for (int it = 0; it < kLpMaxAugment; ++it) {
-    uint32_t dm = 0u;
-    for (int t = 0; t < s; ++t)
-      if (rd[t] > eps) dm |= 1u << t;
-    if (!dm) return true;
-    // adjacency (u -> v when pair {u,v} gives flow to u), 8 bits per token;
-    // sources: tokens of pairs with supply left, each with the first such pair
-    unsigned long long adjw = 0ull, srcp = 0ull;
-    uint32_t srcm = 0u;
-    for (int i = 0; i < s; ++i) {
-      for (int j = i + 1; j < s; ++j) {
-        const int e = pidx(i, j, SM);
-        const float fl = FL[e], fh = FH[e], rs = RS[e];
-        if (fl > eps) adjw |= 1ull << (8 * i + j);
-        if (fh > eps) adjw |= 1ull << (8 * j + i);
-        if (rs > eps) {
-          if (!(srcm >> i & 1u)) {
-            srcm |= 1u << i;
-            srcp |= (unsigned long long)e << (5 * i);
-          }
-          if (!(srcm >> j & 1u)) {
-            srcm |= 1u << j;
-            srcp |= (unsigned long long)e << (5 * j);
-          }
-        }
-      }
-    }
-    if (!srcm) return true;
-    // levels in increasing token order; a token's parent is the first
-    // frontier token reaching it
-    uint32_t visited = srcm, frontier = srcm, hit = srcm & dm, par = 0u;
-    for (int level = 0; level < SM && !hit && frontier; ++level) {
-      uint32_t nxt = 0u;
-      for (uint32_t f = frontier; f; f &= f - 1u) {
-        const int uu = __ffs(f) - 1;
-        const uint32_t nb = (uint32_t)(adjw >> (8 * uu)) & 0xffu & ~(visited | nxt);
-        for (uint32_t g = nb; g; g &= g - 1u) par |= (uint32_t)(uu + 1) << (4 * (__ffs(g) - 1));
-        nxt |= nb;
-      }
-      visited |= nxt;
-      frontier = nxt;
-      hit = nxt & dm;
-    }
-    if (!hit) return true;
-    const int sink = __ffs(hit) - 1;
-    float delta = rd[sink];
-    int t = sink, t0 = sink;
-    for (int g = 0; g < SM; ++g) {
-      const int uu = (int)((par >> (4 * t)) & 15u) - 1;
-      if (uu < 0) {
-        t0 = t;
-        break;
-      }
-      const int e = pidx(uu, t, SM);
-      delta = fminf(delta, (uu < t) ? FL[e] : FH[e]);
-      t = uu;
-    }
-    const int e0 = (int)((srcp >> (5 * t0)) & 31ull);
-    const bool lo0 = pidx_lo(e0, SM) == t0;
-    delta = fminf(delta, RS[e0]);
-    RS[e0] = __fsub_rn(RS[e0], delta);
-    if (lo0)
-      FL[e0] = __fadd_rn(FL[e0], delta);
-    else
-      FH[e0] = __fadd_rn(FH[e0], delta);
-    t = sink;
-    for (int g = 0; g < SM; ++g) {
-      const int uu = (int)((par >> (4 * t)) & 15u) - 1;
-      if (uu < 0) break;
-      const int e = pidx(uu, t, SM);
-      if (uu < t) {
-        FL[e] = __fsub_rn(FL[e], delta);
-        FH[e] = __fadd_rn(FH[e], delta);
-      } else {
-        FH[e] = __fsub_rn(FH[e], delta);
-        FL[e] = __fadd_rn(FL[e], delta);
-      }
-      t = uu;
-    }
-    rd[sink] = __fsub_rn(rd[sink], delta);
-  }
-  return false;
-}
-
-// Stage solve with the direct pass in registers and the augmenting phase on
-// shared-memory pair state (sRS, sFL, sFH: kMaxPairs entries, srd: SM
-// entries, all caller-owned shared memory).  Same result as stage_solve.
-template <int SM>
-__device__ __forceinline__ int stage_solve_split(int s, float A2, float B2, int A, int Btok, float u, const int* om,
-                                                 const float* om_q, const float* om_a, const float* om_b, float* om_x,
-                                                 bool* capped, float* sRS, float* sFL, float* sFH, float* srd) {
-  constexpr int P = SM * (SM - 1) / 2;
-  float RS[P], FL[P], FH[P];
-  float ak[SM], bk[SM], x[SM], rd[SM];
-  float eps = 0.f;
-#pragma unroll
-  for (int t = 0; t < SM; ++t) {
-    ak[t] = om_a[t];
-    bk[t] = om_b[t];
-    const float qk = om_q[t];
-    x[t] = __fadd_rn(__fadd_rn(__fmul_rn(ak[t], bk[t]), __fmul_rn(ak[t], B2)), __fmul_rn(bk[t], A2));
-    rd[t] = (t < s) ? fmaxf(0.f, __fsub_rn(qk, x[t])) : 0.f;
-    if (t < s) eps = __fadd_rn(eps, __fadd_rn(qk, x[t]));
-  }
-  eps = __fmul_rn(eps, kLpEpsRel);
-  // (a) the direct pass, in registers
-#pragma unroll
-  for (int i = 0; i < SM; ++i) {
-#pragma unroll
-    for (int j = i + 1; j < SM; ++j) {
-      const int e = pidx(i, j, SM);
-      RS[e] = (j < s) ? __fadd_rn(__fmul_rn(ak[i], bk[j]), __fmul_rn(ak[j], bk[i])) : 0.f;
-      FL[e] = 0.f;
-      FH[e] = 0.f;
-      if (j >= s) continue;
-      if (RS[e] > eps && rd[i] > eps) {
-        const float d = fminf(RS[e], rd[i]);
-        FL[e] = __fadd_rn(FL[e], d);
-        RS[e] = __fsub_rn(RS[e], d);
-        rd[i] = __fsub_rn(rd[i], d);
-      }
-      if (RS[e] > eps && rd[j] > eps) {
-        const float d = fminf(RS[e], rd[j]);
-        FH[e] = __fadd_rn(FH[e], d);
-        RS[e] = __fsub_rn(RS[e], d);
-        rd[j] = __fsub_rn(rd[j], d);
-      }
-    }
-  }
-  // (b) augmenting paths, only if one exists: a token with demand left
-  // reachable from a pair with supply left along pairs that give flow
-  // (a bitmask closure; the breadth-first search itself runs only then)
-  uint32_t dm = 0u, srcm = 0u;
-  uint32_t adj[SM];
-#pragma unroll
-  for (int t = 0; t < SM; ++t) {
-    adj[t] = 0u;
-    if (t < s && rd[t] > eps) dm |= 1u << t;
-  }
-#pragma unroll
-  for (int i = 0; i < SM; ++i) {
-#pragma unroll
-    for (int j = i + 1; j < SM; ++j) {
-      if (j >= s) continue;
-      const int e = pidx(i, j, SM);
-      if (FL[e] > eps) adj[i] |= 1u << j;
-      if (FH[e] > eps) adj[j] |= 1u << i;
-      if (RS[e] > eps) srcm |= (1u << i) | (1u << j);
-    }
-  }
-  uint32_t reach = srcm;
-  if (dm && srcm) {
-#pragma unroll
-    for (int level = 0; level < SM; ++level) {
-      uint32_t nxt = reach;
-#pragma unroll
-      for (int t = 0; t < SM; ++t)
-        if (reach >> t & 1u) nxt |= adj[t];
-      reach = nxt;
-    }
-  }
-  const bool need = (reach & dm) != 0u;
-  *capped = false;
-  if (need) {
-#pragma unroll
-    for (int e = 0; e < P; ++e) {
-      sRS[e] = RS[e];
-      sFL[e] = FL[e];
-      sFH[e] = FH[e];
-    }
-#pragma unroll
-    for (int t = 0; t < SM; ++t) srd[t] = rd[t];
-    *capped = !lp_augment_smem<SM>(s, sRS, sFL, sFH, srd, eps);
-#pragma unroll
-    for (int e = 0; e < P; ++e) {
-      RS[e] = sRS[e];
-      FL[e] = sFL[e];
-      FH[e] = sFH[e];
-    }
-  }
-  // p_I on Omega_1: base + flow + half of the pair mass left over
-#pragma unroll
-  for (int i = 0; i < SM; ++i) {
-#pragma unroll
-    for (int j = i + 1; j < SM; ++j) {
-      if (j >= s) continue;
-      const int e = pidx(i, j, SM);
-      const float half = __fmul_rn(0.5f, RS[e]);
-      x[i] = __fadd_rn(x[i], __fadd_rn(FL[e], half));
-      x[j] = __fadd_rn(x[j], __fadd_rn(FH[e], half));
-    }
-  }
-#pragma unroll
-  for (int t = 0; t < SM; ++t) om_x[t] = x[t];
-  if (A == Btok) return A;
-  int pa = -1, pb = -1;
-#pragma unroll
-  for (int t = 0; t < SM; ++t) {
-    if (t < s && om[t] == A) pa = t;
-    if (t < s && om[t] == Btok) pb = t;
-  }
-  if (pa >= 0 && pb >= 0) {
-    const int lo = min(pa, pb), hi = max(pa, pb);
-    const int e = pidx(lo, hi, SM);
-    float fl = 0.f, rs = 0.f, alo = 0.f, ahi = 0.f, blo = 0.f, bhi = 0.f;
-#pragma unroll
-    for (int k = 0; k < P; ++k)
-      if (k == e) {
-        fl = FL[k];
-        rs = RS[k];
-      }
-#pragma unroll
-    for (int t = 0; t < SM; ++t) {
-      if (t == lo) {
-        alo = ak[t];
-        blo = bk[t];
-      }
-      if (t == hi) {
-        ahi = ak[t];
-        bhi = bk[t];
-      }
-    }
-    const float m = __fadd_rn(__fmul_rn(alo, bhi), __fmul_rn(ahi, blo));
-    const float wlo = m > 0.f ? __fdiv_rn(__fadd_rn(fl, __fmul_rn(0.5f, rs)), m) : 0.5f;
-    const float wa = (pa < pb) ? wlo : __fsub_rn(1.f, wlo);
-    return (u < wa) ? A : Btok;
-  }
-  if (pa >= 0) return A;
-  if (pb >= 0) return Btok;
-  return (u < 0.5f) ? A : Btok;
-}
-
 // One stage of the weighted scheme given Omega_1 (om[0..s), increasing
 // token ids; entries past s ignored) with q, a, b at those tokens and the
 // Omega_2 masses A2 = a(Omega_2), B2 = b(Omega_2).  Writes p_I on Omega_1 to

@@ -188,7 +188,6 @@ struct DState {                // the decision's working state (shared memory)
   int Y, fast_ok;
   Cand fin[kTopF];
   float lp_rs[kMaxPairs], lp_fl[kMaxPairs], lp_fh[kMaxPairs];   // LP pair state in shared memory
-  float lp_rd[MDS_MAX_S];
   // search
   int seg, cross, lastp, tok;
   float run;
@@ -212,18 +211,15 @@ struct FShared {
   FDesc desc[kNBuf];
   FDesc pend;                  // the scheduler's next task, resolved ahead
   float red[kCW * 2 * kMaxRows];
-  float mrow[kMaxRows];
   float wth[kCW];
   int ncand, last, issued, consumed;
-  int cmb_n, cmb_nv;           // combine of a pass: entries taken, valid entries
+  int cmb_nv;                  // combine of a pass: valid entries
   unsigned cmb_tau;            // ... order key of tau
   float addtau;
   float add[kMaxRows];
   uint32_t bitmap[64];         // one bit per 16-byte unit of a slice holding a special token
   Cand wcand[kCW * kTopF];
   Cand blk[kTopF];
-  float Rs[kMaxSlices];        // slice masses of a search
-  float hm[kMaxSlices];        // slice maxima of the bonus draw
   int flag_ok, flag_ab;
 #ifdef MDS_PHASE_TIMERS
   unsigned long long tm[kPhaseN];
@@ -358,7 +354,7 @@ struct Eng {
 
   // Warp-parallel plan of a sequence's depth-0 pass (every branch valid):
   // lane k < K takes branch k, and a draft model's row is that of its first
-  // branch (the same rows, in the same order, as plan_rows).
+  // branch (the same rows, in the same order, as Dec::plan_warp).
   __device__ void plan_depth0_warp(int b, FPass& P) const {
     const int lane = threadIdx.x & 31;
     const int K = p.K;
@@ -1423,8 +1419,7 @@ template <int DT> __device__ __noinline__ void dec_full_nl(int b);
 template <int DT> __device__ __noinline__ void dec_bonus_nl(int b);
 template <int DT> __device__ __noinline__ void dec_wis0_nl(int b);
 template <int DT> __device__ __noinline__ void dec_accept_nl(int b);
-template <int DT> __device__ __noinline__ bool dec_stage_nl(int A, int Btok, int rb, float u);
-__device__ __noinline__ int lp_solve5(int s, float A2, float B2, int A, int Btok, float u);
+__device__ __forceinline__ int lp_solve5(int s, float A2, float B2, int A, int Btok, float u);
 __device__ __noinline__ int lp_solve8(int s, float A2, float B2, int A, int Btok, float u);
 
 template <int DT>
@@ -1475,88 +1470,6 @@ struct Dec {
   }
 
   // -------------------------------------------------------------- planning
-  // Rows of depth j for the valid branches (the lowest valid branch's target
-  // row, then one row per distinct draft model in branch order) into *P (if
-  // given) and, if X is given, the valid branches, their tokens and rows.
-  // One lane.
-  __device__ void plan_rows(int b, int j, unsigned valid, bool bonus, FPass* P, int* nv, int* vbr, int* X,
-                            int* vrow) const {
-    const int K = p.K, L = p.L, V = p.V;
-    const int kstar = __ffs(valid) - 1;
-    if (P) {
-      P->row[0].ptr = p.target + ((((size_t)b * K + kstar) * (L + 1) + j) * (size_t)V) * p.esize;
-      float tq = p.temps[(size_t)b * (1 + K)];
-      if (!(tq > 0.f) || !(tq < kPosInf)) {
-        atomicOr(p.status, MDS_ST_BADTEMP);
-        tq = 1.f;
-      }
-      P->row[0].c = __fdiv_rn(kLog2e, tq);
-    }
-    int mrow[MDS_MAX_K];
-    for (int m = 0; m < MDS_MAX_K; ++m) mrow[m] = -1;
-    int nr = 1, n = 0;
-    if (!bonus) {
-      for (int k = 0; k < K; ++k) {
-        if (!(valid >> k & 1u)) continue;
-        const int m = p.model_of[k];
-        if (mrow[m] < 0) {
-          mrow[m] = nr;
-          if (P) {
-            P->row[nr].ptr = p.drafts[k] + (((size_t)b * L + j) * (size_t)V) * p.esize;
-            float td = p.temps[(size_t)b * (1 + K) + 1 + k];
-            if (!(td > 0.f) || !(td < kPosInf)) {
-              atomicOr(p.status, MDS_ST_BADTEMP);
-              td = 1.f;
-            }
-            P->row[nr].c = __fdiv_rn(kLog2e, td);
-          }
-          ++nr;
-        }
-        if (X) {
-          int x = p.tokens[((size_t)b * K + k) * L + j];
-          if (x < 0 || x >= V) {
-            atomicOr(p.status, MDS_ST_BADTOKEN);
-            x = 0;
-          }
-          vbr[n] = k;
-          X[n] = x;
-          vrow[n] = mrow[m];
-        }
-        ++n;
-      }
-    }
-    if (nv) *nv = n;
-    if (!P) return;
-    for (int r = 0; r < nr; ++r) {
-      P->row[r].M = 0.f;
-      P->row[r].invZ = 0.f;
-      P->row[r].gamma = 0.f;
-    }
-    P->nrows = nr;
-    P->j = j;
-    P->nspec = 0;
-    P->rb = 0;
-    P->cut = 0.f;
-    P->all0 = 0;
-    if (bonus) {
-      P->kind = kBonus;
-      P->nstream = 1;
-      P->list = 0;
-    } else {
-      P->kind = kStats;
-      if (p.scheme == MDS_WIS0) {
-        P->nstream = 1;
-        P->list = 1;
-      } else if (p.scheme == MDS_WIS) {
-        P->nstream = nr;
-        P->list = (n > 1 && nr <= kListRowsMax && p.ln > 0) ? 1 : 0;
-      } else {
-        P->nstream = min(2, nr);
-        P->list = 0;
-      }
-    }
-  }
-
   // Rows of depth j for the valid branches (the lowest valid branch's target
   // row, then one row per distinct draft model in branch order), one lane per
   // branch; the valid branches, their tokens (tk: the staged tokens of depth
@@ -2032,7 +1945,7 @@ struct Dec {
       const float ul = (lane + 1 < D.nv) ? draw_uniform(p.seed, b, j, kDrawSelect + lane) : 0.f;
       for (; m < D.nv; ++m) {
         const float u = __shfl_sync(FULLM, ul, m - 1);
-        if (!dec_stage_nl<DT>(A, D.X[m], D.vrow[m], u)) break;
+        if (!wis_stage_list(A, D.X[m], D.vrow[m], u)) break;
         A = D.Y;
       }
       if (lane == 0) list_to_table();
@@ -2881,13 +2794,10 @@ template <int DT> __device__ __noinline__ void dec_full_nl(int b) { dec_view<DT>
 template <int DT> __device__ __noinline__ void dec_bonus_nl(int b) { dec_view<DT>().decide_bonus(b); }
 template <int DT> __device__ __noinline__ void dec_wis0_nl(int b) { dec_view<DT>().wis0_decide(b); }
 template <int DT> __device__ __noinline__ void dec_accept_nl(int b) { dec_view<DT>().accept_step(b); }
-template <int DT> __device__ __noinline__ bool dec_stage_nl(int A, int Btok, int rb, float u) {
-  return dec_view<DT>().wis_stage_list(A, Btok, rb, u);
-}
 
 // The stage LP of the calling warp's decision (one lane), on its Omega_1
 // tables: pair state in registers for s <= 5, in shared memory above.
-__device__ __noinline__ int lp_solve5(int s, float A2, float B2, int A, int Btok, float u) {
+__device__ __forceinline__ int lp_solve5(int s, float A2, float B2, int A, int Btok, float u) {
   DState& D = *reinterpret_cast<DState*>(g_dsm + (size_t)(threadIdx.x >> 5) * kDecPerWarp);
   bool capped = false;
   float RS[10], FL[10], FH[10];
