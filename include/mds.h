@@ -68,6 +68,7 @@ extern "C" {
 #define MDS_MAX_IS_MODELS 4  /* distinct draft models for plain IS          */
 #define MDS_MAX_OMEGA0 62 /* |Omega_0| of the truncated alphabet, MDS_WIS0  */
 #define MDS_MAX_OMEGA0_CLUSTER 30 /* ... with a cluster size set (per-sequence engine) */
+#define MDS_MAX_TOPK 16   /* top_k of the top-k restriction                 */
 
 typedef struct mds_ctx mds_ctx;
 
@@ -121,6 +122,16 @@ typedef struct {
                       MDS_SPECTR out_diag[b][j][2] is prod_i R_i, the
                       probability that every round rejects (with 1 the rounds
                       after an acceptance are computed too).                  */
+  int top_k;       /* 0: off.  1..MDS_MAX_TOPK: every row (target and drafts)
+                      is restricted to its top_k largest logits (ties: lower
+                      token id first) and renormalised before verification
+                      (Section 5's top-k runs, Tables 2 and 3); the caller's
+                      draft tokens should come from the restricted draft rows
+                      (a token outside them has p_I = 0 and is accepted, as
+                      Algorithm 1 reads a zero denominator).  Served for
+                      MDS_SINGLE, MDS_WIS and MDS_SPECTR by the top-k kernel
+                      (one CTA per sequence, no cluster); MDS_IS and MDS_WIS0
+                      return MDS_EUNSUP.  acc_prob and out_diag as above.     */
 } mds_config;
 
 /* Create a context on CUDA device `device`.  Allocates the context's device

@@ -17,7 +17,7 @@ BUILD_DIR = os.path.join(ROOT, "_build")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-cudart", "static", "-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I" + os.path.join(ROOT, "include")]
-SOURCES = ["mds_kernel.cu", "mds_flow.cu", "mds_api.cu", "mds_noalloc.cu"]
+SOURCES = ["mds_kernel.cu", "mds_flow.cu", "mds_topk.cu", "mds_api.cu", "mds_noalloc.cu"]
 
 
 def nvcc():

@@ -7,6 +7,7 @@
 
 #include "mds_flow.h"
 #include "mds_internal.h"
+#include "mds_topk.h"
 
 struct mds_ctx {
   mds_config cfg;
@@ -188,6 +189,7 @@ int mds_create(mds_ctx** out, const mds_config* cfg, int device) {
   if (c.omega0 == 0) c.omega0 = 20;
   if (c.omega0 < 1 || c.omega0 > MDS_MAX_OMEGA0) return MDS_EINVAL;
   if (c.acc_prob != 0 && c.acc_prob != 1) return MDS_EINVAL;
+  if (c.top_k < 0 || c.top_k > MDS_MAX_TOPK) return MDS_EINVAL;
   if (c.max_B < 1 || c.K < 1 || c.K > MDS_MAX_K || c.L < 1 || c.L > MDS_MAX_L || c.V < 1 || c.V > (1 << 24))
     return MDS_ESHAPE;
   if (c.dtype != MDS_F32 && c.dtype != MDS_BF16) return MDS_EINVAL;
@@ -296,6 +298,14 @@ static int verify_impl(mds_ctx* ctx, const void* target_logits, const void* cons
     p.drafts[k] = static_cast<const char*>(draft_logits[k]);
   }
   if (scheme == MDS_IS && n_models > MDS_MAX_IS_MODELS) return MDS_EUNSUP;
+  if (c.top_k > 0) {
+    // rows restricted to their top k: the top-k kernel (no workspace)
+    DeviceGuard g(ctx->device);
+    ctx->last_cn = 0;
+    return mds::topk::verify(c, scheme, p.model_of, tma_ok, target_logits, draft_logits, draft_tokens, temperatures,
+                             out_tokens, out_accept_len, out_diag, B, philox_seed, ctx->work,
+                             static_cast<cudaStream_t>(stream));
+  }
   {
     const int frc = flow_verify(ctx, target_logits, draft_logits, p.model_of, n_models, draft_tokens, temperatures,
                                 scheme, philox_seed, out_tokens, out_accept_len, out_diag, B, stream, bulk_ok, tma_ok);

@@ -9,6 +9,7 @@
 
 #include "mds_flow.h"
 #include "mds_internal.h"
+#include "mds_topk.h"
 
 namespace {
 
@@ -68,6 +69,7 @@ extern "C" int mds_verify_noalloc(const mds_config* cfg_in, int device, const vo
   if (c.omega0 == 0) c.omega0 = 20;
   if (c.omega0 < 1 || c.omega0 > MDS_MAX_OMEGA0) return MDS_EINVAL;
   if (c.acc_prob != 0 && c.acc_prob != 1) return MDS_EINVAL;
+  if (c.top_k < 0 || c.top_k > MDS_MAX_TOPK) return MDS_EINVAL;
   if (c.max_B < 1 || c.K < 1 || c.K > MDS_MAX_K || c.L < 1 || c.L > MDS_MAX_L || c.V < 1 || c.V > (1 << 24))
     return MDS_ESHAPE;
   if (c.dtype != MDS_F32 && c.dtype != MDS_BF16) return MDS_EINVAL;
@@ -112,6 +114,20 @@ extern "C" int mds_verify_noalloc(const mds_config* cfg_in, int device, const vo
   int grid = 0;
   if (rc == MDS_OK) rc = scratch_for(device, &scratch, &grid);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (rc == MDS_OK && c.top_k > 0) {
+    // rows restricted to their top k: the top-k kernel, the status word its only scratch
+    if (!mds::topk::serves(scheme)) {
+      rc = MDS_EUNSUP;
+    } else {
+      const cudaError_t e = cudaMemsetAsync(scratch, 0, kHead, st);
+      rc = (e != cudaSuccess) ? mds::record_cuda_error(e, "mds_verify_noalloc launch")
+                              : mds::topk::verify(c, scheme, p.model_of, tma_ok, target_logits, draft_logits,
+                                                  draft_tokens, temperatures, out_tokens, out_accept_len, out_diag, B,
+                                                  philox_seed, reinterpret_cast<unsigned*>(scratch), st);
+    }
+    if (prev >= 0 && prev != device) cudaSetDevice(prev);
+    return rc;
+  }
   if (rc == MDS_OK) {
     // the dataflow engine where mds_verify takes it (same geometry: same results)
     mds::flow::Params fp{};

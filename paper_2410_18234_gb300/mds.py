@@ -29,6 +29,7 @@ MDS_OK, MDS_EINVAL, MDS_ESHAPE, MDS_EVOCAB, MDS_ECUDA, MDS_EUNSUP = 0, -1, -2, -
 MDS_ST_NONFINITE, MDS_ST_BADTEMP, MDS_ST_ZERO_RESID, MDS_ST_TIMEOUT, MDS_ST_LP_CAP, MDS_ST_BADTOKEN = \
     1, 2, 4, 8, 16, 32
 MDS_ST_OMEGA0 = 64
+MDS_MAX_TOPK = 16
 MDS_MAX_K = 16
 MDS_MAX_OMEGA0 = 62
 MDS_MAX_OMEGA0_CLUSTER = 30   # with a cluster size set (the per-sequence engine)
@@ -42,7 +43,8 @@ EXPORTS = ("mds_create", "mds_verify", "mds_verify_host", "mds_verify_noalloc", 
 class MdsConfig(ctypes.Structure):
     _fields_ = [("max_B", ctypes.c_int), ("K", ctypes.c_int), ("L", ctypes.c_int), ("V", ctypes.c_int),
                 ("dtype", ctypes.c_int), ("wis_s", ctypes.c_int), ("is_h", ctypes.c_float),
-                ("cluster", ctypes.c_int), ("omega0", ctypes.c_int), ("acc_prob", ctypes.c_int)]
+                ("cluster", ctypes.c_int), ("omega0", ctypes.c_int), ("acc_prob", ctypes.c_int),
+                ("top_k", ctypes.c_int)]
 
 
 class MdsError(RuntimeError):
@@ -100,9 +102,10 @@ def error_string(code):
 # ----------------------------------------------------------- C entry points
 
 
-def mds_create(max_B, K, L, V, dtype="bf16", wis_s=5, is_h=0.25, cluster=0, device=0, omega0=0, acc_prob=0):
+def mds_create(max_B, K, L, V, dtype="bf16", wis_s=5, is_h=0.25, cluster=0, device=0, omega0=0, acc_prob=0,
+               top_k=0):
     cfg = MdsConfig(int(max_B), int(K), int(L), int(V), DTYPES[dtype] if isinstance(dtype, str) else int(dtype),
-                    int(wis_s), float(is_h), int(cluster), int(omega0), int(acc_prob))
+                    int(wis_s), float(is_h), int(cluster), int(omega0), int(acc_prob), int(top_k))
     h = ctypes.c_void_p()
     rc = _lib.mds_create(ctypes.byref(h), ctypes.byref(cfg), int(device))
     if rc != MDS_OK:
@@ -200,14 +203,14 @@ def mds_verify_host(ctx, target, drafts, model_ids, tokens, temps, scheme, seed,
 
 def mds_verify_noalloc(max_B, K, L, V, target, drafts, model_ids, tokens, temps, scheme, seed, out_tokens,
                        out_accept, out_diag=None, stream=None, dtype="bf16", wis_s=5, is_h=0.25, cluster=0,
-                       device=0, omega0=0, acc_prob=0):
+                       device=0, omega0=0, acc_prob=0, top_k=0):
     """Context-free entry point for callers that cannot allocate device
     memory (see include/mds.h): the configuration is passed directly and the
     kernel's scratch is a static device array inside the library."""
     check_buffers(int(K), int(L), int(V), dtype, target, drafts, model_ids, tokens, temps, out_tokens, out_accept,
                   out_diag, "cuda", device=int(device))
     cfg = MdsConfig(int(max_B), int(K), int(L), int(V), DTYPES[dtype] if isinstance(dtype, str) else int(dtype),
-                    int(wis_s), float(is_h), int(cluster), int(omega0), int(acc_prob))
+                    int(wis_s), float(is_h), int(cluster), int(omega0), int(acc_prob), int(top_k))
     Kn = len(model_ids)
     B = int(tokens.shape[0])
     if stream is None:
@@ -321,11 +324,11 @@ class Verifier:
     """Owns one context; allocates outputs with torch on the context's device."""
 
     def __init__(self, max_B, K, L, V, dtype="bf16", wis_s=5, is_h=0.25, cluster=0, device=0, omega0=0,
-                 acc_prob=0):
+                 acc_prob=0, top_k=0):
         self.max_B, self.K, self.L, self.V = int(max_B), int(K), int(L), int(V)
         self.dtype = dtype
         self.device = torch.device("cuda", device)
-        self.ctx = mds_create(max_B, K, L, V, dtype, wis_s, is_h, cluster, device, omega0, acc_prob)
+        self.ctx = mds_create(max_B, K, L, V, dtype, wis_s, is_h, cluster, device, omega0, acc_prob, top_k)
 
     def verify(self, target, drafts, model_ids, tokens, temps, scheme, seed, diag=False, out=None, stream=None):
         B = int(tokens.shape[0])

@@ -13,7 +13,8 @@ then made equal across branches that share a prefix (and, for draft rows, a
 model), so the dense per-branch buffers are consistent with one tree.  Branch
 k's token at depth j is sampled independently from its own draft
 distribution softmax(l_d / T_k) at its node, by the Gumbel-max rule applied
-to the stored (rounded) logits.
+to the stored (rounded) logits; with top_k set, only the row's top_k logits
+(and any tied with the k-th) take part.
 
 Logits.  target = scale * N(0,1) (plus an optional boost of the largest
 entries), draft = target + sigma * N(0,1), both drawn in fp32 and then
@@ -51,6 +52,7 @@ class WorkloadSpec:
     schemes: List[str] = field(default_factory=list)
     data_seed: int = 0
     verify_seed: int = 1
+    top_k: int = 0                  # > 0: each branch samples from its draft row's top_k logits only
 
     def with_(self, **kw):
         return replace(self, **kw)
@@ -155,7 +157,12 @@ def make_workload(spec: WorkloadSpec, device="cpu", seed=None) -> Workload:
         # each branch samples its own token at its node (Gumbel-max on the stored logits)
         u = torch.rand(B, K, V, generator=g, device=dev).clamp_(min=1e-12)
         gum = -torch.log(-torch.log(u))
-        tk = (d_st.float() / temps[:, 1:, None] + gum).argmax(dim=2)
+        score = d_st.float() / temps[:, 1:, None] + gum
+        if spec.top_k > 0:
+            # sample from the row's top_k logits (every logit tied with the k-th is kept)
+            kth = torch.topk(d_st.float(), min(spec.top_k, V), dim=2).values[:, :, -1:]
+            score = torch.where(d_st.float() >= kth, score, torch.full_like(score, float("-inf")))
+        tk = score.argmax(dim=2)
         tokens[:, :, j] = tk.to(torch.int32)
         same = same & (tk[:, :, None] == tk[:, None, :])
     return Workload(spec, target, drafts, tokens, temps, list(spec.model_ids))
