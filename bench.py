@@ -51,6 +51,7 @@ def parse():
     ap.add_argument("--scheme", default=None)
     ap.add_argument("--cluster", type=int, default=0)
     ap.add_argument("--omega0", type=int, default=20, help="|Omega_0| of the truncated-alphabet scheme WIS0")
+    ap.add_argument("--top-k", type=int, default=0, help="restrict every row to its top k logits (0: off)")
     ap.add_argument("--B", type=int, default=0, help="override the batch (profiling on a small case)")
     ap.add_argument("--K", type=int, default=0, help="override the branch count, keeping the first K branches' "
                                                     "draft models (profiling on a small case)")
@@ -154,10 +155,12 @@ class ClockSampler:
 # ----------------------------------------------------------------- peaks / traffic
 
 
-def kernel_name(scheme, cluster):
-    """The kernel a call ran: the slice-dataflow engine's for single, WIS and
-    WIS0 (the library reports cluster size 0 for it), the per-sequence
-    engine's otherwise."""
+def kernel_name(scheme, cluster, top_k=0):
+    """The kernel a call ran: the top-k kernel for rows restricted to their
+    top k, the slice-dataflow engine's for single, WIS and WIS0 (the library
+    reports cluster size 0 for it), the per-sequence engine's otherwise."""
+    if top_k:
+        return "topk_kernel"
     return "flow_kernel" if cluster == 0 and scheme in ("single", "WIS", "WIS0") else "verify_kernel"
 
 
@@ -170,12 +173,20 @@ def hbm_peak():
         return FALLBACK_HBM, "fallback"
 
 
-def kernel_source_hash():
-    """Hash of the library's code with comments and blank lines removed, so
-    that recorded counters survive edits to comments only."""
+# the translation unit of each kernel and the internal headers it includes
+KERNEL_SOURCES = {
+    "flow_kernel": ["mds_flow.cu", "mds_flow.h", "mds_device.cuh", "mds_internal.h"],
+    "verify_kernel": ["mds_kernel.cu", "mds_internal.h"],
+    "topk_kernel": ["mds_topk.cu", "mds_topk.h", "mds_device.cuh", "mds_internal.h"],
+}
+
+
+def kernel_source_hash(kernel):
+    """Hash of one kernel's sources with comments and blank lines removed, so
+    that recorded counters survive edits to comments and to other kernels."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2410_18234_gb300", "csrc")
-    for name in sorted(os.listdir(csrc)):
+    for name in KERNEL_SOURCES[kernel]:
         text = open(os.path.join(csrc, name), encoding="utf-8").read()
         text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
         text = re.sub(r"//[^\n]*", "", text)
@@ -184,16 +195,16 @@ def kernel_source_hash():
     return h.hexdigest()[:16]
 
 
-def recorded_traffic(workload, scheme):
+def recorded_traffic(workload, scheme, kernel, top_k=0):
     """DRAM bytes per launch from the committed ncu summary, if it was taken
-    on the current kernel source; else None."""
+    on the kernel's current source; else None."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         d = json.load(open(path))
     except (OSError, ValueError):
         return None
-    e = d.get(f"{workload}/{scheme}")
-    if not e or e.get("kernel_hash") != kernel_source_hash():
+    e = d.get(f"{workload}/{scheme}" + (f"/top{top_k}" if top_k else ""))
+    if not e or e.get("kernel") != kernel or e.get("kernel_hash") != kernel_source_hash(kernel):
         return None
     return e.get("dram_bytes_per_launch")
 
@@ -201,7 +212,7 @@ def recorded_traffic(workload, scheme):
 # ----------------------------------------------------------------- oracle leg
 
 
-def oracle_rate(w, scheme, seconds, seqs=None, omega0=20):
+def oracle_rate(w, scheme, seconds, seqs=None, omega0=20, top_k=0):
     """The oracle, as it stands, over a bounded prefix of the workload's
     sequences (host cores).  Returns (vocab_rows/s, sample description,
     outputs) for the sequences it finished."""
@@ -215,7 +226,7 @@ def oracle_rate(w, scheme, seconds, seqs=None, omega0=20):
     for b in order:
         host = host_copy(w, [b])
         t0 = time.perf_counter()
-        o, a, recs = oracle_verify(*host, scheme, spec.verify_seed, seq_ids=[b], omega0=omega0)
+        o, a, recs = oracle_verify(*host, scheme, spec.verify_seed, seq_ids=[b], omega0=omega0, top_k=top_k)
         t_total += time.perf_counter() - t0
         out = np.asarray(o[b])[None]
         r, _ = walk_accounting(host[3], w.model_ids, out, np.array([a[b]]), spec.V, es, scheme, omega0)
@@ -229,15 +240,15 @@ def oracle_rate(w, scheme, seconds, seqs=None, omega0=20):
 
 def _oracle_seq(job):
     """One sequence through the oracle (a worker of the all-core baseline)."""
-    host, scheme, seed, b, omega0, V, es = job
+    host, scheme, seed, b, omega0, V, es, top_k = job
     from oracle.verify import oracle_verify
-    o, a, _ = oracle_verify(*host, scheme, seed, seq_ids=[b], omega0=omega0)
+    o, a, _ = oracle_verify(*host, scheme, seed, seq_ids=[b], omega0=omega0, top_k=top_k)
     out = np.asarray(o[b])[None]
     r, _ = walk_accounting(host[3], host[2], out, np.array([a[b]]), V, es, scheme, omega0)
     return r
 
 
-def oracle_rate_all_cores(w, scheme, seconds, omega0=20, cores=None):
+def oracle_rate_all_cores(w, scheme, seconds, omega0=20, cores=None, top_k=0):
     """The oracle, as it stands, on every host core: one process per core
     (spawned, so no CUDA state is inherited), sequences handed out in order
     until the time budget is spent; the rate is the rows finished over the
@@ -255,7 +266,7 @@ def oracle_rate_all_cores(w, scheme, seconds, omega0=20, cores=None):
         b = 0
         while True:
             while b < spec.B and len(pending) < 2 * cores and time.perf_counter() - t0 < seconds:
-                job = (host_copy(w, [b]), scheme, spec.verify_seed, b, omega0, spec.V, es)
+                job = (host_copy(w, [b]), scheme, spec.verify_seed, b, omega0, spec.V, es, top_k)
                 job = ((job[0][0], job[0][1], job[0][2], job[0][3], job[0][4]), *job[1:])
                 pending.append(pool.apply_async(_oracle_seq, (job,)))
                 b += 1
@@ -319,6 +330,9 @@ TABLE = [("tiny", "IS"), ("llama2-32k", "IS"), ("llama2-32k", "WIS"), ("two-mode
          ("serving-152k", "single"), ("serving-152k", "IS"), ("serving-152k", "WIS"), ("serving-152k", "SpecTr"),
          ("serving-152k-k2", "single"), ("serving-152k-k2", "IS"), ("serving-152k-k2", "WIS"),
          ("serving-152k-k2", "SpecTr")]
+# rows restricted to their top k (Section 5: k = 5 and 10)
+TABLE_TOPK = [("llama3-128k", "WIS", 10), ("llama3-128k", "single", 10), ("llama3-128k", "SpecTr", 10),
+              ("two-models-50k", "WIS", 5), ("serving-152k", "WIS", 5), ("serving-152k-k2", "WIS", 10)]
 
 
 def table(args):
@@ -335,13 +349,15 @@ def table(args):
     flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
     rows_md = []
     want = None if not args.only else set(args.only.split(","))
-    for name, scheme in TABLE:
-        if want and f"{name}/{scheme}" not in want and name not in want:
+    for name, scheme, top_k in [(n, s, 0) for n, s in TABLE] + TABLE_TOPK:
+        tag = f"{name}/{scheme}" + (f"/top{top_k}" if top_k else "")
+        if want and tag not in want and name not in want:
             continue
-        spec = WORKLOADS[name]
+        spec = WORKLOADS[name].with_(top_k=top_k)
         es = 4 if spec.dtype == "f32" else 2
         w = make_workload(spec, device=dev)
-        v = mds.Verifier(spec.B, spec.K, spec.L, spec.V, dtype=spec.dtype, device=0, omega0=args.omega0)
+        v = mds.Verifier(spec.B, spec.K, spec.L, spec.V, dtype=spec.dtype, device=0, omega0=args.omega0,
+                         top_k=top_k)
         out_tokens = torch.empty(spec.B, spec.L + 1, dtype=torch.int32, device=dev)
         out_acc = torch.empty(spec.B, dtype=torch.int32, device=dev)
         stream = torch.cuda.current_stream(dev)
@@ -381,15 +397,15 @@ def table(args):
         o_tok, o_acc = out_tokens.cpu().numpy(), out_acc.cpu().numpy()
         rows, abytes = walk_accounting(tok, w.model_ids, o_tok, o_acc, spec.V, es, scheme, args.omega0)
         gbs = abytes / (ms * 1e-3) / 1e9
-        rate, desc, outs = oracle_rate(w, scheme, args.cpu_seconds, omega0=args.omega0)
+        rate, desc, outs = oracle_rate(w, scheme, args.cpu_seconds, omega0=args.omega0, top_k=top_k)
         par = agreement(o_tok, o_acc, outs)
         bits, _ = v.status()
         cn = v.cluster_size
         v.close()
-        line = {"workload": name, "scheme": scheme, "B": spec.B, "K": spec.K, "L": spec.L, "V": spec.V,
+        line = {"workload": name, "scheme": scheme, "top_k": top_k, "B": spec.B, "K": spec.K, "L": spec.L, "V": spec.V,
                 "logits": spec.dtype, "ms_per_step": ms, "ms_mean": float(np.mean(times)),
                 "rows_per_s": rows / (ms * 1e-3), "vocab_rows_per_step": rows, "gb_per_s": gbs,
-                "hbm_frac": gbs / peak, "peak": peak, "peak_kind": peak_kind, "kernel": kernel_name(scheme, cn),
+                "hbm_frac": gbs / peak, "peak": peak, "peak_kind": peak_kind, "kernel": kernel_name(scheme, cn, top_k),
                 "block_efficiency": float(np.mean(o_acc + 1)), "oracle_agreement": par,
                 "cpu_1core_rows_per_s": rate, "cpu_sample": desc, "status_bits": bits, "ex2_roofline": ex2}
         print(json.dumps(line), flush=True)
@@ -404,7 +420,8 @@ def table(args):
         a = r["oracle_agreement"]
         e = r["ex2_roofline"]
         ex = f"{e['ex2_per_s'] / 1e12:.2f} T ({e['frac']:.3f})" if e else "-"
-        md.append(f"| {r['workload']} | {r['scheme']} | {r['kernel']} | {r['ms_per_step']:.3f} | "
+        sch = r["scheme"] + (f" top-{r['top_k']}" if r["top_k"] else "")
+        md.append(f"| {r['workload']} | {sch} | {r['kernel']} | {r['ms_per_step']:.3f} | "
                   f"{r['rows_per_s'] / 1e6:.2f}M | {r['gb_per_s']:.0f} | {r['hbm_frac']:.3f} | {ex} | "
                   f"{r['block_efficiency']:.2f} | {a['identical']}/{a['band']}/{a['mismatch']} of {a['sequences']} | "
                   f"{r['cpu_1core_rows_per_s']:.1f} |")
@@ -434,7 +451,10 @@ def main():
         spec = spec.with_(B=args.B)
     if args.K:
         spec = spec.with_(K=args.K, model_ids=list(spec.model_ids)[:args.K])
+    if args.top_k:
+        spec = spec.with_(top_k=args.top_k)
     scheme = args.scheme or spec.schemes[0]
+    topk_cfg = {"top_k": args.top_k} if args.top_k else {}
     es = 4 if spec.dtype == "f32" else 2
 
     if args.impl == "reference":
@@ -445,12 +465,12 @@ def main():
         # each step: the oracle over a bounded sample of the workload
         per_step = max(2.0, args.cpu_seconds / max(1, args.steps + args.warmup))
         for _ in range(args.warmup):
-            oracle_rate(w, scheme, per_step / 4, omega0=args.omega0)
+            oracle_rate(w, scheme, per_step / 4, omega0=args.omega0, top_k=args.top_k)
         rates = []
         desc = ""
         t0 = time.perf_counter()
         for _ in range(args.steps):
-            r, desc, _ = oracle_rate(w, scheme, per_step, omega0=args.omega0)
+            r, desc, _ = oracle_rate(w, scheme, per_step, omega0=args.omega0, top_k=args.top_k)
             rates.append(r)
         wall = time.perf_counter() - t0
         value = float(np.mean(rates))
@@ -460,7 +480,7 @@ def main():
                 "data": "synthetic",
                 "config": {"workload": spec.name, "B": spec.B, "K": spec.K, "L": spec.L, "V": spec.V,
                            "logits": spec.dtype, "scheme": scheme,
-                           **({"omega0": args.omega0} if scheme == "WIS0" else {})},
+                           **({"omega0": args.omega0} if scheme == "WIS0" else {}), **topk_cfg},
                 "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
                                  "sample": f"per step {desc}"},
                 "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -477,7 +497,7 @@ def main():
     from paper_2410_18234_gb300 import mds
     w = make_workload(spec, device=dev, seed=rank_seed(spec, rank))
     v = mds.Verifier(spec.B, spec.K, spec.L, spec.V, dtype=spec.dtype, cluster=args.cluster, device=dev.index,
-                     omega0=args.omega0)
+                     omega0=args.omega0, top_k=args.top_k)
     drafts = w.draft_list()
     out_tokens = torch.empty(spec.B, spec.L + 1, dtype=torch.int32, device=dev)
     out_acc = torch.empty(spec.B, dtype=torch.int32, device=dev)
@@ -560,12 +580,13 @@ def main():
     cpu_all = None
     parity = None
     if rank == 0 and world == 1 and not (args.no_cpu_baseline and args.no_parity):
-        rate, desc, outs = oracle_rate(w, scheme, args.cpu_seconds, omega0=args.omega0)
+        rate, desc, outs = oracle_rate(w, scheme, args.cpu_seconds, omega0=args.omega0, top_k=args.top_k)
         parity = agreement(o_tok, o_acc, outs)
         if not args.no_cpu_baseline:
             cpu = {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc}
             if not args.no_cpu_all:
-                r_all, d_all, cores = oracle_rate_all_cores(w, scheme, args.cpu_seconds, omega0=args.omega0)
+                r_all, d_all, cores = oracle_rate_all_cores(w, scheme, args.cpu_seconds, omega0=args.omega0,
+                                                            top_k=args.top_k)
                 cpu_all = {"value": r_all, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": d_all}
 
     bits, msg = v.status()
@@ -579,12 +600,13 @@ def main():
             "vs_baseline": None, "dtype": "f32", "data": "synthetic",
             "config": {"workload": spec.name, "B": spec.B, "K": spec.K, "L": spec.L, "V": spec.V,
                        "logits": spec.dtype, "scheme": scheme, "cluster": cn, "l2_flush": True,
-                       **({"omega0": args.omega0} if scheme == "WIS0" else {}),
+                       **({"omega0": args.omega0} if scheme == "WIS0" else {}), **topk_cfg,
                        "parallelism": f"sequence-sharded x{world}", "seed": spec.verify_seed},
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "peak_kind": peak_kind,
-                         "traffic": None if (args.B or args.K) else recorded_traffic(spec.name, scheme),
-                         "algorithmic_bytes_per_launch": int(abytes), "kernel": kernel_name(scheme, cn)},
+                         "traffic": None if (args.B or args.K) else recorded_traffic(
+                             spec.name, scheme, kernel_name(scheme, cn, args.top_k), args.top_k),
+                         "algorithmic_bytes_per_launch": int(abytes), "kernel": kernel_name(scheme, cn, args.top_k)},
             "cpu_baseline": cpu,
             "cpu_baseline_all_cores": cpu_all,
             "e2e": e2e,

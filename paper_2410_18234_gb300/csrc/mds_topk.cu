@@ -36,6 +36,7 @@ constexpr int kKMax = MDS_MAX_TOPK;
 constexpr int kRowsMax = 1 + MDS_MAX_K;
 constexpr int kEntMax = kRowsMax * kKMax;   // kept entries of one depth, and the largest |U|
 constexpr unsigned FULL = 0xffffffffu;
+constexpr int kPrefixUnits = 4;             // units per thread behind a row's first logit bound
 
 static_assert(kWarps * kKMax == 4 * 32, "the row merge holds four candidates per lane");
 static_assert(kKMax <= 32, "a row's kept entries fit one warp");
@@ -70,6 +71,7 @@ struct Shared {
   float RS[kMaxPairs], FL[kMaxPairs], FH[kMaxPairs];
   int Y;
   int bcast;                              // warp 0's broadcast word
+  float tau0;                             // lower bound on a row's kk-th logit
   // bonus: the target row's kept entries by increasing id
   int bid[kKMax];
   float bw[kKMax];
@@ -92,22 +94,25 @@ __device__ __forceinline__ int key_id(unsigned long long k) { return (int)(0xfff
 __device__ __forceinline__ float key_val(unsigned long long k) { return ord_val((unsigned)(k >> 32)); }
 
 // A thread's running list: its 16 largest keys, decreasing; the k-th entry
-// and its logit bound what can still enter.
+// and its logit (or the row's known floor, if higher) bound what can still
+// enter.  Every array is indexed by
+// compile-time constants only (registers).
 struct TopList {
   unsigned long long e[kKMax];
   unsigned long long kth;
   float bound;
+  float floor;   // a lower bound on the row's kk-th logit known in advance
 
   __device__ __forceinline__ void reset() {
 #pragma unroll
     for (int i = 0; i < kKMax; ++i) e[i] = 0ull;
     kth = 0ull;
     bound = kNegInf;
+    floor = kNegInf;
   }
-  __device__ __forceinline__ void offer(float v, int id, int kk) {
-    if (!(v >= bound)) return;   // below the k-th logit (or NaN)
+  __device__ __forceinline__ void insert(float v, int id, int kk) {
     unsigned long long x = entry_key(v, id);
-    if (x <= kth) return;
+    if (!(v >= bound) || x <= kth) return;
 #pragma unroll
     for (int i = 0; i < kKMax; ++i) {
       const unsigned long long t = e[i];
@@ -118,7 +123,24 @@ struct TopList {
 #pragma unroll
     for (int i = 0; i < kKMax; ++i)
       if (i == kk - 1) kth = e[i];
-    bound = kth ? key_val(kth) : kNegInf;
+    bound = kth ? fmaxf(floor, key_val(kth)) : floor;
+  }
+  // The values of one unit (n of them, ids base, base + 1, ...): a mask of
+  // those at or above the bound, then one insertion site for the (rare) hits.
+  template <int N>
+  __device__ __forceinline__ void offer(const float (&v)[N], int base, int kk) {
+    unsigned m = 0u;
+#pragma unroll
+    for (int i = 0; i < N; ++i) m |= (v[i] >= bound) ? (1u << i) : 0u;
+    while (m) {
+      const int i0 = __ffs(m) - 1;
+      m &= m - 1u;
+      float x = v[0];
+#pragma unroll
+      for (int i = 1; i < N; ++i)
+        if (i == i0) x = v[i];
+      insert(x, base + i0, kk);
+    }
   }
   __device__ __forceinline__ void pop() {
 #pragma unroll
@@ -127,53 +149,101 @@ struct TopList {
   }
 };
 
+template <int DT>
+__device__ __forceinline__ void scan_unit(TopList& T, const uint4& x, int u, int kk) {
+  using E = Elt<DT>;
+  if (!(E::unit_max(x) >= T.bound)) return;
+  float v[E::VE];
+  E::unpack(x, v);
+  T.offer<E::VE>(v, u * E::VE, kk);
+}
 
 // The row's top kk into S.id / S.lg / S.n[r] (all threads; ends synchronised).
 template <int DT>
-__device__ void select_row(const Params& p, Shared& S, int r, int kk) {
+__device__ __noinline__ void select_row(const Params& p, Shared& S, int r, int kk) {
   using E = Elt<DT>;
-  constexpr int VE = E::VE;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const char* row = S.rowp[r];
   TopList T;
   T.reset();
+  // A lower bound on the row's kk-th logit: the kk-th largest of the threads'
+  // maxima over their first units (kk distinct logits reach it), so the
+  // full scan below inserts only logits at or above it.
+  {
+    float mx = kNegInf;
+    if (p.vec) {
+      const uint4* rv = reinterpret_cast<const uint4*>(row);
+      const int nu = (int)(((size_t)p.V * p.esize) / 16);
+#pragma unroll
+      for (int q = 0; q < kPrefixUnits; ++q)
+        if (tid + q * kThreads < nu) mx = fmaxf(mx, E::unit_max(__ldcs(rv + tid + q * kThreads)));
+    } else {
+#pragma unroll
+      for (int q = 0; q < kPrefixUnits; ++q)
+        if (tid + q * kThreads < p.V) mx = fmaxf(mx, E::global(row, tid + q * kThreads));
+    }
+    // kk rounds of a warp maximum over (max, thread) keys, then over the warps'
+    unsigned long long mk = (mx == mx && mx > kNegInf) ? entry_key(mx, tid) : 0ull;
+    for (int t = 0; t < kk; ++t) {
+      const unsigned long long m = warp_max_u64(mk);
+      if (mk == m) mk = 0ull;
+      if (lane == 0) S.wk[warp][t] = m;
+    }
+    __syncthreads();
+    if (warp == 0) {
+      unsigned long long c0, c1, c2, c3;
+      const int e0 = lane, e1 = lane + 32, e2 = lane + 64, e3 = lane + 96;
+      c0 = (e0 % kKMax < kk) ? S.wk[e0 / kKMax][e0 % kKMax] : 0ull;
+      c1 = (e1 % kKMax < kk) ? S.wk[e1 / kKMax][e1 % kKMax] : 0ull;
+      c2 = (e2 % kKMax < kk) ? S.wk[e2 / kKMax][e2 % kKMax] : 0ull;
+      c3 = (e3 % kKMax < kk) ? S.wk[e3 / kKMax][e3 % kKMax] : 0ull;
+      unsigned long long m = 0ull;
+      for (int t = 0; t < kk; ++t) {
+        m = warp_max_u64(max_u64(max_u64(c0, c1), max_u64(c2, c3)));
+        if (m == 0ull) break;
+        if (c0 == m) c0 = 0ull;
+        if (c1 == m) c1 = 0ull;
+        if (c2 == m) c2 = 0ull;
+        if (c3 == m) c3 = 0ull;
+      }
+      // fewer than kk threads saw a logit: no bound
+      if (lane == 0) S.tau0 = (m != 0ull) ? key_val(m) : kNegInf;
+    }
+    __syncthreads();
+    T.floor = S.tau0;
+    T.bound = S.tau0;
+  }
   if (p.vec) {
     // 16-byte units, four in flight per thread
     const uint4* rv = reinterpret_cast<const uint4*>(row);
     const int nu = (int)(((size_t)p.V * p.esize) / 16);
     int u = tid;
     for (; u + 3 * kThreads < nu; u += 4 * kThreads) {
-      uint4 x[4];
-#pragma unroll
-      for (int q = 0; q < 4; ++q) x[q] = __ldcs(rv + u + q * kThreads);
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        if (!(E::unit_max(x[q]) >= T.bound)) continue;
-        float v[VE];
-        E::unpack(x[q], v);
-#pragma unroll
-        for (int e = 0; e < VE; ++e) T.offer(v[e], (u + q * kThreads) * VE + e, kk);
-      }
+      const uint4 x0 = __ldcs(rv + u), x1 = __ldcs(rv + u + kThreads), x2 = __ldcs(rv + u + 2 * kThreads),
+                  x3 = __ldcs(rv + u + 3 * kThreads);
+      scan_unit<DT>(T, x0, u, kk);
+      scan_unit<DT>(T, x1, u + kThreads, kk);
+      scan_unit<DT>(T, x2, u + 2 * kThreads, kk);
+      scan_unit<DT>(T, x3, u + 3 * kThreads, kk);
     }
-    for (; u < nu; u += kThreads) {
-      const uint4 x = __ldcs(rv + u);
-      if (!(E::unit_max(x) >= T.bound)) continue;
-      float v[VE];
-      E::unpack(x, v);
-#pragma unroll
-      for (int e = 0; e < VE; ++e) T.offer(v[e], u * VE + e, kk);
-    }
+    for (; u < nu; u += kThreads) scan_unit<DT>(T, __ldcs(rv + u), u, kk);
   } else {
     // element loads (rows of any length and alignment), four in flight
     int i = tid;
     for (; i + 3 * kThreads < p.V; i += 4 * kThreads) {
-      float v[4];
+      const float v4[4] = {E::global(row, i), E::global(row, i + kThreads), E::global(row, i + 2 * kThreads),
+                           E::global(row, i + 3 * kThreads)};
+      unsigned m = 0u;
 #pragma unroll
-      for (int q = 0; q < 4; ++q) v[q] = E::global(row, i + q * kThreads);
-#pragma unroll
-      for (int q = 0; q < 4; ++q) T.offer(v[q], i + q * kThreads, kk);
+      for (int q = 0; q < 4; ++q) m |= (v4[q] >= T.bound) ? (1u << q) : 0u;
+      while (m) {
+        const int q0 = __ffs(m) - 1;
+        m &= m - 1u;
+        const float x = q0 == 0 ? v4[0] : q0 == 1 ? v4[1] : q0 == 2 ? v4[2] : v4[3];
+        T.insert(x, i + q0 * kThreads, kk);
+      }
     }
-    for (; i < p.V; i += kThreads) T.offer(E::global(row, i), i, kk);
+    for (; i < p.V; i += kThreads) T.insert(E::global(row, i), i, kk);
   }
   // each warp's top kk: kk rounds of a warp maximum over the lists' heads
   for (int t = 0; t < kk; ++t) {
@@ -184,29 +254,23 @@ __device__ void select_row(const Params& p, Shared& S, int r, int kk) {
   __syncthreads();
   if (warp == 0) {
     // the row's top kk from the warps' lists, four candidates per lane
-    unsigned long long c[4];
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const int e = lane + 32 * q, w = e / kKMax, t = e - w * kKMax;
-      c[q] = (t < kk) ? S.wk[w][t] : 0ull;
+    unsigned long long c0, c1, c2, c3;
+    {
+      const int e0 = lane, e1 = lane + 32, e2 = lane + 64, e3 = lane + 96;
+      c0 = (e0 % kKMax < kk) ? S.wk[e0 / kKMax][e0 % kKMax] : 0ull;
+      c1 = (e1 % kKMax < kk) ? S.wk[e1 / kKMax][e1 % kKMax] : 0ull;
+      c2 = (e2 % kKMax < kk) ? S.wk[e2 / kKMax][e2 % kKMax] : 0ull;
+      c3 = (e3 % kKMax < kk) ? S.wk[e3 / kKMax][e3 % kKMax] : 0ull;
     }
     int n = 0;
     for (int t = 0; t < kk; ++t) {
-      unsigned long long best = 0ull;
-      int bq = 0;
-#pragma unroll
-      for (int q = 0; q < 4; ++q)
-        if (c[q] > best) {
-          best = c[q];
-          bq = q;
-        }
+      const unsigned long long best = max_u64(max_u64(c0, c1), max_u64(c2, c3));
       const unsigned long long m = warp_max_u64(best);
       if (m == 0ull) break;
-      if (best == m) {
-#pragma unroll
-        for (int q = 0; q < 4; ++q)
-          if (q == bq) c[q] = 0ull;
-      }
+      if (c0 == m) c0 = 0ull;
+      if (c1 == m) c1 = 0ull;
+      if (c2 == m) c2 = 0ull;
+      if (c3 == m) c3 = 0ull;
       if (lane == 0) {
         S.id[r][t] = key_id(m);
         S.lg[r][t] = key_val(m);
@@ -260,7 +324,8 @@ __device__ void plan(const Params& p, Shared& S, int b, int j, bool bonus) {
       tq = 1.f;
     }
     S.rowc[0] = __fdiv_rn(kLog2e, tq);
-    S.nrows = bonus ? 1 : 1 + __popc(fm);
+    // the single-draft step reads only the first valid branch's model row (row 1)
+    S.nrows = bonus ? 1 : (p.scheme == MDS_SINGLE ? 2 : 1 + __popc(fm));
     S.nv = bonus ? 0 : __popc(vm);
   }
 }
