@@ -89,8 +89,12 @@ typedef struct mds_ctx mds_ctx;
  * renormalised (the non-iid appendix's remark); Algorithm 1 against q / p_a
  * gives Y' (drawn from q / p_a directly when no draft token lies in
  * Omega_0).  Y' is kept with probability p_a (draw 34), otherwise the output
- * is drawn from the tokens outside Omega_0 in proportion to q (draw 35). */
-typedef enum { MDS_SINGLE = 0, MDS_IS = 1, MDS_WIS = 2, MDS_SPECTR = 3, MDS_WIS0 = 4 } mds_scheme;
+ * is drawn from the tokens outside Omega_0 in proportion to q (draw 35).
+ * MDS_WISSORT: MDS_WIS with the sorted rule on Omega_2 (Section 4, Eq. heur
+ * and Eq. p_Ieq; the non-iid appendix): a pair of tokens outside Omega_1
+ * selects the one earlier in key order (larger q - a b, then lower id).
+ * Served with top_k > 0 only (MDS_EUNSUP otherwise). */
+typedef enum { MDS_SINGLE = 0, MDS_IS = 1, MDS_WIS = 2, MDS_SPECTR = 3, MDS_WIS0 = 4, MDS_WISSORT = 5 } mds_scheme;
 
 /* Storage type of the logits. */
 typedef enum { MDS_F32 = 0, MDS_BF16 = 1 } mds_dtype;
@@ -129,7 +133,7 @@ typedef struct {
                       draft tokens should come from the restricted draft rows
                       (a token outside them has p_I = 0 and is accepted, as
                       Algorithm 1 reads a zero denominator).  Served for
-                      MDS_SINGLE, MDS_WIS and MDS_SPECTR by the top-k kernel
+                      MDS_SINGLE, MDS_WIS, MDS_SPECTR and MDS_WISSORT by the top-k kernel
                       (one CTA per sequence, no cluster); MDS_IS and MDS_WIS0
                       return MDS_EUNSUP.  acc_prob and out_diag as above.     */
 } mds_config;

@@ -59,8 +59,7 @@ from . import is_laplace
 from . import truncated
 from . import sorted_lp
 
-SCHEMES = {"single": 0, "IS": 1, "WIS": 2, "SpecTr": 3, "WIS0": 4,
-           "WISsort": None}   # None: no device scheme id (the oracle alone has it)
+SCHEMES = {"single": 0, "IS": 1, "WIS": 2, "SpecTr": 3, "WIS0": 4, "WISsort": 5}
 
 # Band thresholds (absolute, on quantities in [0, 1] or scaled as stated).
 BAND_ACCEPT = 1e-6   # |u - min(1, q(Y)/p_I(Y))|

@@ -273,7 +273,8 @@ static int verify_impl(mds_ctx* ctx, const void* target_logits, const void* cons
                        float* out_diag, int B, void* stream, bool bulk_ok) {
   if (!ctx) return MDS_EINVAL;
   const mds_config& c = ctx->cfg;
-  if (scheme < MDS_SINGLE || scheme > MDS_WIS0) return MDS_EINVAL;
+  if (scheme < MDS_SINGLE || scheme > MDS_WISSORT) return MDS_EINVAL;
+  if (scheme == MDS_WISSORT && c.top_k <= 0) return MDS_EUNSUP;   // the top-k kernel's scheme only
   if (B < 0 || B > c.max_B) return MDS_ESHAPE;
   if (B == 0) return MDS_OK;
   if (!target_logits || !draft_logits || !draft_model_id || !draft_tokens || !temperatures || !out_tokens ||

@@ -1,8 +1,7 @@
-// Device helpers shared by the two verification engines (mds_kernel.cu, the
-// per-sequence engine, and mds_flow.cu, the slice-dataflow engine): inline
-// PTX wrappers, the counter-based random numbers, logit IO, the exponent
-// convention of every probability, and the stage maximum flow of the
-// weighted scheme.  Not part of the public ABI.
+// Device helpers of the slice-dataflow engine (mds_flow.cu) and the top-k
+// kernel (mds_topk.cu): inline PTX wrappers, the counter-based random
+// numbers, logit IO, the exponent convention of every probability, and the
+// stage maximum flow of the weighted scheme.  Not part of the public ABI.
 #pragma once
 #include <cuda_bf16.h>
 

@@ -76,7 +76,8 @@ extern "C" int mds_verify_noalloc(const mds_config* cfg_in, int device, const vo
   if (c.wis_s < 1 || c.wis_s > MDS_MAX_S || !(c.is_h > 0.f) || c.is_h > 4.f) return MDS_EINVAL;
   if (c.cluster != 0 && c.cluster != 1 && c.cluster != 2 && c.cluster != 4 && c.cluster != 8 && c.cluster != 16)
     return MDS_EINVAL;
-  if (scheme < MDS_SINGLE || scheme > MDS_WIS0) return MDS_EINVAL;
+  if (scheme < MDS_SINGLE || scheme > MDS_WISSORT) return MDS_EINVAL;
+  if (scheme == MDS_WISSORT && c.top_k <= 0) return MDS_EUNSUP;   // the top-k kernel's scheme only
   if (B < 0 || B > c.max_B) return MDS_ESHAPE;
   if (device < 0 || device >= kMaxDevices) return MDS_EINVAL;
   if (B == 0) return MDS_OK;

@@ -10,6 +10,10 @@
 //     q - a b over the whole vocabulary (ties to the lower id): the positive
 //     keys of U, then zero keys (tokens outside U and tokens of U with a zero
 //     key) by increasing id, then negative keys;
+//   * WIS with the sorted rule on Omega_2 (Section 4 Eq. heur, Eq. p_Ieq):
+//     the same stages, a pair inside Omega_2 selecting the token earlier in
+//     key order; its Omega_2 law needs each token's key-ordered suffix
+//     masses, a sum over U;
 //   * SpecTr: sequential rejection over the valid drafts.
 // Tokens outside U carry zero mass in every law, so the inverse CDFs in
 // token-id order (residual, bonus) run over U sorted by id.
@@ -55,6 +59,8 @@ struct Shared {
   float law[kRowsMax][kEntMax];
   float cur[kEntMax];                     // running law (stage output law, SpecTr target)
   float key[kEntMax];                     // stage keys q - a b
+  float nxt[kEntMax];                     // the sorted rule's Omega_2 law, before it replaces cur
+  unsigned char in1[kEntMax];             // U entry is in Omega_1 of the current stage
   short rank[kEntMax];                    // position in U of each kept entry
   unsigned char dup[kEntMax];             // entry repeats a token of an earlier entry
   int nU;
@@ -495,8 +501,12 @@ __device__ int next_key(const Shared& S, int sign, float lk, int lid, float* bk_
 // Warp 0: one pairwise stage of the weighted scheme with input laws
 // a = S.cur (the running law) and b = S.law[rb] against q = S.law[0]; ordered
 // inputs (A, Btok) and selection uniform u.  Returns the stage's token and
-// leaves its output law in S.cur.
-__device__ int wis_stage(const Params& p, Shared& S, int A, int Btok, int rb, float u) {
+// leaves its output law in S.cur.  With `sorted`, Omega_2 follows the sorted
+// rule of the truncated LP (Section 4 Eq. heur and Eq. p_Ieq, the non-iid
+// appendix): a pair inside Omega_2 selects the token earlier in key order, so
+// p_I(k) = a_k b_k + b_k A_after(k) + a_k B_after(k) with the Omega_2 masses
+// of the tokens after k; otherwise the variant's 1/2 rule.
+__device__ int wis_stage(const Params& p, Shared& S, int A, int Btok, int rb, float u, bool sorted) {
   const int lane = threadIdx.x & 31;
   const int nU = S.nU;
   const float* q = S.law[0];
@@ -575,12 +585,31 @@ __device__ int wis_stage(const Params& p, Shared& S, int A, int Btok, int rb, fl
   for (int i = lane; i < nU; i += 32) {
     bool in1 = false;
     for (int t = 0; t < s; ++t) in1 |= (S.om_in[t] && S.om_u[t] == i);
+    S.in1[i] = in1 ? 1 : 0;
     if (!in1) {
       sa = __fadd_rn(sa, S.cur[i]);
       sb = __fadd_rn(sb, bl[i]);
     }
   }
   const float A2 = warp_sum(sa), B2 = warp_sum(sb);
+  __syncwarp();
+  if (sorted) {
+    // Omega_2 values of the sorted rule (tokens outside U carry no mass)
+    for (int i = lane; i < nU; i += 32) {
+      if (S.in1[i]) continue;
+      const float ki = S.key[i];
+      const int idi = S.uid[i];
+      float aa = 0.f, ba = 0.f;
+      for (int j = 0; j < nU; ++j)
+        if (!S.in1[j] && better(ki, idi, S.key[j], S.uid[j])) {
+          aa = __fadd_rn(aa, S.cur[j]);
+          ba = __fadd_rn(ba, bl[j]);
+        }
+      const float ai = S.cur[i], bi = bl[i];
+      S.nxt[i] = __fadd_rn(__fadd_rn(__fmul_rn(ai, bi), __fmul_rn(bi, aa)), __fmul_rn(ai, ba));
+    }
+    __syncwarp();
+  }
   if (lane == 0) {
     bool capped = false;
     int y;
@@ -592,15 +621,30 @@ __device__ int wis_stage(const Params& p, Shared& S, int A, int Btok, int rb, fl
                                  S.FH);
     }
     if (capped) atomicOr(p.status, MDS_ST_LP_CAP);
+    if (sorted && A != Btok) {
+      // both inputs in Omega_2: the one earlier in key order (a token outside U has key 0)
+      bool ia = false, ib = false;
+      for (int t = 0; t < s; ++t) {
+        ia |= (S.om[t] == A);
+        ib |= (S.om[t] == Btok);
+      }
+      if (!ia && !ib) {
+        const int ua = find_u(S, A), ub = find_u(S, Btok);
+        const float ka = ua >= 0 ? S.key[ua] : 0.f, kb = ub >= 0 ? S.key[ub] : 0.f;
+        y = better(ka, A, kb, Btok) ? A : Btok;
+      }
+    }
     S.Y = y;
   }
   __syncwarp();
-  // the stage's output law: p_I on Omega_1 from the LP, (a B2 + b A2) / 2 elsewhere
+  // the stage's output law: p_I on Omega_1 from the LP; on Omega_2 the sorted
+  // rule's values or (a B2 + b A2) / 2
   for (int i = lane; i < nU; i += 32) {
     int pos = -1;
     for (int t = 0; t < s; ++t)
       if (S.om_in[t] && S.om_u[t] == i) pos = t;
     S.cur[i] = (pos >= 0) ? S.om_x[pos]
+               : sorted   ? S.nxt[i]
                           : __fmul_rn(0.5f, __fadd_rn(__fmul_rn(S.cur[i], B2), __fmul_rn(bl[i], A2)));
   }
   const int y = S.Y;
@@ -702,12 +746,14 @@ __device__ __noinline__ void decide(const Params& p, Shared& S, int b, int j) {
   } else {
     int Y = S.X[0];
     const float* a = S.law[S.vrow[0]];
-    if (p.scheme == MDS_WIS && nv > 1) {
+    if ((p.scheme == MDS_WIS || p.scheme == MDS_WISSORT) && nv > 1) {
       for (int i = lane; i < S.nU; i += 32) S.cur[i] = a[i];
       __syncwarp();
       // every stage's selection uniform at once (lane m - 1 draws stage m's)
       const float ul = (lane + 1 < nv) ? draw_uniform(p.seed, b, j, kDrawSelect + lane) : 0.f;
-      for (int m = 1; m < nv; ++m) Y = wis_stage(p, S, Y, S.X[m], S.vrow[m], __shfl_sync(FULL, ul, m - 1));
+      const bool sorted = p.scheme == MDS_WISSORT;
+      for (int m = 1; m < nv; ++m)
+        Y = wis_stage(p, S, Y, S.X[m], S.vrow[m], __shfl_sync(FULL, ul, m - 1), sorted);
       a = S.cur;
     }
     Z = accept_resid(p, S, b, j, Y, a, &R, &qY, &pIY);

@@ -34,7 +34,9 @@ struct Params {
 };
 
 // Schemes the kernel serves.
-inline bool serves(int scheme) { return scheme == MDS_SINGLE || scheme == MDS_WIS || scheme == MDS_SPECTR; }
+inline bool serves(int scheme) {
+  return scheme == MDS_SINGLE || scheme == MDS_WIS || scheme == MDS_SPECTR || scheme == MDS_WISSORT;
+}
 
 // One CTA per sequence on `stream`.
 cudaError_t launch(const Params& p, cudaStream_t stream);

@@ -19,8 +19,9 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 # libmds_timers.so); the default is the in-tree libmds.so.
 LIB_PATH = os.environ.get("MDS_LIBRARY") or os.path.join(_HERE, "_lib", "libmds.so")
 
-MDS_SINGLE, MDS_IS, MDS_WIS, MDS_SPECTR, MDS_WIS0 = 0, 1, 2, 3, 4
-SCHEMES = {"single": MDS_SINGLE, "IS": MDS_IS, "WIS": MDS_WIS, "SpecTr": MDS_SPECTR, "WIS0": MDS_WIS0}
+MDS_SINGLE, MDS_IS, MDS_WIS, MDS_SPECTR, MDS_WIS0, MDS_WISSORT = 0, 1, 2, 3, 4, 5
+SCHEMES = {"single": MDS_SINGLE, "IS": MDS_IS, "WIS": MDS_WIS, "SpecTr": MDS_SPECTR, "WIS0": MDS_WIS0,
+           "WISsort": MDS_WISSORT}
 MDS_F32, MDS_BF16 = 0, 1
 DTYPES = {"f32": MDS_F32, "bf16": MDS_BF16}
 TORCH_DTYPES = {MDS_F32: torch.float32, MDS_BF16: torch.bfloat16}

@@ -6,8 +6,9 @@ the lower id) and renormalises (oracle/truncated.py:top_filter) before the
 scheme runs; the top-k kernel selects each visited row's top k and runs the
 scheme on the union of the kept tokens.  Cases: k from 1 to the largest, f32
 and bf16 rows, rows fetched by 16-byte units and by element loads (ragged V),
-one and two draft models, s = 8 (the shared-memory LP), V below k and below
-s (zero-key tokens outside the union fill Omega_1), draft tokens drawn
+one and two draft models, the variant (WIS) and the sorted rule (WISsort) on
+Omega_2, s = 8 (the shared-memory LP), V below k and below s (zero-key tokens
+outside the union fill Omega_1), draft tokens drawn
 without the restriction (p_I(Y) = 0), acc_prob, the allocation-free entry
 point, and sampled sequences of the full-size workload.
 """
@@ -68,35 +69,36 @@ CASES = [
 @pytest.mark.parametrize("top_k", [5, 10])
 def test_paper_top_k_matches_oracle(name, kw, top_k):
     spec = WORKLOADS[name].with_(top_k=top_k, **kw)
-    for scheme in ("WIS", "single", "SpecTr"):
+    for scheme in ("WIS", "WISsort", "single", "SpecTr"):
         ok(run_topk(spec, scheme, seed=7 + top_k, top_k=top_k), scheme)
 
 
 @pytest.mark.parametrize("top_k", [1, 2, 16])
 def test_extreme_k(top_k):
     spec = WORKLOADS["llama2-32k"].with_(B=10, V=4099, K=3, model_ids=[0, 0, 0], top_k=top_k)
-    for scheme in ("WIS", "single", "SpecTr"):
+    for scheme in ("WIS", "WISsort", "single", "SpecTr"):
         ok(run_topk(spec, scheme, seed=3, top_k=top_k), scheme)
 
 
 def test_largest_s_uses_the_shared_memory_lp():
     spec = WORKLOADS["llama3-128k"].with_(B=8, V=6000, top_k=10)
-    ok(run_topk(spec, "WIS", seed=5, top_k=10, wis_s=8), "WIS")
-    ok(run_topk(spec, "WIS", seed=6, top_k=10, wis_s=1), "WIS")
+    for scheme in ("WIS", "WISsort"):
+        ok(run_topk(spec, scheme, seed=5, top_k=10, wis_s=8), scheme)
+        ok(run_topk(spec, scheme, seed=6, top_k=10, wis_s=1), scheme)
 
 
 def test_vocabulary_smaller_than_k_and_s():
     # V = 3: every row keeps the whole vocabulary; s = min(5, V)
     spec = WORKLOADS["tiny"].with_(B=16, V=3, K=4, model_ids=[0, 1, 0, 1], draft_sigma=[0.7, 1.5],
                                    t_draft=[1.0, 0.8], top_k=5)
-    for scheme in ("WIS", "single", "SpecTr"):
+    for scheme in ("WIS", "WISsort", "single", "SpecTr"):
         ok(run_topk(spec, scheme, seed=2, top_k=5), scheme)
 
 
 def test_draft_tokens_outside_the_restriction():
     # tokens drawn from the unrestricted draft rows: p_I(Y) = 0 accepts Y
     spec = WORKLOADS["llama2-32k"].with_(B=12, V=3001)
-    for scheme in ("WIS", "single", "SpecTr"):
+    for scheme in ("WIS", "WISsort", "single", "SpecTr"):
         ok(run_topk(spec, scheme, seed=9, top_k=5), scheme)
 
 
@@ -127,6 +129,13 @@ def test_unserved_schemes_refused():
         with pytest.raises(mds.MdsError) as e:
             v.verify(w.target, w.draft_list(), w.model_ids, w.tokens, w.temps, scheme, 1)
         assert e.value.code == mds.MDS_EUNSUP
+    torch.cuda.synchronize()
+    v.close()
+    # the sorted rule is served on restricted rows only
+    v = mds.Verifier(spec.B, spec.K, spec.L, spec.V, dtype=spec.dtype)
+    with pytest.raises(mds.MdsError) as e:
+        v.verify(w.target, w.draft_list(), w.model_ids, w.tokens, w.temps, "WISsort", 1)
+    assert e.value.code == mds.MDS_EUNSUP
     torch.cuda.synchronize()
     v.close()
 
