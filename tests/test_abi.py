@@ -60,7 +60,8 @@ def test_create_rejects_bad_config_before_touching_a_device():
             mds.mds_create(**c)
         assert e.value.code == mds.MDS_ESHAPE
     for c in (dict(wis_s=9), dict(is_h=-1.0), dict(cluster=3), dict(dtype=7), dict(omega0=-2),
-              dict(omega0=mds.MDS_MAX_OMEGA0 + 1), dict(acc_prob=2), dict(acc_prob=-1)):
+              dict(omega0=mds.MDS_MAX_OMEGA0 + 1), dict(acc_prob=2), dict(acc_prob=-1), dict(top_k=-1),
+              dict(top_k=mds.MDS_MAX_TOPK + 1)):
         with pytest.raises(mds.MdsError) as e:
             mds.mds_create(4, 2, 4, 100, **c)
         assert e.value.code == mds.MDS_EINVAL
@@ -90,6 +91,7 @@ def test_binding_config_matches_the_header():
         assert ids["MDS_" + name.upper()] == sid
     assert int(re.search(r"#define MDS_MAX_OMEGA0 (\d+)", text).group(1)) == mds.MDS_MAX_OMEGA0
     assert int(re.search(r"#define MDS_ST_OMEGA0 (\d+)u", text).group(1)) == mds.MDS_ST_OMEGA0
+    assert int(re.search(r"#define MDS_MAX_TOPK (\d+)", text).group(1)) == mds.MDS_MAX_TOPK
 
 
 def test_header_compiles_as_c_and_matches_the_binding_layout(tmp_path):

@@ -1,6 +1,7 @@
 """Host logic of bench.py: the vocab-row and algorithmic-byte accounting
 replayed from a walk's outputs, for WIS (every visited row streamed) and the
-truncated alphabet (target rows streamed, draft rows read at Omega_0)."""
+truncated alphabet (target rows streamed, draft rows read at Omega_0); the
+kernel a call runs and the recorded DRAM traffic of its current source."""
 import os
 import sys
 
@@ -42,3 +43,22 @@ def test_truncated_alphabet_counts_target_rows_and_point_loads():
     # Omega_0 larger than the vocabulary reads each draft row in full at most
     _, small = bench.walk_accounting(tokens, mids, out, acc, 8, es, "WIS0", M)
     assert small == (rows - draft_rows) * 8 * es + draft_rows * 8 * es + io
+
+
+def test_kernel_names_and_recorded_traffic():
+    assert bench.kernel_name("WIS", 0) == "flow_kernel"
+    assert bench.kernel_name("WIS", 2) == "verify_kernel"
+    assert bench.kernel_name("SpecTr", 0) == "verify_kernel"
+    assert bench.kernel_name("WIS", 0, top_k=10) == "topk_kernel"
+    # every committed record names its kernel and matches that kernel's
+    # current source, so the bench line reports it; another kernel's record
+    # or a stale hash reads as unknown
+    import json
+    d = json.load(open(os.path.join(bench.ROOT, "profiles", "traffic.json")))
+    for key, e in d.items():
+        parts = key.split("/")
+        top_k = int(parts[2][3:]) if len(parts) > 2 else 0
+        assert bench.recorded_traffic(parts[0], parts[1], e["kernel"], top_k) == e["dram_bytes_per_launch"]
+        other = "verify_kernel" if e["kernel"] != "verify_kernel" else "flow_kernel"
+        assert bench.recorded_traffic(parts[0], parts[1], other, top_k) is None
+    assert bench.recorded_traffic("llama3-128k", "WIS", "flow_kernel", 5) is None
