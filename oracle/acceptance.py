@@ -5,10 +5,10 @@ TEST INFRASTRUCTURE ONLY (see ``oracle/__init__``).  Plain fp64 numpy.
 For a target law q and the valid branches' draft laws, the probability that
 a depth accepts one of the draft tokens:
 
-single, IS, WIS   Theorem 1: sum_k min(q_k, p_I(k)) with p_I the law of the
-                  intermediate token (the draft law itself; the Laplace
+single, IS, WIS,  Theorem 1: sum_k min(q_k, p_I(k)) with p_I the law of the
+WISsort           intermediate token (the draft law itself; the Laplace
                   identity of ``is_laplace``; the pairwise stage chain of
-                  ``wis``).
+                  ``wis``, or of ``sorted_lp`` for the sorted rule).
 SpecTr            the sequential-rejection reading: 1 - prod_i R_i, R_i the
                   residual mass left after round i.
 WIS0              the truncated alphabet (Section 4): p_a = q(Omega_0) times
@@ -21,13 +21,13 @@ optimal           Theorem 3 for K = 2 i.i.d. drafts and Remark 2's
 
 Running the module prints these for depth 0 of a few sequences of every
 named synthetic workload (the counterpart of the paper's Table 2 on the
-stand-in rows):  python -m oracle.acceptance [--top-p=0.95] [workload ...]
+stand-in rows):  python -m oracle.acceptance [--top-p=0.95] [--top-k=5] [workload ...]
 """
 import itertools
 
 import numpy as np
 
-from . import enum, is_laplace, theory, truncated
+from . import enum, is_laplace, sorted_lp, theory, truncated
 
 
 def scheme_acceptance(q, dists, mids, scheme, s=5, is_h=0.25):
@@ -38,6 +38,11 @@ def scheme_acceptance(q, dists, mids, scheme, s=5, is_h=0.25):
         return float(np.minimum(q, dists[0]).sum())
     if scheme == "WIS":
         pI = enum.wis_stages(q, dists, s)[-1].pI
+        return float(np.minimum(q, pI).sum())
+    if scheme == "WISsort":
+        pI = np.asarray(dists[0], dtype=np.float64)
+        for d in dists[1:]:
+            pI = sorted_lp.stage(q, pI, d, s).pI
         return float(np.minimum(q, pI).sum())
     if scheme == "IS":
         rows, counts = {}, {}
@@ -96,10 +101,11 @@ def _softmax(x, t):
     return e / e.sum()
 
 
-def table(names=None, seqs=(0, 1, 2, 3), top_p=1.0):
-    """Rows of (workload, sequence, K, single, IS, WIS, WIS0, SpecTr,
-    optimal) at depth 0, every row top-p filtered first when top_p < 1
-    (Section 5); IS is skipped above 60000 tokens (its quadrature costs V x T)."""
+def table(names=None, seqs=(0, 1, 2, 3), top_p=1.0, top_k=0):
+    """Rows of (workload, sequence, K, single, IS, WIS, WISsort, WIS0,
+    SpecTr, optimal) at depth 0, every row top-k / top-p filtered first when
+    set (Section 5); IS is skipped above 60000 tokens (its quadrature costs
+    V x T)."""
     from synth import WORKLOADS, make_workload
     out = []
     for name in names or list(WORKLOADS):
@@ -109,12 +115,12 @@ def table(names=None, seqs=(0, 1, 2, 3), top_p=1.0):
             temps = w.temps[b].double().numpy()
             q = _softmax(w.target[b, 0, 0].float().numpy(), temps[0])
             dists = [_softmax(w.drafts[k, b, 0].float().numpy(), temps[1 + k]) for k in range(spec.K)]
-            if top_p < 1.0:
-                q = truncated.top_filter(q, top_p=top_p)
-                dists = [truncated.top_filter(d, top_p=top_p) for d in dists]
+            if top_p < 1.0 or top_k > 0:
+                q = truncated.top_filter(q, top_k=top_k, top_p=top_p)
+                dists = [truncated.top_filter(d, top_k=top_k, top_p=top_p) for d in dists]
             mids = list(spec.model_ids)
             row = {"workload": name, "b": b, "K": spec.K}
-            for sch in ("single", "IS", "WIS", "SpecTr"):
+            for sch in ("single", "IS", "WIS", "WISsort", "SpecTr"):
                 if sch == "IS" and spec.V > 60000:
                     row[sch] = None
                     continue
@@ -129,13 +135,20 @@ def table(names=None, seqs=(0, 1, 2, 3), top_p=1.0):
 if __name__ == "__main__":
     import sys
     args = sys.argv[1:]
-    tp = 1.0
-    if args and args[0].startswith("--top-p="):
-        tp = float(args.pop(0).split("=", 1)[1])
-    rows = table(args or None, top_p=tp)
-    print("| workload | b | K | single | IS | WIS (s = 5) | WIS0 (M = 20) | SpecTr reading | optimal (Thm 3 / Remark 2) |")
-    print("|---|---|---|---|---|---|---|---|---|")
+    tp, tk = 1.0, 0
+    while args and args[0].startswith("--"):
+        opt, val = args.pop(0).split("=", 1)
+        if opt == "--top-p":
+            tp = float(val)
+        elif opt == "--top-k":
+            tk = int(val)
+        else:
+            raise SystemExit(f"unknown option {opt}")
+    rows = table(args or None, top_p=tp, top_k=tk)
+    print("| workload | b | K | single | IS | WIS (s = 5) | WISsort (s = 5) | WIS0 (M = 20) | SpecTr reading | "
+          "optimal (Thm 3 / Remark 2) |")
+    print("|---|---|---|---|---|---|---|---|---|---|")
     f = lambda v: "—" if v is None else f"{v:.4f}"   # noqa: E731
     for r in rows:
         print(f"| {r['workload']} | {r['b']} | {r['K']} | {f(r['single'])} | {f(r['IS'])} | {f(r['WIS'])} | "
-              f"{f(r['WIS0'])} | {f(r['SpecTr'])} | {f(r['optimal'])} |")
+              f"{f(r['WISsort'])} | {f(r['WIS0'])} | {f(r['SpecTr'])} | {f(r['optimal'])} |")

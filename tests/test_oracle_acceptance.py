@@ -61,7 +61,7 @@ def test_accept_rate_matches(scheme):
 
 
 def test_analytic_evaluator_matches_the_walk_and_the_ceiling():
-    """oracle.acceptance: single / IS / WIS equal 1 - R of the walk's depth 0;
+    """oracle.acceptance: single / IS / WIS / WISsort equal 1 - R of the walk's depth 0;
     every scheme stays below Theorem 3's optimum for K = 2 i.i.d. drafts (the
     optimum over all token-level selection rules)."""
     from oracle import acceptance
@@ -70,7 +70,7 @@ def test_analytic_evaluator_matches_the_walk_and_the_ceiling():
         tl, dr, mids, tok, temps, q, p = _rows(V, B, 2, 1, seed=40 + seed)
         best = theory.thm3_pstar(p, q)
         assert acceptance.optimal_acceptance(q, p, 2) == pytest.approx(best, abs=1e-12)
-        for scheme in ("single", "IS", "WIS", "SpecTr"):
+        for scheme in ("single", "IS", "WIS", "WISsort", "SpecTr"):
             val = acceptance.scheme_acceptance(q, [p, p], [0, 0], scheme)
             assert val <= best + 1e-9, (scheme, val, best)
             if scheme == "SpecTr":
