@@ -122,3 +122,27 @@ def test_truncated_evaluator_matches_enumeration():
             want += pr * sum(by * min(1.0, qt[y] / pI[y]) for y, by in beta.items())
         got = acceptance.truncated_acceptance(q, dists, M, s=2)
         assert got == pytest.approx(pa * want, abs=1e-12)
+
+
+def test_wis_reaches_theorem3_when_the_target_keeps_at_most_s_tokens():
+    """A positive key q - p^2 needs q > 0, so with at most s target tokens
+    every positive key lies in Omega_1; a target token with a negative key
+    already has p_I >= p^2 > q, and tokens outside the target's support add
+    nothing to sum min(q, p_I).  The truncated LP (either Omega_2 rule) then
+    attains the full optimum: Theorem 3 for K = 2 i.i.d. drafts, up to the
+    stage LP's saturation threshold (residuals at or below 1e-6 of the
+    stage's mass count as zero, so a few such residuals may stay unserved).
+    Checked on top-k restricted rows (Section 5's setting) with s = 5."""
+    from oracle import acceptance, truncated
+    rng = np.random.default_rng(21)
+    for trial in range(40):
+        V = int(rng.integers(6, 60))
+        k = int(rng.integers(1, 6))
+        q = truncated.top_filter(rng.dirichlet(np.full(V, 0.5)), top_k=k)
+        p = rng.dirichlet(np.full(V, 0.5))
+        if trial % 2:
+            p = truncated.top_filter(p, top_k=int(rng.integers(1, 12)))
+        best = acceptance.optimal_acceptance(q, p, 2)
+        for scheme in ("WIS", "WISsort"):
+            val = acceptance.scheme_acceptance(q, [p, p], [0, 0], scheme)
+            assert best - 1e-5 <= val <= best + 1e-9, (trial, scheme, val, best)
