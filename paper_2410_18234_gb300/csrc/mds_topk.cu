@@ -20,11 +20,14 @@
 //
 // One CTA of 256 threads verifies one sequence.  Per depth: warp 0 plans the
 // rows (the target row of the lowest valid branch, one draft row per model
-// among the valid branches, read from its lowest valid branch); every thread
-// scans its strided share of a row keeping a sorted list of its 16 largest
-// (logit, -id) keys, the warps merge their lists into the row's top k; warp 0
-// then computes the kept entries' probabilities, the union, the scheme's
-// decision and the walk.
+// among the valid branches, read from its lowest valid branch; the single
+// draft step reads only the first valid branch's).  For each row, every
+// thread first takes the maximum of its first units; the k-th largest of
+// those maxima bounds the row's k-th logit from below.  Then every thread
+// scans its strided share of the row, keeping a sorted list of its 16
+// largest (logit, -id) keys at or above that bound, and the warps merge the
+// lists into the row's top k.  Warp 0 then computes the kept entries'
+// probabilities, the union, the scheme's decision and the walk.
 #include "mds_device.cuh"
 #include "mds_topk.h"
 
